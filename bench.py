@@ -1,0 +1,428 @@
+"""Benchmark of the block-sparse inference hot path on GB300.
+
+Workload: the block-sparse GEMM M = K = N = 4096, bf16, block-based pruning
+with bm = 128 rows x bk = 32 columns keeping 1/4 of the columns of every block
+(4x rate) -- the point on which the effective-TFLOP/s target is stated.  One
+step is one bp_gemm call (gather-GEMM on the tensor cores + fused epilogue)
+on one batch X (4096 x 4096); the weights are pruned (bp_prune) and packed
+(bp_pack) once before timing, their times are reported under "offline".
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+One JSON line on stdout (rank 0).  Under torchrun each rank runs an
+independent replica on its own GPU (no collective on the data path) and the
+value is the work of all ranks divided by the slowest rank's time.
+--impl reference times the CPU oracle (plain fp64 C loops) on a bounded
+sample of the same workload on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "effective TFLOP/s (kept-weight FLOPs)"
+UNIT = "TFLOP/s"
+WORKLOAD = dict(M=4096, K=4096, N=4096, bm=128, bk=32, rate=4.0, dtype="bf16")
+L2_BYTES = 129 * 2 ** 20
+
+
+def workload_name(w=WORKLOAD) -> str:
+    return (f"block-sparse GEMM {w['M']}x{w['K']}x{w['N']} {w['dtype']}, block-based "
+            f"bm={w['bm']} bk={w['bk']}, keep 1/{w['rate']:g} of the columns per block")
+
+
+# ----------------------------------------------------------------------- helpers
+def read_peaks() -> dict:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        d["_source"] = "measured"
+        return d
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "_source": "fallback"}
+
+
+def kernel_source_sha() -> str:
+    h = hashlib.sha256()
+    for f in ("bp_mma.cu", "bp_common.cuh", "bp_internal.h"):
+        with open(os.path.join(ROOT, "paper_2111_11581_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel source; else None."""
+    p = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(workload)
+    if not e or e.get("kernel_src_sha") != kernel_source_sha():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """Samples SM clock and clock-event reasons through NVML (ctypes) while running."""
+    REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
+               0x8: "hw_slowdown", 0x10: "sync_boost", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown",
+               0x100: "display_clock_setting"}
+
+    def __init__(self, index: int, period_s: float = 0.01):
+        self.index, self.period = index, period_s
+        self.samples, self.reasons, self.max_mhz = [], set(), None
+        self._stop = threading.Event()
+        self._nvml = None
+        try:
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() == 0:
+                h = ctypes.c_void_p()
+                if nv.nvmlDeviceGetHandleByIndex_v2(index, ctypes.byref(h)) == 0:
+                    self._nvml, self._h = nv, h
+                    m = ctypes.c_uint()
+                    if nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(m)) == 0:
+                        self.max_mhz = m.value
+        except OSError:
+            self._nvml = None
+
+    def _once(self):
+        nv, h = self._nvml, self._h
+        c = ctypes.c_uint()
+        if nv.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(c)) == 0:
+            self.samples.append(c.value)
+        r = ctypes.c_ulonglong()
+        if nv.nvmlDeviceGetCurrentClocksEventReasons(h, ctypes.byref(r)) == 0:
+            for bit, name in self.REASONS.items():
+                if r.value & bit:
+                    self.reasons.add(name)
+
+    def _run(self):
+        while not self._stop.is_set():
+            self._once()
+            time.sleep(self.period)
+
+    def __enter__(self):
+        if self._nvml is not None:
+            self._t = threading.Thread(target=self._run, daemon=True)
+            self._t.start()
+        return self
+
+    def __exit__(self, *a):
+        if self._nvml is not None:
+            self._stop.set()
+            self._t.join()
+            self._once()
+
+    def summary(self) -> dict:
+        return {"sm_mhz": statistics.median(self.samples) if self.samples else None,
+                "sm_max_mhz": self.max_mhz, "samples": len(self.samples),
+                "reasons": sorted(self.reasons - {"gpu_idle"})}
+
+
+def aggregate(local_seconds: float, local_units: float, world: int, reduce_max, reduce_sum):
+    """Whole-job throughput: units of all ranks / the slowest rank's time."""
+    t = reduce_max(local_seconds)
+    u = reduce_sum(local_units)
+    return u / t, t
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+# ----------------------------------------------------------------------- our arm
+def run_ours(args):
+    import numpy as np
+    import torch
+
+    from paper_2111_11581_gb300 import bp, build, inputs
+
+    world, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    build.build()
+    bp.load()
+    w = WORKLOAD
+    dtype = bp.BF16 if w["dtype"] == "bf16" else bp.F16
+    L = inputs.gemm_point(w["M"], w["K"], w["N"], w["bm"], w["bk"], w["rate"], dtype)
+    W = inputs.layer_weight(L, dtype)
+    X = inputs.layer_input(L, dtype)
+    lay = bp.layout(bp.BLOCK_BASED, dtype, L.M, L.K, L.bm, L.bk)
+    Wd = inputs.as_torch(W, dtype).cuda()
+    # offline: prune + pack (timed once, not part of a step)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    mask = bp.prune(lay, Wd, L.rate)
+    t1 = time.perf_counter()
+    pw = bp.pack(lay, Wd, mask)
+    torch.cuda.synchronize()
+    t2 = time.perf_counter()
+    nnz_vals = int(pw.c.nnz_vals)
+    flops = 2.0 * nnz_vals * L.N
+    # rotating buffer sets: > 2x L2 in total so every step reads from HBM
+    set_bytes = pw.dev.numel() + 2 * L.K * L.N + 2 * L.M * L.N
+    R = max(2, -(-2 * L2_BYTES // set_bytes))
+    Xd0 = inputs.as_torch(X, dtype).cuda()
+    sets = []
+    for i in range(R):
+        dev = pw.dev.clone()
+        c = bp.Packed(pw.c.lay, pw.c.num_rb, pw.c.nnz_cols, pw.c.nnz_vals, pw.c.rb_ptr,
+                      pw.c.col_idx, pw.c.values, dev.data_ptr(), pw.c.dev_bytes)
+        Xi = Xd0.clone()
+        Yi = torch.empty((L.M, L.N), dtype=Xd0.dtype, device="cuda")
+        sets.append((c, dev, Xi, Yi))
+    stream = torch.cuda.current_stream()
+    sp = int(stream.cuda_stream)
+
+    def step(i):
+        c, _, Xi, Yi = sets[i % R]
+        st = bp.bp_gemm(c, Xi.data_ptr(), L.N, L.N, None, 0, Yi.data_ptr(), L.N, sp)
+        if st != bp.OK:
+            raise bp.BpError(st, "bp_gemm")
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    if bp.device_status() != bp.OK:
+        raise RuntimeError("kernel watchdog fired during warm-up")
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with sampler:
+        ev0.record(stream)
+        for i in range(args.steps):
+            step(i)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    ms_total = ev0.elapsed_time(ev1)
+    if bp.device_status() != bp.OK:
+        raise RuntimeError("kernel watchdog fired during the timed region")
+    local_s = ms_total / 1e3
+    if dist:
+        def rmax(v):
+            t = torch.tensor([v], dtype=torch.float64, device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            return float(t.item())
+
+        def rsum(v):
+            t = torch.tensor([v], dtype=torch.float64, device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.SUM)
+            return float(t.item())
+    else:
+        rmax = rsum = (lambda v: v)
+    value_flops, tmax = aggregate(local_s, flops * args.steps, world, rmax, rsum)
+    value = value_flops / 1e12
+    ms_per_step = tmax * 1e3 / args.steps
+    per_launch_s = local_s / args.steps
+
+    # correctness guard on the timed output (sampled rows vs a cuBLAS witness)
+    Yc = sets[(args.steps - 1) % R][3]
+    rows = torch.arange(0, L.M, 257, device="cuda")
+    Wm = (Wd[rows].float() * mask[rows].float())
+    ref = Wm @ sets[(args.steps - 1) % R][2].float()
+    if not bool(((Yc[rows].float() - ref).abs() <= 1e-2 * ref.abs().clamp_min(1)).all()):
+        raise RuntimeError("timed output does not match the cuBLAS witness")
+
+    # dense cuBLAS on the unpruned shape, same rotation
+    dense = [(Wd.clone(), s[2], torch.empty_like(s[3])) for s in sets]
+    for i in range(max(3, args.warmup)):
+        a, b, o = dense[i % R]
+        torch.matmul(a, b, out=o)
+    torch.cuda.synchronize()
+    nd = min(args.steps, 200)
+    ev0.record(stream)
+    for i in range(nd):
+        a, b, o = dense[i % R]
+        torch.matmul(a, b, out=o)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    dense_ms = ev0.elapsed_time(ev1) / nd
+    del dense
+
+    # end to end through the public API: pinned host X -> device, bp_gemm, Y -> pinned host
+    Xh = torch.empty((L.K, L.N), dtype=Xd0.dtype, pin_memory=True)
+    Xh.copy_(Xd0.cpu())
+    Yh = torch.empty((L.M, L.N), dtype=Xd0.dtype, pin_memory=True)
+    ne = max(3, min(args.steps, 30))
+    c0, _, Xe, Ye = sets[0]
+    pwe = bp.PackedWeight(c0, pw.rb_ptr, pw.col_idx, pw.values, sets[0][1])
+    for i in range(2):
+        Xe.copy_(Xh, non_blocking=True)
+        bp.gemm(pwe, Xe, out=Ye)
+        Yh.copy_(Ye, non_blocking=True)
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for i in range(ne):
+        Xe.copy_(Xh, non_blocking=True)
+        bp.gemm(pwe, Xe, out=Ye)
+        Yh.copy_(Ye, non_blocking=True)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = ev0.elapsed_time(ev1) / ne
+    e2e_value = rsum(flops) / 1e12 / (rmax(e2e_ms / 1e3))
+
+    peaks = read_peaks()
+    peak = float(peaks["bf16_tflops"])
+    achieved = flops / per_launch_s / 1e12
+    algo_bytes = (2 * nnz_vals + 4 * pw.c.nnz_cols + 2 * L.K * L.N + 2 * L.M * L.N)
+    bound = "tensor" if flops / algo_bytes > peak * 1e12 / (float(peaks["hbm_gbs"]) * 1e9) \
+        else "hbm"
+    roof = {"bound": bound, "achieved": round(achieved, 2), "peak": peak, "unit": UNIT,
+            "frac": round(achieved / peak, 4), "traffic": recorded_traffic(workload_name()),
+            "peak_source": f"{peaks['_source']} (bf16 burst)",
+            "algorithmic_bytes": algo_bytes,
+            "achieved_gbs": round(algo_bytes / per_launch_s / 1e9, 1)}
+    if bound == "hbm":
+        hbm = float(peaks["hbm_gbs"])
+        roof.update({"achieved": roof["achieved_gbs"], "peak": hbm, "unit": "GB/s",
+                     "frac": round(roof["achieved_gbs"] / hbm, 4)})
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(W, mask.cpu().numpy(), X, dtype, budget_s=args.cpu_seconds)
+
+    out = {
+        "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded W ~ N(0,0.02), X ~ U(-1,1))",
+        "config": {"workload": workload_name(), "M": L.M, "K": L.K, "N": L.N, "bm": L.bm,
+                   "bk": L.bk, "keep": 1.0 / L.rate, "kept_weights": nnz_vals,
+                   "parallelism": f"replicas x{world}",
+                   "l2": f"inputs larger than L2: {R} rotating buffer sets of "
+                         f"{set_bytes / 2 ** 20:.0f} MiB"},
+        "clocks": sampler.summary(),
+        "e2e": {"value": round(e2e_value, 2), "unit": UNIT,
+                "h2d_bytes_per_step": 2 * L.K * L.N, "d2h_bytes_per_step": 2 * L.M * L.N},
+        "gpu_launches": args.steps,
+        "roofline": roof,
+        "cpu_baseline": cpu,
+        "dense_cublas": {"ms": round(dense_ms, 5),
+                         "tflops_dense_flops": round(2.0 * L.M * L.K * L.N / dense_ms / 1e9, 1),
+                         "speedup_vs_dense": round(dense_ms / ms_per_step, 3)},
+        "offline": {"bp_prune_ms": round((t1 - t0) * 1e3, 2),
+                    "bp_pack_ms": round((t2 - t1) * 1e3, 2)},
+    }
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+def cpu_baseline(W, mask, X, dtype, budget_s=15.0):
+    """The oracle's masked GEMM on a bounded sample of the workload's output rows."""
+    import numpy as np
+    import oracle
+
+    M = W.shape[0]
+    kept = mask.sum(axis=1).astype(np.float64)
+    N = X.shape[1]
+    rows_done, flops, t_used, r0, nb = 0, 0.0, 0.0, 0, 8
+    while t_used < budget_s and r0 < M:
+        rows = slice(r0, min(M, r0 + nb))
+        t = time.perf_counter()
+        oracle.masked_gemm(W[rows], mask[rows], X, dtype)
+        dt = time.perf_counter() - t
+        t_used += dt
+        flops += 2.0 * kept[rows].sum() * N
+        rows_done += rows.stop - rows.start
+        r0 = rows.stop
+        if dt < budget_s / 8:
+            nb *= 2
+    return {"value": round(flops / t_used / 1e12, 6), "unit": UNIT, "cores": oracle.max_threads(),
+            "kind": "oracle",
+            "sample": f"{rows_done} of {M} output rows x all {N} columns "
+                      f"({t_used:.1f} s of CPU time)"}
+
+
+# ----------------------------------------------------------------------- reference arm
+def run_reference(args):
+    world, rank, _ = dist_setup()
+    if rank != 0:
+        return
+    import numpy as np
+    import oracle
+    from paper_2111_11581_gb300 import inputs
+
+    w = WORKLOAD
+    dtype = inputs.BF16 if w["dtype"] == "bf16" else inputs.F16
+    L = inputs.gemm_point(w["M"], w["K"], w["N"], w["bm"], w["bk"], w["rate"], dtype)
+    W = inputs.layer_weight(L, dtype)
+    X = inputs.layer_input(L, dtype)
+    mask = oracle.prune(W, dtype, inputs.BLOCK_BASED, L.bm, L.bk, L.rate)
+    kept = mask.sum(axis=1).astype(np.float64)
+    # size one step's sample so that warm-up + timed steps take about 2 minutes
+    per_step = 120.0 / max(1, args.steps + args.warmup)
+    t = time.perf_counter()
+    oracle.masked_gemm(W[:4], mask[:4], X, dtype)
+    row_s = (time.perf_counter() - t) / 4
+    nrows = int(max(1, min(L.M, per_step / max(row_s, 1e-9))))
+    for i in range(args.warmup):
+        r = (i * nrows) % (L.M - nrows + 1)
+        oracle.masked_gemm(W[r:r + nrows], mask[r:r + nrows], X, dtype)
+    flops, t_used = 0.0, 0.0
+    for i in range(args.steps):
+        r = (i * nrows) % (L.M - nrows + 1)
+        t = time.perf_counter()
+        oracle.masked_gemm(W[r:r + nrows], mask[r:r + nrows], X, dtype)
+        t_used += time.perf_counter() - t
+        flops += 2.0 * kept[r:r + nrows].sum() * L.N
+    value = flops / t_used / 1e12
+    sample = f"{nrows} of {L.M} output rows x all {L.N} columns per step"
+    out = {"metric": METRIC, "value": round(value, 6), "unit": UNIT, "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": round(t_used * 1e3 / args.steps, 3), "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "impl": "reference",
+           "config": {"workload": workload_name(), "M": L.M, "K": L.K, "N": L.N, "bm": L.bm,
+                      "bk": L.bk, "keep": 1.0 / L.rate},
+           "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "kind": "oracle",
+                            "cores": oracle.max_threads(), "sample": sample},
+           "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,176 @@
+/*
+ * bp.h -- C ABI of libbp.so: inference of layers pruned with the block-based
+ * (FC / GEMM view) and block-punched (CONV) schemes of arXiv 2111.11581,
+ * on one NVIDIA GB300 (sm_103a).
+ *
+ *   bp_prune     keep the highest-norm columns / kernel positions of every
+ *                block at a given rate                (Sec. 4.1, Eq. column,
+ *                                                       Eq. punched, Sec. 5.1)
+ *   bp_pack      dense weight + mask -> compact per-row-block storage (Sec. 4.3)
+ *   bp_gemm      block-sparse GEMM  Y = (W o mask) X, fused bias/ReLU/cast
+ *   bp_conv2d    block-sparse implicit-GEMM convolution, same epilogue
+ *
+ * Conventions shared by every call:
+ *   - All tensor pointers are DEVICE pointers allocated by the caller; the
+ *     library never allocates device memory.  Host pointers are only the
+ *     scalar outputs named "host" below.
+ *   - 16-bit float tensors are fp16 or bf16 per bp_layout.dtype.  Weights,
+ *     activations and outputs of one call all use that dtype; biases are fp32.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Calls are
+ *     asynchronous on it unless they say they synchronize.
+ *   - Every call returns a bp_status.  Argument, shape and alignment problems
+ *     are reported synchronously and launch nothing.  A kernel whose bounded
+ *     wait ran out (it never hangs) records BP_ERR_TIMEOUT in a device status
+ *     word that bp_device_status() reads.  CUDA launch errors map to
+ *     BP_ERR_CUDA.
+ *   - Pointers passed to bp_gemm / bp_conv2d must be 16-byte aligned and the
+ *     leading dimensions multiples of 8 elements.
+ */
+#ifndef BP_H_
+#define BP_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    BP_OK = 0,
+    BP_ERR_INVALID_ARG = 1,   /* bad pointer, size, rate, alignment or mask */
+    BP_ERR_UNSUPPORTED = 2,   /* valid but not implemented (e.g. bm > 256 not a multiple of 128) */
+    BP_ERR_NONFINITE = 3,     /* bp_prune: a weight is Inf or NaN */
+    BP_ERR_WORKSPACE = 4,     /* workspace missing or smaller than bp_workspace_size() */
+    BP_ERR_CUDA = 5,          /* a CUDA runtime call or launch failed */
+    BP_ERR_TIMEOUT = 6        /* a kernel's bounded wait expired; its output is invalid */
+} bp_status;
+
+typedef enum { BP_F16 = 0, BP_BF16 = 1 } bp_dtype;
+
+typedef enum {
+    BP_BLOCK_BASED = 0,   /* Sec. 4.1.1: bm x bk blocks of the M x K matrix keep whole columns */
+    BP_BLOCK_PUNCHED = 1  /* Sec. 4.1.2: bm filters x bk channels keep the same kh*kw positions */
+} bp_scheme;
+
+/* Shape of a prunable layer in GEMM view (Sec. 4.2: W_i is P x Q for FC,
+ * P x Q x Kh x Kw for CONV; here M = P filters / out-features and
+ * K = Q*Kh*Kw, the OIHW weight flattened so column k = c*kh*kw + i*kw + j).
+ * Block-based: row-blocks of bm rows, column-blocks of bk columns of the
+ *   M x K matrix (kh, kw only describe the conv for bp_conv2d).
+ * Block-punched: blocks of bm filters x bk input channels; a block's units
+ *   are its kh*kw kernel positions.
+ * Partial last blocks keep their real size. */
+typedef struct {
+    int32_t scheme;   /* bp_scheme */
+    int32_t dtype;    /* bp_dtype */
+    int64_t M;        /* rows (filters / out-features), >= 1 */
+    int64_t K;        /* columns = C*kh*kw, >= 1 */
+    int32_t kh, kw;   /* kernel size, 1 x 1 for FC layers */
+    int32_t bm;       /* rows per row-block, >= 1 */
+    int32_t bk;       /* columns (block-based) or channels (punched) per block, >= 1 */
+} bp_layout;
+
+/* Compact storage of a pruned weight (Blocked Compressed Storage, Sec. 4.3).
+ * All rows of a row-block keep the same columns, so one column list per
+ * row-block replaces BCS's per-row column stride + occurrence arrays.
+ * Filled by bp_pack_size (rb_ptr) and bp_pack (the rest); all arrays are
+ * device memory owned by the caller and must stay alive while used.
+ *   rb_ptr [num_rb+1]  int64: row-block rb's columns are col_idx[rb_ptr[rb] .. rb_ptr[rb+1])
+ *   col_idx[nnz_cols]  int32: kept GEMM-view columns, ascending within a row-block
+ *   values [nnz_vals]  16-bit: row-block rb is a bm_rb x K'_rb row-major block
+ *                      starting at element bm*rb_ptr[rb] (bm_rb = rows of rb)
+ *   dev    [dev_bytes] the same weights re-tiled for the tensor-core kernels
+ *                      (k-chunks of 64 columns, zero padded, pre-swizzled) plus
+ *                      their padded index lists; opaque to callers. */
+typedef struct {
+    bp_layout lay;
+    int64_t num_rb;
+    int64_t nnz_cols;
+    int64_t nnz_vals;
+    int64_t *rb_ptr;
+    int32_t *col_idx;
+    void *values;
+    void *dev;
+    int64_t dev_bytes;
+} bp_packed;
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char *bp_status_string(int status);
+
+/* Library ABI version: (major << 16) | minor. */
+int bp_version(void);
+
+/* Device workspace bytes bp_prune needs for `lay` (host output). */
+bp_status bp_workspace_size(const bp_layout *lay, size_t *bytes);
+
+/* One-shot magnitude pruning by block (Sec. 5.1 with the block regularities
+ * of Sec. 4.1).  Scores are the squared L2 norms of Eq. (column) (block-based:
+ * each column of each block) and Eq. (punched) (each kernel position of each
+ * filters x channels block), accumulated in fp64 in ascending row (resp.
+ * filter, then channel) order.  Rate r >= 1 is the parameter-reduction
+ * factor: block b with P_b units keeps its floor(P_b / r) best units, and the
+ * T - sum floor(P_b / r) best remaining units of the whole layer are kept as
+ * well, T = floor(sum P_b / r + 0.5).  Ties prefer the lower unit index
+ * (row-block, then column-block, then column / position).
+ *   W     device, M x K 16-bit weights (OIHW for convolutions)
+ *   rate  >= 1, finite
+ *   mask  device, M x K uint8 output, 1 = kept
+ *   ws    device workspace of at least bp_workspace_size() bytes, 256-B aligned
+ * Synchronizes `stream` (it reads back counts); returns BP_ERR_NONFINITE if a
+ * weight is Inf/NaN (mask then undefined). */
+bp_status bp_prune(const bp_layout *lay, const void *W, double rate, uint8_t *mask, void *ws,
+                   size_t ws_bytes, void *stream);
+
+/* First half of packing: checks that every row of each row-block keeps the
+ * same columns as the row-block's first row (BP_ERR_INVALID_ARG otherwise)
+ * and writes rb_ptr (device, num_rb+1 int64, caller-allocated).  Host
+ * outputs: nnz_cols, nnz_vals and dev_bytes, the sizes the caller allocates
+ * for col_idx, values and dev.  Synchronizes `stream`. */
+bp_status bp_pack_size(const bp_layout *lay, const uint8_t *mask, int64_t *rb_ptr,
+                       int64_t *nnz_cols, int64_t *nnz_vals, int64_t *dev_bytes, void *stream);
+
+/* Second half: fills out->col_idx, out->values and out->dev from W and mask.
+ * `out` must carry lay, rb_ptr (from bp_pack_size), the sizes returned by
+ * bp_pack_size and caller-allocated arrays of those sizes (dev 16-B aligned).
+ * num_rb, nnz_cols, nnz_vals and dev_bytes are checked against the layout. */
+bp_status bp_pack(const bp_layout *lay, const void *W, const uint8_t *mask, bp_packed *out,
+                  void *stream);
+
+/* Block-sparse GEMM (the FC layer of Sec. 4.2 with pruned weights skipped,
+ * Sec. 4.3):  Y[m, n] = act( sum over kept k of W[m,k] * X[k,n] + bias[m] ),
+ * fp32 accumulation on the tensor cores, one round-to-nearest-even cast.
+ *   X     device, K x N row-major (leading dimension ldx >= N, multiple of 8)
+ *   N     >= 0 columns (tokens)
+ *   bias  device fp32 [M] or NULL
+ *   relu  0 / 1
+ *   Y     device, M x N row-major (ldy >= N, multiple of 8)
+ * Supported bm: 1..256, or any multiple of 128. */
+bp_status bp_gemm(const bp_packed *P, const void *X, int64_t N, int64_t ldx, const float *bias,
+                  int relu, void *Y, int64_t ldy, void *stream);
+
+/* Block-sparse convolution as an implicit GEMM over the GEMM view of
+ * bp_layout (kept column k = c*kh*kw + i*kw + j), NCHW input and output:
+ *   out[b,f,oh,ow] = act( sum over kept (c,i,j) of W[f,c,i,j] *
+ *                         in[b, c, oh*stride_h + i - pad_h, ow*stride_w + j - pad_w]
+ *                         + bias[f] ),  zero outside the input.
+ *   in    device, Nb x C x H x W;   out  device, Nb x M x Ho x Wo with
+ *   Ho = (H + 2 pad_h - kh) / stride_h + 1, Wo likewise.
+ * Requires C*kh*kw == lay.K; dilation and groups are not supported. */
+bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, int64_t H,
+                    int64_t W, int pad_h, int pad_w, int stride_h, int stride_w,
+                    const float *bias, int relu, void *out, void *stream);
+
+/* Synchronizes `stream`, then returns BP_ERR_TIMEOUT if any kernel of this
+ * library recorded an expired wait since the previous call (and clears the
+ * record), else BP_OK. */
+bp_status bp_device_status(void *stream);
+
+/* Upper bound, in nanoseconds, on every wait inside the kernels launched
+ * after this call (default 2e9).  0 restores the default. */
+bp_status bp_set_watchdog_ns(uint64_t ns);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* BP_H_ */

@@ -1,0 +1,385 @@
+// C ABI of libbp (declared in include/bp.h): argument checking, host-side
+// counting and the launch sequences of bp_prune / bp_pack_size / bp_pack /
+// bp_gemm / bp_conv2d.  No call allocates device memory.
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "bp_common.cuh"
+
+namespace bp {
+
+// Device status word: kernels OR kDevTimeout into it when a bounded wait ran
+// out; bp_device_status() reads and clears it.
+__device__ unsigned g_dev_status;
+// Flag word of bp_pack_size's row-block consistency check (calls serialised).
+__device__ int g_pack_bad;
+
+namespace {
+constexpr uint64_t kDefaultWatchdogNs = 2000000000ull;
+uint64_t g_watchdog_ns = kDefaultWatchdogNs;
+std::mutex g_mu;            // guards the per-device caches and g_pack_bad
+constexpr int kMaxDev = 64;
+unsigned *g_status_ptr[kMaxDev];
+int g_sms[kMaxDev];
+
+int cur_dev() {
+    int d = 0;
+    cudaGetDevice(&d);
+    return d < 0 || d >= kMaxDev ? 0 : d;
+}
+
+int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bp_status cuda_status(cudaError_t e) { return e == cudaSuccess ? BP_OK : BP_ERR_CUDA; }
+
+bool layout_ok(const bp_layout *l) {
+    if (!l) return false;
+    if (l->scheme != BP_BLOCK_BASED && l->scheme != BP_BLOCK_PUNCHED) return false;
+    if (l->dtype != BP_F16 && l->dtype != BP_BF16) return false;
+    if (l->M < 1 || l->K < 1 || l->kh < 1 || l->kw < 1 || l->bm < 1 || l->bk < 1) return false;
+    if (l->K % ((int64_t)l->kh * l->kw) != 0) return false;
+    if (l->M > (int64_t)1 << 40 || l->K > ((int64_t)1 << 31) - 1) return false;
+    return true;
+}
+
+// units and per-layer keep counts (Sec. 4.1 / 5.1 reading: floor(P_b / r) per
+// block, T = floor(sum P_b / r + 0.5) per layer)
+struct Counts {
+    int64_t U, sum_base, T, E;
+};
+
+Counts host_counts(const bp_layout &l, double rate) {
+    Counts c{};
+    const int64_t RB = cdiv(l.M, l.bm);
+    const int64_t KK = (int64_t)l.kh * l.kw;
+    int64_t per_rb_base = 0, per_rb_units = 0;
+    if (l.scheme == BP_BLOCK_BASED) {
+        const int64_t full = l.K / l.bk, tail = l.K % l.bk;
+        per_rb_base = full * (int64_t)std::floor((double)l.bk / rate) +
+                      (tail ? (int64_t)std::floor((double)tail / rate) : 0);
+        per_rb_units = l.K;
+    } else {
+        const int64_t CB = cdiv(l.K / KK, l.bk);
+        per_rb_base = CB * (int64_t)std::floor((double)KK / rate);
+        per_rb_units = CB * KK;
+    }
+    c.U = RB * per_rb_units;
+    c.sum_base = RB * per_rb_base;
+    c.T = (int64_t)std::floor((double)c.U / rate + 0.5);
+    c.E = c.T - c.sum_base;
+    return c;
+}
+
+struct PruneWs {
+    int64_t off_scores, off_hist, off_chunks, off_flag, off_keep, total;
+};
+
+int64_t align_up(int64_t v, int64_t a) { return (v + a - 1) / a * a; }
+
+PruneWs prune_ws(const bp_layout &l) {
+    const Counts c = host_counts(l, 1.0);
+    PruneWs w;
+    w.off_scores = 0;
+    w.off_hist = align_up(c.U * 8, 256);
+    w.off_chunks = w.off_hist + 1024;
+    w.off_flag = align_up(w.off_chunks + 8 * threshold_chunks(c.U), 256);
+    w.off_keep = w.off_flag + 256;
+    w.total = align_up(w.off_keep + c.U, 256);
+    return w;
+}
+
+}  // namespace
+
+uint64_t watchdog_ns() { return g_watchdog_ns; }
+
+unsigned *device_status_ptr() {
+    std::lock_guard<std::mutex> lk(g_mu);
+    const int d = cur_dev();
+    if (!g_status_ptr[d]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_dev_status) == cudaSuccess)
+            g_status_ptr[d] = static_cast<unsigned *>(p);
+    }
+    return g_status_ptr[d];
+}
+
+int num_sms() {
+    const int d = cur_dev();
+    if (!g_sms[d]) {
+        int v = 0;
+        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, d);
+        g_sms[d] = v > 0 ? v : 1;
+    }
+    return g_sms[d];
+}
+
+bool checked_mode() {
+    const char *e = std::getenv("BP_CHECKED");
+    return e && e[0] == '1';
+}
+
+Orientation orientation_for(int64_t bm) {
+    if (bm % kSlab == 0) return kWeightA;
+    if (bm <= 256) return kWeightB;
+    return kNoTensorCore;
+}
+
+int64_t rows_pad_for(int64_t bm) {
+    switch (orientation_for(bm)) {
+    case kWeightA: return bm;
+    case kWeightB: return align_up(bm, 16);
+    default: return 0;
+    }
+}
+
+DevLayout dev_layout(const bp_layout &lay, const int64_t *rb_ptr_host) {
+    DevLayout d{};
+    d.orient = orientation_for(lay.bm);
+    d.rows_pad = rows_pad_for(lay.bm);
+    d.num_rb = cdiv(lay.M, lay.bm);
+    d.off_chunks = align_up(8 * (d.num_rb + 1), 256);
+    d.tile_bytes = d.rows_pad * kBK * 2;
+    d.chunk_bytes = d.tile_bytes + kBK * 4;
+    d.kc_total = -1;
+    d.bytes = -1;
+    if (rb_ptr_host) {
+        int64_t kc = 0;
+        for (int64_t rb = 0; rb < d.num_rb; ++rb) kc += cdiv(rb_ptr_host[rb + 1] - rb_ptr_host[rb], kBK);
+        d.kc_total = kc;
+        d.bytes = d.orient == kNoTensorCore ? 0 : d.off_chunks + kc * d.chunk_bytes;
+    }
+    return d;
+}
+
+}  // namespace bp
+
+using namespace bp;
+
+extern "C" {
+
+const char *bp_status_string(int status) {
+    switch (status) {
+    case BP_OK: return "ok";
+    case BP_ERR_INVALID_ARG: return "invalid argument";
+    case BP_ERR_UNSUPPORTED: return "unsupported configuration";
+    case BP_ERR_NONFINITE: return "non-finite weight";
+    case BP_ERR_WORKSPACE: return "workspace too small";
+    case BP_ERR_CUDA: return "CUDA error";
+    case BP_ERR_TIMEOUT: return "kernel wait timed out";
+    default: return "unknown status";
+    }
+}
+
+int bp_version(void) { return (1 << 16) | 0; }
+
+bp_status bp_workspace_size(const bp_layout *lay, size_t *bytes) {
+    if (!layout_ok(lay) || !bytes) return BP_ERR_INVALID_ARG;
+    *bytes = (size_t)prune_ws(*lay).total;
+    return BP_OK;
+}
+
+bp_status bp_prune(const bp_layout *lay, const void *W, double rate, uint8_t *mask, void *ws,
+                   size_t ws_bytes, void *stream) {
+    if (!layout_ok(lay) || !W || !mask) return BP_ERR_INVALID_ARG;
+    if (!(rate >= 1.0) || !std::isfinite(rate)) return BP_ERR_INVALID_ARG;
+    const PruneWs w = prune_ws(*lay);
+    if (!ws || ws_bytes < (size_t)w.total || (reinterpret_cast<uintptr_t>(ws) & 255u))
+        return BP_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint8_t *base = static_cast<uint8_t *>(ws);
+    double *scores = reinterpret_cast<double *>(base + w.off_scores);
+    unsigned *hist = reinterpret_cast<unsigned *>(base + w.off_hist);
+    int64_t *chunks = reinterpret_cast<int64_t *>(base + w.off_chunks);
+    int *flag = reinterpret_cast<int *>(base + w.off_flag);
+    uint8_t *keep = base + w.off_keep;
+    const Counts c = host_counts(*lay, rate);
+
+    cudaError_t e = cudaMemsetAsync(flag, 0, sizeof(int), s);
+    if (e == cudaSuccess) e = launch_scores(*lay, W, scores, flag, s);
+    if (e == cudaSuccess) e = launch_base_select(*lay, scores, rate, keep, s);
+    int nonfinite = 0;
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&nonfinite, flag, sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return BP_ERR_CUDA;
+    if (nonfinite) return BP_ERR_NONFINITE;
+
+    if (c.E > 0) {
+        // most-significant-digit radix select of the E-th best remaining unit
+        uint64_t prefix = 0;
+        int64_t need = c.E;
+        unsigned h[256];
+        for (int shift = 56; shift >= 0; shift -= 8) {
+            e = cudaMemsetAsync(hist, 0, 256 * sizeof(unsigned), s);
+            if (e == cudaSuccess) e = launch_radix_hist(c.U, scores, keep, prefix, shift, hist, s);
+            if (e == cudaSuccess) e = cudaMemcpyAsync(h, hist, sizeof(h), cudaMemcpyDeviceToHost, s);
+            if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+            if (e != cudaSuccess) return BP_ERR_CUDA;
+            int d = 255;
+            for (; d > 0; --d) {
+                if ((int64_t)h[d] >= need) break;
+                need -= h[d];
+            }
+            prefix |= (uint64_t)d << shift;
+        }
+        e = launch_threshold_select(c.U, scores, keep, prefix, need, chunks, s);
+        if (e != cudaSuccess) return BP_ERR_CUDA;
+    }
+    e = launch_write_mask(*lay, keep, mask, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    return cuda_status(e);
+}
+
+bp_status bp_pack_size(const bp_layout *lay, const uint8_t *mask, int64_t *rb_ptr,
+                       int64_t *nnz_cols, int64_t *nnz_vals, int64_t *dev_bytes, void *stream) {
+    if (!layout_ok(lay) || !mask || !rb_ptr || !nnz_cols || !nnz_vals || !dev_bytes)
+        return BP_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int64_t RB = cdiv(lay->M, lay->bm);
+    if (RB > 65535) return BP_ERR_UNSUPPORTED;
+    std::lock_guard<std::mutex> lk(g_mu);
+    int *bad = nullptr;
+    if (cudaGetSymbolAddress(reinterpret_cast<void **>(&bad), g_pack_bad) != cudaSuccess)
+        return BP_ERR_CUDA;
+    std::vector<int64_t> h(RB + 1);
+    int hbad = 0;
+    cudaError_t e = cudaMemsetAsync(bad, 0, sizeof(int), s);
+    if (e == cudaSuccess) e = launch_rb_counts(*lay, mask, rb_ptr, bad, s);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(h.data(), rb_ptr, 8 * (RB + 1), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&hbad, bad, sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return BP_ERR_CUDA;
+    if (hbad) return BP_ERR_INVALID_ARG;
+    int64_t nv = 0;
+    for (int64_t rb = 0; rb < RB; ++rb) {
+        const int64_t rows = std::min<int64_t>(lay->bm, lay->M - rb * lay->bm);
+        nv += rows * (h[rb + 1] - h[rb]);
+    }
+    *nnz_cols = h[RB];
+    *nnz_vals = nv;
+    *dev_bytes = dev_layout(*lay, h.data()).bytes;
+    return BP_OK;
+}
+
+bp_status bp_pack(const bp_layout *lay, const void *W, const uint8_t *mask, bp_packed *out,
+                  void *stream) {
+    if (!layout_ok(lay) || !W || !mask || !out || !out->rb_ptr) return BP_ERR_INVALID_ARG;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int64_t RB = cdiv(lay->M, lay->bm);
+    if (RB > 65535) return BP_ERR_UNSUPPORTED;
+    if (out->num_rb != RB) return BP_ERR_INVALID_ARG;
+    std::vector<int64_t> h(RB + 1);
+    cudaError_t e = cudaMemcpyAsync(h.data(), out->rb_ptr, 8 * (RB + 1), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return BP_ERR_CUDA;
+    if (h[0] != 0) return BP_ERR_INVALID_ARG;
+    int64_t nv = 0;
+    for (int64_t rb = 0; rb < RB; ++rb) {
+        const int64_t kp = h[rb + 1] - h[rb];
+        if (kp < 0 || kp > lay->K) return BP_ERR_INVALID_ARG;
+        nv += std::min<int64_t>(lay->bm, lay->M - rb * lay->bm) * kp;
+    }
+    if (out->nnz_cols != h[RB] || out->nnz_vals != nv) return BP_ERR_INVALID_ARG;
+    if ((h[RB] > 0 && !out->col_idx) || (nv > 0 && !out->values)) return BP_ERR_INVALID_ARG;
+    const DevLayout dl = dev_layout(*lay, h.data());
+    if (out->dev_bytes != dl.bytes) return BP_ERR_INVALID_ARG;
+    if (dl.bytes > 0 && (!out->dev || !aligned16(out->dev))) return BP_ERR_INVALID_ARG;
+    out->lay = *lay;
+    std::vector<int64_t> kc(RB + 1, 0);
+    for (int64_t rb = 0; rb < RB; ++rb) kc[rb + 1] = kc[rb] + cdiv(h[rb + 1] - h[rb], kBK);
+    if (dl.bytes > 0)
+        e = cudaMemcpyAsync(out->dev, kc.data(), 8 * (RB + 1), cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess) e = launch_pack(*lay, W, mask, *out, dl, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    return cuda_status(e);
+}
+
+static bp_status check_packed(const bp_packed *P, DevLayout *dl) {
+    if (!P || !layout_ok(&P->lay) || !P->dev || !aligned16(P->dev)) return BP_ERR_INVALID_ARG;
+    if (P->num_rb != cdiv(P->lay.M, P->lay.bm)) return BP_ERR_INVALID_ARG;
+    *dl = dev_layout(P->lay, nullptr);
+    if (dl->orient == kNoTensorCore) return BP_ERR_UNSUPPORTED;
+    if (P->dev_bytes < dl->off_chunks) return BP_ERR_INVALID_ARG;
+    return BP_OK;
+}
+
+static bp_status finish_launch(cudaError_t e, cudaStream_t s) {
+    if (e != cudaSuccess) return BP_ERR_CUDA;
+    if (checked_mode()) return bp_device_status(s);
+    return BP_OK;
+}
+
+bp_status bp_gemm(const bp_packed *P, const void *X, int64_t N, int64_t ldx, const float *bias,
+                  int relu, void *Y, int64_t ldy, void *stream) {
+    DevLayout dl;
+    bp_status st = check_packed(P, &dl);
+    if (st != BP_OK) return st;
+    if (N < 0 || !X || !Y || ldx < N || ldy < N || ldx % 8 || ldy % 8) return BP_ERR_INVALID_ARG;
+    if (!aligned16(X) || !aligned16(Y)) return BP_ERR_INVALID_ARG;
+    if (bias && (reinterpret_cast<uintptr_t>(bias) & 3u)) return BP_ERR_INVALID_ARG;
+    if (N == 0) return BP_OK;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    return finish_launch(launch_mma(*P, dl, X, N, ldx, bias, relu, Y, ldy, nullptr, s), s);
+}
+
+bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, int64_t H,
+                    int64_t W, int pad_h, int pad_w, int stride_h, int stride_w,
+                    const float *bias, int relu, void *out, void *stream) {
+    DevLayout dl;
+    bp_status st = check_packed(P, &dl);
+    if (st != BP_OK) return st;
+    const bp_layout &l = P->lay;
+    if (!in || !out || Nb < 0 || C < 1 || H < 1 || W < 1) return BP_ERR_INVALID_ARG;
+    if (pad_h < 0 || pad_w < 0 || stride_h < 1 || stride_w < 1) return BP_ERR_INVALID_ARG;
+    if (C * l.kh * l.kw != l.K) return BP_ERR_INVALID_ARG;
+    if (H + 2 * pad_h < l.kh || W + 2 * pad_w < l.kw) return BP_ERR_INVALID_ARG;
+    if (!aligned16(in) || !aligned16(out)) return BP_ERR_INVALID_ARG;
+    if (bias && (reinterpret_cast<uintptr_t>(bias) & 3u)) return BP_ERR_INVALID_ARG;
+    if (dl.rows_pad > 256) return BP_ERR_UNSUPPORTED;
+    if (H > (1 << 28) || W > (1 << 28)) return BP_ERR_UNSUPPORTED;
+    ConvShape cs;
+    cs.Nb = Nb;
+    cs.C = C;
+    cs.H = H;
+    cs.W = W;
+    cs.Ho = (H + 2 * pad_h - l.kh) / stride_h + 1;
+    cs.Wo = (W + 2 * pad_w - l.kw) / stride_w + 1;
+    cs.kh = l.kh;
+    cs.kw = l.kw;
+    cs.ph = pad_h;
+    cs.pw = pad_w;
+    cs.sh = stride_h;
+    cs.sw = stride_w;
+    const int64_t N = Nb * cs.Ho * cs.Wo;
+    if (N == 0) return BP_OK;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    return finish_launch(launch_mma(*P, dl, in, N, 0, bias, relu, out, 0, &cs, s), s);
+}
+
+bp_status bp_device_status(void *stream) {
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(s) != cudaSuccess) return BP_ERR_CUDA;
+    unsigned *p = device_status_ptr();
+    if (!p) return BP_ERR_CUDA;
+    unsigned v = 0;
+    if (cudaMemcpy(&v, p, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return BP_ERR_CUDA;
+    if (v) {
+        const unsigned zero = 0;
+        if (cudaMemcpy(p, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess)
+            return BP_ERR_CUDA;
+        return BP_ERR_TIMEOUT;
+    }
+    return BP_OK;
+}
+
+bp_status bp_set_watchdog_ns(uint64_t ns) {
+    g_watchdog_ns = ns ? ns : kDefaultWatchdogNs;
+    return BP_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,549 @@
+// Block-sparse GEMM / implicit-GEMM convolution on the sm_103a tensor cores.
+//
+// Each work item is one row-block (or one 128-row slab of it) times one tile
+// of activation columns.  The row-block's compact weights Wc (bm x K'_rb,
+// Sec. 4.3) multiply the activation rows selected by its kept-column list, so
+// pruned weights never enter the product.  Per k-chunk of 64 kept columns:
+//
+//   producer warps 0-3  copy the pre-swizzled weight tile (cp.async) and
+//                       gather the 64 activation rows named by the chunk's
+//                       column list into a 128-byte-swizzled MN-major tile
+//                       (GEMM: rows of X; conv: im2col rows built on the fly,
+//                       zero outside the image);
+//   MMA warp 4          issues tcgen05.mma (K = 16 per instruction) into an
+//                       fp32 accumulator in tensor memory, double-buffered
+//                       across work items;
+//   epilogue warps 5-8  read the accumulator (tcgen05.ld), add the bias,
+//                       apply ReLU, round to fp16/bf16 and store.
+//
+// Two operand orientations:
+//   kWeightA (bm a multiple of 128): D[128 weight rows x 256 tokens]
+//            = Wc tile (A, K-major) * gathered X (B, MN-major);
+//   kWeightB (bm <= 256): D[128 tokens x rows_pad] = gathered X^T (A,
+//            MN-major) * Wc^T (B, K-major), rows_pad = bm rounded up to 16.
+//
+// Every wait is bounded (see mbar_wait); on expiry the kernel records
+// kDevTimeout in the device status word, drains its own copies and tensor
+// core work, frees tensor memory and returns.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include <mutex>
+
+#include "bp_common.cuh"
+
+namespace bp {
+namespace {
+
+constexpr int kThreads = 288;          // 9 warps
+constexpr int kProducerThreads = 128;
+constexpr int kMmaWarp = 4;
+constexpr int kLag = 2;                // cp.async groups in flight per producer thread
+constexpr uint64_t kDrainNs = 1000000000ull;
+
+struct Params {
+    int dtype;
+    int relu;
+    int64_t M, bm, rows_pad, num_rb, nslab;
+    int64_t N;              // tokens (GEMM) or Nb*Ho*Wo pixels (conv)
+    int64_t n_tiles, num_items;
+    int64_t stages;
+    uint32_t w_tile_bytes, x_tile_bytes, tmem_cols, acc_cols;
+    const int64_t *kc_ptr;
+    const uint8_t *chunks;       // k-chunks: weight tile, then 64 int32 column indices
+    int64_t tile_bytes, chunk_bytes;
+    const uint16_t *X;
+    int64_t ldx;
+    uint16_t *Y;
+    int64_t ldy;
+    const float *bias;
+    // convolution
+    int64_t C, H, W, Ho, Wo, HoWo, KK;
+    int kw, ph, pw, sh, sw;
+    uint64_t watchdog_ns;
+    unsigned *status;
+};
+
+__device__ __forceinline__ uint32_t pack2(float a, float b, int dtype) {
+    if (dtype == BP_BF16) {
+        const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+        return *reinterpret_cast<const uint32_t *>(&h);
+    }
+    const __half2 h = __floats2half2_rn(a, b);
+    return *reinterpret_cast<const uint32_t *>(&h);
+}
+
+__device__ __forceinline__ uint16_t cvt1(float a, int dtype) {
+    if (dtype == BP_BF16) return __bfloat16_as_ushort(__float2bfloat16_rn(a));
+    return __half_as_ushort(__float2half_rn(a));
+}
+
+struct Smem {
+    uint8_t *w;          // stages x w_tile_bytes
+    uint8_t *x;          // stages x x_tile_bytes
+    uint64_t *full;      // [stages]
+    uint64_t *empty;     // [stages]
+    uint64_t *tfull;     // [2]
+    uint64_t *tempty;    // [2]
+    uint64_t *drain;     // [1]
+    uint32_t *tmem_base;
+    int *abort_flag;
+};
+
+__device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
+    Smem s;
+    uint8_t *base = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    s.w = base;
+    s.x = base + p.stages * p.w_tile_bytes;
+    uint8_t *b = s.x + p.stages * p.x_tile_bytes;
+    s.full = reinterpret_cast<uint64_t *>(b);
+    s.empty = s.full + p.stages;
+    s.tfull = s.empty + p.stages;
+    s.tempty = s.tfull + 2;
+    s.drain = s.tempty + 2;
+    s.tmem_base = reinterpret_cast<uint32_t *>(s.drain + 1);
+    s.abort_flag = reinterpret_cast<int *>(s.tmem_base + 1);
+    return s;
+}
+
+__device__ __forceinline__ void raise_timeout(const Params &p, const Smem &s) {
+    *reinterpret_cast<volatile int *>(s.abort_flag) = 1;
+    atomicOr(p.status, kDevTimeout);
+}
+
+struct Item {
+    int64_t rb, slab, n0, kc0, nkc, rows;   // rows = real rows of the row-block
+};
+
+__device__ __forceinline__ Item decode(const Params &p, int64_t it, bool wa) {
+    Item t;
+    const int64_t R = p.num_rb * p.nslab;
+    const int64_t rs = it % R;
+    t.n0 = (it / R) * (wa ? 256 : 128);
+    t.rb = rs / p.nslab;
+    t.slab = rs % p.nslab;
+    t.kc0 = p.kc_ptr[t.rb];
+    t.nkc = p.kc_ptr[t.rb + 1] - t.kc0;
+    t.rows = min(p.bm, p.M - t.rb * p.bm);
+    return t;
+}
+
+// ------------------------------------------------------------------ producer
+template <bool WA, bool CONV>
+__device__ void producer(const Params &p, const Smem &s) {
+    const int tid = threadIdx.x;            // 0..127
+    const int warp = tid >> 5, lane = tid & 31;
+    volatile int *abort_flag = s.abort_flag;
+    int stage = 0;
+    uint32_t phase = 0;
+    int pend[kLag + 1];
+    int npend = 0;
+    bool ok = true;
+    const uint32_t w_units = p.w_tile_bytes >> 4;
+
+    for (int64_t it = blockIdx.x; it < p.num_items && ok; it += gridDim.x) {
+        const Item t = decode(p, it, WA);
+        if (t.nkc == 0) continue;
+        // convolution: this thread's 8 pixels are fixed for the whole tile
+        int64_t pbase[8];
+        int ih0[8], iw0[8];
+        const int u16 = lane & 15;           // 16-byte unit within a 128-token row
+        if (CONV) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const int64_t pix = t.n0 + u16 * 8 + e;
+                if (pix < p.N) {
+                    const int64_t b = pix / p.HoWo, hw = pix % p.HoWo;
+                    const int oh = (int)(hw / p.Wo), ow = (int)(hw % p.Wo);
+                    pbase[e] = b * p.C * p.H * p.W;
+                    ih0[e] = oh * p.sh - p.ph;
+                    iw0[e] = ow * p.sw - p.pw;
+                } else {
+                    pbase[e] = 0;
+                    ih0[e] = -(1 << 29);     // never inside the image
+                    iw0[e] = 0;
+                }
+            }
+        }
+        for (int64_t kc = 0; kc < t.nkc; ++kc) {
+            if (!mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)) {
+                raise_timeout(p, s);
+                ok = false;
+                break;
+            }
+            const uint32_t ws = smem_u32(s.w + stage * p.w_tile_bytes);
+            const uint32_t xs = smem_u32(s.x + stage * p.x_tile_bytes);
+            // weight tile: contiguous pre-swizzled bytes
+            const uint8_t *chunk = p.chunks + (t.kc0 + kc) * p.chunk_bytes;
+            const uint8_t *wsrc = chunk + t.slab * (kSlab * kBK * 2);
+            for (uint32_t u = tid; u < w_units; u += kProducerThreads)
+                cp_async_16(ws + u * 16, wsrc + (size_t)u * 16, 16);
+            const int32_t *cl = reinterpret_cast<const int32_t *>(chunk + p.tile_bytes);
+            if (!CONV) {
+                if (WA) {
+                    // 64 rows x 32 units (256 tokens); one warp covers one row
+                    const int cn = lane >> 3, j = lane & 7;
+                    const int64_t n = t.n0 + lane * 8;
+                    const uint32_t nb = n < p.N ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
+#pragma unroll 4
+                    for (int i = 0; i < 16; ++i) {
+                        const int r = warp + 4 * i;
+                        const int32_t idx = cl[r];
+                        const bool live = idx >= 0 && nb > 0;
+                        const uint16_t *src = live ? p.X + idx * p.ldx + n : p.X;
+                        cp_async_16(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4), src,
+                                    live ? nb : 0u);
+                    }
+                } else {
+                    // 64 rows x 16 units (128 tokens); one warp covers two rows
+                    const int cn = u16 >> 3, j = u16 & 7;
+                    const int64_t n = t.n0 + u16 * 8;
+                    const uint32_t nb = n < p.N ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
+#pragma unroll 4
+                    for (int i = 0; i < 8; ++i) {
+                        const int r = 2 * (warp + 4 * i) + (lane >> 4);
+                        const int32_t idx = cl[r];
+                        const bool live = idx >= 0 && nb > 0;
+                        const uint16_t *src = live ? p.X + idx * p.ldx + n : p.X;
+                        cp_async_16(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4), src,
+                                    live ? nb : 0u);
+                    }
+                }
+                cp_async_commit();
+                pend[npend++] = stage;
+                if (npend > kLag) {
+                    cp_async_wait_group<kLag>();
+                    fence_proxy_async_smem();
+                    mbar_arrive(&s.full[pend[0]]);
+#pragma unroll
+                    for (int q = 0; q < kLag; ++q) pend[q] = pend[q + 1];
+                    --npend;
+                }
+            } else {
+                // im2col rows of 128 pixels, built in registers
+                const int cn = u16 >> 3, j = u16 & 7;
+#pragma unroll 2
+                for (int i = 0; i < 8; ++i) {
+                    const int r = 2 * (warp + 4 * i) + (lane >> 4);
+                    const int32_t idx = cl[r];
+                    uint32_t v[4] = {0u, 0u, 0u, 0u};
+                    if (idx >= 0) {
+                        const int64_t c = idx / p.KK;
+                        const int rs = (int)(idx - c * p.KK);
+                        const int di = rs / p.kw, dj = rs - (rs / p.kw) * p.kw;
+                        const uint16_t *plane = p.X + c * p.H * p.W;
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            const int ih = ih0[e] + di, iw = iw0[e] + dj;
+                            uint32_t h = 0u;
+                            if ((unsigned)ih < (unsigned)p.H && (unsigned)iw < (unsigned)p.W)
+                                h = __ldg(plane + pbase[e] + (int64_t)ih * p.W + iw);
+                            v[e >> 1] |= h << ((e & 1) * 16);
+                        }
+                    }
+                    st_shared_v4(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4),
+                                 make_uint4(v[0], v[1], v[2], v[3]));
+                }
+                cp_async_wait_all();
+                fence_proxy_async_smem();
+                mbar_arrive(&s.full[stage]);
+            }
+            if (++stage == p.stages) {
+                stage = 0;
+                phase ^= 1u;
+            }
+        }
+    }
+    cp_async_wait_all();
+    fence_proxy_async_smem();
+    if (ok)
+        for (int q = 0; q < npend; ++q) mbar_arrive(&s.full[pend[q]]);
+}
+
+// ------------------------------------------------------------------ MMA issuer
+template <bool WA>
+__device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
+    volatile int *abort_flag = s.abort_flag;
+    const bool bf16 = p.dtype == BP_BF16;
+    const uint32_t idesc = WA ? make_idesc(bf16, false, true, 128, 256)
+                              : make_idesc(bf16, true, false, 128, (int)p.rows_pad);
+    int stage = 0;
+    uint32_t phase = 0;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    bool ok = true;
+    for (int64_t it = blockIdx.x; it < p.num_items && ok; it += gridDim.x) {
+        const Item t = decode(p, it, WA);
+        if (t.nkc == 0) continue;
+        if (!mbar_wait(&s.tempty[acc], acc_phase ^ 1u, p.watchdog_ns, abort_flag)) {
+            raise_timeout(p, s);
+            break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem + acc * p.acc_cols;
+        for (int64_t kc = 0; kc < t.nkc; ++kc) {
+            if (!mbar_wait(&s.full[stage], phase, p.watchdog_ns, abort_flag)) {
+                raise_timeout(p, s);
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t ws = smem_u32(s.w + stage * p.w_tile_bytes);
+            const uint32_t xs = smem_u32(s.x + stage * p.x_tile_bytes);
+#pragma unroll
+            for (int kk = 0; kk < kBK / 16; ++kk) {
+                const uint64_t wdesc = make_sdesc_sw128(ws + kk * 32, 16, 1024);
+                const uint64_t xdesc = make_sdesc_sw128(xs + kk * 2048, 8192, 1024);
+                const uint32_t accum = (kc > 0 || kk > 0) ? 1u : 0u;
+                if (WA) umma_f16_ss(d, wdesc, xdesc, idesc, accum);
+                else umma_f16_ss(d, xdesc, wdesc, idesc, accum);
+            }
+            umma_commit(&s.empty[stage]);
+            if (++stage == p.stages) {
+                stage = 0;
+                phase ^= 1u;
+            }
+        }
+        if (!ok) break;
+        umma_commit(&s.tfull[acc]);
+        if (++acc == 2) {
+            acc = 0;
+            acc_phase ^= 1u;
+        }
+    }
+    // all issued tensor-core work must finish before tensor memory is freed
+    umma_commit(s.drain);
+    if (!mbar_wait(s.drain, 0, kDrainNs, nullptr)) atomicOr(p.status, kDevTimeout);
+}
+
+// ------------------------------------------------------------------ epilogue
+template <bool WA, bool CONV>
+__device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
+    volatile int *abort_flag = s.abort_flag;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int q = warp & 3;                  // tensor-memory lane quadrant of this warp
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int64_t it = blockIdx.x; it < p.num_items; it += gridDim.x) {
+        const Item t = decode(p, it, WA);
+        const bool has = t.nkc > 0;
+        if (has) {
+            if (!mbar_wait(&s.tfull[acc], acc_phase, p.watchdog_ns, abort_flag)) {
+                raise_timeout(p, s);
+                break;
+            }
+            tc_fence_after();
+        }
+        const uint32_t tacc = tmem + ((uint32_t)(32 * q) << 16) + acc * p.acc_cols;
+        if (WA) {
+            const int64_t row = t.slab * kSlab + 32 * q + lane;
+            const bool vrow = row < t.rows;
+            const int64_t m = t.rb * p.bm + row;
+            const float bv = (p.bias && vrow) ? p.bias[m] : 0.f;
+            uint16_t *yrow = p.Y + (vrow ? m : 0) * p.ldy;
+            for (int c0 = 0; c0 < 256; c0 += 16) {
+                uint32_t r[16];
+                if (has) {
+                    tmem_ld_32x32b_x16(tacc + c0, r);
+                    tmem_ld_wait();
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) r[e] = 0u;
+                }
+                const int64_t n = t.n0 + c0;
+                if (!vrow || n >= p.N) continue;
+                float f[16];
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    float v = __uint_as_float(r[e]) + bv;
+                    f[e] = (p.relu && v < 0.f) ? 0.f : v;
+                }
+                if (n + 16 <= p.N) {
+                    uint4 a, b;
+                    a.x = pack2(f[0], f[1], p.dtype);
+                    a.y = pack2(f[2], f[3], p.dtype);
+                    a.z = pack2(f[4], f[5], p.dtype);
+                    a.w = pack2(f[6], f[7], p.dtype);
+                    b.x = pack2(f[8], f[9], p.dtype);
+                    b.y = pack2(f[10], f[11], p.dtype);
+                    b.z = pack2(f[12], f[13], p.dtype);
+                    b.w = pack2(f[14], f[15], p.dtype);
+                    uint4 *dst = reinterpret_cast<uint4 *>(yrow + n);
+                    dst[0] = a;
+                    dst[1] = b;
+                } else {
+                    for (int e = 0; e < 16 && n + e < p.N; ++e) yrow[n + e] = cvt1(f[e], p.dtype);
+                }
+            }
+        } else {
+            const int64_t n = t.n0 + 32 * q + lane;
+            const bool vcol = n < p.N;
+            int64_t obase = 0;                 // output offset of this token / pixel
+            int64_t ostride = p.ldy;           // between consecutive output rows
+            if (CONV) {
+                const int64_t b = vcol ? n / p.HoWo : 0, hw = vcol ? n % p.HoWo : 0;
+                obase = b * p.M * p.HoWo + hw;
+                ostride = p.HoWo;
+            } else {
+                obase = n;
+            }
+            for (int c0 = 0; c0 < p.rows_pad; c0 += 16) {
+                uint32_t r[16];
+                if (has) {
+                    tmem_ld_32x32b_x16(tacc + c0, r);
+                    tmem_ld_wait();
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) r[e] = 0u;
+                }
+                if (!vcol) continue;
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const int64_t row = c0 + e;
+                    if (row < t.rows) {
+                        const int64_t m = t.rb * p.bm + row;
+                        float v = __uint_as_float(r[e]) + (p.bias ? p.bias[m] : 0.f);
+                        if (p.relu && v < 0.f) v = 0.f;
+                        p.Y[obase + m * ostride] = cvt1(v, p.dtype);
+                    }
+                }
+            }
+        }
+        if (has) {
+            tc_fence_before();
+            mbar_arrive(&s.tempty[acc]);
+            if (++acc == 2) {
+                acc = 0;
+                acc_phase ^= 1u;
+            }
+        }
+    }
+}
+
+template <bool WA, bool CONV>
+__global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_constant__ Params p) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    const Smem s = carve(smem_raw, p);
+    const int warp = threadIdx.x >> 5;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < p.stages; ++i) {
+            mbar_init(&s.full[i], kProducerThreads);
+            mbar_init(&s.empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&s.tfull[i], 1);
+            mbar_init(&s.tempty[i], 128);
+        }
+        mbar_init(s.drain, 1);
+        *s.abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == kMmaWarp) {
+        tmem_alloc(s.tmem_base, p.tmem_cols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *s.tmem_base;
+
+    if (warp < 4) {
+        producer<WA, CONV>(p, s);
+    } else if (warp == kMmaWarp) {
+        if ((threadIdx.x & 31) == 0) mma_issuer<WA>(p, s, tmem);
+        __syncwarp();
+    } else {
+        epilogue<WA, CONV>(p, s, tmem);
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == kMmaWarp) tmem_dealloc(tmem, p.tmem_cols);
+}
+
+uint32_t pow2_at_least(uint32_t v) {
+    uint32_t r = 32;
+    while (r < v) r <<= 1;
+    return r;
+}
+
+template <bool WA, bool CONV>
+cudaError_t launch_variant(Params &p, cudaStream_t st) {
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [] {
+        attr_err = cudaFuncSetAttribute(bp_mma_kernel<WA, CONV>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
+    });
+    if (attr_err != cudaSuccess) return attr_err;
+    const size_t smem = 1024 + (size_t)p.stages * (p.w_tile_bytes + p.x_tile_bytes) +
+                        (2 * (size_t)p.stages + 5) * 8 + 16;
+    const int64_t grid = p.num_items < num_sms() ? p.num_items : num_sms();
+    bp_mma_kernel<WA, CONV><<<(unsigned)grid, kThreads, smem, st>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, int64_t N,
+                       int64_t ldx, const float *bias, int relu, void *Y, int64_t ldy,
+                       const ConvShape *conv, cudaStream_t st) {
+    Params p{};
+    // GEMMs put 128-row weight slabs on the MMA M side when bm allows it;
+    // convolutions (and bm not a multiple of 128) put 128 pixels / tokens there.
+    // Both read the same device image when rows_pad <= 256.
+    const bool wa = conv == nullptr && dl.orient == kWeightA;
+    if (!wa && dl.rows_pad > 256) return cudaErrorInvalidValue;
+    const uint8_t *dev = static_cast<const uint8_t *>(P.dev);
+    p.dtype = P.lay.dtype;
+    p.relu = relu;
+    p.M = P.lay.M;
+    p.bm = P.lay.bm;
+    p.rows_pad = dl.rows_pad;
+    p.num_rb = P.num_rb;
+    p.nslab = wa ? dl.rows_pad / kSlab : 1;
+    p.N = N;
+    const int64_t nt = wa ? 256 : 128;
+    p.n_tiles = (N + nt - 1) / nt;
+    p.num_items = p.n_tiles * p.num_rb * p.nslab;
+    p.w_tile_bytes = (uint32_t)((wa ? kSlab : dl.rows_pad) * kBK * 2);
+    p.x_tile_bytes = (uint32_t)(nt * kBK * 2);
+    const int64_t budget = 200 * 1024;
+    int64_t stages = budget / (p.w_tile_bytes + p.x_tile_bytes);
+    if (stages > 8) stages = 8;
+    p.stages = stages;
+    p.acc_cols = pow2_at_least(wa ? 256u : (uint32_t)dl.rows_pad);
+    p.tmem_cols = 2 * p.acc_cols;
+    p.kc_ptr = reinterpret_cast<const int64_t *>(dev);
+    p.chunks = dev + dl.off_chunks;
+    p.tile_bytes = dl.tile_bytes;
+    p.chunk_bytes = dl.chunk_bytes;
+    p.X = static_cast<const uint16_t *>(X);
+    p.ldx = ldx;
+    p.Y = static_cast<uint16_t *>(Y);
+    p.ldy = ldy;
+    p.bias = bias;
+    p.watchdog_ns = watchdog_ns();
+    p.status = device_status_ptr();
+    if (conv) {
+        p.C = conv->C;
+        p.H = conv->H;
+        p.W = conv->W;
+        p.Ho = conv->Ho;
+        p.Wo = conv->Wo;
+        p.HoWo = conv->Ho * conv->Wo;
+        p.KK = (int64_t)conv->kh * conv->kw;
+        p.kw = conv->kw;
+        p.ph = conv->ph;
+        p.pw = conv->pw;
+        p.sh = conv->sh;
+        p.sw = conv->sw;
+    }
+    if (p.num_items == 0) return cudaSuccess;
+    if (conv) return launch_variant<false, true>(p, st);
+    return wa ? launch_variant<true, false>(p, st) : launch_variant<false, false>(p, st);
+}
+
+}  // namespace bp

@@ -1,0 +1,112 @@
+"""The C-ABI library loads on the CPU, exports every symbol include/bp.h
+declares, its ctypes mirror matches the C structs, and argument checks that
+run on the host reject bad calls without touching a GPU."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+from paper_2111_11581_gb300 import bp, build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "bp.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return bp.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(bp_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_header_declares_the_binding_exports():
+    assert declared_functions() == sorted(bp.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    out = subprocess.run(["nm", "-D", "--defined-only", bp.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (bp_\w+)", out))
+    for name in declared_functions():
+        assert name in exported, name
+        assert hasattr(lib, name)
+
+
+def test_ctypes_structs_match_header(tmp_path):
+    src = tmp_path / "sz.c"
+    src.write_text('#include "bp.h"\n#include <stdio.h>\n#include <stddef.h>\n'
+                   'int main(void){printf("%zu %zu %zu %zu %zu %zu\\n", sizeof(bp_layout),'
+                   ' offsetof(bp_layout, K), offsetof(bp_layout, bk), sizeof(bp_packed),'
+                   ' offsetof(bp_packed, rb_ptr), offsetof(bp_packed, dev_bytes)); return 0;}\n')
+    exe = tmp_path / "sz"
+    subprocess.run(["gcc", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)],
+                   check=True)
+    got = list(map(int, subprocess.run([str(exe)], capture_output=True, text=True,
+                                       check=True).stdout.split()))
+    want = [ctypes.sizeof(bp.Layout), bp.Layout.K.offset, bp.Layout.bk.offset,
+            ctypes.sizeof(bp.Packed), bp.Packed.rb_ptr.offset, bp.Packed.dev_bytes.offset]
+    assert got == want
+
+
+def test_status_strings_and_version(lib):
+    assert bp.status_string(bp.OK) == "ok"
+    assert bp.status_string(bp.ERR_TIMEOUT) == "kernel wait timed out"
+    assert bp.bp_version() >> 16 == 1
+
+
+def test_workspace_size_is_host_only(lib):
+    lay = bp.layout(bp.BLOCK_BASED, bp.BF16, 4096, 4096, 128, 32)
+    n = bp.bp_workspace_size(lay)
+    # fp64 score + keep byte per unit (RB * K units) plus small tables
+    assert n >= 32 * 4096 * 9
+    with pytest.raises(bp.BpError):
+        bp.bp_workspace_size(bp.layout(bp.BLOCK_BASED, bp.BF16, 0, 16, 16, 16))
+
+
+@pytest.mark.parametrize("bad", [
+    dict(scheme=2), dict(dtype=7), dict(M=0), dict(K=0), dict(bm=0), dict(bk=0),
+    dict(kh=3, kw=3, K=10),            # K not a multiple of kh*kw
+])
+def test_host_argument_checks(lib, bad):
+    args = dict(scheme=0, dtype=1, M=64, K=64, bm=16, bk=16, kh=1, kw=1)
+    args.update(bad)
+    lay = bp.Layout(args["scheme"], args["dtype"], args["M"], args["K"], args["kh"], args["kw"],
+                    args["bm"], args["bk"])
+    assert bp.bp_prune(lay, 16, 2.0, 16, 256, 1 << 20, 0) == bp.ERR_INVALID_ARG
+
+
+def test_rate_below_one_rejected_on_host(lib):
+    lay = bp.layout(bp.BLOCK_BASED, bp.F16, 64, 64, 16, 16)
+    assert bp.bp_prune(lay, 16, 0.5, 16, 256, 1 << 20, 0) == bp.ERR_INVALID_ARG
+    assert bp.bp_prune(lay, 16, float("nan"), 16, 256, 1 << 20, 0) == bp.ERR_INVALID_ARG
+    assert bp.bp_prune(lay, 16, 2.0, 16, 256, 16, 0) == bp.ERR_WORKSPACE
+
+
+def test_gemm_argument_checks_on_host(lib):
+    lay = bp.layout(bp.BLOCK_BASED, bp.F16, 64, 64, 16, 16)
+    P = bp.Packed(lay, 4, 0, 0, 16, 16, 16, 256, 1 << 12)
+    # ldx not a multiple of 8, misaligned X, N > ldx, null packed
+    assert bp.bp_gemm(P, 256, 10, 10, None, 0, 256, 16, 0) == bp.ERR_INVALID_ARG
+    assert bp.bp_gemm(P, 258, 8, 8, None, 0, 256, 8, 0) == bp.ERR_INVALID_ARG
+    assert bp.bp_gemm(P, 256, 16, 8, None, 0, 256, 16, 0) == bp.ERR_INVALID_ARG
+    assert bp.load().bp_gemm(None, 256, 8, 8, None, 0, 256, 8, None) == bp.ERR_INVALID_ARG
+    # bm > 256 and not a multiple of 128 has no tensor-core path
+    lay2 = bp.layout(bp.BLOCK_BASED, bp.F16, 600, 64, 300, 16)
+    P2 = bp.Packed(lay2, 2, 0, 0, 16, 16, 16, 256, 1 << 12)
+    assert bp.bp_gemm(P2, 256, 8, 8, None, 0, 256, 8, 0) == bp.ERR_UNSUPPORTED
+
+
+def test_conv_argument_checks_on_host(lib):
+    lay = bp.layout(bp.BLOCK_PUNCHED, bp.F16, 16, 8 * 9, 8, 4, 3, 3)
+    P = bp.Packed(lay, 2, 0, 0, 16, 16, 16, 256, 1 << 12)
+    # C*kh*kw != K, negative pad, zero stride
+    assert bp.bp_conv2d(P, 256, 2, 7, 8, 8, 1, 1, 1, 1, None, 0, 256, 0) == bp.ERR_INVALID_ARG
+    assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, -1, 1, 1, 1, None, 0, 256, 0) == bp.ERR_INVALID_ARG
+    assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, 1, 1, 0, 1, None, 0, 256, 0) == bp.ERR_INVALID_ARG

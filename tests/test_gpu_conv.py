@@ -1,0 +1,66 @@
+"""GPU parity of bp_conv2d against the CPU oracle's masked direct convolution."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2111_11581_gb300 import bp, inputs
+from tests._util import assert_close, dev16, host_bits
+
+pytestmark = pytest.mark.gpu
+BB, BPU = bp.BLOCK_BASED, bp.BLOCK_PUNCHED
+
+
+def _run(F, C, kh, kw, Nb, H, W_, pad, stride, scheme, bm, bk, rate, dtype, seed, bias=True,
+         relu=True, oracle_images=None):
+    Wt = inputs.normal((F, C, kh, kw), inputs.kaiming_std(C * kh * kw), dtype, seed)
+    x = inputs.normal((Nb, C, H, W_), 1.0, dtype, seed + 1)
+    b = inputs.bias(F, 0.01, seed + 2) if bias else None
+    lay = bp.layout(scheme, dtype, F, C * kh * kw, bm, bk, kh, kw)
+    Wd = dev16(Wt.reshape(F, -1), dtype)
+    mask = bp.prune(lay, Wd, rate)
+    pw = bp.pack(lay, Wd, mask)
+    xd = dev16(x, dtype)
+    bd = torch.from_numpy(b).cuda() if b is not None else None
+    out = bp.conv2d(pw, xd, pad=(pad, pad), stride=(stride, stride), bias=bd, relu=relu)
+    torch.cuda.synchronize()
+    assert bp.device_status() == bp.OK
+    m = mask.cpu().numpy()
+    nb = Nb if oracle_images is None else oracle_images
+    ref = oracle.masked_conv2d(Wt, m, x[:nb], dtype, pad=(pad, pad), stride=(stride, stride),
+                               bias=b, relu=relu)
+    assert_close(host_bits(out)[:nb], ref, dtype, "bp_conv2d")
+    return out, Wd, mask, xd, bd
+
+
+CASES = [
+    # F, C, kh, kw, Nb, H, W, pad, stride, scheme, bm, bk, rate, dtype
+    (16, 8, 3, 3, 2, 8, 8, 1, 1, BPU, 8, 4, 3.0, bp.F16),
+    (24, 12, 3, 3, 3, 11, 9, 1, 2, BPU, 8, 4, 8.0, bp.BF16),     # stride 2, odd sizes, extras
+    (40, 20, 3, 3, 2, 14, 14, 1, 1, BPU, 16, 8, 8.0, bp.BF16),   # partial filter/channel blocks
+    (64, 32, 1, 1, 2, 7, 7, 0, 1, BB, 32, 32, 8.0, bp.BF16),     # 1x1 as block-based
+    (64, 48, 1, 1, 2, 14, 14, 0, 2, BB, 32, 32, 6.0, bp.F16),    # 1x1 stride 2 (downsample)
+    (16, 3, 7, 7, 2, 20, 20, 3, 2, BPU, 8, 2, 4.0, bp.BF16),     # 7x7 stride 2
+    (20, 8, 3, 3, 1, 5, 6, 2, 1, BB, 4, 16, 2.0, bp.F16),        # block-based on a 3x3 view
+    (128, 16, 3, 3, 2, 9, 9, 1, 1, BPU, 128, 4, 3.0, bp.BF16),   # bm = 128 filters
+    (8, 8, 3, 3, 4, 4, 4, 1, 1, BPU, 8, 4, 9.0, bp.F16),         # keep 1 of 9
+]
+
+
+@pytest.mark.parametrize("case", CASES, ids=lambda c: f"F{c[0]}C{c[1]}k{c[2]}s{c[8]}_b{c[10]}x{c[11]}_r{c[12]:g}")
+def test_conv_matches_oracle(case):
+    F, C, kh, kw, Nb, H, W_, pad, stride, scheme, bm, bk, rate, dtype = case
+    _run(F, C, kh, kw, Nb, H, W_, pad, stride, scheme, bm, bk, rate, dtype, seed=F * C + H)
+
+
+def test_conv3x3_full_size():
+    """3x3 CONV, N=128, C=F=128, 16x16, pad 1, blocks 8 filters x 4 channels keep 3
+    of 9 positions, bias, ReLU.  The oracle recomputes 16 of the 128 images; the
+    whole batch is also checked against cuDNN on the masked weight."""
+    L = inputs.conv3x3_128()
+    out, Wd, mask, xd, bd = _run(L.M, L.C, 3, 3, L.N, L.H, L.W, 1, 1, BPU, L.bm, L.bk, L.rate,
+                                 bp.F16, seed=L.seed, oracle_images=16)
+    wm = (Wd.float() * mask.float()).reshape(L.M, L.C, 3, 3)
+    ref = torch.relu(torch.nn.functional.conv2d(xd.float(), wm, bd, padding=1))
+    err = (out.float() - ref).abs()
+    assert bool((err <= 1e-2 * ref.abs().clamp_min(1.0)).all())

@@ -1,0 +1,140 @@
+"""GPU parity of bp_prune / bp_pack_size / bp_pack against the CPU oracle:
+masks, rb_ptr, col_idx and values must match bit for bit, and the tiled
+device image must decode back to the same weights and column lists."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2111_11581_gb300 import bp, inputs
+from tests._util import dev16
+
+pytestmark = pytest.mark.gpu
+BB, BP_ = bp.BLOCK_BASED, bp.BLOCK_PUNCHED
+
+CASES = [
+    # scheme, dtype, M, K, kh, kw, bm, bk, rate
+    (BB, bp.F16, 512, 512, 1, 1, 16, 16, 4.0),            # FC 512x512, keep 4 of 16
+    (BP_, bp.F16, 128, 128 * 9, 3, 3, 8, 4, 3.0),         # 3x3 CONV, keep 3 of 9
+    (BP_, bp.F16, 256, 128 * 9, 3, 3, 8, 4, 8.0),         # VGG layer: base 1 + extras
+    (BP_, bp.BF16, 64, 64 * 9, 3, 3, 16, 8, 8.0),         # ResNet 3x3 blocks
+    (BB, bp.BF16, 256, 64, 1, 1, 32, 32, 8.0),            # ResNet 1x1 reduce
+    (BB, bp.BF16, 10, 512, 1, 1, 16, 16, 8.0),            # FC 512->10, one partial row-block
+    (BB, bp.BF16, 1000, 2048, 1, 1, 32, 32, 6.0),         # FC 2048->1000, partial last block
+    (BB, bp.BF16, 768, 3072, 1, 1, 128, 8, 16.0),         # bk*keep < 1: all kept units are extras
+    (BB, bp.F16, 100, 96, 1, 1, 16, 10, 8.0 / 3.0),       # partial row/col blocks, base + extras
+    (BB, bp.F16, 64, 80, 1, 1, 1, 1, 3.0),                # unstructured special case
+    (BB, bp.BF16, 48, 256, 1, 1, 48, 8, 4.0),             # structured special case (bm = M)
+    (BB, bp.BF16, 384, 256, 1, 1, 128, 32, 2.0),          # bm = 128 (weight-as-A tiles)
+    (BB, bp.F16, 512, 192, 1, 1, 256, 16, 4.0),           # bm = 256
+    (BP_, bp.F16, 24, 5 * 49, 7, 7, 8, 2, 5.0),           # 7x7 kernels, partial channel block
+]
+
+
+def _ids(c):
+    return f"s{c[0]}_d{c[1]}_{c[2]}x{c[3]}_k{c[4]}{c[5]}_b{c[6]}x{c[7]}_r{c[8]:.3g}"
+
+
+@pytest.mark.parametrize("case", CASES, ids=_ids)
+def test_prune_and_pack_bit_exact(case):
+    scheme, dtype, M, K, kh, kw, bm, bk, rate = case
+    W = inputs.normal((M, K), 0.05, dtype, seed=M * 7 + K)
+    lay = bp.layout(scheme, dtype, M, K, bm, bk, kh, kw)
+    Wd = dev16(W, dtype)
+    mask = bp.prune(lay, Wd, rate)
+    torch.cuda.synchronize()
+    ref_mask = oracle.prune(W, dtype, scheme, bm, bk, rate, kh, kw)
+    got = mask.cpu().numpy()
+    assert (got == ref_mask).all(), f"{int((got != ref_mask).sum())} mask bytes differ"
+
+    pw = bp.pack(lay, Wd, mask)
+    rb_ptr, col_idx, values = oracle.pack(W, ref_mask, bm)
+    assert (pw.rb_ptr.cpu().numpy() == rb_ptr).all()
+    assert (pw.col_idx.cpu().numpy() == col_idx).all()
+    assert (pw.values.cpu().view(torch.int16).numpy().view(np.uint16) == values).all()
+    _check_device_image(pw, rb_ptr, col_idx, values, M, bm)
+
+
+def _sw128(row, k):
+    return (row >> 3) * 1024 + (row & 7) * 128 + (((k >> 3) ^ (row & 7)) << 4) + (k & 7) * 2
+
+
+def _check_device_image(pw, rb_ptr, col_idx, values, M, bm):
+    """Decode the tiled image on the host: weights and padded column lists."""
+    if bm % 128 == 0:
+        rows_pad = bm
+    elif bm <= 256:
+        rows_pad = (bm + 15) // 16 * 16
+    else:
+        return
+    img = pw.dev.cpu().numpy()
+    RB = len(rb_ptr) - 1
+    kc_ptr = img[:8 * (RB + 1)].view(np.int64)
+    off = (8 * (RB + 1) + 255) // 256 * 256
+    tile_bytes = rows_pad * 128
+    chunk = tile_bytes + 256
+    assert img.size == off + kc_ptr[-1] * chunk
+    rows = np.arange(rows_pad)[:, None]
+    ks = np.arange(64)[None, :]
+    offs = _sw128(rows, ks)
+    for rb in range(RB):
+        kp = rb_ptr[rb + 1] - rb_ptr[rb]
+        nkc = kc_ptr[rb + 1] - kc_ptr[rb]
+        assert nkc == -(-kp // 64)
+        r_rb = min(bm, M - rb * bm)
+        vals = values[bm * rb_ptr[rb]: bm * rb_ptr[rb] + r_rb * kp].reshape(r_rb, kp)
+        for kc in range(nkc):
+            base = off + (kc_ptr[rb] + kc) * chunk
+            t = img[base:base + tile_bytes]
+            dec = t.view(np.uint16)[offs // 2]
+            want = np.zeros((rows_pad, 64), np.uint16)
+            seg = vals[:, kc * 64: (kc + 1) * 64]
+            want[:r_rb, :seg.shape[1]] = seg
+            assert (dec == want).all(), (rb, kc)
+            cl = img[base + tile_bytes: base + chunk].view(np.int32)
+            wl = np.full(64, -1, np.int32)
+            s = col_idx[rb_ptr[rb] + kc * 64: min(rb_ptr[rb] + (kc + 1) * 64, rb_ptr[rb + 1])]
+            wl[:s.size] = s
+            assert (cl == wl).all(), (rb, kc)
+
+
+def test_prune_ties_resolved_like_oracle():
+    # every weight equal: all scores tie, so only the tie rule decides
+    M, K = 64, 96
+    W = oracle.round_to(np.full((M, K), 0.25), bp.F16)
+    for scheme, kh, kw, bm, bk, rate in [(BB, 1, 1, 16, 16, 2.5), (BB, 1, 1, 1, 1, 7.0),
+                                         (BP_, 3, 3, 8, 4, 8.0)]:
+        Kx = K if scheme == BB else 8 * 9
+        Wx = W[:, :Kx].copy()
+        lay = bp.layout(scheme, bp.F16, M, Kx, bm, bk, kh, kw)
+        mask = bp.prune(lay, dev16(Wx, bp.F16), rate).cpu().numpy()
+        assert (mask == oracle.prune(Wx, bp.F16, scheme, bm, bk, rate, kh, kw)).all()
+
+
+def test_prune_rejects_nonfinite():
+    W = inputs.normal((32, 32), 1.0, bp.F16, seed=3)
+    W[5, 7] = 0x7c00                     # +inf
+    lay = bp.layout(BB, bp.F16, 32, 32, 8, 8)
+    with pytest.raises(bp.BpError) as e:
+        bp.prune(lay, dev16(W, bp.F16), 2.0)
+    assert e.value.status == bp.ERR_NONFINITE
+
+
+def test_pack_rejects_rows_that_disagree():
+    lay = bp.layout(BB, bp.F16, 32, 32, 8, 8)
+    mask = torch.ones((32, 32), dtype=torch.uint8, device="cuda")
+    mask[3, 5] = 0                        # row 3 differs from row 0 of its row-block
+    rb_ptr = torch.empty(5, dtype=torch.int64, device="cuda")
+    st, *_ = bp.bp_pack_size(lay, mask.data_ptr(), rb_ptr.data_ptr(), 0)
+    assert st == bp.ERR_INVALID_ARG
+
+
+def test_rate_one_keeps_everything_and_all_pruned_layer():
+    W = inputs.normal((40, 24), 1.0, bp.BF16, seed=4)
+    lay = bp.layout(BB, bp.BF16, 40, 24, 8, 8)
+    assert bp.prune(lay, dev16(W, bp.BF16), 1.0).cpu().numpy().all()
+    # rate so high that T rounds to 0: nothing kept, every K'_rb = 0
+    mask = bp.prune(lay, dev16(W, bp.BF16), 1e9)
+    assert int(mask.sum()) == 0
+    pw = bp.pack(lay, dev16(W, bp.BF16), mask)
+    assert int(pw.c.nnz_cols) == 0
