@@ -170,6 +170,14 @@ bp_status bp_device_status(void *stream);
  * after this call (default 2e9).  0 restores the default. */
 bp_status bp_set_watchdog_ns(uint64_t ns);
 
+/* Fault injection for tests of the bounded waits: from the next launch on,
+ * CTA 0 of every bp_gemm / bp_conv2d kernel skips filling its pipeline stage
+ * number `stage` (0-based, counted over the CTA's whole run), so the tensor-
+ * core warp waits for data that never comes, its wait expires after the
+ * watchdog budget, the kernel records BP_ERR_TIMEOUT and returns (the output
+ * is then invalid).  -1 (the default) turns it off.  Nothing faults. */
+bp_status bp_debug_drop_stage(int64_t stage);
+
 #ifdef __cplusplus
 }
 #endif

@@ -35,7 +35,8 @@ class Packed(ctypes.Structure):
 
 
 EXPORTS = ("bp_status_string", "bp_version", "bp_workspace_size", "bp_prune", "bp_pack_size",
-           "bp_pack", "bp_gemm", "bp_conv2d", "bp_device_status", "bp_set_watchdog_ns")
+           "bp_pack", "bp_gemm", "bp_conv2d", "bp_device_status", "bp_set_watchdog_ns",
+           "bp_debug_drop_stage")
 
 _lib = None
 _lock = threading.Lock()
@@ -72,6 +73,7 @@ def load(path: str = LIB_PATH):
                                 vp]),
             "bp_device_status": (i32, [vp]),
             "bp_set_watchdog_ns": (i32, [ctypes.c_uint64]),
+            "bp_debug_drop_stage": (i32, [i64]),
         }
         for name, (res, args) in sig.items():
             f = getattr(lib, name)
@@ -134,6 +136,10 @@ def bp_device_status(stream: int = 0) -> int:
 
 def bp_set_watchdog_ns(ns: int) -> int:
     return load().bp_set_watchdog_ns(int(ns))
+
+
+def bp_debug_drop_stage(stage: int) -> int:
+    return load().bp_debug_drop_stage(int(stage))
 
 
 # ------------------------------------------------------------------ torch marshalling

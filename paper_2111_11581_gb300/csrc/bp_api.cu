@@ -20,6 +20,7 @@ __device__ int g_pack_bad;
 namespace {
 constexpr uint64_t kDefaultWatchdogNs = 2000000000ull;
 uint64_t g_watchdog_ns = kDefaultWatchdogNs;
+int64_t g_drop_stage = -1;
 std::mutex g_mu;            // guards the per-device caches and g_pack_bad
 constexpr int kMaxDev = 64;
 unsigned *g_status_ptr[kMaxDev];
@@ -96,6 +97,7 @@ PruneWs prune_ws(const bp_layout &l) {
 }  // namespace
 
 uint64_t watchdog_ns() { return g_watchdog_ns; }
+int64_t debug_drop_stage() { return g_drop_stage; }
 
 unsigned *device_status_ptr() {
     std::lock_guard<std::mutex> lk(g_mu);
@@ -379,6 +381,12 @@ bp_status bp_device_status(void *stream) {
 
 bp_status bp_set_watchdog_ns(uint64_t ns) {
     g_watchdog_ns = ns ? ns : kDefaultWatchdogNs;
+    return BP_OK;
+}
+
+bp_status bp_debug_drop_stage(int64_t stage) {
+    if (stage < -1) return BP_ERR_INVALID_ARG;
+    g_drop_stage = stage;
     return BP_OK;
 }
 

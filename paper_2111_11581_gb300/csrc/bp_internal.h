@@ -28,7 +28,8 @@ enum Orientation { kWeightA = 0, kWeightB = 1, kNoTensorCore = 2 };
 //   off_chunks + c*chunk_bytes  k-chunk c: its (rows_pad x 64) 16-bit weight
 //                               tile in K-major 128-byte-swizzled order,
 //                               followed by its 64 int32 column indices
-//                               (-1 = padding, read as zeros).
+//                               (padding repeats the last kept column; its
+//                               weights are zero).
 struct DevLayout {
     Orientation orient;
     int64_t rows_pad;     // rows per k-chunk tile
@@ -48,6 +49,7 @@ DevLayout dev_layout(const bp_layout &lay, const int64_t *rb_ptr_host);
 
 // Library-wide settings.
 uint64_t watchdog_ns();
+int64_t debug_drop_stage();     // -1 = no fault injection
 unsigned *device_status_ptr();   // device address of the status word
 int num_sms();
 bool checked_mode();

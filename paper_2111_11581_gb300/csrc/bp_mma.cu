@@ -3,18 +3,22 @@
 // Each work item is one row-block (or one 128-row slab of it) times one tile
 // of activation columns.  The row-block's compact weights Wc (bm x K'_rb,
 // Sec. 4.3) multiply the activation rows selected by its kept-column list, so
-// pruned weights never enter the product.  Per k-chunk of 64 kept columns:
+// pruned weights never enter the product.  Per k-chunk of 64 kept columns a
+// pipeline stage holds the chunk's pre-swizzled weight tile and the 64
+// activation rows it names, laid out as a 128-byte-swizzled MN-major tile:
 //
-//   producer warps 0-3  copy the pre-swizzled weight tile (cp.async) and
-//                       gather the 64 activation rows named by the chunk's
-//                       column list into a 128-byte-swizzled MN-major tile
-//                       (GEMM: rows of X; conv: im2col rows built on the fly,
-//                       zero outside the image);
-//   MMA warp 4          issues tcgen05.mma (K = 16 per instruction) into an
-//                       fp32 accumulator in tensor memory, double-buffered
-//                       across work items;
-//   epilogue warps 5-8  read the accumulator (tcgen05.ld), add the bias,
-//                       apply ReLU, round to fp16/bf16 and store.
+//   warps 0-3   producers.  Thread 0 copies the weight tile with one TMA
+//               bulk copy (completion counted in bytes on the stage's
+//               weight barrier).  GEMM: the 128 threads gather the rows of X
+//               with 16-byte cp.async (one 512- or 256-byte row segment per
+//               warp instruction) and arrive on the stage's data barrier
+//               when their copies land, without blocking.  CONV: im2col rows
+//               are built in registers (zero outside the image) and stored.
+//               (TMA tile::gather4 moves 4 x 128 B per instruction and
+//               measured about 6x slower per byte than this path.)
+//   warp 4      MMA issuer: tcgen05.mma (K = 16 per instruction) into an
+//               fp32 accumulator in tensor memory, double-buffered;
+//   warps 5-8   epilogue: tcgen05.ld, + bias, ReLU, round to fp16/bf16, store.
 //
 // Two operand orientations:
 //   kWeightA (bm a multiple of 128): D[128 weight rows x 256 tokens]
@@ -35,22 +39,22 @@
 namespace bp {
 namespace {
 
-constexpr int kThreads = 288;          // 9 warps
-constexpr int kProducerThreads = 128;
-constexpr int kMmaWarp = 4;
-constexpr int kLag = 2;                // cp.async groups in flight per producer thread
 constexpr uint64_t kDrainNs = 1000000000ull;
+constexpr int kMaxStages = 8;
+constexpr int kPrefetch = 6;           // index lists loaded this many stages ahead
+constexpr int kMaxCachedRb = 2047;     // kc_ptr kept in shared memory up to this many row-blocks
 
 struct Params {
     int dtype;
     int relu;
     int64_t M, bm, rows_pad, num_rb, nslab;
     int64_t N;              // tokens (GEMM) or Nb*Ho*Wo pixels (conv)
-    int64_t n_tiles, num_items;
+    int64_t num_items;
     int64_t stages;
     uint32_t w_tile_bytes, x_tile_bytes, tmem_cols, acc_cols;
     const int64_t *kc_ptr;
-    const uint8_t *chunks;       // k-chunks: weight tile, then 64 int32 column indices
+    int64_t kc_cached;      // entries of kc_ptr copied to shared memory (0 = none)
+    const uint8_t *chunks;  // k-chunks: weight tile, then 64 int32 column indices
     int64_t tile_bytes, chunk_bytes;
     const uint16_t *X;
     int64_t ldx;
@@ -61,8 +65,14 @@ struct Params {
     int64_t C, H, W, Ho, Wo, HoWo, KK;
     int kw, ph, pw, sh, sw;
     uint64_t watchdog_ns;
+    int64_t drop_stage;     // fault injection: CTA 0 never fills this stage (-1 = off)
     unsigned *status;
 };
+
+constexpr int kProducerWarps = 4;
+constexpr int kMmaWarp = 4;
+constexpr int kThreads = 288;
+constexpr uint32_t kProducerThreads = 128;
 
 __device__ __forceinline__ uint32_t pack2(float a, float b, int dtype) {
     if (dtype == BP_BF16) {
@@ -81,13 +91,15 @@ __device__ __forceinline__ uint16_t cvt1(float a, int dtype) {
 struct Smem {
     uint8_t *w;          // stages x w_tile_bytes
     uint8_t *x;          // stages x x_tile_bytes
-    uint64_t *full;      // [stages]
-    uint64_t *empty;     // [stages]
+    uint64_t *full;      // [stages] activation tile landed (128 producer arrivals)
+    uint64_t *wfull;     // [stages] weight tile landed (TMA byte count)
+    uint64_t *empty;     // [stages] tensor cores done with the stage
     uint64_t *tfull;     // [2]
     uint64_t *tempty;    // [2]
     uint64_t *drain;     // [1]
     uint32_t *tmem_base;
     int *abort_flag;
+    int64_t *kc;         // [kc_cached] copy of kc_ptr, or nullptr
 };
 
 __device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
@@ -98,12 +110,14 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
     s.x = base + p.stages * p.w_tile_bytes;
     uint8_t *b = s.x + p.stages * p.x_tile_bytes;
     s.full = reinterpret_cast<uint64_t *>(b);
-    s.empty = s.full + p.stages;
+    s.wfull = s.full + p.stages;
+    s.empty = s.wfull + p.stages;
     s.tfull = s.empty + p.stages;
     s.tempty = s.tfull + 2;
     s.drain = s.tempty + 2;
     s.tmem_base = reinterpret_cast<uint32_t *>(s.drain + 1);
     s.abort_flag = reinterpret_cast<int *>(s.tmem_base + 1);
+    s.kc = p.kc_cached ? reinterpret_cast<int64_t *>(s.drain + 2) : nullptr;
     return s;
 }
 
@@ -116,54 +130,183 @@ struct Item {
     int64_t rb, slab, n0, kc0, nkc, rows;   // rows = real rows of the row-block
 };
 
-__device__ __forceinline__ Item decode(const Params &p, int64_t it, bool wa) {
+__device__ __forceinline__ Item decode(const Params &p, const int64_t *kc, int64_t it, bool wa) {
     Item t;
     const int64_t R = p.num_rb * p.nslab;
     const int64_t rs = it % R;
     t.n0 = (it / R) * (wa ? 256 : 128);
     t.rb = rs / p.nslab;
     t.slab = rs % p.nslab;
-    t.kc0 = p.kc_ptr[t.rb];
-    t.nkc = p.kc_ptr[t.rb + 1] - t.kc0;
+    t.kc0 = kc[t.rb];
+    t.nkc = kc[t.rb + 1] - t.kc0;
     t.rows = min(p.bm, p.M - t.rb * p.bm);
     return t;
 }
 
-// ------------------------------------------------------------------ producer
-template <bool WA, bool CONV>
-__device__ void producer(const Params &p, const Smem &s) {
+// Walks this CTA's (work item, k-chunk) sequence, skipping empty row-blocks.
+struct Cursor {
+    int64_t it;
+    int64_t kc;
+    Item t;
+    __device__ __forceinline__ void first(const Params &p, const int64_t *kcp, bool wa) {
+        kc = 0;
+        for (it = blockIdx.x; it < p.num_items; it += gridDim.x) {
+            t = decode(p, kcp, it, wa);
+            if (t.nkc > 0) return;
+        }
+    }
+    __device__ __forceinline__ void next(const Params &p, const int64_t *kcp, bool wa) {
+        if (++kc < t.nkc) return;
+        kc = 0;
+        for (it += gridDim.x; it < p.num_items; it += gridDim.x) {
+            t = decode(p, kcp, it, wa);
+            if (t.nkc > 0) return;
+        }
+    }
+    __device__ __forceinline__ bool valid(const Params &p) const { return it < p.num_items; }
+};
+
+// ------------------------------------------------------------------ producers
+// Weight tile of a stage: thread 0 of the producers, TMA bulk copy.
+struct WeightCopier {
+    uint32_t last_phase[kMaxStages];
+    bool issued[kMaxStages];
+    __device__ __forceinline__ void init() {
+        for (int i = 0; i < kMaxStages; ++i) issued[i] = false;
+    }
+    __device__ __forceinline__ void copy(const Params &p, const Smem &s, int stage, uint32_t phase,
+                                         const uint8_t *src) {
+        mbar_arrive_expect_tx(&s.wfull[stage], p.w_tile_bytes);
+        bulk_g2s(smem_u32(s.w + stage * p.w_tile_bytes), src, p.w_tile_bytes, &s.wfull[stage]);
+        issued[stage] = true;
+        last_phase[stage] = phase;
+    }
+    // the CTA is unwinding: let every weight copy already issued land first
+    __device__ __forceinline__ void drain(const Params &p, const Smem &s) {
+        for (int i = 0; i < p.stages; ++i)
+            if (issued[i] && !mbar_wait(&s.wfull[i], last_phase[i], kDrainNs, nullptr))
+                atomicOr(p.status, kDevTimeout);
+    }
+};
+
+template <bool WA>
+__device__ void producer_gather(const Params &p, const Smem &s) {
+    const int tid = threadIdx.x;            // 0..127
+    const int warp = tid >> 5, lane = tid & 31;
+    const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
+    volatile int *abort_flag = s.abort_flag;
+    WeightCopier wc;
+    wc.init();
+    auto load_idx = [&](const Cursor &c) {
+        const int32_t *cl = reinterpret_cast<const int32_t *>(
+            p.chunks + (c.t.kc0 + c.kc) * p.chunk_bytes + p.tile_bytes);
+        return make_int2(__ldg(cl + lane), __ldg(cl + lane + 32));
+    };
+    // ring[i]: this lane's two entries of the index list i chunks after the next one
+    Cursor cur, look;
+    cur.first(p, kcp, WA);
+    look = cur;
+    int2 ring[kPrefetch];
+#pragma unroll
+    for (int i = 0; i < kPrefetch; ++i) {
+        ring[i] = look.valid(p) ? load_idx(look) : make_int2(0, 0);
+        if (look.valid(p)) look.next(p, kcp, WA);
+    }
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    int64_t count = 0;
+    while (cur.valid(p)) {
+        const Item t = cur.t;
+        const int64_t kc = cur.kc;
+        const int2 iv = ring[0];
+#pragma unroll
+        for (int i = 0; i + 1 < kPrefetch; ++i) ring[i] = ring[i + 1];
+        ring[kPrefetch - 1] = look.valid(p) ? load_idx(look) : make_int2(0, 0);
+        if (look.valid(p)) look.next(p, kcp, WA);
+        cur.next(p, kcp, WA);
+        const bool drop = blockIdx.x == 0 && count++ == p.drop_stage;
+        if (!mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)) {
+            raise_timeout(p, s);
+            ok = false;
+            break;
+        }
+        if (!drop) {
+            const uint8_t *chunk = p.chunks + (t.kc0 + kc) * p.chunk_bytes;
+            if (tid == 0) wc.copy(p, s, stage, phase, chunk + t.slab * (kSlab * kBK * 2));
+            const uint32_t xs = smem_u32(s.x + stage * p.x_tile_bytes);
+            if (WA) {
+                // 64 rows x 256 tokens: one warp instruction per row segment of 512 B
+                const int cn = lane >> 3, j = lane & 7;
+                const int64_t n = t.n0 + lane * 8;
+                const uint32_t nb = n < p.N ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
+                const uint16_t *xcol = p.X + (nb ? n : 0);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int r = warp + 4 * i;
+                    const int idx = __shfl_sync(0xffffffffu, i < 8 ? iv.x : iv.y, r & 31);
+                    cp_async_16(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4),
+                                xcol + (int64_t)idx * p.ldx, nb);
+                }
+            } else {
+                // 64 rows x 128 tokens: one warp instruction covers two rows
+                const int u16 = lane & 15, cn = u16 >> 3, j = u16 & 7;
+                const int64_t n = t.n0 + u16 * 8;
+                const uint32_t nb = n < p.N ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
+                const uint16_t *xcol = p.X + (nb ? n : 0);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int r = 2 * (warp + 4 * i) + (lane >> 4);
+                    const int idx = __shfl_sync(0xffffffffu, i < 4 ? iv.x : iv.y, r & 31);
+                    cp_async_16(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4),
+                                xcol + (int64_t)idx * p.ldx, nb);
+                }
+            }
+            cp_async_arrive_noinc(&s.full[stage]);
+        }
+        if (++stage == p.stages) {
+            stage = 0;
+            phase ^= 1u;
+        }
+    }
+    cp_async_wait_all();
+    if (!ok && tid == 0) wc.drain(p, s);
+}
+
+// ------------------------------------------------------------------ CONV producer (im2col)
+__device__ void producer_im2col(const Params &p, const Smem &s) {
+    const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     const int tid = threadIdx.x;            // 0..127
     const int warp = tid >> 5, lane = tid & 31;
     volatile int *abort_flag = s.abort_flag;
     int stage = 0;
     uint32_t phase = 0;
-    int pend[kLag + 1];
-    int npend = 0;
     bool ok = true;
-    const uint32_t w_units = p.w_tile_bytes >> 4;
+    const int u16 = lane & 15;           // 16-byte unit (8 pixels) within a 128-pixel row
+    const int cn = u16 >> 3, j = u16 & 7;
+    int64_t count = 0;
+    WeightCopier wc;
+    wc.init();
 
     for (int64_t it = blockIdx.x; it < p.num_items && ok; it += gridDim.x) {
-        const Item t = decode(p, it, WA);
+        const Item t = decode(p, kcp, it, false);
         if (t.nkc == 0) continue;
-        // convolution: this thread's 8 pixels are fixed for the whole tile
+        // this thread's 8 pixels are fixed for the whole tile
         int64_t pbase[8];
         int ih0[8], iw0[8];
-        const int u16 = lane & 15;           // 16-byte unit within a 128-token row
-        if (CONV) {
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                const int64_t pix = t.n0 + u16 * 8 + e;
-                if (pix < p.N) {
-                    const int64_t b = pix / p.HoWo, hw = pix % p.HoWo;
-                    const int oh = (int)(hw / p.Wo), ow = (int)(hw % p.Wo);
-                    pbase[e] = b * p.C * p.H * p.W;
-                    ih0[e] = oh * p.sh - p.ph;
-                    iw0[e] = ow * p.sw - p.pw;
-                } else {
-                    pbase[e] = 0;
-                    ih0[e] = -(1 << 29);     // never inside the image
-                    iw0[e] = 0;
-                }
+        for (int e = 0; e < 8; ++e) {
+            const int64_t pix = t.n0 + u16 * 8 + e;
+            if (pix < p.N) {
+                const int64_t b = pix / p.HoWo, hw = pix % p.HoWo;
+                const int oh = (int)(hw / p.Wo), ow = (int)(hw % p.Wo);
+                pbase[e] = b * p.C * p.H * p.W;
+                ih0[e] = oh * p.sh - p.ph;
+                iw0[e] = ow * p.sw - p.pw;
+            } else {
+                pbase[e] = 0;
+                ih0[e] = -(1 << 29);     // never inside the image
+                iw0[e] = 0;
             }
         }
         for (int64_t kc = 0; kc < t.nkc; ++kc) {
@@ -172,98 +315,52 @@ __device__ void producer(const Params &p, const Smem &s) {
                 ok = false;
                 break;
             }
-            const uint32_t ws = smem_u32(s.w + stage * p.w_tile_bytes);
-            const uint32_t xs = smem_u32(s.x + stage * p.x_tile_bytes);
-            // weight tile: contiguous pre-swizzled bytes
-            const uint8_t *chunk = p.chunks + (t.kc0 + kc) * p.chunk_bytes;
-            const uint8_t *wsrc = chunk + t.slab * (kSlab * kBK * 2);
-            for (uint32_t u = tid; u < w_units; u += kProducerThreads)
-                cp_async_16(ws + u * 16, wsrc + (size_t)u * 16, 16);
-            const int32_t *cl = reinterpret_cast<const int32_t *>(chunk + p.tile_bytes);
-            if (!CONV) {
-                if (WA) {
-                    // 64 rows x 32 units (256 tokens); one warp covers one row
-                    const int cn = lane >> 3, j = lane & 7;
-                    const int64_t n = t.n0 + lane * 8;
-                    const uint32_t nb = n < p.N ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
-#pragma unroll 4
-                    for (int i = 0; i < 16; ++i) {
-                        const int r = warp + 4 * i;
-                        const int32_t idx = cl[r];
-                        const bool live = idx >= 0 && nb > 0;
-                        const uint16_t *src = live ? p.X + idx * p.ldx + n : p.X;
-                        cp_async_16(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4), src,
-                                    live ? nb : 0u);
-                    }
-                } else {
-                    // 64 rows x 16 units (128 tokens); one warp covers two rows
-                    const int cn = u16 >> 3, j = u16 & 7;
-                    const int64_t n = t.n0 + u16 * 8;
-                    const uint32_t nb = n < p.N ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
-#pragma unroll 4
-                    for (int i = 0; i < 8; ++i) {
-                        const int r = 2 * (warp + 4 * i) + (lane >> 4);
-                        const int32_t idx = cl[r];
-                        const bool live = idx >= 0 && nb > 0;
-                        const uint16_t *src = live ? p.X + idx * p.ldx + n : p.X;
-                        cp_async_16(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4), src,
-                                    live ? nb : 0u);
-                    }
+            if (blockIdx.x == 0 && count++ == p.drop_stage) {   // injected lost stage
+                if (++stage == p.stages) {
+                    stage = 0;
+                    phase ^= 1u;
                 }
-                cp_async_commit();
-                pend[npend++] = stage;
-                if (npend > kLag) {
-                    cp_async_wait_group<kLag>();
-                    fence_proxy_async_smem();
-                    mbar_arrive(&s.full[pend[0]]);
-#pragma unroll
-                    for (int q = 0; q < kLag; ++q) pend[q] = pend[q + 1];
-                    --npend;
-                }
-            } else {
-                // im2col rows of 128 pixels, built in registers
-                const int cn = u16 >> 3, j = u16 & 7;
-#pragma unroll 2
-                for (int i = 0; i < 8; ++i) {
-                    const int r = 2 * (warp + 4 * i) + (lane >> 4);
-                    const int32_t idx = cl[r];
-                    uint32_t v[4] = {0u, 0u, 0u, 0u};
-                    if (idx >= 0) {
-                        const int64_t c = idx / p.KK;
-                        const int rs = (int)(idx - c * p.KK);
-                        const int di = rs / p.kw, dj = rs - (rs / p.kw) * p.kw;
-                        const uint16_t *plane = p.X + c * p.H * p.W;
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            const int ih = ih0[e] + di, iw = iw0[e] + dj;
-                            uint32_t h = 0u;
-                            if ((unsigned)ih < (unsigned)p.H && (unsigned)iw < (unsigned)p.W)
-                                h = __ldg(plane + pbase[e] + (int64_t)ih * p.W + iw);
-                            v[e >> 1] |= h << ((e & 1) * 16);
-                        }
-                    }
-                    st_shared_v4(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4),
-                                 make_uint4(v[0], v[1], v[2], v[3]));
-                }
-                cp_async_wait_all();
-                fence_proxy_async_smem();
-                mbar_arrive(&s.full[stage]);
+                continue;
             }
+            const uint32_t xs = smem_u32(s.x + stage * p.x_tile_bytes);
+            const uint8_t *chunk = p.chunks + (t.kc0 + kc) * p.chunk_bytes;
+            if (tid == 0) wc.copy(p, s, stage, phase, chunk);
+            const int32_t *cl = reinterpret_cast<const int32_t *>(chunk + p.tile_bytes);
+#pragma unroll 2
+            for (int i = 0; i < 8; ++i) {
+                const int r = 2 * (warp + 4 * i) + (lane >> 4);
+                const int32_t idx = cl[r];
+                uint32_t v[4] = {0u, 0u, 0u, 0u};
+                const int64_t c = idx / p.KK;
+                const int rs = (int)(idx - c * p.KK);
+                const int di = rs / p.kw, dj = rs - (rs / p.kw) * p.kw;
+                const uint16_t *plane = p.X + c * p.H * p.W;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const int ih = ih0[e] + di, iw = iw0[e] + dj;
+                    uint32_t h = 0u;
+                    if ((unsigned)ih < (unsigned)p.H && (unsigned)iw < (unsigned)p.W)
+                        h = __ldg(plane + pbase[e] + (int64_t)ih * p.W + iw);
+                    v[e >> 1] |= h << ((e & 1) * 16);
+                }
+                st_shared_v4(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4),
+                             make_uint4(v[0], v[1], v[2], v[3]));
+            }
+            fence_proxy_async_smem();
+            mbar_arrive(&s.full[stage]);
             if (++stage == p.stages) {
                 stage = 0;
                 phase ^= 1u;
             }
         }
     }
-    cp_async_wait_all();
-    fence_proxy_async_smem();
-    if (ok)
-        for (int q = 0; q < npend; ++q) mbar_arrive(&s.full[pend[q]]);
+    if (!ok && tid == 0) wc.drain(p, s);
 }
 
 // ------------------------------------------------------------------ MMA issuer
 template <bool WA>
 __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
+    const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
     const bool bf16 = p.dtype == BP_BF16;
     const uint32_t idesc = WA ? make_idesc(bf16, false, true, 128, 256)
@@ -274,7 +371,7 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
     uint32_t acc_phase = 0;
     bool ok = true;
     for (int64_t it = blockIdx.x; it < p.num_items && ok; it += gridDim.x) {
-        const Item t = decode(p, it, WA);
+        const Item t = decode(p, kcp, it, WA);
         if (t.nkc == 0) continue;
         if (!mbar_wait(&s.tempty[acc], acc_phase ^ 1u, p.watchdog_ns, abort_flag)) {
             raise_timeout(p, s);
@@ -283,11 +380,15 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
         tc_fence_after();
         const uint32_t d = tmem + acc * p.acc_cols;
         for (int64_t kc = 0; kc < t.nkc; ++kc) {
-            if (!mbar_wait(&s.full[stage], phase, p.watchdog_ns, abort_flag)) {
+            if (!mbar_wait(&s.full[stage], phase, p.watchdog_ns, abort_flag) ||
+                !mbar_wait(&s.wfull[stage], phase, p.watchdog_ns, abort_flag)) {
                 raise_timeout(p, s);
                 ok = false;
                 break;
             }
+            // the activation tile was written through the generic proxy (cp.async or
+            // st.shared); order it before the tensor core's async-proxy reads
+            fence_proxy_async_smem();
             tc_fence_after();
             const uint32_t ws = smem_u32(s.w + stage * p.w_tile_bytes);
             const uint32_t xs = smem_u32(s.x + stage * p.x_tile_bytes);
@@ -320,13 +421,14 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
 // ------------------------------------------------------------------ epilogue
 template <bool WA, bool CONV>
 __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
+    const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int q = warp & 3;                  // tensor-memory lane quadrant of this warp
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int64_t it = blockIdx.x; it < p.num_items; it += gridDim.x) {
-        const Item t = decode(p, it, WA);
+        const Item t = decode(p, kcp, it, WA);
         const bool has = t.nkc > 0;
         if (has) {
             if (!mbar_wait(&s.tfull[acc], acc_phase, p.watchdog_ns, abort_flag)) {
@@ -429,6 +531,7 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     if (threadIdx.x == 0) {
         for (int i = 0; i < p.stages; ++i) {
             mbar_init(&s.full[i], kProducerThreads);
+            mbar_init(&s.wfull[i], 1);
             mbar_init(&s.empty[i], 1);
         }
         for (int i = 0; i < 2; ++i) {
@@ -439,6 +542,8 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
         *s.abort_flag = 0;
         fence_mbar_init();
     }
+    if (s.kc)
+        for (int64_t i = threadIdx.x; i < p.kc_cached; i += kThreads) s.kc[i] = p.kc_ptr[i];
     if (warp == kMmaWarp) {
         tmem_alloc(s.tmem_base, p.tmem_cols);
         tmem_relinquish();
@@ -448,8 +553,9 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     tc_fence_after();
     const uint32_t tmem = *s.tmem_base;
 
-    if (warp < 4) {
-        producer<WA, CONV>(p, s);
+    if (warp < kProducerWarps) {
+        if (CONV) producer_im2col(p, s);
+        else producer_gather<WA>(p, s);
     } else if (warp == kMmaWarp) {
         if ((threadIdx.x & 31) == 0) mma_issuer<WA>(p, s, tmem);
         __syncwarp();
@@ -479,7 +585,7 @@ cudaError_t launch_variant(Params &p, cudaStream_t st) {
     });
     if (attr_err != cudaSuccess) return attr_err;
     const size_t smem = 1024 + (size_t)p.stages * (p.w_tile_bytes + p.x_tile_bytes) +
-                        (2 * (size_t)p.stages + 5) * 8 + 16;
+                        (3 * (size_t)p.stages + 7) * 8 + 8 * (size_t)p.kc_cached;
     const int64_t grid = p.num_items < num_sms() ? p.num_items : num_sms();
     bp_mma_kernel<WA, CONV><<<(unsigned)grid, kThreads, smem, st>>>(p);
     return cudaGetLastError();
@@ -506,17 +612,16 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     p.nslab = wa ? dl.rows_pad / kSlab : 1;
     p.N = N;
     const int64_t nt = wa ? 256 : 128;
-    p.n_tiles = (N + nt - 1) / nt;
-    p.num_items = p.n_tiles * p.num_rb * p.nslab;
+    p.num_items = (N + nt - 1) / nt * p.num_rb * p.nslab;
     p.w_tile_bytes = (uint32_t)((wa ? kSlab : dl.rows_pad) * kBK * 2);
     p.x_tile_bytes = (uint32_t)(nt * kBK * 2);
-    const int64_t budget = 200 * 1024;
-    int64_t stages = budget / (p.w_tile_bytes + p.x_tile_bytes);
-    if (stages > 8) stages = 8;
+    int64_t stages = (200 * 1024) / (p.w_tile_bytes + p.x_tile_bytes);
+    if (stages > kMaxStages) stages = kMaxStages;
     p.stages = stages;
     p.acc_cols = pow2_at_least(wa ? 256u : (uint32_t)dl.rows_pad);
     p.tmem_cols = 2 * p.acc_cols;
     p.kc_ptr = reinterpret_cast<const int64_t *>(dev);
+    p.kc_cached = p.num_rb + 1 <= kMaxCachedRb + 1 ? p.num_rb + 1 : 0;
     p.chunks = dev + dl.off_chunks;
     p.tile_bytes = dl.tile_bytes;
     p.chunk_bytes = dl.chunk_bytes;
@@ -526,7 +631,9 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     p.ldy = ldy;
     p.bias = bias;
     p.watchdog_ns = watchdog_ns();
+    p.drop_stage = debug_drop_stage();
     p.status = device_status_ptr();
+    if (p.num_items == 0) return cudaSuccess;
     if (conv) {
         p.C = conv->C;
         p.H = conv->H;
@@ -540,9 +647,8 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
         p.pw = conv->pw;
         p.sh = conv->sh;
         p.sw = conv->sw;
+        return launch_variant<false, true>(p, st);
     }
-    if (p.num_items == 0) return cudaSuccess;
-    if (conv) return launch_variant<false, true>(p, st);
     return wa ? launch_variant<true, false>(p, st) : launch_variant<false, false>(p, st);
 }
 

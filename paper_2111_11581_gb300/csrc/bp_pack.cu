@@ -3,8 +3,7 @@
 // Sec. 4.3), then col_idx / values (the canonical compact arrays) and the
 // device image the tensor-core kernels stream: per row-block k-chunks of 64
 // kept columns, each a (rows_pad x 64) K-major tile already in the 128-byte
-// swizzled shared-memory order, plus the padded column list of every chunk
-// (-1 marks padding, which the kernels turn into zeros).
+// swizzled shared-memory order, plus the padded column list of every chunk.
 #include "bp_common.cuh"
 
 namespace bp {
@@ -101,7 +100,8 @@ __global__ void values_kernel(int64_t M, int64_t K, int64_t bm,
 }
 
 // Padded column list of every k-chunk: entry r of chunk kc of row-block rb is
-// its (kc*64 + r)-th kept column, or -1 past K'_rb.
+// its (kc*64 + r)-th kept column; past K'_rb it repeats the row-block's last
+// kept column (a valid row to load, multiplied by the zero-padded weights).
 __global__ void cidx_kernel(const int64_t *__restrict__ rb_ptr, const int64_t *__restrict__ kc_ptr,
                             const int32_t *__restrict__ col_idx, uint8_t *__restrict__ chunks,
                             int64_t tile_bytes, int64_t chunk_bytes) {
@@ -110,7 +110,7 @@ __global__ void cidx_kernel(const int64_t *__restrict__ rb_ptr, const int64_t *_
     const int64_t c0 = kc_ptr[rb], nkc = kc_ptr[rb + 1] - c0;
     for (int64_t t = threadIdx.x; t < nkc * kBK; t += blockDim.x) {
         int32_t *cl = reinterpret_cast<int32_t *>(chunks + (c0 + t / kBK) * chunk_bytes + tile_bytes);
-        cl[t % kBK] = t < kp ? col_idx[p0 + t] : -1;
+        cl[t % kBK] = col_idx[p0 + (t < kp ? t : kp - 1)];
     }
 }
 

@@ -92,8 +92,8 @@ def _check_device_image(pw, rb_ptr, col_idx, values, M, bm):
             want[:r_rb, :seg.shape[1]] = seg
             assert (dec == want).all(), (rb, kc)
             cl = img[base + tile_bytes: base + chunk].view(np.int32)
-            wl = np.full(64, -1, np.int32)
             s = col_idx[rb_ptr[rb] + kc * 64: min(rb_ptr[rb] + (kc + 1) * 64, rb_ptr[rb + 1])]
+            wl = np.full(64, col_idx[rb_ptr[rb + 1] - 1], np.int32)   # padding: last kept column
             wl[:s.size] = s
             assert (cl == wl).all(), (rb, kc)
 
