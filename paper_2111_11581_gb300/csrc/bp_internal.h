@@ -5,7 +5,7 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
-#include "../../include/bp.h"
+#include "bp.h"
 
 namespace bp {
 

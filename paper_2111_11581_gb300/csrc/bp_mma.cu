@@ -18,7 +18,10 @@
 //               measured about 6x slower per byte than this path.)
 //   warp 4      MMA issuer: tcgen05.mma (K = 16 per instruction) into an
 //               fp32 accumulator in tensor memory, double-buffered;
-//   warps 5-8   epilogue: tcgen05.ld, + bias, ReLU, round to fp16/bf16, store.
+//   warps 5-8   epilogue: tcgen05.ld, + bias, ReLU, round to fp16/bf16, store
+//               (weight-as-A tiles: through a swizzled shared-memory staging
+//               buffer and TMA tensor stores of 32 x 32 boxes, which keeps the
+//               output off the load/store unit the gather needs).
 //
 // Two operand orientations:
 //   kWeightA (bm a multiple of 128): D[128 weight rows x 256 tokens]
@@ -29,8 +32,10 @@
 // Every wait is bounded (see mbar_wait); on expiry the kernel records
 // kDevTimeout in the device status word, drains its own copies and tensor
 // core work, frees tensor memory and returns.
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
+#include <cudaTypedefs.h>
 
 #include <mutex>
 
@@ -43,15 +48,17 @@ constexpr uint64_t kDrainNs = 1000000000ull;
 constexpr int kMaxStages = 8;
 constexpr int kPrefetch = 6;           // index lists loaded this many stages ahead
 constexpr int kMaxCachedRb = 2047;     // kc_ptr kept in shared memory up to this many row-blocks
+constexpr int64_t kMaxSmem = 232448;   // dynamic shared memory per CTA (227 KB)
 
-struct Params {
+struct alignas(64) Params {
+    CUtensorMap ymap;       // weight-as-A GEMM: Y as a 2-D tensor, box 32 x 32, 64-byte swizzle
     int dtype;
     int relu;
     int64_t M, bm, rows_pad, num_rb, nslab;
     int64_t N;              // tokens (GEMM) or Nb*Ho*Wo pixels (conv)
     int64_t num_items;
     int64_t stages;
-    uint32_t w_tile_bytes, x_tile_bytes, tmem_cols, acc_cols;
+    uint32_t w_tile_bytes, x_tile_bytes, tmem_cols, acc_cols, ystage_bytes;
     const int64_t *kc_ptr;
     int64_t kc_cached;      // entries of kc_ptr copied to shared memory (0 = none)
     const uint8_t *chunks;  // k-chunks: weight tile, then 64 int32 column indices
@@ -91,6 +98,7 @@ __device__ __forceinline__ uint16_t cvt1(float a, int dtype) {
 struct Smem {
     uint8_t *w;          // stages x w_tile_bytes
     uint8_t *x;          // stages x x_tile_bytes
+    uint8_t *ystage;     // weight-as-A: 4 epilogue warps x 2 buffers x 2 KB
     uint64_t *full;      // [stages] activation tile landed (128 producer arrivals)
     uint64_t *wfull;     // [stages] weight tile landed (TMA byte count)
     uint64_t *empty;     // [stages] tensor cores done with the stage
@@ -108,7 +116,8 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
         (reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023));
     s.w = base;
     s.x = base + p.stages * p.w_tile_bytes;
-    uint8_t *b = s.x + p.stages * p.x_tile_bytes;
+    s.ystage = s.x + p.stages * p.x_tile_bytes;
+    uint8_t *b = s.ystage + p.ystage_bytes;
     s.full = reinterpret_cast<uint64_t *>(b);
     s.wfull = s.full + p.stages;
     s.empty = s.wfull + p.stages;
@@ -439,43 +448,43 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
         }
         const uint32_t tacc = tmem + ((uint32_t)(32 * q) << 16) + acc * p.acc_cols;
         if (WA) {
-            const int64_t row = t.slab * kSlab + 32 * q + lane;
-            const bool vrow = row < t.rows;
-            const int64_t m = t.rb * p.bm + row;
-            const float bv = (p.bias && vrow) ? p.bias[m] : 0.f;
-            uint16_t *yrow = p.Y + (vrow ? m : 0) * p.ldy;
-            for (int c0 = 0; c0 < 256; c0 += 16) {
-                uint32_t r[16];
+            // lane = output row; 32 x 32 boxes staged in shared memory (64-byte swizzle:
+            // 16-byte chunk c of row r sits at chunk c ^ ((r >> 1) & 3)), then TMA-stored
+            const int64_t row0 = t.slab * kSlab + 32 * q;
+            const bool vrow = row0 + lane < t.rows;
+            const float bv = (p.bias && vrow) ? p.bias[t.rb * p.bm + row0 + lane] : 0.f;
+            const uint32_t stg = smem_u32(s.ystage + (warp - kMmaWarp - 1) * 4096);
+            for (int c0 = 0; c0 < 256 && t.n0 + c0 < p.N; c0 += 32) {
+                uint32_t r[32];
                 if (has) {
-                    tmem_ld_32x32b_x16(tacc + c0, r);
+                    tmem_ld_32x32b_x32(tacc + c0, r);
                     tmem_ld_wait();
                 } else {
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) r[e] = 0u;
+                    for (int e = 0; e < 32; ++e) r[e] = 0u;
                 }
-                const int64_t n = t.n0 + c0;
-                if (!vrow || n >= p.N) continue;
-                float f[16];
+                uint32_t pk[16];
 #pragma unroll
                 for (int e = 0; e < 16; ++e) {
-                    float v = __uint_as_float(r[e]) + bv;
-                    f[e] = (p.relu && v < 0.f) ? 0.f : v;
+                    float a = __uint_as_float(r[2 * e]) + bv, b = __uint_as_float(r[2 * e + 1]) + bv;
+                    if (p.relu) {
+                        a = fmaxf(a, 0.f);
+                        b = fmaxf(b, 0.f);
+                    }
+                    pk[e] = pack2(a, b, p.dtype);
                 }
-                if (n + 16 <= p.N) {
-                    uint4 a, b;
-                    a.x = pack2(f[0], f[1], p.dtype);
-                    a.y = pack2(f[2], f[3], p.dtype);
-                    a.z = pack2(f[4], f[5], p.dtype);
-                    a.w = pack2(f[6], f[7], p.dtype);
-                    b.x = pack2(f[8], f[9], p.dtype);
-                    b.y = pack2(f[10], f[11], p.dtype);
-                    b.z = pack2(f[12], f[13], p.dtype);
-                    b.w = pack2(f[14], f[15], p.dtype);
-                    uint4 *dst = reinterpret_cast<uint4 *>(yrow + n);
-                    dst[0] = a;
-                    dst[1] = b;
-                } else {
-                    for (int e = 0; e < 16 && n + e < p.N; ++e) yrow[n + e] = cvt1(f[e], p.dtype);
+                const uint32_t sb = stg + ((c0 >> 5) & 1) * 2048;
+                if (lane == 0) bulk_wait_read<1>();     // the store that used this buffer is done
+                __syncwarp();
+#pragma unroll
+                for (int ch = 0; ch < 4; ++ch)
+                    st_shared_v4(sb + lane * 64 + ((ch ^ ((lane >> 1) & 3)) << 4),
+                                 make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]));
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_2d(&p.ymap, sb, (int32_t)(t.n0 + c0), (int32_t)(t.rb * p.bm + row0));
+                    bulk_commit();
                 }
             }
         } else {
@@ -521,6 +530,7 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             }
         }
     }
+    if (WA && lane == 0) bulk_wait_all();       // staged output fully written before exit
 }
 
 template <bool WA, bool CONV>
@@ -575,17 +585,31 @@ uint32_t pow2_at_least(uint32_t v) {
     return r;
 }
 
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    });
+    return fn;
+}
+
 template <bool WA, bool CONV>
 cudaError_t launch_variant(Params &p, cudaStream_t st) {
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [] {
         attr_err = cudaFuncSetAttribute(bp_mma_kernel<WA, CONV>,
-                                        cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxSmem);
     });
     if (attr_err != cudaSuccess) return attr_err;
     const size_t smem = 1024 + (size_t)p.stages * (p.w_tile_bytes + p.x_tile_bytes) +
-                        (3 * (size_t)p.stages + 7) * 8 + 8 * (size_t)p.kc_cached;
+                        p.ystage_bytes + (3 * (size_t)p.stages + 7) * 8 + 8 * (size_t)p.kc_cached;
     const int64_t grid = p.num_items < num_sms() ? p.num_items : num_sms();
     bp_mma_kernel<WA, CONV><<<(unsigned)grid, kThreads, smem, st>>>(p);
     return cudaGetLastError();
@@ -615,13 +639,20 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     p.num_items = (N + nt - 1) / nt * p.num_rb * p.nslab;
     p.w_tile_bytes = (uint32_t)((wa ? kSlab : dl.rows_pad) * kBK * 2);
     p.x_tile_bytes = (uint32_t)(nt * kBK * 2);
-    int64_t stages = (200 * 1024) / (p.w_tile_bytes + p.x_tile_bytes);
-    if (stages > kMaxStages) stages = kMaxStages;
-    p.stages = stages;
+    p.ystage_bytes = wa ? 4 * 2 * 2048 : 0;
+    p.kc_cached = p.num_rb + 1 <= kMaxCachedRb + 1 ? p.num_rb + 1 : 0;
+    // shared memory: stages + output staging + barriers + kc_ptr copy, within 227 KB
+    auto stages_for = [&](int64_t kc) {
+        const int64_t avail = kMaxSmem - 1024 - p.ystage_bytes - 8 * 32 - 8 * kc;
+        const int64_t st = avail / (p.w_tile_bytes + p.x_tile_bytes);
+        return st > kMaxStages ? (int64_t)kMaxStages : st;
+    };
+    if (stages_for(p.kc_cached) < 3) p.kc_cached = 0;
+    p.stages = stages_for(p.kc_cached);
+    if (p.stages < 2) return cudaErrorInvalidValue;
     p.acc_cols = pow2_at_least(wa ? 256u : (uint32_t)dl.rows_pad);
     p.tmem_cols = 2 * p.acc_cols;
     p.kc_ptr = reinterpret_cast<const int64_t *>(dev);
-    p.kc_cached = p.num_rb + 1 <= kMaxCachedRb + 1 ? p.num_rb + 1 : 0;
     p.chunks = dev + dl.off_chunks;
     p.tile_bytes = dl.tile_bytes;
     p.chunk_bytes = dl.chunk_bytes;
@@ -649,7 +680,21 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
         p.sw = conv->sw;
         return launch_variant<false, true>(p, st);
     }
-    return wa ? launch_variant<true, false>(p, st) : launch_variant<false, false>(p, st);
+    if (!wa) return launch_variant<false, false>(p, st);
+    // Y as a 2-D tensor (N inner, M rows) for the epilogue's 32 x 32 box stores
+    PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    const cuuint64_t gdim[2] = {(cuuint64_t)N, (cuuint64_t)P.lay.M};
+    const cuuint64_t gstride[1] = {(cuuint64_t)ldy * 2};
+    const cuuint32_t box[2] = {32, 32};
+    const cuuint32_t estride[2] = {1, 1};
+    if (enc(&p.ymap,
+            P.lay.dtype == BP_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16,
+            2, Y, gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return cudaErrorInvalidValue;
+    return launch_variant<true, false>(p, st);
 }
 
 }  // namespace bp
