@@ -76,10 +76,15 @@ struct alignas(64) Params {
     unsigned *status;
 };
 
-constexpr int kProducerWarps = 4;
-constexpr int kMmaWarp = 4;
-constexpr int kThreads = 288;
-constexpr uint32_t kProducerThreads = 128;
+// Warp roles: producers, then one MMA warp, then four epilogue warps.
+constexpr int kGemmProducerWarps = 4;
+template <bool CONV>
+struct Roles {
+    static constexpr int kProducerWarps = CONV ? 4 : kGemmProducerWarps;
+    static constexpr int kMmaWarp = kProducerWarps;
+    static constexpr int kThreads = (kProducerWarps + 5) * 32;
+    static constexpr uint32_t kProducerThreads = kProducerWarps * 32;
+};
 
 __device__ __forceinline__ uint32_t pack2(float a, float b, int dtype) {
     if (dtype == BP_BF16) {
@@ -200,7 +205,8 @@ struct WeightCopier {
 
 template <bool WA>
 __device__ void producer_gather(const Params &p, const Smem &s) {
-    const int tid = threadIdx.x;            // 0..127
+    constexpr int PW = kGemmProducerWarps;
+    const int tid = threadIdx.x;            // 0 .. 32*PW-1
     const int warp = tid >> 5, lane = tid & 31;
     const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
@@ -251,9 +257,9 @@ __device__ void producer_gather(const Params &p, const Smem &s) {
                 const uint32_t nb = n < p.N ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
                 const uint16_t *xcol = p.X + (nb ? n : 0);
 #pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const int r = warp + 4 * i;
-                    const int idx = __shfl_sync(0xffffffffu, i < 8 ? iv.x : iv.y, r & 31);
+                for (int i = 0; i < 64 / PW; ++i) {
+                    const int r = warp + PW * i;
+                    const int idx = __shfl_sync(0xffffffffu, r < 32 ? iv.x : iv.y, r & 31);
                     cp_async_16(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4),
                                 xcol + (int64_t)idx * p.ldx, nb);
                 }
@@ -264,9 +270,9 @@ __device__ void producer_gather(const Params &p, const Smem &s) {
                 const uint32_t nb = n < p.N ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
                 const uint16_t *xcol = p.X + (nb ? n : 0);
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int r = 2 * (warp + 4 * i) + (lane >> 4);
-                    const int idx = __shfl_sync(0xffffffffu, i < 4 ? iv.x : iv.y, r & 31);
+                for (int i = 0; i < 32 / PW; ++i) {
+                    const int r = 2 * (warp + PW * i) + (lane >> 4);
+                    const int idx = __shfl_sync(0xffffffffu, r < 32 ? iv.x : iv.y, r & 31);
                     cp_async_16(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4),
                                 xcol + (int64_t)idx * p.ldx, nb);
                 }
@@ -453,7 +459,7 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             const int64_t row0 = t.slab * kSlab + 32 * q;
             const bool vrow = row0 + lane < t.rows;
             const float bv = (p.bias && vrow) ? p.bias[t.rb * p.bm + row0 + lane] : 0.f;
-            const uint32_t stg = smem_u32(s.ystage + (warp - kMmaWarp - 1) * 4096);
+            const uint32_t stg = smem_u32(s.ystage + (warp - Roles<CONV>::kMmaWarp - 1) * 4096);
             for (int c0 = 0; c0 < 256 && t.n0 + c0 < p.N; c0 += 32) {
                 uint32_t r[32];
                 if (has) {
@@ -534,13 +540,15 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
 }
 
 template <bool WA, bool CONV>
-__global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_constant__ Params p) {
+__global__ void __launch_bounds__(Roles<CONV>::kThreads, 1)
+    bp_mma_kernel(const __grid_constant__ Params p) {
+    using R = Roles<CONV>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     const Smem s = carve(smem_raw, p);
     const int warp = threadIdx.x >> 5;
     if (threadIdx.x == 0) {
         for (int i = 0; i < p.stages; ++i) {
-            mbar_init(&s.full[i], kProducerThreads);
+            mbar_init(&s.full[i], R::kProducerThreads);
             mbar_init(&s.wfull[i], 1);
             mbar_init(&s.empty[i], 1);
         }
@@ -553,8 +561,8 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
         fence_mbar_init();
     }
     if (s.kc)
-        for (int64_t i = threadIdx.x; i < p.kc_cached; i += kThreads) s.kc[i] = p.kc_ptr[i];
-    if (warp == kMmaWarp) {
+        for (int64_t i = threadIdx.x; i < p.kc_cached; i += R::kThreads) s.kc[i] = p.kc_ptr[i];
+    if (warp == R::kMmaWarp) {
         tmem_alloc(s.tmem_base, p.tmem_cols);
         tmem_relinquish();
     }
@@ -563,10 +571,10 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     tc_fence_after();
     const uint32_t tmem = *s.tmem_base;
 
-    if (warp < kProducerWarps) {
+    if (warp < R::kProducerWarps) {
         if (CONV) producer_im2col(p, s);
         else producer_gather<WA>(p, s);
-    } else if (warp == kMmaWarp) {
+    } else if (warp == R::kMmaWarp) {
         if ((threadIdx.x & 31) == 0) mma_issuer<WA>(p, s, tmem);
         __syncwarp();
     } else {
@@ -576,7 +584,7 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == kMmaWarp) tmem_dealloc(tmem, p.tmem_cols);
+    if (warp == R::kMmaWarp) tmem_dealloc(tmem, p.tmem_cols);
 }
 
 uint32_t pow2_at_least(uint32_t v) {
@@ -611,7 +619,7 @@ cudaError_t launch_variant(Params &p, cudaStream_t st) {
     const size_t smem = 1024 + (size_t)p.stages * (p.w_tile_bytes + p.x_tile_bytes) +
                         p.ystage_bytes + (3 * (size_t)p.stages + 7) * 8 + 8 * (size_t)p.kc_cached;
     const int64_t grid = p.num_items < num_sms() ? p.num_items : num_sms();
-    bp_mma_kernel<WA, CONV><<<(unsigned)grid, kThreads, smem, st>>>(p);
+    bp_mma_kernel<WA, CONV><<<(unsigned)grid, Roles<CONV>::kThreads, smem, st>>>(p);
     return cudaGetLastError();
 }
 
