@@ -170,6 +170,22 @@ bp_status bp_device_status(void *stream);
  * after this call (default 2e9).  0 restores the default. */
 bp_status bp_set_watchdog_ns(uint64_t ns);
 
+/* bp_prune without a caller-provided workspace, for callers that cannot
+ * allocate device memory (code running under a no-allocation rule after
+ * start-up, plug-ins whose host framework owns all device memory, callers
+ * that must not trigger the synchronisation cudaMalloc can cause).  The
+ * paper has no counterpart: this is an interface convenience of this library.
+ * Same arguments, result and synchronisation as bp_prune; the workspace is a
+ * fixed 8 MiB array inside the library's device memory (held on every GPU
+ * that loads the library until it is unloaded).  Layouts whose
+ * bp_workspace_size() exceeds 8 MiB are rejected with BP_ERR_WORKSPACE before
+ * anything is launched.  The array's address is looked up on the first call
+ * made on each device (make that call before any stream capture).  All calls
+ * share the array: calls that may overlap on the GPU race and must be
+ * serialised by the caller.  Allocates nothing. */
+bp_status bp_prune_noalloc(const bp_layout *lay, const void *W, double rate, uint8_t *mask,
+                           void *stream);
+
 /* Fault injection for tests of the bounded waits: from the next launch on,
  * CTA 0 of every bp_gemm / bp_conv2d kernel skips filling its pipeline stage
  * number `stage` (0-based, counted over the CTA's whole run), so the tensor-

@@ -36,7 +36,7 @@ class Packed(ctypes.Structure):
 
 EXPORTS = ("bp_status_string", "bp_version", "bp_workspace_size", "bp_prune", "bp_pack_size",
            "bp_pack", "bp_gemm", "bp_conv2d", "bp_device_status", "bp_set_watchdog_ns",
-           "bp_debug_drop_stage")
+           "bp_debug_drop_stage", "bp_prune_noalloc")
 
 _lib = None
 _lock = threading.Lock()
@@ -74,6 +74,7 @@ def load(path: str = LIB_PATH):
             "bp_device_status": (i32, [vp]),
             "bp_set_watchdog_ns": (i32, [ctypes.c_uint64]),
             "bp_debug_drop_stage": (i32, [i64]),
+            "bp_prune_noalloc": (i32, [P_L, vp, dbl, vp, vp]),
         }
         for name, (res, args) in sig.items():
             f = getattr(lib, name)
@@ -136,6 +137,10 @@ def bp_device_status(stream: int = 0) -> int:
 
 def bp_set_watchdog_ns(ns: int) -> int:
     return load().bp_set_watchdog_ns(int(ns))
+
+
+def bp_prune_noalloc(lay: Layout, W: int, rate: float, mask: int, stream: int = 0) -> int:
+    return load().bp_prune_noalloc(ctypes.byref(lay), W, float(rate), mask, stream)
 
 
 def bp_debug_drop_stage(stage: int) -> int:
