@@ -46,7 +46,7 @@ namespace {
 
 constexpr uint64_t kDrainNs = 1000000000ull;
 constexpr int kMaxStages = 8;
-constexpr int kPrefetch = 6;           // index lists loaded this many stages ahead
+constexpr int kIdxSlots = 8;           // index lists copied to shared memory this many chunks ahead
 constexpr int kMaxCachedRb = 2047;     // kc_ptr kept in shared memory up to this many row-blocks
 constexpr int64_t kMaxSmem = 232448;   // dynamic shared memory per CTA (227 KB)
 
@@ -76,14 +76,17 @@ struct alignas(64) Params {
     unsigned *status;
 };
 
-// Warp roles: producers, then one MMA warp, then four epilogue warps.
-constexpr int kGemmProducerWarps = 4;
+// Warp roles.  GEMM: 8 gather warps, 1 control warp (index lists + weight
+// tiles through TMA), 1 MMA warp, 4 epilogue warps.  CONV: 4 im2col warps
+// (thread 0 also copies weight tiles), 1 MMA warp, 4 epilogue warps.
 template <bool CONV>
 struct Roles {
-    static constexpr int kProducerWarps = CONV ? 4 : kGemmProducerWarps;
-    static constexpr int kMmaWarp = kProducerWarps;
-    static constexpr int kThreads = (kProducerWarps + 5) * 32;
-    static constexpr uint32_t kProducerThreads = kProducerWarps * 32;
+    static constexpr int kGatherWarps = CONV ? 4 : 8;
+    static constexpr int kCtrlWarp = CONV ? -1 : 8;
+    static constexpr int kMmaWarp = CONV ? 4 : 9;
+    static constexpr int kEpiWarp0 = kMmaWarp + 1;
+    static constexpr int kThreads = (kEpiWarp0 + 4) * 32;
+    static constexpr uint32_t kGatherThreads = kGatherWarps * 32;
 };
 
 __device__ __forceinline__ uint32_t pack2(float a, float b, int dtype) {
@@ -110,6 +113,9 @@ struct Smem {
     uint64_t *tfull;     // [2]
     uint64_t *tempty;    // [2]
     uint64_t *drain;     // [1]
+    uint64_t *ifull;     // [kIdxSlots] index list of a chunk landed (TMA byte count)
+    uint64_t *iempty;    // [kIdxSlots] all producer threads have read the slot
+    int32_t *idx;        // [kIdxSlots][64] index lists of upcoming chunks
     uint32_t *tmem_base;
     int *abort_flag;
     int64_t *kc;         // [kc_cached] copy of kc_ptr, or nullptr
@@ -129,9 +135,14 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
     s.tfull = s.empty + p.stages;
     s.tempty = s.tfull + 2;
     s.drain = s.tempty + 2;
-    s.tmem_base = reinterpret_cast<uint32_t *>(s.drain + 1);
+    s.ifull = s.drain + 1;
+    s.iempty = s.ifull + kIdxSlots;
+    s.tmem_base = reinterpret_cast<uint32_t *>(s.iempty + kIdxSlots);
     s.abort_flag = reinterpret_cast<int *>(s.tmem_base + 1);
-    s.kc = p.kc_cached ? reinterpret_cast<int64_t *>(s.drain + 2) : nullptr;
+    // TMA bulk copies need a 16-byte-aligned destination: round up to 128 bytes
+    const uintptr_t after = reinterpret_cast<uintptr_t>(s.iempty + kIdxSlots + 2);
+    s.idx = reinterpret_cast<int32_t *>((after + 127) & ~static_cast<uintptr_t>(127));
+    s.kc = p.kc_cached ? reinterpret_cast<int64_t *>(s.idx + kIdxSlots * kBK) : nullptr;
     return s;
 }
 
@@ -203,62 +214,102 @@ struct WeightCopier {
     }
 };
 
+// Index lists of upcoming chunks, copied by TMA (256 B each) into a ring of
+// kIdxSlots shared-memory slots up to kIdxSlots chunks ahead of their use, so
+// the producers never wait on a global load for them.  Every producer thread
+// arrives on the slot's iempty barrier once it has read the list; thread 0
+// refills a slot only after that (bounded wait), one chunk later.
+struct IndexRing {
+    Cursor look;         // next chunk whose list is to be fetched (thread 0)
+    int64_t fetched;     // lists fetched so far
+    uint32_t last_phase[kIdxSlots];
+    bool pending[kIdxSlots];
+    __device__ __forceinline__ void fetch_one(const Params &p, const Smem &s, const int64_t *kcp,
+                                              bool wa) {
+        const int slot = (int)(fetched % kIdxSlots);
+        const uint32_t ph = (uint32_t)((fetched / kIdxSlots) & 1);
+        mbar_arrive_expect_tx(&s.ifull[slot], kBK * 4);
+        bulk_g2s(smem_u32(s.idx + slot * kBK),
+                 p.chunks + (look.t.kc0 + look.kc) * p.chunk_bytes + p.tile_bytes, kBK * 4,
+                 &s.ifull[slot]);
+        pending[slot] = true;
+        last_phase[slot] = ph;
+        ++fetched;
+        look.next(p, kcp, wa);
+    }
+    // thread 0: start the first kIdxSlots fetches
+    __device__ __forceinline__ void start(const Params &p, const Smem &s, const int64_t *kcp,
+                                          bool wa, const Cursor &first) {
+        look = first;
+        fetched = 0;
+        for (int i = 0; i < kIdxSlots; ++i) pending[i] = false;
+        for (int i = 0; i < kIdxSlots && look.valid(p); ++i) fetch_one(p, s, kcp, wa);
+    }
+    // thread 0, after the list of chunk `used` was read by everyone: refill its slot
+    __device__ __forceinline__ bool refill(const Params &p, const Smem &s, const int64_t *kcp,
+                                           bool wa, int64_t used, volatile int *abort_flag) {
+        const int slot = (int)(used % kIdxSlots);
+        pending[slot] = false;
+        if (!look.valid(p)) return true;
+        if (!mbar_wait(&s.iempty[slot], (uint32_t)((used / kIdxSlots) & 1), p.watchdog_ns,
+                       abort_flag))
+            return false;
+        fence_proxy_async_smem();   // the reads of the old list precede the TMA overwrite
+        fetch_one(p, s, kcp, wa);
+        return true;
+    }
+    // the CTA is unwinding: let every list copy in flight land first
+    __device__ __forceinline__ void drain(const Params &p, const Smem &s) {
+        for (int i = 0; i < kIdxSlots; ++i)
+            if (pending[i] && !mbar_wait(&s.ifull[i], last_phase[i], kDrainNs, nullptr))
+                atomicOr(p.status, kDevTimeout);
+    }
+};
+
+// Gather warps (GEMM): per chunk, read the chunk's index list from the shared
+// ring, then copy the 64 activation rows it names into the stage with 16-byte
+// cp.async straight into the swizzled layout; arrive on the stage's data
+// barrier when the copies land (no blocking).
 template <bool WA>
-__device__ void producer_gather(const Params &p, const Smem &s) {
-    constexpr int PW = kGemmProducerWarps;
-    const int tid = threadIdx.x;            // 0 .. 32*PW-1
-    const int warp = tid >> 5, lane = tid & 31;
+__device__ void gather_warps(const Params &p, const Smem &s) {
+    constexpr int GW = Roles<false>::kGatherWarps;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
-    WeightCopier wc;
-    wc.init();
-    auto load_idx = [&](const Cursor &c) {
-        const int32_t *cl = reinterpret_cast<const int32_t *>(
-            p.chunks + (c.t.kc0 + c.kc) * p.chunk_bytes + p.tile_bytes);
-        return make_int2(__ldg(cl + lane), __ldg(cl + lane + 32));
-    };
-    // ring[i]: this lane's two entries of the index list i chunks after the next one
-    Cursor cur, look;
+    Cursor cur;
     cur.first(p, kcp, WA);
-    look = cur;
-    int2 ring[kPrefetch];
-#pragma unroll
-    for (int i = 0; i < kPrefetch; ++i) {
-        ring[i] = look.valid(p) ? load_idx(look) : make_int2(0, 0);
-        if (look.valid(p)) look.next(p, kcp, WA);
-    }
     int stage = 0;
     uint32_t phase = 0;
-    bool ok = true;
     int64_t count = 0;
     while (cur.valid(p)) {
         const Item t = cur.t;
-        const int64_t kc = cur.kc;
-        const int2 iv = ring[0];
-#pragma unroll
-        for (int i = 0; i + 1 < kPrefetch; ++i) ring[i] = ring[i + 1];
-        ring[kPrefetch - 1] = look.valid(p) ? load_idx(look) : make_int2(0, 0);
-        if (look.valid(p)) look.next(p, kcp, WA);
         cur.next(p, kcp, WA);
-        const bool drop = blockIdx.x == 0 && count++ == p.drop_stage;
+        const int slot = (int)(count % kIdxSlots);
+        if (!mbar_wait(&s.ifull[slot], (uint32_t)((count / kIdxSlots) & 1), p.watchdog_ns,
+                       abort_flag)) {
+            raise_timeout(p, s);
+            break;
+        }
+        // two entries of the list per lane, broadcast below by shuffles
+        const int2 iv = make_int2(s.idx[slot * kBK + lane], s.idx[slot * kBK + 32 + lane]);
+        mbar_arrive(&s.iempty[slot]);
+        const int64_t seq = count++;
+        const bool drop = blockIdx.x == 0 && seq == p.drop_stage;
         if (!mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)) {
             raise_timeout(p, s);
-            ok = false;
             break;
         }
         if (!drop) {
-            const uint8_t *chunk = p.chunks + (t.kc0 + kc) * p.chunk_bytes;
-            if (tid == 0) wc.copy(p, s, stage, phase, chunk + t.slab * (kSlab * kBK * 2));
             const uint32_t xs = smem_u32(s.x + stage * p.x_tile_bytes);
             if (WA) {
-                // 64 rows x 256 tokens: one warp instruction per row segment of 512 B
+                // 64 rows x 256 tokens: one warp instruction per 512-byte row segment
                 const int cn = lane >> 3, j = lane & 7;
                 const int64_t n = t.n0 + lane * 8;
                 const uint32_t nb = n < p.N ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
                 const uint16_t *xcol = p.X + (nb ? n : 0);
 #pragma unroll
-                for (int i = 0; i < 64 / PW; ++i) {
-                    const int r = warp + PW * i;
+                for (int i = 0; i < 64 / GW; ++i) {
+                    const int r = warp + GW * i;
                     const int idx = __shfl_sync(0xffffffffu, r < 32 ? iv.x : iv.y, r & 31);
                     cp_async_16(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4),
                                 xcol + (int64_t)idx * p.ldx, nb);
@@ -270,13 +321,17 @@ __device__ void producer_gather(const Params &p, const Smem &s) {
                 const uint32_t nb = n < p.N ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
                 const uint16_t *xcol = p.X + (nb ? n : 0);
 #pragma unroll
-                for (int i = 0; i < 32 / PW; ++i) {
-                    const int r = 2 * (warp + PW * i) + (lane >> 4);
+                for (int i = 0; i < 32 / GW; ++i) {
+                    const int r = 2 * (warp + GW * i) + (lane >> 4);
                     const int idx = __shfl_sync(0xffffffffu, r < 32 ? iv.x : iv.y, r & 31);
                     cp_async_16(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4),
                                 xcol + (int64_t)idx * p.ldx, nb);
                 }
             }
+            // Signal the stage once this thread's copies have landed, without
+            // blocking.  The tile was written through the generic proxy; the
+            // tensor-core thread orders it before its async-proxy reads with a
+            // proxy fence after acquiring the barrier.
             cp_async_arrive_noinc(&s.full[stage]);
         }
         if (++stage == p.stages) {
@@ -285,7 +340,52 @@ __device__ void producer_gather(const Params &p, const Smem &s) {
         }
     }
     cp_async_wait_all();
-    if (!ok && tid == 0) wc.drain(p, s);
+}
+
+// Control thread (GEMM, lane 0 of the control warp): keeps the index-list ring
+// kIdxSlots chunks ahead and copies each stage's weight tile (TMA bulk) as
+// soon as the stage is free.
+template <bool WA>
+__device__ void control_thread(const Params &p, const Smem &s) {
+    const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
+    volatile int *abort_flag = s.abort_flag;
+    WeightCopier wc;
+    wc.init();
+    Cursor cur;
+    cur.first(p, kcp, WA);
+    IndexRing ring;
+    ring.start(p, s, kcp, WA, cur);
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    int64_t count = 0;
+    while (cur.valid(p)) {
+        const Item t = cur.t;
+        const int64_t kc = cur.kc;
+        cur.next(p, kcp, WA);
+        const int64_t seq = count++;
+        if (!mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)) {
+            raise_timeout(p, s);
+            ok = false;
+            break;
+        }
+        if (!(blockIdx.x == 0 && seq == p.drop_stage))
+            wc.copy(p, s, stage, phase,
+                    p.chunks + (t.kc0 + kc) * p.chunk_bytes + t.slab * (kSlab * kBK * 2));
+        if (seq > 0 && !ring.refill(p, s, kcp, WA, seq - 1, abort_flag)) {
+            raise_timeout(p, s);
+            ok = false;
+            break;
+        }
+        if (++stage == p.stages) {
+            stage = 0;
+            phase ^= 1u;
+        }
+    }
+    if (!ok) {
+        wc.drain(p, s);
+        ring.drain(p, s);
+    }
 }
 
 // ------------------------------------------------------------------ CONV producer (im2col)
@@ -330,7 +430,8 @@ __device__ void producer_im2col(const Params &p, const Smem &s) {
                 ok = false;
                 break;
             }
-            if (blockIdx.x == 0 && count++ == p.drop_stage) {   // injected lost stage
+            const int64_t seq = count++;
+            if (blockIdx.x == 0 && seq == p.drop_stage) {       // injected lost stage
                 if (++stage == p.stages) {
                     stage = 0;
                     phase ^= 1u;
@@ -401,8 +502,9 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
                 ok = false;
                 break;
             }
-            // the activation tile was written through the generic proxy (cp.async or
-            // st.shared); order it before the tensor core's async-proxy reads
+            // the activation tile was written through the generic proxy (cp.async /
+            // st.shared): order those writes, acquired through the barrier, before
+            // the tensor core's async-proxy reads
             fence_proxy_async_smem();
             tc_fence_after();
             const uint32_t ws = smem_u32(s.w + stage * p.w_tile_bytes);
@@ -459,7 +561,7 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             const int64_t row0 = t.slab * kSlab + 32 * q;
             const bool vrow = row0 + lane < t.rows;
             const float bv = (p.bias && vrow) ? p.bias[t.rb * p.bm + row0 + lane] : 0.f;
-            const uint32_t stg = smem_u32(s.ystage + (warp - Roles<CONV>::kMmaWarp - 1) * 4096);
+            const uint32_t stg = smem_u32(s.ystage + (warp - Roles<CONV>::kEpiWarp0) * 4096);
             for (int c0 = 0; c0 < 256 && t.n0 + c0 < p.N; c0 += 32) {
                 uint32_t r[32];
                 if (has) {
@@ -548,7 +650,7 @@ __global__ void __launch_bounds__(Roles<CONV>::kThreads, 1)
     const int warp = threadIdx.x >> 5;
     if (threadIdx.x == 0) {
         for (int i = 0; i < p.stages; ++i) {
-            mbar_init(&s.full[i], R::kProducerThreads);
+            mbar_init(&s.full[i], R::kGatherThreads);
             mbar_init(&s.wfull[i], 1);
             mbar_init(&s.empty[i], 1);
         }
@@ -557,6 +659,10 @@ __global__ void __launch_bounds__(Roles<CONV>::kThreads, 1)
             mbar_init(&s.tempty[i], 128);
         }
         mbar_init(s.drain, 1);
+        for (int i = 0; i < kIdxSlots; ++i) {
+            mbar_init(&s.ifull[i], 1);
+            mbar_init(&s.iempty[i], R::kGatherThreads);
+        }
         *s.abort_flag = 0;
         fence_mbar_init();
     }
@@ -571,9 +677,12 @@ __global__ void __launch_bounds__(Roles<CONV>::kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *s.tmem_base;
 
-    if (warp < R::kProducerWarps) {
+    if (warp < R::kGatherWarps) {
         if (CONV) producer_im2col(p, s);
-        else producer_gather<WA>(p, s);
+        else gather_warps<WA>(p, s);
+    } else if (warp == R::kCtrlWarp) {
+        if ((threadIdx.x & 31) == 0) control_thread<WA>(p, s);
+        __syncwarp();
     } else if (warp == R::kMmaWarp) {
         if ((threadIdx.x & 31) == 0) mma_issuer<WA>(p, s, tmem);
         __syncwarp();
@@ -617,7 +726,8 @@ cudaError_t launch_variant(Params &p, cudaStream_t st) {
     });
     if (attr_err != cudaSuccess) return attr_err;
     const size_t smem = 1024 + (size_t)p.stages * (p.w_tile_bytes + p.x_tile_bytes) +
-                        p.ystage_bytes + (3 * (size_t)p.stages + 7) * 8 + 8 * (size_t)p.kc_cached;
+                        p.ystage_bytes + (3 * (size_t)p.stages + 7 + 2 * kIdxSlots) * 8 +
+                        128 + (size_t)kIdxSlots * kBK * 4 + 8 * (size_t)p.kc_cached;
     const int64_t grid = p.num_items < num_sms() ? p.num_items : num_sms();
     bp_mma_kernel<WA, CONV><<<(unsigned)grid, Roles<CONV>::kThreads, smem, st>>>(p);
     return cudaGetLastError();
@@ -651,7 +761,8 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     p.kc_cached = p.num_rb + 1 <= kMaxCachedRb + 1 ? p.num_rb + 1 : 0;
     // shared memory: stages + output staging + barriers + kc_ptr copy, within 227 KB
     auto stages_for = [&](int64_t kc) {
-        const int64_t avail = kMaxSmem - 1024 - p.ystage_bytes - 8 * 32 - 8 * kc;
+        const int64_t avail =
+            kMaxSmem - 1024 - p.ystage_bytes - 8 * 48 - 128 - kIdxSlots * kBK * 4 - 8 * kc;
         const int64_t st = avail / (p.w_tile_bytes + p.x_tile_bytes);
         return st > kMaxStages ? (int64_t)kMaxStages : st;
     };
