@@ -254,7 +254,8 @@ struct IndexRing {
         if (!mbar_wait(&s.iempty[slot], (uint32_t)((used / kIdxSlots) & 1), p.watchdog_ns,
                        abort_flag))
             return false;
-        fence_proxy_async_smem();   // the reads of the old list precede the TMA overwrite
+        // the readers' loads completed before their (release) arrivals, which the
+        // wait above acquired, so the TMA overwrite cannot overtake them
         fetch_one(p, s, kcp, wa);
         return true;
     }

@@ -39,6 +39,9 @@ CASES = [
     (33, 70, 7, 1, 1, 4.0, bp.F16, False, False),               # unstructured, N < 8
     (48, 512, 256, 48, 8, 8.0, bp.BF16, False, False),          # structured (bm = M)
     (128, 64, 1, 16, 16, 1.0, bp.F16, True, False),             # N = 1, nothing pruned
+    # 16 row-blocks x 11 column tiles = 176 tiles: more than one wave of CTAs,
+    # and the last column tile is ragged (100 of 256 tokens)
+    (2048, 512, 2660, 128, 32, 4.0, bp.BF16, True, True),
 ]
 
 
