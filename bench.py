@@ -407,6 +407,117 @@ def run_reference(args):
     print(json.dumps(out), flush=True)
 
 
+# ----------------------------------------------------------------------- other workloads
+def _layer_step(layer, dtype, flush, reps=5):
+    """Prune + pack one layer, then time its bp_conv2d / bp_gemm launch (device
+    time, median of `reps`, L2 flushed before each launch) and the dense cuDNN /
+    cuBLAS call on the unpruned weight the same way.  Returns a dict."""
+    import torch
+    from paper_2111_11581_gb300 import bp, inputs
+
+    W = inputs.layer_weight(layer, dtype)
+    x = inputs.layer_input(layer, dtype)
+    b = inputs.layer_bias(layer)
+    Wd = inputs.as_torch(W.reshape(layer.M, -1), dtype).cuda()
+    xd = inputs.as_torch(x, dtype).cuda()
+    bd = torch.from_numpy(b).cuda() if b is not None else None
+    dense = layer.scheme < 0
+    if not dense:
+        lay = bp.layout(layer.scheme, dtype, layer.M, layer.K, layer.bm, layer.bk, layer.kh,
+                        layer.kw)
+        mask = bp.prune(lay, Wd, layer.rate)
+        pw = bp.pack(lay, Wd, mask)
+        kept = int(pw.c.nnz_vals)
+    else:
+        kept = layer.M * layer.K
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+
+    def timed(fn):
+        ts = []
+        for _ in range(reps + 1):
+            flush.zero_()
+            ev[0].record()
+            fn()
+            ev[1].record()
+            torch.cuda.synchronize()
+            ts.append(ev[0].elapsed_time(ev[1]) * 1e3)
+        return statistics.median(ts[1:])
+
+    if layer.kind == "conv":
+        wc = Wd.reshape(layer.M, layer.C, layer.kh, layer.kw)
+        bdd = bd.to(xd.dtype) if bd is not None else None
+        dense_fn = lambda: torch.nn.functional.conv2d(xd, wc, bdd, stride=layer.stride,  # noqa
+                                                      padding=layer.pad)
+        if not dense:
+            pad, stride = (layer.pad, layer.pad), (layer.stride, layer.stride)
+            ws = bp.conv2d_workspace(pw, tuple(xd.shape), pad, stride)
+            yo = bp.conv2d(pw, xd, pad=pad, stride=stride, bias=bd, relu=layer.relu, ws=ws)
+            ours_fn = lambda: bp.conv2d(pw, xd, pad=pad, stride=stride, bias=bd,  # noqa
+                                        relu=layer.relu, out=yo, ws=ws)
+        else:
+            ours_fn = dense_fn
+    else:
+        dense_fn = lambda: torch.matmul(Wd, xd)  # noqa
+        ours_fn = (lambda: bp.gemm(pw, xd, bias=bd, relu=layer.relu)) if not dense else dense_fn
+    t_ours = timed(ours_fn)
+    t_dense = timed(dense_fn)
+    if bp.device_status() != bp.OK:
+        raise RuntimeError("kernel watchdog fired")
+    n = layer.gemm_n
+    return {"layer": layer.name, "kind": layer.kind, "M": layer.M, "K": layer.K, "N": n,
+            "bm": layer.bm, "bk": layer.bk, "rate": layer.rate, "pruned": not dense,
+            "kept_flop": 2.0 * kept * n, "us": round(t_ours, 2), "dense_us": round(t_dense, 2)}
+
+
+def run_workload(args):
+    import torch
+    from paper_2111_11581_gb300 import bp, build, inputs
+
+    torch.cuda.set_device(0)
+    build.build()
+    bp.load()
+    flush = torch.empty(256 * 2 ** 20 // 4, dtype=torch.float32, device="cuda")
+    name = args.workload
+    if name == "fc512":
+        layers, dtype = [inputs.fc512()], inputs.F16
+    elif name == "conv3x3":
+        layers, dtype = [inputs.conv3x3_128()], inputs.F16
+    elif name == "vgg16":
+        layers, dtype = inputs.vgg16_cifar(), inputs.F16
+    elif name == "resnet50":
+        layers, dtype = inputs.resnet50_imagenet(), inputs.BF16
+    elif name == "sweep":
+        layers, dtype = [], None
+        for dt in (inputs.BF16, inputs.F16):
+            for (M, K, N) in inputs.GEMM_SHAPES:
+                for bm in inputs.SWEEP_BM:
+                    for bk in inputs.SWEEP_BK:
+                        for r in inputs.SWEEP_KEEP:
+                            layers.append((inputs.gemm_point(M, K, N, bm, bk, r, dt), dt))
+        if args.sweep_subset:
+            layers = [l for l in layers if l[0].bk == 32 and l[0].M == 4096] + \
+                     [l for l in layers if l[0].bk == 32 and l[0].M != 4096 and l[1] == inputs.BF16]
+    else:
+        raise SystemExit(f"unknown workload {name}")
+    rows = []
+    for item in layers:
+        layer, dt = item if isinstance(item, tuple) else (item, dtype)
+        rows.append(_layer_step(layer, dt, flush))
+        r = rows[-1]
+        print(f"# {r['layer']:40s} {r['us']:9.2f} us (dense {r['dense_us']:9.2f})"
+              f"  {r['kept_flop'] / r['us'] / 1e6:8.1f} TFLOP/s", file=sys.stderr, flush=True)
+    pr = [r for r in rows if r["pruned"]]
+    t = sum(r["us"] for r in pr)
+    fl = sum(r["kept_flop"] for r in pr)
+    td = sum(r["dense_us"] for r in pr)
+    out = {"metric": METRIC, "value": round(fl / t / 1e6, 2), "unit": UNIT, "n_gpus": 1,
+           "workload": name, "pruned_layers": len(pr), "sum_us": round(t, 2),
+           "dense_sum_us": round(td, 2), "speedup_vs_dense": round(td / t, 3),
+           "timing": "per-layer device time, median of 5, L2 flushed (256 MiB write) before each launch",
+           "layers": rows}
+    print(json.dumps(out), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -415,10 +526,16 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default=None,
+                    help="fc512 | conv3x3 | vgg16 | resnet50 | sweep: per-layer timings "
+                         "of another workload (one JSON line), instead of the default step")
+    ap.add_argument("--sweep-subset", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.impl == "reference":
+    if args.workload:
+        run_workload(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)

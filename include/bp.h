@@ -8,7 +8,7 @@
  *                                                       Eq. punched, Sec. 5.1)
  *   bp_pack      dense weight + mask -> compact per-row-block storage (Sec. 4.3)
  *   bp_gemm      block-sparse GEMM  Y = (W o mask) X, fused bias/ReLU/cast
- *   bp_conv2d    block-sparse implicit-GEMM convolution, same epilogue
+ *   bp_conv2d    block-sparse convolution (im2col + the same product), same epilogue
  *
  * Conventions shared by every call:
  *   - All tensor pointers are DEVICE pointers allocated by the caller; the
@@ -39,7 +39,7 @@ extern "C" {
 typedef enum {
     BP_OK = 0,
     BP_ERR_INVALID_ARG = 1,   /* bad pointer, size, rate, alignment or mask */
-    BP_ERR_UNSUPPORTED = 2,   /* valid but not implemented (e.g. bm > 256 not a multiple of 128) */
+    BP_ERR_UNSUPPORTED = 2,   /* valid but beyond the implemented limits (e.g. M > 1,048,576) */
     BP_ERR_NONFINITE = 3,     /* bp_prune: a weight is Inf or NaN */
     BP_ERR_WORKSPACE = 4,     /* workspace missing or smaller than bp_workspace_size() */
     BP_ERR_CUDA = 5,          /* a CUDA runtime call or launch failed */
@@ -80,9 +80,12 @@ typedef struct {
  *   col_idx[nnz_cols]  int32: kept GEMM-view columns, ascending within a row-block
  *   values [nnz_vals]  16-bit: row-block rb is a bm_rb x K'_rb row-major block
  *                      starting at element bm*rb_ptr[rb] (bm_rb = rows of rb)
- *   dev    [dev_bytes] the same weights re-tiled for the tensor-core kernels
- *                      (k-chunks of 64 columns, zero padded, pre-swizzled) plus
- *                      their padded index lists; opaque to callers. */
+ *   dev    [dev_bytes] the same weights re-tiled for the tensor-core kernel:
+ *                      slabs of 128 rows, each with the union of its rows'
+ *                      kept columns in chunks of 64 (pre-swizzled tiles, zero
+ *                      weights where a row prunes a column), their index lists
+ *                      and load plans; opaque to callers, its size fixed by
+ *                      the layout and the mask (bp_pack_size). */
 typedef struct {
     bp_layout lay;
     int64_t num_rb;
@@ -145,21 +148,36 @@ bp_status bp_pack(const bp_layout *lay, const void *W, const uint8_t *mask, bp_p
  *   bias  device fp32 [M] or NULL
  *   relu  0 / 1
  *   Y     device, M x N row-major (ldy >= N, multiple of 8)
- * Supported bm: 1..256, or any multiple of 128. */
+ * Any bm: weights are processed in slabs of 128 rows (see bp_packed::dev).
+ * X must be finite: rows of X that a slab lists may meet zero weights of rows
+ * that prune them (0 * Inf is NaN).  The launch is a programmatic dependent
+ * of the previous kernel in `stream` (its set-up overlaps that kernel's end;
+ * it reads and writes nothing before that kernel has completed). */
 bp_status bp_gemm(const bp_packed *P, const void *X, int64_t N, int64_t ldx, const float *bias,
                   int relu, void *Y, int64_t ldy, void *stream);
 
-/* Block-sparse convolution as an implicit GEMM over the GEMM view of
- * bp_layout (kept column k = c*kh*kw + i*kw + j), NCHW input and output:
+/* Block-sparse convolution over the GEMM view of bp_layout (kept column
+ * k = c*kh*kw + i*kw + j), NCHW input and output:
  *   out[b,f,oh,ow] = act( sum over kept (c,i,j) of W[f,c,i,j] *
  *                         in[b, c, oh*stride_h + i - pad_h, ow*stride_w + j - pad_w]
  *                         + bias[f] ),  zero outside the input.
  *   in    device, Nb x C x H x W;   out  device, Nb x M x Ho x Wo with
  *   Ho = (H + 2 pad_h - kh) / stride_h + 1, Wo likewise.
- * Requires C*kh*kw == lay.K; dilation and groups are not supported. */
+ *   ws    device workspace of at least bp_conv2d_workspace_size() bytes
+ *         (16-B aligned): the input expanded to the K x (Nb*Ho*Wo) matrix
+ *         (im2col), which the block-sparse product then reads.
+ * Requires C*kh*kw == lay.K; dilation and groups are not supported.  The
+ * input must be finite (see bp_gemm). */
 bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, int64_t H,
                     int64_t W, int pad_h, int pad_w, int stride_h, int stride_w,
-                    const float *bias, int relu, void *out, void *stream);
+                    const float *bias, int relu, void *out, void *ws, size_t ws_bytes,
+                    void *stream);
+
+/* Device workspace bytes bp_conv2d needs for this packed weight and input
+ * shape (host output): 2 * K * (Nb*Ho*Wo rounded up to 8). */
+bp_status bp_conv2d_workspace_size(const bp_packed *P, int64_t Nb, int64_t C, int64_t H,
+                                   int64_t W, int pad_h, int pad_w, int stride_h, int stride_w,
+                                   size_t *bytes);
 
 /* Synchronizes `stream`, then returns BP_ERR_TIMEOUT if any kernel of this
  * library recorded an expired wait since the previous call (and clears the

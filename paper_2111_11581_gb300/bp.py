@@ -35,7 +35,7 @@ class Packed(ctypes.Structure):
 
 
 EXPORTS = ("bp_status_string", "bp_version", "bp_workspace_size", "bp_prune", "bp_pack_size",
-           "bp_pack", "bp_gemm", "bp_conv2d", "bp_device_status", "bp_set_watchdog_ns",
+           "bp_pack", "bp_gemm", "bp_conv2d", "bp_conv2d_workspace_size", "bp_device_status", "bp_set_watchdog_ns",
            "bp_debug_drop_stage", "bp_prune_noalloc")
 
 _lib = None
@@ -70,7 +70,9 @@ def load(path: str = LIB_PATH):
             "bp_pack": (i32, [P_L, vp, vp, P_P, vp]),
             "bp_gemm": (i32, [P_P, vp, i64, i64, vp, i32, vp, i64, vp]),
             "bp_conv2d": (i32, [P_P, vp, i64, i64, i64, i64, i32, i32, i32, i32, vp, i32, vp,
-                                vp]),
+                                vp, sz, vp]),
+            "bp_conv2d_workspace_size": (i32, [P_P, i64, i64, i64, i64, i32, i32, i32, i32,
+                                               ctypes.POINTER(sz)]),
             "bp_device_status": (i32, [vp]),
             "bp_set_watchdog_ns": (i32, [ctypes.c_uint64]),
             "bp_debug_drop_stage": (i32, [i64]),
@@ -126,9 +128,17 @@ def bp_gemm(packed: Packed, X: int, N: int, ldx: int, bias: int | None, relu: in
 
 def bp_conv2d(packed: Packed, x: int, Nb: int, C: int, H: int, W: int, pad_h: int, pad_w: int,
               stride_h: int, stride_w: int, bias: int | None, relu: int, out: int,
-              stream: int = 0) -> int:
+              ws: int | None, ws_bytes: int, stream: int = 0) -> int:
     return load().bp_conv2d(ctypes.byref(packed), x, Nb, C, H, W, pad_h, pad_w, stride_h,
-                            stride_w, bias, int(relu), out, stream)
+                            stride_w, bias, int(relu), out, ws, ws_bytes, stream)
+
+
+def bp_conv2d_workspace_size(packed: Packed, Nb: int, C: int, H: int, W: int, pad_h: int,
+                             pad_w: int, stride_h: int, stride_w: int):
+    n = ctypes.c_size_t()
+    st = load().bp_conv2d_workspace_size(ctypes.byref(packed), Nb, C, H, W, pad_h, pad_w,
+                                         stride_h, stride_w, ctypes.byref(n))
+    return st, n.value
 
 
 def bp_device_status(stream: int = 0) -> int:
@@ -223,9 +233,19 @@ def gemm(pw: PackedWeight, X, bias=None, relu: bool = False, out=None, stream=No
     return out
 
 
+def conv2d_workspace(pw: PackedWeight, shape, pad=(0, 0), stride=(1, 1), device="cuda"):
+    """Device workspace bp_conv2d needs for an NCHW input of `shape` (its im2col matrix)."""
+    torch = _torch()
+    Nb, C, H, W = shape
+    st, n = bp_conv2d_workspace_size(pw.c, Nb, C, H, W, pad[0], pad[1], stride[0], stride[1])
+    _chk(st, "bp_conv2d_workspace_size")
+    return torch.empty(max(n, 16), dtype=torch.uint8, device=device)
+
+
 def conv2d(pw: PackedWeight, x, pad=(0, 0), stride=(1, 1), bias=None, relu: bool = False,
-           out=None, stream=None):
-    """NCHW block-sparse convolution through bp_conv2d."""
+           out=None, ws=None, stream=None):
+    """NCHW block-sparse convolution through bp_conv2d (`ws` from conv2d_workspace,
+    allocated here when not given)."""
     torch = _torch()
     Nb, C, H, W = x.shape
     lay = pw.lay
@@ -233,9 +253,11 @@ def conv2d(pw: PackedWeight, x, pad=(0, 0), stride=(1, 1), bias=None, relu: bool
     Wo = (W + 2 * pad[1] - lay.kw) // stride[1] + 1
     if out is None:
         out = torch.empty((Nb, lay.M, Ho, Wo), dtype=x.dtype, device=x.device)
+    if ws is None:
+        ws = conv2d_workspace(pw, x.shape, pad, stride, x.device)
     st = bp_conv2d(pw.c, x.data_ptr(), Nb, C, H, W, pad[0], pad[1], stride[0], stride[1],
                    None if bias is None else bias.data_ptr(), int(relu), out.data_ptr(),
-                   _stream(stream))
+                   ws.data_ptr(), ws.numel() * ws.element_size(), _stream(stream))
     _chk(st, "bp_conv2d")
     return out
 

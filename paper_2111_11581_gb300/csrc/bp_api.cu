@@ -14,8 +14,10 @@ namespace bp {
 // Device status word: kernels OR kDevTimeout into it when a bounded wait ran
 // out; bp_device_status() reads and clears it.
 __device__ unsigned g_dev_status;
-// Flag word of bp_pack_size's row-block consistency check (calls serialised).
+// Flag word of bp_pack_size's row-block consistency check and per-slab block
+// counts of the device image (pack calls are serialised by g_mu).
 __device__ int g_pack_bad;
+__device__ int64_t g_slab_info[2 * kMaxSlabs];
 
 namespace {
 constexpr uint64_t kDefaultWatchdogNs = 2000000000ull;
@@ -125,37 +127,39 @@ bool checked_mode() {
     return e && e[0] == '1';
 }
 
-Orientation orientation_for(int64_t bm) {
-    if (bm % kSlab == 0) return kWeightA;
-    if (bm <= 256) return kWeightB;
-    return kNoTensorCore;
-}
-
-int64_t rows_pad_for(int64_t bm) {
-    switch (orientation_for(bm)) {
-    case kWeightA: return bm;
-    case kWeightB: return align_up(bm, 16);
-    default: return 0;
-    }
-}
-
-DevLayout dev_layout(const bp_layout &lay, const int64_t *rb_ptr_host) {
+DevLayout dev_layout(const bp_layout &lay, const int64_t *slab_chunks_host) {
     DevLayout d{};
-    d.orient = orientation_for(lay.bm);
-    d.rows_pad = rows_pad_for(lay.bm);
-    d.num_rb = cdiv(lay.M, lay.bm);
-    d.off_chunks = align_up(8 * (d.num_rb + 1), 256);
-    d.tile_bytes = d.rows_pad * kBK * 2;
-    d.chunk_bytes = d.tile_bytes + kBK * 4;
+    d.num_slabs = cdiv(lay.M, kSlab);
+    d.off_tiles = align_up(8 * (d.num_slabs + 1), 256);
+    d.tile_bytes = (int64_t)kSlab * kBK * 2;
     d.kc_total = -1;
+    d.off_meta = -1;
     d.bytes = -1;
-    if (rb_ptr_host) {
+    if (slab_chunks_host) {
         int64_t kc = 0;
-        for (int64_t rb = 0; rb < d.num_rb; ++rb) kc += cdiv(rb_ptr_host[rb + 1] - rb_ptr_host[rb], kBK);
+        for (int64_t s = 0; s < d.num_slabs; ++s) kc += slab_chunks_host[s];
         d.kc_total = kc;
-        d.bytes = d.orient == kNoTensorCore ? 0 : d.off_chunks + kc * d.chunk_bytes;
+        d.off_meta = d.off_tiles + kc * d.tile_bytes;
+        d.bytes = d.off_meta + kc * kMetaBytes;
     }
     return d;
+}
+
+// Per-slab chunk counts of the device image (device pass + read-back; syncs).
+static bp_status slab_chunk_counts(const bp_layout &lay, const uint8_t *mask, cudaStream_t s,
+                                   std::vector<int64_t> &chunks) {
+    const int64_t S = cdiv(lay.M, kSlab);
+    int64_t *info = nullptr;
+    if (cudaGetSymbolAddress(reinterpret_cast<void **>(&info), g_slab_info) != cudaSuccess)
+        return BP_ERR_CUDA;
+    std::vector<int64_t> h(2 * S);
+    cudaError_t e = launch_slab_counts(lay, mask, info, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(h.data(), info, 16 * S, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return BP_ERR_CUDA;
+    chunks.resize(S);
+    for (int64_t i = 0; i < S; ++i) chunks[i] = h[2 * i] + cdiv(h[2 * i + 1], kBK);
+    return BP_OK;
 }
 
 }  // namespace bp
@@ -262,9 +266,13 @@ bp_status bp_pack_size(const bp_layout *lay, const uint8_t *mask, int64_t *rb_pt
         const int64_t rows = std::min<int64_t>(lay->bm, lay->M - rb * lay->bm);
         nv += rows * (h[rb + 1] - h[rb]);
     }
+    if (cdiv(lay->M, kSlab) > kMaxSlabs) return BP_ERR_UNSUPPORTED;
+    std::vector<int64_t> sc;
+    const bp_status st = slab_chunk_counts(*lay, mask, s, sc);
+    if (st != BP_OK) return st;
     *nnz_cols = h[RB];
     *nnz_vals = nv;
-    *dev_bytes = dev_layout(*lay, h.data()).bytes;
+    *dev_bytes = dev_layout(*lay, sc.data()).bytes;
     return BP_OK;
 }
 
@@ -288,14 +296,18 @@ bp_status bp_pack(const bp_layout *lay, const void *W, const uint8_t *mask, bp_p
     }
     if (out->nnz_cols != h[RB] || out->nnz_vals != nv) return BP_ERR_INVALID_ARG;
     if ((h[RB] > 0 && !out->col_idx) || (nv > 0 && !out->values)) return BP_ERR_INVALID_ARG;
-    const DevLayout dl = dev_layout(*lay, h.data());
+    if (cdiv(lay->M, kSlab) > kMaxSlabs) return BP_ERR_UNSUPPORTED;
+    std::lock_guard<std::mutex> lk(g_mu);
+    std::vector<int64_t> sc;
+    const bp_status st = slab_chunk_counts(*lay, mask, s, sc);
+    if (st != BP_OK) return st;
+    const DevLayout dl = dev_layout(*lay, sc.data());
     if (out->dev_bytes != dl.bytes) return BP_ERR_INVALID_ARG;
-    if (dl.bytes > 0 && (!out->dev || !aligned16(out->dev))) return BP_ERR_INVALID_ARG;
+    if (!out->dev || !aligned16(out->dev)) return BP_ERR_INVALID_ARG;
     out->lay = *lay;
-    std::vector<int64_t> kc(RB + 1, 0);
-    for (int64_t rb = 0; rb < RB; ++rb) kc[rb + 1] = kc[rb] + cdiv(h[rb + 1] - h[rb], kBK);
-    if (dl.bytes > 0)
-        e = cudaMemcpyAsync(out->dev, kc.data(), 8 * (RB + 1), cudaMemcpyHostToDevice, s);
+    std::vector<int64_t> kc(dl.num_slabs + 1, 0);
+    for (int64_t i = 0; i < dl.num_slabs; ++i) kc[i + 1] = kc[i] + sc[i];
+    e = cudaMemcpyAsync(out->dev, kc.data(), 8 * (dl.num_slabs + 1), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = launch_pack(*lay, W, mask, *out, dl, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     return cuda_status(e);
@@ -304,9 +316,14 @@ bp_status bp_pack(const bp_layout *lay, const void *W, const uint8_t *mask, bp_p
 static bp_status check_packed(const bp_packed *P, DevLayout *dl) {
     if (!P || !layout_ok(&P->lay) || !P->dev || !aligned16(P->dev)) return BP_ERR_INVALID_ARG;
     if (P->num_rb != cdiv(P->lay.M, P->lay.bm)) return BP_ERR_INVALID_ARG;
+    if (cdiv(P->lay.M, kSlab) > kMaxSlabs) return BP_ERR_UNSUPPORTED;
     *dl = dev_layout(P->lay, nullptr);
-    if (dl->orient == kNoTensorCore) return BP_ERR_UNSUPPORTED;
-    if (P->dev_bytes < dl->off_chunks) return BP_ERR_INVALID_ARG;
+    // the chunk count follows from the image size: tiles + list/plan records
+    const int64_t rest = P->dev_bytes - dl->off_tiles, per = dl->tile_bytes + kMetaBytes;
+    if (rest < 0 || rest % per) return BP_ERR_INVALID_ARG;
+    dl->kc_total = rest / per;
+    dl->off_meta = dl->off_tiles + dl->kc_total * dl->tile_bytes;
+    dl->bytes = P->dev_bytes;
     return BP_OK;
 }
 
@@ -329,38 +346,64 @@ bp_status bp_gemm(const bp_packed *P, const void *X, int64_t N, int64_t ldx, con
     return finish_launch(launch_mma(*P, dl, X, N, ldx, bias, relu, Y, ldy, nullptr, s), s);
 }
 
-bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, int64_t H,
-                    int64_t W, int pad_h, int pad_w, int stride_h, int stride_w,
-                    const float *bias, int relu, void *out, void *stream) {
-    DevLayout dl;
-    bp_status st = check_packed(P, &dl);
+static bp_status conv_shape(const bp_packed *P, int64_t Nb, int64_t C, int64_t H, int64_t W,
+                            int pad_h, int pad_w, int stride_h, int stride_w, ConvShape *cs,
+                            DevLayout *dl) {
+    bp_status st = check_packed(P, dl);
     if (st != BP_OK) return st;
     const bp_layout &l = P->lay;
-    if (!in || !out || Nb < 0 || C < 1 || H < 1 || W < 1) return BP_ERR_INVALID_ARG;
+    if (Nb < 0 || C < 1 || H < 1 || W < 1) return BP_ERR_INVALID_ARG;
     if (pad_h < 0 || pad_w < 0 || stride_h < 1 || stride_w < 1) return BP_ERR_INVALID_ARG;
     if (C * l.kh * l.kw != l.K) return BP_ERR_INVALID_ARG;
     if (H + 2 * pad_h < l.kh || W + 2 * pad_w < l.kw) return BP_ERR_INVALID_ARG;
-    if (!aligned16(in) || !aligned16(out)) return BP_ERR_INVALID_ARG;
-    if (bias && (reinterpret_cast<uintptr_t>(bias) & 3u)) return BP_ERR_INVALID_ARG;
-    if (dl.rows_pad > 256) return BP_ERR_UNSUPPORTED;
     if (H > (1 << 28) || W > (1 << 28)) return BP_ERR_UNSUPPORTED;
+    cs->Nb = Nb;
+    cs->C = C;
+    cs->H = H;
+    cs->W = W;
+    cs->Ho = (H + 2 * pad_h - l.kh) / stride_h + 1;
+    cs->Wo = (W + 2 * pad_w - l.kw) / stride_w + 1;
+    cs->kh = l.kh;
+    cs->kw = l.kw;
+    cs->ph = pad_h;
+    cs->pw = pad_w;
+    cs->sh = stride_h;
+    cs->sw = stride_w;
+    return BP_OK;
+}
+
+bp_status bp_conv2d_workspace_size(const bp_packed *P, int64_t Nb, int64_t C, int64_t H,
+                                   int64_t W, int pad_h, int pad_w, int stride_h, int stride_w,
+                                   size_t *bytes) {
     ConvShape cs;
-    cs.Nb = Nb;
-    cs.C = C;
-    cs.H = H;
-    cs.W = W;
-    cs.Ho = (H + 2 * pad_h - l.kh) / stride_h + 1;
-    cs.Wo = (W + 2 * pad_w - l.kw) / stride_w + 1;
-    cs.kh = l.kh;
-    cs.kw = l.kw;
-    cs.ph = pad_h;
-    cs.pw = pad_w;
-    cs.sh = stride_h;
-    cs.sw = stride_w;
+    DevLayout dl;
+    if (!bytes) return BP_ERR_INVALID_ARG;
+    const bp_status st = conv_shape(P, Nb, C, H, W, pad_h, pad_w, stride_h, stride_w, &cs, &dl);
+    if (st != BP_OK) return st;
+    const int64_t N = Nb * cs.Ho * cs.Wo;
+    *bytes = (size_t)(P->lay.K * align_up(N, 8) * 2);
+    return BP_OK;
+}
+
+bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, int64_t H,
+                    int64_t W, int pad_h, int pad_w, int stride_h, int stride_w,
+                    const float *bias, int relu, void *out, void *ws, size_t ws_bytes,
+                    void *stream) {
+    ConvShape cs;
+    DevLayout dl;
+    const bp_status st =
+        conv_shape(P, Nb, C, H, W, pad_h, pad_w, stride_h, stride_w, &cs, &dl);
+    if (st != BP_OK) return st;
+    if (!in || !out || !aligned16(in) || !aligned16(out)) return BP_ERR_INVALID_ARG;
+    if (bias && (reinterpret_cast<uintptr_t>(bias) & 3u)) return BP_ERR_INVALID_ARG;
     const int64_t N = Nb * cs.Ho * cs.Wo;
     if (N == 0) return BP_OK;
+    const int64_t ldx = align_up(N, 8);
+    if (!ws || !aligned16(ws) || ws_bytes < (size_t)(P->lay.K * ldx * 2)) return BP_ERR_WORKSPACE;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    return finish_launch(launch_mma(*P, dl, in, N, 0, bias, relu, out, 0, &cs, s), s);
+    cudaError_t e = launch_im2col(cs, ldx, in, ws, s);
+    if (e != cudaSuccess) return BP_ERR_CUDA;
+    return finish_launch(launch_mma(*P, dl, ws, N, ldx, bias, relu, out, 0, &cs, s), s);
 }
 
 bp_status bp_device_status(void *stream) {

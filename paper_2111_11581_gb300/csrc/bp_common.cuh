@@ -21,6 +21,18 @@ __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// ---------------------------------------------------------------- programmatic dependent launch
+// Block until the grids this one depends on have completed and their memory
+// operations are visible (a no-op when launched without the attribute).
+__device__ __forceinline__ void grid_dependency_wait() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+// Allow the next grid in the stream to be scheduled (it still waits for this
+// one's completion before touching memory).
+__device__ __forceinline__ void grid_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
@@ -32,6 +44,13 @@ __device__ __forceinline__ void fence_mbar_init() {
 
 __device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
     asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
+
+// `count` arrivals at once.
+__device__ __forceinline__ void mbar_arrive_cnt(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+                 "r"(count)
                  : "memory");
 }
 
@@ -68,20 +87,24 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t *bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Bounded wait on phase `parity` of an mbarrier.  Gives up after `limit_ns`
-// of global-timer time, or early when another role of the CTA raised
-// `*abort` (pass nullptr to ignore it); returns false then and the caller
-// records the timeout and unwinds.
+// Bounded wait on phase `parity` of an mbarrier.  Gives up once `limit_ns`
+// of global-timer time have passed since its 64th unsuccessful probe, or early
+// when another role of the CTA raised `*abort` (pass nullptr to ignore it);
+// returns false then and the caller records the timeout and unwinds.  Each
+// probe (try_wait) suspends the thread for a bounded time at most.  The timer
+// is read only every 64 probes: it is slow to read, and a read on every wait
+// would sit on the pipeline's critical path.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint64_t limit_ns,
                                           volatile int *abort) {
     const uint32_t a = smem_u32(bar);
-    if (mbar_try_wait(a, parity)) return true;
-    const uint64_t deadline = globaltimer_ns() + limit_ns;
+    uint64_t deadline = 0;
     for (uint32_t it = 1;; ++it) {
         if (mbar_try_wait(a, parity)) return true;
         if ((it & 63u) == 0u) {
             if (abort != nullptr && *abort) return false;
-            if (globaltimer_ns() > deadline) return false;
+            const uint64_t now = globaltimer_ns();
+            if (deadline == 0) deadline = now + limit_ns;
+            else if (now > deadline) return false;
         }
     }
 }
@@ -105,6 +128,20 @@ __device__ __forceinline__ void tma_store_2d(const void *tmap, uint32_t src, int
                      tmap),
                  "r"(src), "r"(x), "r"(y)
                  : "memory");
+}
+// 2-D tile load global -> shared through a tensor map; completion counted in
+// bytes on `bar`, out-of-range elements of the box read as zero.  x (the
+// innermost coordinate) times the element size must be a multiple of 16.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const void *tmap, int32_t x, int32_t y,
+                                            uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"(tmap), "r"(x), "r"(y), "r"(smem_u32(bar))
+        : "memory");
+}
+__device__ __forceinline__ void prefetch_tmap(const void *tmap) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(tmap) : "memory");
 }
 __device__ __forceinline__ void bulk_commit() {
     asm volatile("cp.async.bulk.commit_group;" ::: "memory");

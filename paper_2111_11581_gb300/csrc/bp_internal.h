@@ -12,40 +12,52 @@ namespace bp {
 // Device status bits recorded by kernels (read by bp_device_status).
 constexpr unsigned kDevTimeout = 1u;
 
-// Tile geometry of the tensor-core kernels.
+// Tile geometry of the tensor-core kernel.
 constexpr int kBK = 64;            // GEMM-view columns per k-chunk (one 128-B swizzle row)
-constexpr int kSlab = 128;         // weight rows per MMA when W is the A operand
+constexpr int kSlab = 128;         // weight rows per slab (the MMA's M)
 
-// Which operand the compact weights are in the tensor-core product.
-//   kWeightA: W rows are the MMA M dimension (bm a multiple of 128), the
-//             gathered activations are the N = 256 operand.
-//   kWeightB: 128 gathered activation columns (tokens / pixels) are the MMA M
-//             dimension, W rows are N (bm <= 256, padded to a multiple of 16).
-enum Orientation { kWeightA = 0, kWeightB = 1, kNoTensorCore = 2 };
+constexpr int kDenseMin = 48;      // a 64-column block whose union keeps >= this many columns is stored whole
+constexpr int64_t kMaxSlabs = 8192;  // 128-row slabs per layer (M <= 1,048,576)
+constexpr int kListBytes = kBK * 4;  // a chunk's 64 int32 column indices
+constexpr int kPlanBytes = 64;       // a chunk's load plan
+constexpr int kMetaBytes = kListBytes + kPlanBytes;   // list + plan record of a chunk
+constexpr int kMaxBoxes = 8;         // tile loads in a chunk's plan at most
 
-// Device image inside bp_packed::dev (all offsets in bytes):
-//   [0, 8*(num_rb+1))         int64 kc_ptr: first k-chunk of each row-block
-//   off_chunks + c*chunk_bytes  k-chunk c: its (rows_pad x 64) 16-bit weight
-//                               tile in K-major 128-byte-swizzled order,
-//                               followed by its 64 int32 column indices
-//                               (padding repeats the last kept column; its
-//                               weights are zero).
+// Device image inside bp_packed::dev, the form the tensor-core kernel streams.
+// Rows are grouped in slabs of 128 (slab s = rows 128s .. 128s+127); a slab's
+// column list is the union of the kept columns of its rows (all rows of a
+// row-block keep the same columns, so for bm a multiple of 128 it is exactly
+// the row-block's list).  Aligned 64-column blocks whose union holds at least
+// kDenseMin columns are listed whole (64 consecutive columns, weights zero
+// where a row prunes them); the other union columns follow in ascending
+// order, 64 per k-chunk.  All offsets in bytes, C = total k-chunks:
+//   [0, 8*(S+1))                 int64 kc_ptr: first k-chunk of each slab
+//   off_tiles + c*16384          k-chunk c's 128 x 64 16-bit weight tile in
+//                                K-major 128-byte-swizzled order
+//   off_meta + c*kMetaBytes      k-chunk c's record:
+//     [0, 256)                   its 64 int32 column indices (a partial last
+//                                chunk repeats its last index; the weights of
+//                                such repeats are zero);
+//     [256, 320)                 its load plan, int32 words: [0] = number of
+//                                tile loads B (0: gather the rows one by one),
+//                                [1 + b] = first column of load b, [9], [10] =
+//                                one byte per load: bits 0-2 = first list
+//                                position / 8, bits 4-5 = log2(rows / 8); the
+//                                loads cover the 64 list positions in order,
+//                                and each live entry of a load's range is its
+//                                first column plus its offset (repeats read
+//                                other rows, against zero weights).
 struct DevLayout {
-    Orientation orient;
-    int64_t rows_pad;     // rows per k-chunk tile
-    int64_t num_rb;
-    int64_t kc_total;     // total k-chunks over all row-blocks (-1 if unknown)
-    int64_t off_chunks;
-    int64_t tile_bytes;   // rows_pad * 64 * 2
-    int64_t chunk_bytes;  // tile_bytes + 64 * 4
+    int64_t num_slabs;
+    int64_t kc_total;     // total k-chunks (-1 if unknown)
+    int64_t off_tiles;
+    int64_t off_meta;     // (when kc_total is known)
+    int64_t tile_bytes;   // 128 * 64 * 2
     int64_t bytes;        // total image size (when kc_total is known)
 };
 
-Orientation orientation_for(int64_t bm);
-int64_t rows_pad_for(int64_t bm);
-// Image layout for a layout and its per-row-block kept-column counts
-// (rb_ptr_host = host copy of rb_ptr, or nullptr to leave kc_total unknown).
-DevLayout dev_layout(const bp_layout &lay, const int64_t *rb_ptr_host);
+// Image layout; slab_chunks_host = per-slab chunk counts (host) or nullptr.
+DevLayout dev_layout(const bp_layout &lay, const int64_t *slab_chunks_host);
 
 // Library-wide settings.
 uint64_t watchdog_ns();
@@ -70,6 +82,10 @@ int64_t threshold_chunks(int64_t U);
 
 cudaError_t launch_rb_counts(const bp_layout &lay, const uint8_t *mask, int64_t *rb_ptr,
                              int *bad, cudaStream_t s);
+// Per slab: number of whole (dense) 64-column blocks and of remaining union
+// columns, written to info[2*s], info[2*s+1] (device).
+cudaError_t launch_slab_counts(const bp_layout &lay, const uint8_t *mask, int64_t *info,
+                               cudaStream_t s);
 cudaError_t launch_pack(const bp_layout &lay, const void *W, const uint8_t *mask,
                         const bp_packed &P, const DevLayout &dl, cudaStream_t s);
 
@@ -77,6 +93,13 @@ struct ConvShape {
     int64_t Nb, C, H, W, Ho, Wo;
     int kh, kw, ph, pw, sh, sw;
 };
+// im2col of an NCHW input: Xcol[k][n] (K x N row-major, leading dimension ldx),
+// k = c*kh*kw + i*kw + j, n = b*Ho*Wo + oh*Wo + ow, zero outside the image.
+cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void *xcol,
+                          cudaStream_t s);
+// The block-sparse product on the tensor cores: Y = act(W_packed X + bias).
+// conv == nullptr: Y is M x N row-major (ldy).  Otherwise Y is the NCHW output
+// of the convolution and X its im2col matrix.
 cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, int64_t N,
                        int64_t ldx, const float *bias, int relu, void *Y, int64_t ldy,
                        const ConvShape *conv, cudaStream_t s);

@@ -1,33 +1,31 @@
-// Block-sparse GEMM / implicit-GEMM convolution on the sm_103a tensor cores.
+// Block-sparse product on the sm_103a tensor cores (bp_gemm, and bp_conv2d on
+// its im2col matrix).
 //
-// Each work item is one row-block (or one 128-row slab of it) times one tile
-// of activation columns.  The row-block's compact weights Wc (bm x K'_rb,
-// Sec. 4.3) multiply the activation rows selected by its kept-column list, so
-// pruned weights never enter the product.  Per k-chunk of 64 kept columns a
-// pipeline stage holds the chunk's pre-swizzled weight tile and the 64
-// activation rows it names, laid out as a 128-byte-swizzled MN-major tile:
+// The packed weight is a sequence of 128-row slabs; a slab's column list is
+// the union of its rows' kept columns (Sec. 4.3: the rows of a row-block keep
+// the same columns, so for bm a multiple of 128 the list is the row-block's
+// own).  A work unit is one slab times one tile of 256 activation columns
+// (tokens / pixels).  Per k-chunk of 64 listed columns a pipeline stage holds
+// the chunk's pre-swizzled weight tile (the MMA's A operand, K-major) and the
+// 64 activation rows the chunk names (the B operand, MN-major, 128-byte
+// swizzle), so columns no row of the slab keeps never enter the product:
 //
-//   warps 0-3   producers.  Thread 0 copies the weight tile with one TMA
-//               bulk copy (completion counted in bytes on the stage's
-//               weight barrier).  GEMM: the 128 threads gather the rows of X
-//               with 16-byte cp.async (one 512- or 256-byte row segment per
-//               warp instruction) and arrive on the stage's data barrier
-//               when their copies land, without blocking.  CONV: im2col rows
-//               are built in registers (zero outside the image) and stored.
-//               (TMA tile::gather4 moves 4 x 128 B per instruction and
-//               measured about 6x slower per byte than this path.)
-//   warp 4      MMA issuer: tcgen05.mma (K = 16 per instruction) into an
-//               fp32 accumulator in tensor memory, double-buffered;
-//   warps 5-8   epilogue: tcgen05.ld, + bias, ReLU, round to fp16/bf16, store
-//               (weight-as-A tiles: through a swizzled shared-memory staging
-//               buffer and TMA tensor stores of 32 x 32 boxes, which keeps the
-//               output off the load/store unit the gather needs).
-//
-// Two operand orientations:
-//   kWeightA (bm a multiple of 128): D[128 weight rows x 256 tokens]
-//            = Wc tile (A, K-major) * gathered X (B, MN-major);
-//   kWeightB (bm <= 256): D[128 tokens x rows_pad] = gathered X^T (A,
-//            MN-major) * Wc^T (B, K-major), rows_pad = bm rounded up to 16.
+//   warps 0-7   gather: for chunks without a load plan, the activation rows,
+//               16-byte cp.async straight into the swizzled layout (one
+//               512-byte row segment per warp instruction), signalled with
+//               cp.async.mbarrier.arrive.noinc so no thread blocks on them;
+//   warp 8      control (one thread): copies the chunks' records (index list
+//               + load plan) into shared memory a window of kWin chunks at a
+//               time, one window ahead (TMA bulk copies), copies each stage's
+//               weight tile (TMA bulk), and when a chunk's list is made of runs
+//               of consecutive columns (its plan, built at pack time) loads the
+//               activation rows of each run with TMA tile loads;
+//   warp 9      MMA issuer: tcgen05.mma 128 x 256 x 16 into one of two fp32
+//               accumulators in tensor memory (the epilogue of a tile
+//               overlaps the MMAs of the next);
+//   warps 10-13 epilogue: tcgen05.ld, + bias, ReLU, round to fp16/bf16, then
+//               TMA tensor stores of 32 x 32 boxes staged in shared memory
+//               (GEMM), or direct stores into the NCHW output (convolution).
 //
 // Every wait is bounded (see mbar_wait); on expiry the kernel records
 // kDevTimeout in the device status word, drains its own copies and tensor
@@ -37,6 +35,8 @@
 #include <cuda_fp16.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
+#include <cstdint>
 #include <mutex>
 
 #include "bp_common.cuh"
@@ -46,47 +46,49 @@ namespace {
 
 constexpr uint64_t kDrainNs = 1000000000ull;
 constexpr int kMaxStages = 8;
-constexpr int kIdxSlots = 8;           // index lists copied to shared memory this many chunks ahead
-constexpr int kMaxCachedRb = 2047;     // kc_ptr kept in shared memory up to this many row-blocks
+constexpr int kWin = 16;               // chunk records per shared-memory window
+constexpr int kWinBufs = 3;            // windows in shared memory (one being filled ahead)
+constexpr uint32_t kWinBytes = kWin * kMetaBytes;
+constexpr int64_t kMaxCachedKc = 2048; // kc_ptr entries kept in shared memory at most
 constexpr int64_t kMaxSmem = 232448;   // dynamic shared memory per CTA (227 KB)
+constexpr int kNT = 256;               // activation columns per tile at most (the MMA's N)
+constexpr uint32_t kWTileBytes = kSlab * kBK * 2;   // 16 KB
+constexpr uint32_t kXTileBytes = kNT * kBK * 2;     // 32 KB
 
-struct alignas(64) Params {
-    CUtensorMap ymap;       // weight-as-A GEMM: Y as a 2-D tensor, box 32 x 32, 64-byte swizzle
+// Warp roles.
+constexpr int kGatherWarps = 8;
+constexpr int kCtrlWarp = 8;
+constexpr int kMmaWarp = 9;
+constexpr int kEpiWarp0 = 10;
+constexpr int kThreads = (kEpiWarp0 + 4) * 32;
+constexpr uint32_t kGatherThreads = kGatherWarps * 32;
+
+struct Params {
+    CUtensorMap ymap;       // GEMM output Y as a 2-D tensor, box 32 x 32, 64-byte swizzle
+    CUtensorMap xmap[4];    // activations X (N inner, K rows), boxes 64 x (8 << i), 128-byte swizzle
     int dtype;
     int relu;
-    int64_t M, bm, rows_pad, num_rb, nslab;
+    int conv;               // 1: Y is the NCHW output of a convolution
+    int64_t M, num_slabs;
     int64_t N;              // tokens (GEMM) or Nb*Ho*Wo pixels (conv)
+    int nt;                 // activation columns per tile: a multiple of 32, 64 .. 256
+    int xboxes;             // 64-column TMA boxes per activation row: ceil(nt / 64)
     int64_t num_items;
     int64_t stages;
-    uint32_t w_tile_bytes, x_tile_bytes, tmem_cols, acc_cols, ystage_bytes;
+    uint32_t tmem_cols, acc_cols, ystage_bytes;
     const int64_t *kc_ptr;
     int64_t kc_cached;      // entries of kc_ptr copied to shared memory (0 = none)
-    const uint8_t *chunks;  // k-chunks: weight tile, then 64 int32 column indices
-    int64_t tile_bytes, chunk_bytes;
+    const uint8_t *tiles;   // k-chunk weight tiles (16 KB each)
+    const uint8_t *meta;    // k-chunk records: index list + load plan (kMetaBytes each)
     const uint16_t *X;
     int64_t ldx;
     uint16_t *Y;
     int64_t ldy;
+    int64_t HoWo;           // conv: output pixels per image
     const float *bias;
-    // convolution
-    int64_t C, H, W, Ho, Wo, HoWo, KK;
-    int kw, ph, pw, sh, sw;
     uint64_t watchdog_ns;
     int64_t drop_stage;     // fault injection: CTA 0 never fills this stage (-1 = off)
     unsigned *status;
-};
-
-// Warp roles.  GEMM: 8 gather warps, 1 control warp (index lists + weight
-// tiles through TMA), 1 MMA warp, 4 epilogue warps.  CONV: 4 im2col warps
-// (thread 0 also copies weight tiles), 1 MMA warp, 4 epilogue warps.
-template <bool CONV>
-struct Roles {
-    static constexpr int kGatherWarps = CONV ? 4 : 8;
-    static constexpr int kCtrlWarp = CONV ? -1 : 8;
-    static constexpr int kMmaWarp = CONV ? 4 : 9;
-    static constexpr int kEpiWarp0 = kMmaWarp + 1;
-    static constexpr int kThreads = (kEpiWarp0 + 4) * 32;
-    static constexpr uint32_t kGatherThreads = kGatherWarps * 32;
 };
 
 __device__ __forceinline__ uint32_t pack2(float a, float b, int dtype) {
@@ -98,26 +100,23 @@ __device__ __forceinline__ uint32_t pack2(float a, float b, int dtype) {
     return *reinterpret_cast<const uint32_t *>(&h);
 }
 
-__device__ __forceinline__ uint16_t cvt1(float a, int dtype) {
-    if (dtype == BP_BF16) return __bfloat16_as_ushort(__float2bfloat16_rn(a));
-    return __half_as_ushort(__float2half_rn(a));
-}
-
 struct Smem {
-    uint8_t *w;          // stages x w_tile_bytes
-    uint8_t *x;          // stages x x_tile_bytes
-    uint8_t *ystage;     // weight-as-A: 4 epilogue warps x 2 buffers x 2 KB
-    uint64_t *full;      // [stages] activation tile landed (128 producer arrivals)
-    uint64_t *wfull;     // [stages] weight tile landed (TMA byte count)
+    uint8_t *w;          // stages x kWTileBytes
+    uint8_t *x;          // stages x kXTileBytes
+    uint8_t *ystage;     // GEMM: 4 epilogue warps x 2 buffers x 2 KB
+    uint64_t *full;      // [stages] gathered activation rows landed (256 arrivals; used by
+                         // chunks without a load plan only)
+    uint64_t *wfull;     // [stages] weight tile (+ TMA-loaded activations) landed
     uint64_t *empty;     // [stages] tensor cores done with the stage
-    uint64_t *tfull;     // [2]
-    uint64_t *tempty;    // [2]
+    uint64_t *tfull;     // [2] accumulator ready for the epilogue
+    uint64_t *tempty;    // [2] accumulator drained
     uint64_t *drain;     // [1]
-    uint64_t *ifull;     // [kIdxSlots] index list of a chunk landed (TMA byte count)
-    uint64_t *iempty;    // [kIdxSlots] all producer threads have read the slot
-    int32_t *idx;        // [kIdxSlots][64] index lists of upcoming chunks
+    uint64_t *pfull;     // [kWinBufs] a window of chunk records landed (TMA byte count)
+    uint64_t *pempty;    // [kWinBufs] the gather warps and the control thread are done with it
+    uint32_t *skind;     // [stages] 1: the stage's activations come from TMA tile loads
     uint32_t *tmem_base;
     int *abort_flag;
+    uint8_t *win;        // [kWinBufs][kWinBytes] chunk records of the current windows
     int64_t *kc;         // [kc_cached] copy of kc_ptr, or nullptr
 };
 
@@ -126,8 +125,8 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
     uint8_t *base = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023));
     s.w = base;
-    s.x = base + p.stages * p.w_tile_bytes;
-    s.ystage = s.x + p.stages * p.x_tile_bytes;
+    s.x = base + p.stages * kWTileBytes;
+    s.ystage = s.x + p.stages * kXTileBytes;
     uint8_t *b = s.ystage + p.ystage_bytes;
     s.full = reinterpret_cast<uint64_t *>(b);
     s.wfull = s.full + p.stages;
@@ -135,15 +134,22 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
     s.tfull = s.empty + p.stages;
     s.tempty = s.tfull + 2;
     s.drain = s.tempty + 2;
-    s.ifull = s.drain + 1;
-    s.iempty = s.ifull + kIdxSlots;
-    s.tmem_base = reinterpret_cast<uint32_t *>(s.iempty + kIdxSlots);
+    s.pfull = s.drain + 1;
+    s.pempty = s.pfull + kWinBufs;
+    s.skind = reinterpret_cast<uint32_t *>(s.pempty + kWinBufs);
+    s.tmem_base = s.skind + p.stages;
     s.abort_flag = reinterpret_cast<int *>(s.tmem_base + 1);
     // TMA bulk copies need a 16-byte-aligned destination: round up to 128 bytes
-    const uintptr_t after = reinterpret_cast<uintptr_t>(s.iempty + kIdxSlots + 2);
-    s.idx = reinterpret_cast<int32_t *>((after + 127) & ~static_cast<uintptr_t>(127));
-    s.kc = p.kc_cached ? reinterpret_cast<int64_t *>(s.idx + kIdxSlots * kBK) : nullptr;
+    const uintptr_t after = reinterpret_cast<uintptr_t>(s.abort_flag + 1);
+    s.win = reinterpret_cast<uint8_t *>((after + 127) & ~static_cast<uintptr_t>(127));
+    s.kc = p.kc_cached ? reinterpret_cast<int64_t *>(s.win + kWinBufs * kWinBytes) : nullptr;
     return s;
+}
+
+size_t smem_bytes(int64_t stages, uint32_t ystage_bytes, int64_t kc_cached) {
+    return 1024 + (size_t)stages * (kWTileBytes + kXTileBytes) + ystage_bytes +
+           (3 * (size_t)stages + 5 + 2 * kWinBufs) * 8 + 4 * (size_t)stages + 8 + 128 +
+           (size_t)kWinBufs * kWinBytes + 8 * (size_t)kc_cached;
 }
 
 __device__ __forceinline__ void raise_timeout(const Params &p, const Smem &s) {
@@ -152,377 +158,308 @@ __device__ __forceinline__ void raise_timeout(const Params &p, const Smem &s) {
 }
 
 struct Item {
-    int64_t rb, slab, n0, kc0, nkc, rows;   // rows = real rows of the row-block
+    int64_t slab, n0, kc0, nkc, rows;   // rows = real rows of the slab
 };
 
-__device__ __forceinline__ Item decode(const Params &p, const int64_t *kc, int64_t it, bool wa) {
+// Work unit u -> (slab, 256-column tile), slab fastest.
+__device__ __forceinline__ Item decode(const Params &p, const int64_t *kc, int64_t u) {
     Item t;
-    const int64_t R = p.num_rb * p.nslab;
-    const int64_t rs = it % R;
-    t.n0 = (it / R) * (wa ? 256 : 128);
-    t.rb = rs / p.nslab;
-    t.slab = rs % p.nslab;
-    t.kc0 = kc[t.rb];
-    t.nkc = kc[t.rb + 1] - t.kc0;
-    t.rows = min(p.bm, p.M - t.rb * p.bm);
+    t.slab = u % p.num_slabs;
+    t.n0 = (u / p.num_slabs) * p.nt;
+    t.kc0 = kc[t.slab];
+    t.nkc = kc[t.slab + 1] - t.kc0;
+    t.rows = min((int64_t)kSlab, p.M - t.slab * kSlab);
     return t;
 }
 
-// Walks this CTA's (work item, k-chunk) sequence, skipping empty row-blocks.
-struct Cursor {
-    int64_t it;
-    int64_t kc;
+// Walks this CTA's windows: runs of up to kWin consecutive k-chunks of one
+// work unit, in the order the CTA processes them (units with no chunk skipped).
+struct Window {
+    int64_t it;          // work unit
+    int64_t k0, cnt;     // first chunk of the window within the unit, chunks in it
     Item t;
-    __device__ __forceinline__ void first(const Params &p, const int64_t *kcp, bool wa) {
-        kc = 0;
+    __device__ __forceinline__ void first(const Params &p, const int64_t *kcp) {
+        k0 = 0;
         for (it = blockIdx.x; it < p.num_items; it += gridDim.x) {
-            t = decode(p, kcp, it, wa);
-            if (t.nkc > 0) return;
+            t = decode(p, kcp, it);
+            if (t.nkc > 0) break;
         }
+        cnt = valid(p) ? min((int64_t)kWin, t.nkc) : 0;
     }
-    __device__ __forceinline__ void next(const Params &p, const int64_t *kcp, bool wa) {
-        if (++kc < t.nkc) return;
-        kc = 0;
-        for (it += gridDim.x; it < p.num_items; it += gridDim.x) {
-            t = decode(p, kcp, it, wa);
-            if (t.nkc > 0) return;
+    __device__ __forceinline__ void next(const Params &p, const int64_t *kcp) {
+        k0 += kWin;
+        if (k0 >= t.nkc) {
+            k0 = 0;
+            for (it += gridDim.x; it < p.num_items; it += gridDim.x) {
+                t = decode(p, kcp, it);
+                if (t.nkc > 0) break;
+            }
         }
+        cnt = valid(p) ? min((int64_t)kWin, t.nkc - k0) : 0;
     }
     __device__ __forceinline__ bool valid(const Params &p) const { return it < p.num_items; }
 };
 
-// ------------------------------------------------------------------ producers
-// Weight tile of a stage: thread 0 of the producers, TMA bulk copy.
-struct WeightCopier {
-    uint32_t last_phase[kMaxStages];
-    bool issued[kMaxStages];
-    __device__ __forceinline__ void init() {
-        for (int i = 0; i < kMaxStages; ++i) issued[i] = false;
-    }
-    __device__ __forceinline__ void copy(const Params &p, const Smem &s, int stage, uint32_t phase,
-                                         const uint8_t *src) {
-        mbar_arrive_expect_tx(&s.wfull[stage], p.w_tile_bytes);
-        bulk_g2s(smem_u32(s.w + stage * p.w_tile_bytes), src, p.w_tile_bytes, &s.wfull[stage]);
-        issued[stage] = true;
-        last_phase[stage] = phase;
-    }
-    // the CTA is unwinding: let every weight copy already issued land first
-    __device__ __forceinline__ void drain(const Params &p, const Smem &s) {
-        for (int i = 0; i < p.stages; ++i)
-            if (issued[i] && !mbar_wait(&s.wfull[i], last_phase[i], kDrainNs, nullptr))
-                atomicOr(p.status, kDevTimeout);
-    }
-};
+// Load plan of a chunk record (see DevLayout): number of tile loads.
+__device__ __forceinline__ int plan_loads(const uint8_t *rec) {
+    return *reinterpret_cast<const volatile int32_t *>(rec + kListBytes);
+}
 
-// Index lists of upcoming chunks, copied by TMA (256 B each) into a ring of
-// kIdxSlots shared-memory slots up to kIdxSlots chunks ahead of their use, so
-// the producers never wait on a global load for them.  Every producer thread
-// arrives on the slot's iempty barrier once it has read the list; thread 0
-// refills a slot only after that (bounded wait), one chunk later.
-struct IndexRing {
-    Cursor look;         // next chunk whose list is to be fetched (thread 0)
-    int64_t fetched;     // lists fetched so far
-    uint32_t last_phase[kIdxSlots];
-    bool pending[kIdxSlots];
-    __device__ __forceinline__ void fetch_one(const Params &p, const Smem &s, const int64_t *kcp,
-                                              bool wa) {
-        const int slot = (int)(fetched % kIdxSlots);
-        const uint32_t ph = (uint32_t)((fetched / kIdxSlots) & 1);
-        mbar_arrive_expect_tx(&s.ifull[slot], kBK * 4);
-        bulk_g2s(smem_u32(s.idx + slot * kBK),
-                 p.chunks + (look.t.kc0 + look.kc) * p.chunk_bytes + p.tile_bytes, kBK * 4,
-                 &s.ifull[slot]);
-        pending[slot] = true;
-        last_phase[slot] = ph;
-        ++fetched;
-        look.next(p, kcp, wa);
-    }
-    // thread 0: start the first kIdxSlots fetches
-    __device__ __forceinline__ void start(const Params &p, const Smem &s, const int64_t *kcp,
-                                          bool wa, const Cursor &first) {
-        look = first;
-        fetched = 0;
-        for (int i = 0; i < kIdxSlots; ++i) pending[i] = false;
-        for (int i = 0; i < kIdxSlots && look.valid(p); ++i) fetch_one(p, s, kcp, wa);
-    }
-    // thread 0, after the list of chunk `used` was read by everyone: refill its slot
-    __device__ __forceinline__ bool refill(const Params &p, const Smem &s, const int64_t *kcp,
-                                           bool wa, int64_t used, volatile int *abort_flag) {
-        const int slot = (int)(used % kIdxSlots);
-        pending[slot] = false;
-        if (!look.valid(p)) return true;
-        if (!mbar_wait(&s.iempty[slot], (uint32_t)((used / kIdxSlots) & 1), p.watchdog_ns,
-                       abort_flag))
-            return false;
-        // the readers' loads completed before their (release) arrivals, which the
-        // wait above acquired, so the TMA overwrite cannot overtake them
-        fetch_one(p, s, kcp, wa);
-        return true;
-    }
-    // the CTA is unwinding: let every list copy in flight land first
-    __device__ __forceinline__ void drain(const Params &p, const Smem &s) {
-        for (int i = 0; i < kIdxSlots; ++i)
-            if (pending[i] && !mbar_wait(&s.ifull[i], last_phase[i], kDrainNs, nullptr))
-                atomicOr(p.status, kDevTimeout);
-    }
-};
-
-// Gather warps (GEMM): per chunk, read the chunk's index list from the shared
-// ring, then copy the 64 activation rows it names into the stage with 16-byte
-// cp.async straight into the swizzled layout; arrive on the stage's data
-// barrier when the copies land (no blocking).
-template <bool WA>
+// ------------------------------------------------------------------ gather warps
 __device__ void gather_warps(const Params &p, const Smem &s) {
-    constexpr int GW = Roles<false>::kGatherWarps;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
-    Cursor cur;
-    cur.first(p, kcp, WA);
+    Window win;
+    win.first(p, kcp);
     int stage = 0;
     uint32_t phase = 0;
-    int64_t count = 0;
-    while (cur.valid(p)) {
-        const Item t = cur.t;
-        cur.next(p, kcp, WA);
-        const int slot = (int)(count % kIdxSlots);
-        if (!mbar_wait(&s.ifull[slot], (uint32_t)((count / kIdxSlots) & 1), p.watchdog_ns,
-                       abort_flag)) {
-            raise_timeout(p, s);
-            break;
-        }
-        // two entries of the list per lane, broadcast below by shuffles
-        const int2 iv = make_int2(s.idx[slot * kBK + lane], s.idx[slot * kBK + 32 + lane]);
-        mbar_arrive(&s.iempty[slot]);
-        const int64_t seq = count++;
-        const bool drop = blockIdx.x == 0 && seq == p.drop_stage;
-        if (!mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)) {
-            raise_timeout(p, s);
-            break;
-        }
-        if (!drop) {
-            const uint32_t xs = smem_u32(s.x + stage * p.x_tile_bytes);
-            if (WA) {
-                // 64 rows x 256 tokens: one warp instruction per 512-byte row segment
-                const int cn = lane >> 3, j = lane & 7;
-                const int64_t n = t.n0 + lane * 8;
-                const uint32_t nb = n < p.N ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
-                const uint16_t *xcol = p.X + (nb ? n : 0);
-#pragma unroll
-                for (int i = 0; i < 64 / GW; ++i) {
-                    const int r = warp + GW * i;
-                    const int idx = __shfl_sync(0xffffffffu, r < 32 ? iv.x : iv.y, r & 31);
-                    cp_async_16(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4),
-                                xcol + (int64_t)idx * p.ldx, nb);
-                }
-            } else {
-                // 64 rows x 128 tokens: one warp instruction covers two rows
-                const int u16 = lane & 15, cn = u16 >> 3, j = u16 & 7;
-                const int64_t n = t.n0 + u16 * 8;
-                const uint32_t nb = n < p.N ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
-                const uint16_t *xcol = p.X + (nb ? n : 0);
-#pragma unroll
-                for (int i = 0; i < 32 / GW; ++i) {
-                    const int r = 2 * (warp + GW * i) + (lane >> 4);
-                    const int idx = __shfl_sync(0xffffffffu, r < 32 ? iv.x : iv.y, r & 31);
-                    cp_async_16(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4),
-                                xcol + (int64_t)idx * p.ldx, nb);
-                }
-            }
-            // Signal the stage once this thread's copies have landed, without
-            // blocking.  The tile was written through the generic proxy; the
-            // tensor-core thread orders it before its async-proxy reads with a
-            // proxy fence after acquiring the barrier.
-            cp_async_arrive_noinc(&s.full[stage]);
-        }
-        if (++stage == p.stages) {
-            stage = 0;
-            phase ^= 1u;
-        }
-    }
-    cp_async_wait_all();
-}
-
-// Control thread (GEMM, lane 0 of the control warp): keeps the index-list ring
-// kIdxSlots chunks ahead and copies each stage's weight tile (TMA bulk) as
-// soon as the stage is free.
-template <bool WA>
-__device__ void control_thread(const Params &p, const Smem &s) {
-    const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
-    volatile int *abort_flag = s.abort_flag;
-    WeightCopier wc;
-    wc.init();
-    Cursor cur;
-    cur.first(p, kcp, WA);
-    IndexRing ring;
-    ring.start(p, s, kcp, WA, cur);
-    int stage = 0;
-    uint32_t phase = 0;
+    int64_t count = 0, wseq = 0;
     bool ok = true;
-    int64_t count = 0;
-    while (cur.valid(p)) {
-        const Item t = cur.t;
-        const int64_t kc = cur.kc;
-        cur.next(p, kcp, WA);
-        const int64_t seq = count++;
-        if (!mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)) {
-            raise_timeout(p, s);
-            ok = false;
-            break;
-        }
-        if (!(blockIdx.x == 0 && seq == p.drop_stage))
-            wc.copy(p, s, stage, phase,
-                    p.chunks + (t.kc0 + kc) * p.chunk_bytes + t.slab * (kSlab * kBK * 2));
-        if (seq > 0 && !ring.refill(p, s, kcp, WA, seq - 1, abort_flag)) {
-            raise_timeout(p, s);
-            ok = false;
-            break;
-        }
-        if (++stage == p.stages) {
-            stage = 0;
-            phase ^= 1u;
-        }
-    }
-    if (!ok) {
-        wc.drain(p, s);
-        ring.drain(p, s);
-    }
-}
-
-// ------------------------------------------------------------------ CONV producer (im2col)
-__device__ void producer_im2col(const Params &p, const Smem &s) {
-    const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
-    const int tid = threadIdx.x;            // 0..127
-    const int warp = tid >> 5, lane = tid & 31;
-    volatile int *abort_flag = s.abort_flag;
-    int stage = 0;
-    uint32_t phase = 0;
-    bool ok = true;
-    const int u16 = lane & 15;           // 16-byte unit (8 pixels) within a 128-pixel row
-    const int cn = u16 >> 3, j = u16 & 7;
-    int64_t count = 0;
-    WeightCopier wc;
-    wc.init();
-
-    for (int64_t it = blockIdx.x; it < p.num_items && ok; it += gridDim.x) {
-        const Item t = decode(p, kcp, it, false);
-        if (t.nkc == 0) continue;
-        // this thread's 8 pixels are fixed for the whole tile
-        int64_t pbase[8];
-        int ih0[8], iw0[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            const int64_t pix = t.n0 + u16 * 8 + e;
-            if (pix < p.N) {
-                const int64_t b = pix / p.HoWo, hw = pix % p.HoWo;
-                const int oh = (int)(hw / p.Wo), ow = (int)(hw % p.Wo);
-                pbase[e] = b * p.C * p.H * p.W;
-                ih0[e] = oh * p.sh - p.ph;
-                iw0[e] = ow * p.sw - p.pw;
-            } else {
-                pbase[e] = 0;
-                ih0[e] = -(1 << 29);     // never inside the image
-                iw0[e] = 0;
-            }
-        }
-        for (int64_t kc = 0; kc < t.nkc; ++kc) {
-            if (!mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)) {
-                raise_timeout(p, s);
-                ok = false;
-                break;
-            }
+    for (; win.valid(p) && ok; win.next(p, kcp), ++wseq) {
+        const int buf = (int)(wseq % kWinBufs);
+        // outcomes of waits are made warp-uniform, so the warp leaves the loop as one
+        ok = __all_sync(0xffffffffu, mbar_wait(&s.pfull[buf], (uint32_t)((wseq / kWinBufs) & 1),
+                                              p.watchdog_ns, abort_flag));
+        if (!ok) break;
+        const uint8_t *recs = s.win + buf * kWinBytes;
+        for (int64_t j = 0; j < win.cnt; ++j) {
+            const uint8_t *rec = recs + j * kMetaBytes;
+            const bool tma = plan_loads(rec) > 0;
             const int64_t seq = count++;
-            if (blockIdx.x == 0 && seq == p.drop_stage) {       // injected lost stage
-                if (++stage == p.stages) {
-                    stage = 0;
-                    phase ^= 1u;
-                }
-                continue;
-            }
-            const uint32_t xs = smem_u32(s.x + stage * p.x_tile_bytes);
-            const uint8_t *chunk = p.chunks + (t.kc0 + kc) * p.chunk_bytes;
-            if (tid == 0) wc.copy(p, s, stage, phase, chunk);
-            const int32_t *cl = reinterpret_cast<const int32_t *>(chunk + p.tile_bytes);
-#pragma unroll 2
-            for (int i = 0; i < 8; ++i) {
-                const int r = 2 * (warp + 4 * i) + (lane >> 4);
-                const int32_t idx = cl[r];
-                uint32_t v[4] = {0u, 0u, 0u, 0u};
-                const int64_t c = idx / p.KK;
-                const int rs = (int)(idx - c * p.KK);
-                const int di = rs / p.kw, dj = rs - (rs / p.kw) * p.kw;
-                const uint16_t *plane = p.X + c * p.H * p.W;
+            const bool drop = blockIdx.x == 0 && seq == p.drop_stage;
+            // source rows of this warp's 8 list positions, read before the stage is
+            // free: 16 bytes (8 columns) per lane, lanes past the tile's width idle
+            const uint16_t *src[kBK / kGatherWarps];
+            uint32_t nb = 0;
+            if (!tma) {
+                const int32_t *l = reinterpret_cast<const int32_t *>(rec);
+                const int64_t n = win.t.n0 + lane * 8;
+                nb = (lane * 8 < p.nt && n < p.N) ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
+                const uint16_t *xcol = p.X + (nb ? n : 0);
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const int ih = ih0[e] + di, iw = iw0[e] + dj;
-                    uint32_t h = 0u;
-                    if ((unsigned)ih < (unsigned)p.H && (unsigned)iw < (unsigned)p.W)
-                        h = __ldg(plane + pbase[e] + (int64_t)ih * p.W + iw);
-                    v[e >> 1] |= h << ((e & 1) * 16);
-                }
-                st_shared_v4(xs + cn * 8192 + r * 128 + ((j ^ (r & 7)) << 4),
-                             make_uint4(v[0], v[1], v[2], v[3]));
+                for (int i = 0; i < kBK / kGatherWarps; ++i)
+                    src[i] = xcol + (int64_t)l[warp + kGatherWarps * i] * p.ldx;
             }
-            fence_proxy_async_smem();
-            mbar_arrive(&s.full[stage]);
+            // A planned chunk is loaded and signalled by the control thread; the
+            // warp still waits for its stage (lane 0 alone), which keeps it at most
+            // one phase of the stage barriers ahead of the tensor cores.
+            ok = __all_sync(0xffffffffu,
+                            (!tma || lane == 0)
+                                ? mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)
+                                : true);
+            if (!ok) break;
+            if (!tma && !drop) {
+                // 64 rows x nt columns: one warp instruction per row segment
+                const uint32_t xs = smem_u32(s.x + stage * kXTileBytes);
+                const int cn = lane >> 3, jj = lane & 7;
+                if (lane * 8 < p.nt) {
+#pragma unroll
+                    for (int i = 0; i < kBK / kGatherWarps; ++i) {
+                        const int r = warp + kGatherWarps * i;
+                        cp_async_16(xs + cn * 8192 + r * 128 + ((jj ^ (r & 7)) << 4), src[i], nb);
+                    }
+                }
+                // Signal the stage once this thread's copies have landed, without
+                // blocking.  The tile was written through the generic proxy; the
+                // tensor-core thread orders it before its async-proxy reads with a
+                // proxy fence after acquiring the barrier.
+                cp_async_arrive_noinc(&s.full[stage]);
+            }
             if (++stage == p.stages) {
                 stage = 0;
                 phase ^= 1u;
             }
         }
+        if (!ok) break;
+        __syncwarp();        // the lanes' reads of the window precede lane 0's release
+        if (lane == 0) mbar_arrive(&s.pempty[buf]);
     }
-    if (!ok && tid == 0) wc.drain(p, s);
+    if (!ok) raise_timeout(p, s);
+    cp_async_wait_all();
+}
+
+// ------------------------------------------------------------------ control thread
+struct WindowFiller {
+    Window ahead;        // next window to copy into shared memory
+    int64_t filled;      // windows copied so far
+    __device__ __forceinline__ void fill(const Params &p, const Smem &s, const int64_t *kcp) {
+        const int buf = (int)(filled % kWinBufs);
+        const uint32_t bytes = (uint32_t)ahead.cnt * kMetaBytes;
+        mbar_arrive_expect_tx(&s.pfull[buf], bytes);
+        bulk_g2s(smem_u32(s.win + buf * kWinBytes),
+                 p.meta + (ahead.t.kc0 + ahead.k0) * kMetaBytes, bytes, &s.pfull[buf]);
+        ++filled;
+        ahead.next(p, kcp);
+    }
+    // the CTA is unwinding: let the window copies that may be in flight land first
+    __device__ __forceinline__ void drain(const Params &p, const Smem &s) {
+        for (int64_t q = filled > kWinBufs ? filled - kWinBufs : 0; q < filled; ++q)
+            if (!mbar_wait(&s.pfull[q % kWinBufs], (uint32_t)((q / kWinBufs) & 1), kDrainNs,
+                           nullptr))
+                atomicOr(p.status, kDevTimeout);
+    }
+};
+
+__device__ void control_thread(const Params &p, const Smem &s) {
+    const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
+    volatile int *abort_flag = s.abort_flag;
+    Window win;
+    win.first(p, kcp);
+    WindowFiller wf;
+    wf.ahead = win;
+    wf.filled = 0;
+    if (wf.ahead.valid(p)) wf.fill(p, s, kcp);
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    int64_t count = 0, wseq = 0;
+    for (; win.valid(p) && ok; win.next(p, kcp), ++wseq) {
+        const int buf = (int)(wseq % kWinBufs);
+        // copy the next window into the buffer released by window wseq - 2
+        if (wf.ahead.valid(p)) {
+            const int64_t prev = wf.filled - kWinBufs;
+            if (prev >= 0 && !mbar_wait(&s.pempty[prev % kWinBufs],
+                                        (uint32_t)((prev / kWinBufs) & 1), p.watchdog_ns,
+                                        abort_flag)) {
+                ok = false;
+                break;
+            }
+            wf.fill(p, s, kcp);
+        }
+        if (!mbar_wait(&s.pfull[buf], (uint32_t)((wseq / kWinBufs) & 1), p.watchdog_ns,
+                       abort_flag)) {
+            ok = false;
+            break;
+        }
+        const uint8_t *recs = s.win + buf * kWinBytes;
+        for (int64_t j = 0; j < win.cnt; ++j) {
+            const int64_t seq = count;
+            if (!mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)) {
+                ok = false;
+                break;
+            }
+            // the plan: words 0..11 in three 16-byte loads
+            const uint4 *pv = reinterpret_cast<const uint4 *>(recs + j * kMetaBytes + kListBytes);
+            const uint4 q0 = pv[0], q1 = pv[1], q2 = pv[2];
+            const int nb = (int)q0.x;
+            const bool tma = nb > 0;
+            ++count;
+            if (!(blockIdx.x == 0 && seq == p.drop_stage)) {
+                s.skind[stage] = tma ? 1u : 0u;    // read by the MMA thread after wfull
+                mbar_arrive_expect_tx(&s.wfull[stage],
+                                      kWTileBytes + (tma ? (uint32_t)p.xboxes * (kBK * 128) : 0u));
+                bulk_g2s(smem_u32(s.w + stage * kWTileBytes),
+                         p.tiles + (win.t.kc0 + win.k0 + j) * (int64_t)kWTileBytes, kWTileBytes,
+                         &s.wfull[stage]);
+                if (tma) {
+                    // load b: rows y[b] .. + (8 << lg) - 1 of X into list positions
+                    // 8g ..; x = a multiple of 64 tokens (16-byte aligned), and
+                    // columns past N, rows past K read as zero
+                    const uint32_t ys[8] = {q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w, q2.x};
+                    const uint32_t xs = smem_u32(s.x + stage * kXTileBytes);
+#pragma unroll
+                    for (int b = 0; b < kMaxBoxes; ++b) {
+                        if (b >= nb) break;
+                        const uint32_t d = ((b < 4 ? q2.y : q2.z) >> (8 * (b & 3))) & 0xffu;
+                        const uint32_t dst = xs + (d & 7u) * 1024;
+                        const CUtensorMap *map = &p.xmap[(d >> 4) & 3u];
+#pragma unroll
+                        for (int cn = 0; cn < p.xboxes; ++cn)
+                            tma_load_2d(dst + cn * 8192, map, (int32_t)(win.t.n0 + cn * 64),
+                                        (int32_t)ys[b], &s.wfull[stage]);
+                    }
+                }
+            }
+            if (++stage == p.stages) {
+                stage = 0;
+                phase ^= 1u;
+            }
+        }
+        if (!ok) break;
+        mbar_arrive(&s.pempty[buf]);
+    }
+    if (!ok) {
+        raise_timeout(p, s);
+        // unwinding: the copies of the last stages and the window copies may still
+        // be in flight; let them land before the CTA exits
+        for (int64_t q = count > p.stages ? count - p.stages : 0; q < count; ++q)
+            if (!(blockIdx.x == 0 && q == p.drop_stage) &&
+                !mbar_wait(&s.wfull[q % p.stages], (uint32_t)((q / p.stages) & 1), kDrainNs,
+                           nullptr))
+                atomicOr(p.status, kDevTimeout);
+        wf.drain(p, s);
+    }
 }
 
 // ------------------------------------------------------------------ MMA issuer
-template <bool WA>
 __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
+    // Everything the loop needs lives in registers: the per-chunk path is a
+    // chain of dependent barrier probes and issues, so any reload from the
+    // parameter bank or shared memory adds to every chunk.
     const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
-    const bool bf16 = p.dtype == BP_BF16;
-    const uint32_t idesc = WA ? make_idesc(bf16, false, true, 128, 256)
-                              : make_idesc(bf16, true, false, 128, (int)p.rows_pad);
+    const uint64_t wdog = p.watchdog_ns;
+    const int nst = (int)p.stages;
+    const int64_t nitems = p.num_items;
+    const uint32_t acc_cols = p.acc_cols;
+    uint64_t *const wfull = s.wfull, *const full = s.full, *const empty = s.empty;
+    const volatile uint32_t *const skind = s.skind;
+    const uint32_t idesc = make_idesc(p.dtype == BP_BF16, false, true, kSlab, p.nt);
+    // descriptors of stage 0; a stage / K=16 step adds its byte offset / 16 to
+    // the start-address field (shared addresses stay below 256 KB: no carry)
+    const uint64_t wdesc0 = make_sdesc_sw128(smem_u32(s.w), 16, 1024);
+    const uint64_t xdesc0 = make_sdesc_sw128(smem_u32(s.x), 8192, 1024);
     int stage = 0;
     uint32_t phase = 0;
+    uint32_t gphase = 0;     // per stage: parity of the next gathered fill (bit = stage)
     int acc = 0;
     uint32_t acc_phase = 0;
     bool ok = true;
-    for (int64_t it = blockIdx.x; it < p.num_items && ok; it += gridDim.x) {
-        const Item t = decode(p, kcp, it, WA);
+    for (int64_t it = blockIdx.x; it < nitems && ok; it += gridDim.x) {
+        const Item t = decode(p, kcp, it);
         if (t.nkc == 0) continue;
-        if (!mbar_wait(&s.tempty[acc], acc_phase ^ 1u, p.watchdog_ns, abort_flag)) {
+        if (!mbar_wait(&s.tempty[acc], acc_phase ^ 1u, wdog, abort_flag)) {
             raise_timeout(p, s);
             break;
         }
         tc_fence_after();
-        const uint32_t d = tmem + acc * p.acc_cols;
+        const uint32_t d = tmem + acc * acc_cols;
+        bool ready = mbar_test_wait(&wfull[stage], phase);
         for (int64_t kc = 0; kc < t.nkc; ++kc) {
-            if (!mbar_wait(&s.full[stage], phase, p.watchdog_ns, abort_flag) ||
-                !mbar_wait(&s.wfull[stage], phase, p.watchdog_ns, abort_flag)) {
+            if (!ready && !mbar_wait(&wfull[stage], phase, wdog, abort_flag)) {
                 raise_timeout(p, s);
                 ok = false;
                 break;
             }
-            // the activation tile was written through the generic proxy (cp.async /
-            // st.shared): order those writes, acquired through the barrier, before
-            // the tensor core's async-proxy reads
-            fence_proxy_async_smem();
+            if (skind[stage] == 0u) {
+                // gathered rows: wait for them, then order their generic-proxy
+                // (cp.async) writes, acquired through the barrier, before the tensor
+                // core's async-proxy reads
+                if (!mbar_wait(&full[stage], (gphase >> stage) & 1u, wdog, abort_flag)) {
+                    raise_timeout(p, s);
+                    ok = false;
+                    break;
+                }
+                gphase ^= 1u << stage;
+                fence_proxy_async_smem();
+            }
+            // order the MMAs below after the barrier waits above
             tc_fence_after();
-            const uint32_t ws = smem_u32(s.w + stage * p.w_tile_bytes);
-            const uint32_t xs = smem_u32(s.x + stage * p.x_tile_bytes);
+            const uint64_t wd = wdesc0 + (uint32_t)(stage * (kWTileBytes >> 4));
+            const uint64_t xd = xdesc0 + (uint32_t)(stage * (kXTileBytes >> 4));
+            const int nstage = stage + 1 == nst ? 0 : stage + 1;
+            const uint32_t nphase = stage + 1 == nst ? phase ^ 1u : phase;
+            // probe the next chunk's barrier now: the answer is needed only after
+            // the MMAs below have been issued
+            ready = kc + 1 < t.nkc && mbar_test_wait(&wfull[nstage], nphase);
 #pragma unroll
-            for (int kk = 0; kk < kBK / 16; ++kk) {
-                const uint64_t wdesc = make_sdesc_sw128(ws + kk * 32, 16, 1024);
-                const uint64_t xdesc = make_sdesc_sw128(xs + kk * 2048, 8192, 1024);
-                const uint32_t accum = (kc > 0 || kk > 0) ? 1u : 0u;
-                if (WA) umma_f16_ss(d, wdesc, xdesc, idesc, accum);
-                else umma_f16_ss(d, xdesc, wdesc, idesc, accum);
-            }
-            umma_commit(&s.empty[stage]);
-            if (++stage == p.stages) {
-                stage = 0;
-                phase ^= 1u;
-            }
+            for (int kk = 0; kk < kBK / 16; ++kk)
+                umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * (2048 >> 4), idesc,
+                            (kc > 0 || kk > 0) ? 1u : 0u);
+            umma_commit(&empty[stage]);
+            stage = nstage;
+            phase = nphase;
         }
         if (!ok) break;
         umma_commit(&s.tfull[acc]);
@@ -537,97 +474,89 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
 }
 
 // ------------------------------------------------------------------ epilogue
-template <bool WA, bool CONV>
 __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
     const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int q = warp & 3;                  // tensor-memory lane quadrant of this warp
+    const int q = warp & 3;                  // tensor-memory lane quadrant this warp may read
+    const uint32_t stg = smem_u32(s.ystage + (warp - kEpiWarp0) * 4096);
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int64_t it = blockIdx.x; it < p.num_items; it += gridDim.x) {
-        const Item t = decode(p, kcp, it, WA);
+        const Item t = decode(p, kcp, it);
         const bool has = t.nkc > 0;
         if (has) {
-            if (!mbar_wait(&s.tfull[acc], acc_phase, p.watchdog_ns, abort_flag)) {
+            // warp-uniform outcome: tcgen05.ld below is a warp-collective instruction
+            const bool ok = mbar_wait(&s.tfull[acc], acc_phase, p.watchdog_ns, abort_flag);
+            if (!__all_sync(0xffffffffu, ok)) {
                 raise_timeout(p, s);
                 break;
             }
             tc_fence_after();
         }
         const uint32_t tacc = tmem + ((uint32_t)(32 * q) << 16) + acc * p.acc_cols;
-        if (WA) {
-            // lane = output row; 32 x 32 boxes staged in shared memory (64-byte swizzle:
-            // 16-byte chunk c of row r sits at chunk c ^ ((r >> 1) & 3)), then TMA-stored
-            const int64_t row0 = t.slab * kSlab + 32 * q;
-            const bool vrow = row0 + lane < t.rows;
-            const float bv = (p.bias && vrow) ? p.bias[t.rb * p.bm + row0 + lane] : 0.f;
-            const uint32_t stg = smem_u32(s.ystage + (warp - Roles<CONV>::kEpiWarp0) * 4096);
-            for (int c0 = 0; c0 < 256 && t.n0 + c0 < p.N; c0 += 32) {
-                uint32_t r[32];
-                if (has) {
-                    tmem_ld_32x32b_x32(tacc + c0, r);
-                    tmem_ld_wait();
-                } else {
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) r[e] = 0u;
-                }
-                uint32_t pk[16];
-#pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    float a = __uint_as_float(r[2 * e]) + bv, b = __uint_as_float(r[2 * e + 1]) + bv;
-                    if (p.relu) {
-                        a = fmaxf(a, 0.f);
-                        b = fmaxf(b, 0.f);
-                    }
-                    pk[e] = pack2(a, b, p.dtype);
-                }
-                const uint32_t sb = stg + ((c0 >> 5) & 1) * 2048;
-                if (lane == 0) bulk_wait_read<1>();     // the store that used this buffer is done
-                __syncwarp();
-#pragma unroll
-                for (int ch = 0; ch < 4; ++ch)
-                    st_shared_v4(sb + lane * 64 + ((ch ^ ((lane >> 1) & 3)) << 4),
-                                 make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]));
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) {
-                    tma_store_2d(&p.ymap, sb, (int32_t)(t.n0 + c0), (int32_t)(t.rb * p.bm + row0));
-                    bulk_commit();
-                }
-            }
-        } else {
-            const int64_t n = t.n0 + 32 * q + lane;
-            const bool vcol = n < p.N;
-            int64_t obase = 0;                 // output offset of this token / pixel
-            int64_t ostride = p.ldy;           // between consecutive output rows
-            if (CONV) {
-                const int64_t b = vcol ? n / p.HoWo : 0, hw = vcol ? n % p.HoWo : 0;
-                obase = b * p.M * p.HoWo + hw;
-                ostride = p.HoWo;
+        // lane = output row of the slab; tensor-memory columns = the tile's columns
+        const int64_t row0 = 32 * q;
+        const bool vrow = row0 + lane < t.rows;
+        const int64_t m = t.slab * kSlab + row0 + lane;
+        const float bv = (p.bias && vrow) ? p.bias[m] : 0.f;
+        for (int c0 = 0; c0 < p.nt && t.n0 + c0 < p.N; c0 += 32) {
+            uint32_t r[32];
+            if (has) {
+                tmem_ld_32x32b_x32(tacc + c0, r);
+                tmem_ld_wait();
             } else {
-                obase = n;
+#pragma unroll
+                for (int e = 0; e < 32; ++e) r[e] = 0u;
             }
-            for (int c0 = 0; c0 < p.rows_pad; c0 += 16) {
-                uint32_t r[16];
-                if (has) {
-                    tmem_ld_32x32b_x16(tacc + c0, r);
-                    tmem_ld_wait();
-                } else {
+            uint32_t pk[16];
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) r[e] = 0u;
+            for (int e = 0; e < 16; ++e) {
+                float a = __uint_as_float(r[2 * e]) + bv, b = __uint_as_float(r[2 * e + 1]) + bv;
+                if (p.relu) {
+                    a = fmaxf(a, 0.f);
+                    b = fmaxf(b, 0.f);
                 }
-                if (!vcol) continue;
+                pk[e] = pack2(a, b, p.dtype);
+            }
+            const int64_t n = t.n0 + c0;
+            if (p.conv) {
+                // NCHW output: pixel n = b*HoWo + hw is element (b, m, hw)
+                if (!vrow) continue;
+                int64_t bb = n / p.HoWo, hw = n - bb * p.HoWo;
+                if (hw + 32 <= p.HoWo && (p.HoWo & 7) == 0) {
+                    // hw is a multiple of 8 here, so the row segment is 16-byte aligned
+                    uint4 *d4 = reinterpret_cast<uint4 *>(p.Y + (bb * p.M + m) * p.HoWo + hw);
 #pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    const int64_t row = c0 + e;
-                    if (row < t.rows) {
-                        const int64_t m = t.rb * p.bm + row;
-                        float v = __uint_as_float(r[e]) + (p.bias ? p.bias[m] : 0.f);
-                        if (p.relu && v < 0.f) v = 0.f;
-                        p.Y[obase + m * ostride] = cvt1(v, p.dtype);
+                    for (int ch = 0; ch < 4; ++ch)
+                        d4[ch] = make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2],
+                                            pk[4 * ch + 3]);
+                } else {
+                    for (int e = 0; e < 32 && n + e < p.N; ++e) {
+                        p.Y[(bb * p.M + m) * p.HoWo + hw] = (uint16_t)(pk[e >> 1] >> ((e & 1) * 16));
+                        if (++hw == p.HoWo) {
+                            hw = 0;
+                            ++bb;
+                        }
                     }
                 }
+                continue;
+            }
+            // GEMM: 32 x 32 box staged in shared memory (64-byte swizzle: 16-byte
+            // chunk c of row r sits at chunk c ^ ((r >> 1) & 3)), then TMA-stored;
+            // rows past M and columns past N of the box are not written
+            const uint32_t sb = stg + ((c0 >> 5) & 1) * 2048;
+            if (lane == 0) bulk_wait_read<1>();     // the store that used this buffer is done
+            __syncwarp();
+#pragma unroll
+            for (int ch = 0; ch < 4; ++ch)
+                st_shared_v4(sb + lane * 64 + ((ch ^ ((lane >> 1) & 3)) << 4),
+                             make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]));
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                tma_store_2d(&p.ymap, sb, (int32_t)n, (int32_t)(t.slab * kSlab + row0));
+                bulk_commit();
             }
         }
         if (has) {
@@ -639,19 +568,16 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             }
         }
     }
-    if (WA && lane == 0) bulk_wait_all();       // staged output fully written before exit
+    if (!p.conv && lane == 0) bulk_wait_all();   // staged output fully written before exit
 }
 
-template <bool WA, bool CONV>
-__global__ void __launch_bounds__(Roles<CONV>::kThreads, 1)
-    bp_mma_kernel(const __grid_constant__ Params p) {
-    using R = Roles<CONV>;
+__global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_constant__ Params p) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     const Smem s = carve(smem_raw, p);
     const int warp = threadIdx.x >> 5;
     if (threadIdx.x == 0) {
         for (int i = 0; i < p.stages; ++i) {
-            mbar_init(&s.full[i], R::kGatherThreads);
+            mbar_init(&s.full[i], kGatherThreads);
             mbar_init(&s.wfull[i], 1);
             mbar_init(&s.empty[i], 1);
         }
@@ -660,47 +586,70 @@ __global__ void __launch_bounds__(Roles<CONV>::kThreads, 1)
             mbar_init(&s.tempty[i], 128);
         }
         mbar_init(s.drain, 1);
-        for (int i = 0; i < kIdxSlots; ++i) {
-            mbar_init(&s.ifull[i], 1);
-            mbar_init(&s.iempty[i], R::kGatherThreads);
+        for (int i = 0; i < kWinBufs; ++i) {
+            mbar_init(&s.pfull[i], 1);
+            mbar_init(&s.pempty[i], kGatherWarps + 1);
         }
         *s.abort_flag = 0;
         fence_mbar_init();
     }
-    if (s.kc)
-        for (int64_t i = threadIdx.x; i < p.kc_cached; i += R::kThreads) s.kc[i] = p.kc_ptr[i];
-    if (warp == R::kMmaWarp) {
+    if (warp == kMmaWarp) {
         tmem_alloc(s.tmem_base, p.tmem_cols);
         tmem_relinquish();
     }
+    if (warp == kCtrlWarp && (threadIdx.x & 31) == 0)
+        for (int i = 0; i < 4; ++i) prefetch_tmap(&p.xmap[i]);
+    // Launched as a programmatic dependent: everything above overlaps the end of
+    // the previous kernel in the stream; wait for it before touching global
+    // memory (it may have written the inputs, or still read the output), then
+    // let the next kernel start its own set-up as SMs come free.
+    grid_dependency_wait();
+    grid_launch_dependents();
+    if (s.kc)
+        for (int64_t i = threadIdx.x; i < p.kc_cached; i += kThreads) s.kc[i] = p.kc_ptr[i];
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *s.tmem_base;
 
-    if (warp < R::kGatherWarps) {
-        if (CONV) producer_im2col(p, s);
-        else gather_warps<WA>(p, s);
-    } else if (warp == R::kCtrlWarp) {
-        if ((threadIdx.x & 31) == 0) control_thread<WA>(p, s);
+    if (warp < kGatherWarps) {
+        gather_warps(p, s);
+    } else if (warp == kCtrlWarp) {
+        if ((threadIdx.x & 31) == 0) control_thread(p, s);
         __syncwarp();
-    } else if (warp == R::kMmaWarp) {
-        if ((threadIdx.x & 31) == 0) mma_issuer<WA>(p, s, tmem);
+    } else if (warp == kMmaWarp) {
+        if ((threadIdx.x & 31) == 0) mma_issuer(p, s, tmem);
         __syncwarp();
     } else {
-        epilogue<WA, CONV>(p, s, tmem);
+        epilogue(p, s, tmem);
     }
 
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == R::kMmaWarp) tmem_dealloc(tmem, p.tmem_cols);
+    if (warp == kMmaWarp) tmem_dealloc(tmem, p.tmem_cols);
 }
 
-uint32_t pow2_at_least(uint32_t v) {
-    uint32_t r = 32;
-    while (r < v) r <<= 1;
-    return r;
+// Activation columns per tile (the MMA's N; a multiple of 32, the epilogue's
+// column group, from 64 to 256).  A chunk costs about the same whatever the
+// width: its 64 activation rows take one gather instruction per row and warp,
+// however many columns the lanes cover.  Persistent CTAs take work units in
+// waves, each unit the same number of chunks, so the kernel lasts about
+// (waves x chunks per unit): pick the widest tile with the fewest waves, no
+// wider than N needs (the MMA's time does grow with the width).
+int pick_tile_width(int64_t N, int64_t slabs, int sms) {
+    const int widest = (int)std::max<int64_t>(64, std::min<int64_t>(kNT, (N + 31) / 32 * 32));
+    int best = widest;
+    int64_t best_waves = INT64_MAX;
+    for (int nt = widest; nt >= 64; nt -= 32) {
+        const int64_t items = (N + nt - 1) / nt * slabs;
+        const int64_t waves = (items + sms - 1) / sms;
+        if (waves < best_waves) {
+            best_waves = waves;
+            best = nt;
+        }
+    }
+    return best;
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -717,104 +666,98 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-template <bool WA, bool CONV>
-cudaError_t launch_variant(Params &p, cudaStream_t st) {
-    static std::once_flag once;
-    static cudaError_t attr_err = cudaSuccess;
-    std::call_once(once, [] {
-        attr_err = cudaFuncSetAttribute(bp_mma_kernel<WA, CONV>,
-                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxSmem);
-    });
-    if (attr_err != cudaSuccess) return attr_err;
-    const size_t smem = 1024 + (size_t)p.stages * (p.w_tile_bytes + p.x_tile_bytes) +
-                        p.ystage_bytes + (3 * (size_t)p.stages + 7 + 2 * kIdxSlots) * 8 +
-                        128 + (size_t)kIdxSlots * kBK * 4 + 8 * (size_t)p.kc_cached;
-    const int64_t grid = p.num_items < num_sms() ? p.num_items : num_sms();
-    bp_mma_kernel<WA, CONV><<<(unsigned)grid, Roles<CONV>::kThreads, smem, st>>>(p);
-    return cudaGetLastError();
-}
-
 }  // namespace
 
 cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, int64_t N,
                        int64_t ldx, const float *bias, int relu, void *Y, int64_t ldy,
                        const ConvShape *conv, cudaStream_t st) {
     Params p{};
-    // GEMMs put 128-row weight slabs on the MMA M side when bm allows it;
-    // convolutions (and bm not a multiple of 128) put 128 pixels / tokens there.
-    // Both read the same device image when rows_pad <= 256.
-    const bool wa = conv == nullptr && dl.orient == kWeightA;
-    if (!wa && dl.rows_pad > 256) return cudaErrorInvalidValue;
     const uint8_t *dev = static_cast<const uint8_t *>(P.dev);
     p.dtype = P.lay.dtype;
     p.relu = relu;
+    p.conv = conv ? 1 : 0;
     p.M = P.lay.M;
-    p.bm = P.lay.bm;
-    p.rows_pad = dl.rows_pad;
-    p.num_rb = P.num_rb;
-    p.nslab = wa ? dl.rows_pad / kSlab : 1;
+    p.num_slabs = dl.num_slabs;
     p.N = N;
-    const int64_t nt = wa ? 256 : 128;
-    p.num_items = (N + nt - 1) / nt * p.num_rb * p.nslab;
-    p.w_tile_bytes = (uint32_t)((wa ? kSlab : dl.rows_pad) * kBK * 2);
-    p.x_tile_bytes = (uint32_t)(nt * kBK * 2);
-    p.ystage_bytes = wa ? 4 * 2 * 2048 : 0;
-    p.kc_cached = p.num_rb + 1 <= kMaxCachedRb + 1 ? p.num_rb + 1 : 0;
-    // shared memory: stages + output staging + barriers + kc_ptr copy, within 227 KB
+    p.nt = pick_tile_width(N, p.num_slabs, num_sms());
+    p.xboxes = (p.nt + 63) / 64;
+    p.num_items = (N + p.nt - 1) / p.nt * p.num_slabs;
+    if (p.num_items == 0) return cudaSuccess;
+    p.ystage_bytes = conv ? 0 : 4 * 2 * 2048;
+    // shared memory: stages, output staging, barriers, index ring, and a copy of
+    // kc_ptr when that costs no pipeline stage
     auto stages_for = [&](int64_t kc) {
-        const int64_t avail =
-            kMaxSmem - 1024 - p.ystage_bytes - 8 * 48 - 128 - kIdxSlots * kBK * 4 - 8 * kc;
-        const int64_t st = avail / (p.w_tile_bytes + p.x_tile_bytes);
-        return st > kMaxStages ? (int64_t)kMaxStages : st;
+        int64_t n = kMaxStages;
+        while (n > 0 && (int64_t)smem_bytes(n, p.ystage_bytes, kc) > kMaxSmem) --n;
+        return n;
     };
-    if (stages_for(p.kc_cached) < 3) p.kc_cached = 0;
-    p.stages = stages_for(p.kc_cached);
+    p.stages = stages_for(0);
     if (p.stages < 2) return cudaErrorInvalidValue;
-    p.acc_cols = pow2_at_least(wa ? 256u : (uint32_t)dl.rows_pad);
-    p.tmem_cols = 2 * p.acc_cols;
+    const int64_t kc_entries = p.num_slabs + 1;
+    p.kc_cached = (kc_entries <= kMaxCachedKc && stages_for(kc_entries) == p.stages) ? kc_entries : 0;
+    p.acc_cols = kNT;
+    p.tmem_cols = 2 * kNT;
     p.kc_ptr = reinterpret_cast<const int64_t *>(dev);
-    p.chunks = dev + dl.off_chunks;
-    p.tile_bytes = dl.tile_bytes;
-    p.chunk_bytes = dl.chunk_bytes;
+    p.tiles = dev + dl.off_tiles;
+    p.meta = dev + dl.off_meta;
     p.X = static_cast<const uint16_t *>(X);
     p.ldx = ldx;
     p.Y = static_cast<uint16_t *>(Y);
     p.ldy = ldy;
+    p.HoWo = conv ? conv->Ho * conv->Wo : 0;
     p.bias = bias;
     p.watchdog_ns = watchdog_ns();
     p.drop_stage = debug_drop_stage();
     p.status = device_status_ptr();
-    if (p.num_items == 0) return cudaSuccess;
-    if (conv) {
-        p.C = conv->C;
-        p.H = conv->H;
-        p.W = conv->W;
-        p.Ho = conv->Ho;
-        p.Wo = conv->Wo;
-        p.HoWo = conv->Ho * conv->Wo;
-        p.KK = (int64_t)conv->kh * conv->kw;
-        p.kw = conv->kw;
-        p.ph = conv->ph;
-        p.pw = conv->pw;
-        p.sh = conv->sh;
-        p.sw = conv->sw;
-        return launch_variant<false, true>(p, st);
-    }
-    if (!wa) return launch_variant<false, false>(p, st);
-    // Y as a 2-D tensor (N inner, M rows) for the epilogue's 32 x 32 box stores
+
     PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
     if (!enc) return cudaErrorNotSupported;
-    const cuuint64_t gdim[2] = {(cuuint64_t)N, (cuuint64_t)P.lay.M};
-    const cuuint64_t gstride[1] = {(cuuint64_t)ldy * 2};
-    const cuuint32_t box[2] = {32, 32};
-    const cuuint32_t estride[2] = {1, 1};
-    if (enc(&p.ymap,
-            P.lay.dtype == BP_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16,
-            2, Y, gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
-            CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-        return cudaErrorInvalidValue;
-    return launch_variant<true, false>(p, st);
+    const CUtensorMapDataType tdt =
+        P.lay.dtype == BP_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
+    for (int i = 0; i < 4; ++i) {
+        // X (N inner, K rows): 64-token x (8 << i)-row boxes for runs of consecutive columns
+        const cuuint64_t gdim[2] = {(cuuint64_t)N, (cuuint64_t)P.lay.K};
+        const cuuint64_t gstride[1] = {(cuuint64_t)ldx * 2};
+        const cuuint32_t box[2] = {64, (cuuint32_t)(8 << i)};
+        const cuuint32_t estride[2] = {1, 1};
+        if (enc(&p.xmap[i], tdt, 2, const_cast<void *>(X), gdim, gstride, box, estride,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    if (!conv) {
+        // Y (N inner, M rows) for the epilogue's 32 x 32 box stores
+        const cuuint64_t gdim[2] = {(cuuint64_t)N, (cuuint64_t)P.lay.M};
+        const cuuint64_t gstride[1] = {(cuuint64_t)ldy * 2};
+        const cuuint32_t box[2] = {32, 32};
+        const cuuint32_t estride[2] = {1, 1};
+        if (enc(&p.ymap, tdt, 2, Y, gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [] {
+        attr_err = cudaFuncSetAttribute(bp_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        (int)kMaxSmem);
+    });
+    if (attr_err != cudaSuccess) return attr_err;
+    const int64_t grid = p.num_items < num_sms() ? p.num_items : num_sms();
+    // programmatic dependent launch: the kernel's set-up may overlap the tail of
+    // the previous kernel in the stream (the kernel waits for it before any
+    // global memory access)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem_bytes(p.stages, p.ystage_bytes, p.kc_cached);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, bp_mma_kernel, p);
 }
 
 }  // namespace bp

@@ -1,9 +1,8 @@
 // Packing kernels: mask -> per-row-block kept-column counts (with the check
 // that all rows of a row-block agree, the BCS occurrence property of
-// Sec. 4.3), then col_idx / values (the canonical compact arrays) and the
-// device image the tensor-core kernels stream: per row-block k-chunks of 64
-// kept columns, each a (rows_pad x 64) K-major tile already in the 128-byte
-// swizzled shared-memory order, plus the padded column list of every chunk.
+// Sec. 4.3), then col_idx / values (the canonical compact arrays), the device
+// image the tensor-core kernel streams (128-row slabs, see DevLayout), and the
+// im2col expansion used by convolutions.
 #include "bp_common.cuh"
 
 namespace bp {
@@ -99,51 +98,217 @@ __global__ void values_kernel(int64_t M, int64_t K, int64_t bm,
     }
 }
 
-// Padded column list of every k-chunk: entry r of chunk kc of row-block rb is
-// its (kc*64 + r)-th kept column; past K'_rb it repeats the row-block's last
-// kept column (a valid row to load, multiplied by the zero-padded weights).
-__global__ void cidx_kernel(const int64_t *__restrict__ rb_ptr, const int64_t *__restrict__ kc_ptr,
-                            const int32_t *__restrict__ col_idx, uint8_t *__restrict__ chunks,
-                            int64_t tile_bytes, int64_t chunk_bytes) {
-    const int64_t rb = blockIdx.x;
-    const int64_t p0 = rb_ptr[rb], kp = rb_ptr[rb + 1] - p0;
-    const int64_t c0 = kc_ptr[rb], nkc = kc_ptr[rb + 1] - c0;
-    for (int64_t t = threadIdx.x; t < nkc * kBK; t += blockDim.x) {
-        int32_t *cl = reinterpret_cast<int32_t *>(chunks + (c0 + t / kBK) * chunk_bytes + tile_bytes);
-        cl[t % kBK] = col_idx[p0 + (t < kp ? t : kp - 1)];
+// Is column k kept by any row of slab s?  (rows of a row-block are identical,
+// so the first row of each row-block the slab touches decides)
+__device__ __forceinline__ bool slab_keeps(const uint8_t *__restrict__ mask, int64_t M, int64_t K,
+                                           int64_t bm, int64_t s, int64_t k) {
+    const int64_t r0 = s * kSlab, r1 = min(r0 + kSlab, M);
+    for (int64_t rb = r0 / bm; rb * bm < r1; ++rb)
+        if (mask[rb * bm * K + k]) return true;
+    return false;
+}
+
+// One block per slab, one warp per aligned 64-column block at a time.
+__global__ void slab_counts_kernel(int64_t M, int64_t K, int64_t bm,
+                                   const uint8_t *__restrict__ mask, int64_t *__restrict__ info) {
+    const int64_t s = blockIdx.x;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nwarps = blockDim.x >> 5;
+    int64_t dense = 0, sparse = 0;
+    for (int64_t blk = warp; blk * kBK < K; blk += nwarps) {
+        const int64_t k0 = blk * kBK;
+        const bool a = k0 + lane < K && slab_keeps(mask, M, K, bm, s, k0 + lane);
+        const bool b = k0 + 32 + lane < K && slab_keeps(mask, M, K, bm, s, k0 + 32 + lane);
+        const int u = __popc(__ballot_sync(0xffffffffu, a)) + __popc(__ballot_sync(0xffffffffu, b));
+        const bool whole = u >= kDenseMin && k0 + kBK <= K;
+        if (whole) ++dense;
+        else sparse += u;
+    }
+    __shared__ unsigned long long sd, ss;
+    if (threadIdx.x == 0) sd = ss = 0;
+    __syncthreads();
+    if (lane == 0) {
+        atomicAdd(&sd, (unsigned long long)dense);
+        atomicAdd(&ss, (unsigned long long)sparse);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        info[2 * s] = (int64_t)sd;
+        info[2 * s + 1] = (int64_t)ss;
     }
 }
 
-// Tiles: one thread per 16-byte unit (8 consecutive k of one row).
-__global__ void tiles_kernel(int64_t M, int64_t bm, int64_t rows_pad,
-                             const int64_t *__restrict__ rb_ptr,
-                             const int64_t *__restrict__ kc_ptr,
-                             const uint16_t *__restrict__ values, uint8_t *__restrict__ chunks,
-                             int64_t chunk_bytes) {
-    const int64_t rb = blockIdx.y;
-    const int64_t p0 = rb_ptr[rb], kp = rb_ptr[rb + 1] - p0;
-    const int64_t c0 = kc_ptr[rb], nkc = kc_ptr[rb + 1] - c0;
-    const int64_t rows = min(bm, M - rb * bm);
-    const int64_t units = nkc * rows_pad * (kBK / 8);
+// One warp per slab: the slab's chunk column lists, dense blocks first (in
+// block order), then the remaining union columns ascending, 64 per chunk; the
+// last chunk's unused entries repeat its last index.
+__global__ void slab_lists_kernel(int64_t M, int64_t K, int64_t bm, const uint8_t *__restrict__ mask,
+                                  const int64_t *__restrict__ kc_ptr, uint8_t *__restrict__ meta) {
+    const int64_t s = blockIdx.x;
+    const int lane = threadIdx.x;
+    const int64_t c0 = kc_ptr[s], nkc = kc_ptr[s + 1] - c0;
+    if (nkc == 0) return;
+    auto list = [&](int64_t c) {
+        return reinterpret_cast<int32_t *>(meta + (c0 + c) * kMetaBytes);
+    };
+    int64_t ndense = 0;
+    for (int64_t k0 = 0; k0 < K; k0 += kBK) {
+        const bool a = k0 + lane < K && slab_keeps(mask, M, K, bm, s, k0 + lane);
+        const bool b = k0 + 32 + lane < K && slab_keeps(mask, M, K, bm, s, k0 + 32 + lane);
+        const int u = __popc(__ballot_sync(0xffffffffu, a)) + __popc(__ballot_sync(0xffffffffu, b));
+        if (u >= kDenseMin && k0 + kBK <= K) {
+            int32_t *l = list(ndense++);
+            l[lane] = (int32_t)(k0 + lane);
+            l[lane + 32] = (int32_t)(k0 + 32 + lane);
+        }
+    }
+    int64_t pos = ndense * kBK;        // next free slot (chunk-major)
+    int32_t last = 0;
+    for (int64_t k0 = 0; k0 < K; k0 += kBK) {
+        const bool a = k0 + lane < K && slab_keeps(mask, M, K, bm, s, k0 + lane);
+        const bool b = k0 + 32 + lane < K && slab_keeps(mask, M, K, bm, s, k0 + 32 + lane);
+        const unsigned ba = __ballot_sync(0xffffffffu, a), bb = __ballot_sync(0xffffffffu, b);
+        const int u = __popc(ba) + __popc(bb);
+        if (u == 0 || (u >= kDenseMin && k0 + kBK <= K)) continue;
+        const unsigned below = (1u << lane) - 1u;
+        if (a) {
+            const int64_t q = pos + __popc(ba & below);
+            list(q / kBK)[q % kBK] = (int32_t)(k0 + lane);
+        }
+        if (b) {
+            const int64_t q = pos + __popc(ba) + __popc(bb & below);
+            list(q / kBK)[q % kBK] = (int32_t)(k0 + 32 + lane);
+        }
+        const int hi = bb ? 32 + (31 - __clz(bb)) : 31 - __clz(ba);
+        last = (int32_t)(k0 + hi);
+        pos += u;
+    }
+    __syncwarp();
+    // pad the last sparse chunk
+    const int64_t end = nkc * kBK;
+    for (int64_t q = pos + lane; q < end; q += 32) list(q / kBK)[q % kBK] = last;
+}
+
+// Tiles: one thread per 16-byte unit (8 consecutive list entries of one row).
+// Entry e of a chunk is live when e == 0 or its index differs from entry e-1
+// (lists ascend; padding repeats); dead entries and pruned weights are 0.
+__global__ void tiles_kernel(int64_t M, int64_t K, const uint16_t *__restrict__ W,
+                             const uint8_t *__restrict__ mask, const int64_t *__restrict__ kc_ptr,
+                             uint8_t *__restrict__ tiles, const uint8_t *__restrict__ meta,
+                             int64_t tile_bytes) {
+    const int64_t s = blockIdx.y;
+    const int64_t c0 = kc_ptr[s], nkc = kc_ptr[s + 1] - c0;
+    const int64_t units = nkc * kSlab * (kBK / 8);
     for (int64_t u = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; u < units;
          u += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t kc = u / (rows_pad * (kBK / 8));
-        const int64_t rem = u % (rows_pad * (kBK / 8));
+        const int64_t kc = u / (kSlab * (kBK / 8));
+        const int64_t rem = u % (kSlab * (kBK / 8));
         const uint32_t row = (uint32_t)(rem / (kBK / 8));
         const uint32_t ch = (uint32_t)(rem % (kBK / 8));
+        uint8_t *chunk = tiles + (c0 + kc) * tile_bytes;
+        const int32_t *l = reinterpret_cast<const int32_t *>(meta + (c0 + kc) * kMetaBytes);
+        const int64_t r = s * kSlab + row;
         uint16_t v[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-            const int64_t k = kc * kBK + ch * 8 + e;
-            v[e] = (row < rows && k < kp) ? values[bm * p0 + row * kp + k] : (uint16_t)0;
+            const int q = (int)ch * 8 + e;
+            const int32_t k = l[q];
+            const bool live = q == 0 || k != l[q - 1];
+            v[e] = (live && r < M && mask[r * K + k]) ? W[r * K + k] : (uint16_t)0;
         }
         uint4 pk;
         pk.x = v[0] | ((uint32_t)v[1] << 16);
         pk.y = v[2] | ((uint32_t)v[3] << 16);
         pk.z = v[4] | ((uint32_t)v[5] << 16);
         pk.w = v[6] | ((uint32_t)v[7] << 16);
-        uint8_t *tile = chunks + (c0 + kc) * chunk_bytes;
-        *reinterpret_cast<uint4 *>(tile + sw128_kmajor_offset(row, ch * 8)) = pk;
+        *reinterpret_cast<uint4 *>(chunk + sw128_kmajor_offset(row, ch * 8)) = pk;
+    }
+}
+
+// Load plans: one thread per chunk.  The 64 list positions form 8 groups of 8;
+// a group can be one tile load when each live entry (first occurrence of its
+// index) is the group's first column plus its offset.  When every group can,
+// maximal runs of groups that continue one another (first column 8 past the
+// previous group's, or no live entry at all: padding, whose rows meet zero
+// weights) become loads of 64, 32, 16 or 8 rows; otherwise the plan is empty
+// and the kernel gathers the chunk's rows one by one.
+__global__ void plans_kernel(int64_t kc_total, uint8_t *__restrict__ meta_all) {
+    for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < kc_total;
+         c += (int64_t)gridDim.x * blockDim.x) {
+        uint8_t *meta = meta_all + c * kMetaBytes;
+        const int32_t *l = reinterpret_cast<const int32_t *>(meta);
+        int32_t first[8];
+        bool ok = true;
+        for (int g = 0; g < 8; ++g) {
+            first[g] = l[8 * g];
+            for (int i = 1; i < 8; ++i) {
+                const int q = 8 * g + i;
+                if (l[q] != l[q - 1] && l[q] != first[g] + i) ok = false;
+            }
+        }
+        int32_t w[kPlanBytes / 4];
+        for (int i = 0; i < kPlanBytes / 4; ++i) w[i] = 0;
+        if (ok) {
+            int nb = 0;
+            uint32_t desc[2] = {0u, 0u};
+            for (int g = 0; g < 8;) {
+                int run = 1;
+                while (g + run < 8 && (first[g + run] == first[g] + 8 * run ||
+                                       l[8 * (g + run)] == l[8 * (g + run) - 1]))
+                    ++run;
+                const int lg = run >= 8 ? 3 : run >= 4 ? 2 : run >= 2 ? 1 : 0;
+                w[1 + nb] = first[g];
+                desc[nb >> 2] |= (uint32_t)(g | (lg << 4)) << (8 * (nb & 3));
+                ++nb;
+                g += 1 << lg;
+            }
+            w[0] = nb;
+            w[9] = (int32_t)desc[0];
+            w[10] = (int32_t)desc[1];
+        }
+        int32_t *plan = reinterpret_cast<int32_t *>(meta + kListBytes);
+        for (int i = 0; i < kPlanBytes / 4; ++i) plan[i] = w[i];
+    }
+}
+
+// im2col: one thread per 8 consecutive columns n of one row k.
+__global__ void im2col_kernel(ConvShape cs, int64_t ldx, const uint16_t *__restrict__ in,
+                              uint16_t *__restrict__ xcol) {
+    const int64_t K = cs.C * cs.kh * cs.kw;
+    const int64_t N = cs.Nb * cs.Ho * cs.Wo;
+    const int64_t HoWo = cs.Ho * cs.Wo;
+    const int64_t units_per_row = (N + 7) / 8;
+    for (int64_t u = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; u < K * units_per_row;
+         u += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t k = u / units_per_row, n0 = (u % units_per_row) * 8;
+        const int64_t c = k / (cs.kh * cs.kw);
+        const int rs = (int)(k % (cs.kh * cs.kw));
+        const int i = rs / cs.kw, j = rs % cs.kw;
+        int64_t b = n0 / HoWo, hw = n0 % HoWo;
+        int oh = (int)(hw / cs.Wo), ow = (int)(hw % cs.Wo);
+        uint16_t v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            uint16_t x = 0;
+            if (n0 + e < N) {
+                const int ih = oh * cs.sh + i - cs.ph, iw = ow * cs.sw + j - cs.pw;
+                if ((unsigned)ih < (unsigned)cs.H && (unsigned)iw < (unsigned)cs.W)
+                    x = __ldg(in + ((b * cs.C + c) * cs.H + ih) * cs.W + iw);
+            }
+            v[e] = x;
+            if (++ow == cs.Wo) {
+                ow = 0;
+                if (++oh == cs.Ho) {
+                    oh = 0;
+                    ++b;
+                }
+            }
+        }
+        uint4 pk;
+        pk.x = v[0] | ((uint32_t)v[1] << 16);
+        pk.y = v[2] | ((uint32_t)v[3] << 16);
+        pk.z = v[4] | ((uint32_t)v[5] << 16);
+        pk.w = v[6] | ((uint32_t)v[7] << 16);
+        *reinterpret_cast<uint4 *>(xcol + k * ldx + n0) = pk;
     }
 }
 
@@ -161,6 +326,13 @@ cudaError_t launch_rb_counts(const bp_layout &lay, const uint8_t *mask, int64_t 
     return cudaGetLastError();
 }
 
+cudaError_t launch_slab_counts(const bp_layout &lay, const uint8_t *mask, int64_t *info,
+                               cudaStream_t s) {
+    const int64_t S = (lay.M + kSlab - 1) / kSlab;
+    slab_counts_kernel<<<(unsigned)S, 256, 0, s>>>(lay.M, lay.K, lay.bm, mask, info);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_pack(const bp_layout &lay, const void *W, const uint8_t *mask,
                         const bp_packed &P, const DevLayout &dl, cudaStream_t s) {
     const int64_t RB = P.num_rb;
@@ -172,18 +344,34 @@ cudaError_t launch_pack(const bp_layout &lay, const void *W, const uint8_t *mask
                                                static_cast<const uint16_t *>(W), P.rb_ptr,
                                                P.col_idx, static_cast<uint16_t *>(P.values));
     e = cudaGetLastError();
-    if (e != cudaSuccess || dl.orient == kNoTensorCore) return e;
+    if (e != cudaSuccess || dl.kc_total == 0) return e;
     uint8_t *dev = static_cast<uint8_t *>(P.dev);
     const int64_t *kc_ptr = reinterpret_cast<const int64_t *>(dev);
-    uint8_t *chunks = dev + dl.off_chunks;
-    cidx_kernel<<<(unsigned)RB, 256, 0, s>>>(P.rb_ptr, kc_ptr, P.col_idx, chunks, dl.tile_bytes,
-                                             dl.chunk_bytes);
+    uint8_t *tiles = dev + dl.off_tiles;
+    uint8_t *meta = dev + dl.off_meta;
+    slab_lists_kernel<<<(unsigned)dl.num_slabs, 32, 0, s>>>(lay.M, lay.K, lay.bm, mask, kc_ptr,
+                                                           meta);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    dim3 grid(8, (unsigned)RB);
-    tiles_kernel<<<grid, 256, 0, s>>>(lay.M, lay.bm, dl.rows_pad, P.rb_ptr, kc_ptr,
-                                      static_cast<const uint16_t *>(P.values), chunks,
-                                      dl.chunk_bytes);
+    int64_t pblocks = (dl.kc_total + 127) / 128;
+    if (pblocks > 1024) pblocks = 1024;
+    plans_kernel<<<(unsigned)pblocks, 128, 0, s>>>(dl.kc_total, meta);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    dim3 grid(16, (unsigned)dl.num_slabs);
+    tiles_kernel<<<grid, 256, 0, s>>>(lay.M, lay.K, static_cast<const uint16_t *>(W), mask, kc_ptr,
+                                      tiles, meta, dl.tile_bytes);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void *xcol,
+                          cudaStream_t s) {
+    const int64_t K = cs.C * cs.kh * cs.kw, N = cs.Nb * cs.Ho * cs.Wo;
+    const int64_t units = K * ((N + 7) / 8);
+    int64_t blocks = (units + 255) / 256;
+    if (blocks > 152 * 64) blocks = 152 * 64;
+    im2col_kernel<<<(unsigned)blocks, 256, 0, s>>>(cs, ldx, static_cast<const uint16_t *>(in),
+                                                   static_cast<uint16_t *>(xcol));
     return cudaGetLastError();
 }
 

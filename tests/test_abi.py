@@ -91,22 +91,41 @@ def test_rate_below_one_rejected_on_host(lib):
 
 def test_gemm_argument_checks_on_host(lib):
     lay = bp.layout(bp.BLOCK_BASED, bp.F16, 64, 64, 16, 16)
-    P = bp.Packed(lay, 4, 0, 0, 16, 16, 16, 256, 1 << 12)
+    P = bp.Packed(lay, 4, 0, 0, 16, 16, 16, 256, 256 + 16384 + 320)
     # ldx not a multiple of 8, misaligned X, N > ldx, null packed
     assert bp.bp_gemm(P, 256, 10, 10, None, 0, 256, 16, 0) == bp.ERR_INVALID_ARG
     assert bp.bp_gemm(P, 258, 8, 8, None, 0, 256, 8, 0) == bp.ERR_INVALID_ARG
     assert bp.bp_gemm(P, 256, 16, 8, None, 0, 256, 16, 0) == bp.ERR_INVALID_ARG
     assert bp.load().bp_gemm(None, 256, 8, 8, None, 0, 256, 8, None) == bp.ERR_INVALID_ARG
-    # bm > 256 and not a multiple of 128 has no tensor-core path
-    lay2 = bp.layout(bp.BLOCK_BASED, bp.F16, 600, 64, 300, 16)
-    P2 = bp.Packed(lay2, 2, 0, 0, 16, 16, 16, 256, 1 << 12)
+    # an image size that is not kc_ptr + whole (tile, record) chunks
+    Pbad = bp.Packed(lay, 4, 0, 0, 16, 16, 16, 256, 256 + 16384)
+    assert bp.bp_gemm(Pbad, 256, 8, 8, None, 0, 256, 8, 0) == bp.ERR_INVALID_ARG
+    # more than 8192 slabs of 128 rows (M > 1,048,576) is beyond the device image
+    M2 = (1 << 20) + 128
+    lay2 = bp.layout(bp.BLOCK_BASED, bp.F16, M2, 64, 16, 16)
+    P2 = bp.Packed(lay2, M2 // 16, 0, 0, 16, 16, 16, 256, 1 << 20)
     assert bp.bp_gemm(P2, 256, 8, 8, None, 0, 256, 8, 0) == bp.ERR_UNSUPPORTED
 
 
 def test_conv_argument_checks_on_host(lib):
     lay = bp.layout(bp.BLOCK_PUNCHED, bp.F16, 16, 8 * 9, 8, 4, 3, 3)
-    P = bp.Packed(lay, 2, 0, 0, 16, 16, 16, 256, 1 << 12)
+    P = bp.Packed(lay, 2, 0, 0, 16, 16, 16, 256, 256 + 16384 + 320)
     # C*kh*kw != K, negative pad, zero stride
-    assert bp.bp_conv2d(P, 256, 2, 7, 8, 8, 1, 1, 1, 1, None, 0, 256, 0) == bp.ERR_INVALID_ARG
-    assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, -1, 1, 1, 1, None, 0, 256, 0) == bp.ERR_INVALID_ARG
-    assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, 1, 1, 0, 1, None, 0, 256, 0) == bp.ERR_INVALID_ARG
+    ws = 1 << 16
+    assert bp.bp_conv2d(P, 256, 2, 7, 8, 8, 1, 1, 1, 1, None, 0, 256, ws, 1 << 20, 0) == \
+        bp.ERR_INVALID_ARG
+    assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, -1, 1, 1, 1, None, 0, 256, ws, 1 << 20, 0) == \
+        bp.ERR_INVALID_ARG
+    assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, 1, 1, 0, 1, None, 0, 256, ws, 1 << 20, 0) == \
+        bp.ERR_INVALID_ARG
+    # the im2col workspace: K x roundup8(Nb*Ho*Wo) 16-bit values = 72 x 128 x 2 bytes
+    assert bp.bp_conv2d_workspace_size(P, 2, 8, 8, 8, 1, 1, 1, 1) == (bp.OK, 72 * 128 * 2)
+    assert bp.bp_conv2d_workspace_size(P, 3, 8, 7, 5, 0, 0, 2, 1) == (bp.OK, 72 * 32 * 2)
+    assert bp.bp_conv2d_workspace_size(P, 2, 7, 8, 8, 1, 1, 1, 1)[0] == bp.ERR_INVALID_ARG
+    # too small, missing or misaligned workspace
+    assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, 1, 1, 1, 1, None, 0, 256, ws, 72 * 128 * 2 - 1, 0) \
+        == bp.ERR_WORKSPACE
+    assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, 1, 1, 1, 1, None, 0, 256, None, 1 << 20, 0) == \
+        bp.ERR_WORKSPACE
+    assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, 1, 1, 1, 1, None, 0, 256, ws + 8, 1 << 20, 0) == \
+        bp.ERR_WORKSPACE

@@ -52,50 +52,100 @@ def test_prune_and_pack_bit_exact(case):
     assert (pw.rb_ptr.cpu().numpy() == rb_ptr).all()
     assert (pw.col_idx.cpu().numpy() == col_idx).all()
     assert (pw.values.cpu().view(torch.int16).numpy().view(np.uint16) == values).all()
-    _check_device_image(pw, rb_ptr, col_idx, values, M, bm)
+    _check_device_image(pw, ref_mask.astype(bool), W, M, K)
 
 
 def _sw128(row, k):
     return (row >> 3) * 1024 + (row & 7) * 128 + (((k >> 3) ^ (row & 7)) << 4) + (k & 7) * 2
 
 
-def _check_device_image(pw, rb_ptr, col_idx, values, M, bm):
-    """Decode the tiled image on the host: weights and padded column lists."""
-    if bm % 128 == 0:
-        rows_pad = bm
-    elif bm <= 256:
-        rows_pad = (bm + 15) // 16 * 16
-    else:
-        return
+def _plan(l):
+    """Expected load plan of a chunk list: tile loads of 8 << lg rows for runs of
+    8-position groups whose live entries are consecutive columns (a group with
+    no live entry, padding, continues any run)."""
+    w = np.zeros(16, np.int32)
+    live = np.concatenate([[True], l[1:] != l[:-1]])
+    first = l[::8]
+    for g in range(8):
+        for i in range(1, 8):
+            q = 8 * g + i
+            if live[q] and l[q] != first[g] + i:
+                return w
+    boxes, g = [], 0
+    while g < 8:
+        run = 1
+        while g + run < 8 and (first[g + run] == first[g] + 8 * run or not live[8 * (g + run)]):
+            run += 1
+        lg = 3 if run >= 8 else 2 if run >= 4 else 1 if run >= 2 else 0
+        boxes.append((int(first[g]), g | (lg << 4)))
+        g += 1 << lg
+    w[0] = len(boxes)
+    desc = 0
+    for b, (y, d) in enumerate(boxes):
+        w[1 + b] = y
+        desc |= d << (8 * b)
+    w[9:11] = np.array([desc & 0xffffffff, desc >> 32], np.uint32).view(np.int32)
+    # the loads cover the 64 list positions in order, and every live entry is
+    # its load's first column plus its offset
+    pos = 0
+    for b, (y, d) in enumerate(boxes):
+        assert (d & 7) == pos // 8
+        rows = 8 << (d >> 4)
+        seg = slice(pos, pos + rows)
+        assert (l[seg][live[seg]] == (y + np.arange(rows))[live[seg]]).all()
+        pos += rows
+    assert pos == 64
+    return w
+
+
+def _check_device_image(pw, mask, W, M, K):
+    """Decode the device image on the host, from the mask and weights alone:
+    per 128-row slab, aligned 64-column blocks whose union of kept columns has
+    at least 48 entries are listed whole, the other union columns follow in
+    ascending order 64 per chunk (a partial last chunk repeats its last index);
+    each chunk's 128 x 64 weight tile is K-major 128-byte swizzled and holds
+    W where the row keeps the column (first occurrence of an index only)."""
     img = pw.dev.cpu().numpy()
-    RB = len(rb_ptr) - 1
-    kc_ptr = img[:8 * (RB + 1)].view(np.int64)
-    off = (8 * (RB + 1) + 255) // 256 * 256
-    tile_bytes = rows_pad * 128
-    chunk = tile_bytes + 256
-    assert img.size == off + kc_ptr[-1] * chunk
-    rows = np.arange(rows_pad)[:, None]
-    ks = np.arange(64)[None, :]
-    offs = _sw128(rows, ks)
-    for rb in range(RB):
-        kp = rb_ptr[rb + 1] - rb_ptr[rb]
-        nkc = kc_ptr[rb + 1] - kc_ptr[rb]
-        assert nkc == -(-kp // 64)
-        r_rb = min(bm, M - rb * bm)
-        vals = values[bm * rb_ptr[rb]: bm * rb_ptr[rb] + r_rb * kp].reshape(r_rb, kp)
-        for kc in range(nkc):
-            base = off + (kc_ptr[rb] + kc) * chunk
-            t = img[base:base + tile_bytes]
-            dec = t.view(np.uint16)[offs // 2]
-            want = np.zeros((rows_pad, 64), np.uint16)
-            seg = vals[:, kc * 64: (kc + 1) * 64]
-            want[:r_rb, :seg.shape[1]] = seg
-            assert (dec == want).all(), (rb, kc)
-            cl = img[base + tile_bytes: base + chunk].view(np.int32)
-            s = col_idx[rb_ptr[rb] + kc * 64: min(rb_ptr[rb] + (kc + 1) * 64, rb_ptr[rb + 1])]
-            wl = np.full(64, col_idx[rb_ptr[rb + 1] - 1], np.int32)   # padding: last kept column
-            wl[:s.size] = s
-            assert (cl == wl).all(), (rb, kc)
+    S = -(-M // 128)
+    kc_ptr = img[:8 * (S + 1)].view(np.int64)
+    off = (8 * (S + 1) + 255) // 256 * 256
+    tile_bytes = 128 * 128
+    C = int(kc_ptr[-1])
+    meta_off = off + C * tile_bytes
+    assert kc_ptr[0] == 0
+    assert img.size == meta_off + C * 320
+    offs = _sw128(np.arange(128)[:, None], np.arange(64)[None, :])
+    for s in range(S):
+        r0, r1 = 128 * s, min(128 * s + 128, M)
+        union = mask[r0:r1].any(axis=0)
+        lists = []
+        for k0 in range(0, K, 64):
+            if k0 + 64 <= K and union[k0:k0 + 64].sum() >= 48:
+                lists.append(np.arange(k0, k0 + 64, dtype=np.int32))
+        dense = np.zeros(K, bool)
+        for l in lists:
+            dense[l] = True
+        rest = np.flatnonzero(union & ~dense).astype(np.int32)
+        for c in range(0, rest.size, 64):
+            l = np.full(64, rest[min(c + 63, rest.size - 1)], np.int32)
+            seg = rest[c:c + 64]
+            l[:seg.size] = seg
+            lists.append(l)
+        assert kc_ptr[s + 1] - kc_ptr[s] == len(lists), s
+        for i, l in enumerate(lists):
+            c = int(kc_ptr[s]) + i
+            base = off + c * tile_bytes
+            rec = meta_off + c * 320
+            assert (img[rec: rec + 256].view(np.int32) == l).all(), (s, i)
+            plan = img[rec + 256: rec + 320].view(np.int32)
+            assert (plan == _plan(l)).all(), (s, i, plan[:11], _plan(l)[:11])
+            live = np.concatenate([[True], l[1:] != l[:-1]])
+            want = np.zeros((128, 64), np.uint16)
+            rows = np.arange(r0, r1)
+            keep = mask[rows][:, l] & live[None, :]
+            want[:r1 - r0] = np.where(keep, W[rows][:, l], 0)
+            dec = img[base:base + tile_bytes].view(np.uint16)[offs // 2]
+            assert (dec == want).all(), (s, i)
 
 
 def test_prune_ties_resolved_like_oracle():
