@@ -167,7 +167,9 @@ bp_status bp_gemm(const bp_packed *P, const void *X, int64_t N, int64_t ldx, con
  *         (16-B aligned): the input expanded to the K x (Nb*Ho*Wo) matrix
  *         (im2col), which the block-sparse product then reads.
  * Requires C*kh*kw == lay.K; dilation and groups are not supported.  The
- * input must be finite (see bp_gemm). */
+ * input must be finite (see bp_gemm).  BP_ERR_UNSUPPORTED when kh input
+ * rows padded to W + 2 pad_w exceed 12288 values, when Wo > 4096, Nb > 65535
+ * or Nb*Ho*Wo >= 2^31. */
 bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, int64_t H,
                     int64_t W, int pad_h, int pad_w, int stride_h, int stride_w,
                     const float *bias, int relu, void *out, void *ws, size_t ws_bytes,

@@ -357,6 +357,10 @@ static bp_status conv_shape(const bp_packed *P, int64_t Nb, int64_t C, int64_t H
     if (C * l.kh * l.kw != l.K) return BP_ERR_INVALID_ARG;
     if (H + 2 * pad_h < l.kh || W + 2 * pad_w < l.kw) return BP_ERR_INVALID_ARG;
     if (H > (1 << 28) || W > (1 << 28)) return BP_ERR_UNSUPPORTED;
+
+    // 32-bit pixel indexing in the im2col pass
+    const int64_t Ho = (H + 2 * pad_h - l.kh) / stride_h + 1, Wo = (W + 2 * pad_w - l.kw) / stride_w + 1;
+    if (Nb * Ho * Wo > INT32_MAX - 8 || Nb * C * H * W > ((int64_t)1 << 40)) return BP_ERR_UNSUPPORTED;
     cs->Nb = Nb;
     cs->C = C;
     cs->H = H;
@@ -369,6 +373,9 @@ static bp_status conv_shape(const bp_packed *P, int64_t Nb, int64_t C, int64_t H
     cs->pw = pad_w;
     cs->sh = stride_h;
     cs->sw = stride_w;
+    // the im2col pass stages kh padded input rows in 24 KB of shared memory
+    if (im2col_row_width(*cs) * l.kh > 12288 || cs->Wo > 4096 || Nb > 65535)
+        return BP_ERR_UNSUPPORTED;
     return BP_OK;
 }
 

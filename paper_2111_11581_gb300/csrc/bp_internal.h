@@ -97,6 +97,7 @@ struct ConvShape {
 // k = c*kh*kw + i*kw + j, n = b*Ho*Wo + oh*Wo + ow, zero outside the image.
 cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void *xcol,
                           cudaStream_t s);
+int64_t im2col_row_width(const ConvShape &cs);   // staged input row length (elements)
 // The block-sparse product on the tensor cores: Y = act(W_packed X + bias).
 // conv == nullptr: Y is M x N row-major (ldy).  Otherwise Y is the NCHW output
 // of the convolution and X its im2col matrix.

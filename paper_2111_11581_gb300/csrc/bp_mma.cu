@@ -521,24 +521,37 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             }
             const int64_t n = t.n0 + c0;
             if (p.conv) {
-                // NCHW output: pixel n = b*HoWo + hw is element (b, m, hw)
-                if (!vrow) continue;
-                int64_t bb = n / p.HoWo, hw = n - bb * p.HoWo;
-                if (hw + 32 <= p.HoWo && (p.HoWo & 7) == 0) {
-                    // hw is a multiple of 8 here, so the row segment is 16-byte aligned
-                    uint4 *d4 = reinterpret_cast<uint4 *>(p.Y + (bb * p.M + m) * p.HoWo + hw);
+                // NCHW output, pixel n = b*HoWo + hw is element (b, m, hw): stage the
+                // 32 x 32 box (lane = channel row, 80-byte rows), then write it with
+                // lanes along the pixels, one coalesced 64-byte store per channel
+                if ((p.HoWo & 7) == 0 && (n % p.HoWo) + 32 <= p.HoWo && n + 32 <= p.N) {
+                    // the 32 pixels are consecutive in one image, 16-byte aligned:
+                    // each lane stores its channel's 64-byte row segment directly
+                    if (vrow) {
+                        const int64_t bb = n / p.HoWo, hw = n - bb * p.HoWo;
+                        uint4 *d4 = reinterpret_cast<uint4 *>(p.Y + (bb * p.M + m) * p.HoWo + hw);
 #pragma unroll
-                    for (int ch = 0; ch < 4; ++ch)
-                        d4[ch] = make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2],
-                                            pk[4 * ch + 3]);
-                } else {
-                    for (int e = 0; e < 32 && n + e < p.N; ++e) {
-                        p.Y[(bb * p.M + m) * p.HoWo + hw] = (uint16_t)(pk[e >> 1] >> ((e & 1) * 16));
-                        if (++hw == p.HoWo) {
-                            hw = 0;
-                            ++bb;
-                        }
+                        for (int ch = 0; ch < 4; ++ch)
+                            d4[ch] = make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2],
+                                                pk[4 * ch + 3]);
                     }
+                    continue;
+                }
+                uint8_t *box = s.ystage + (warp - kEpiWarp0) * 4096;
+                __syncwarp();                      // the previous box has been read
+#pragma unroll
+                for (int ch = 0; ch < 4; ++ch)
+                    st_shared_v4(smem_u32(box + lane * 80 + ch * 16),
+                                 make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]));
+                __syncwarp();
+                const int64_t nn = n + lane;
+                const int rmax = (int)min((int64_t)32, t.rows - row0);
+                if (nn < p.N && rmax > 0) {
+                    const uint32_t bb = (uint32_t)nn / (uint32_t)p.HoWo;
+                    const uint32_t hw = (uint32_t)nn - bb * (uint32_t)p.HoWo;
+                    uint16_t *dst = p.Y + ((int64_t)bb * p.M + t.slab * kSlab + row0) * p.HoWo + hw;
+                    const uint16_t *src = reinterpret_cast<const uint16_t *>(box) + lane;
+                    for (int r = 0; r < rmax; ++r) dst[r * p.HoWo] = src[r * 40];
                 }
                 continue;
             }
@@ -683,7 +696,7 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     p.xboxes = (p.nt + 63) / 64;
     p.num_items = (N + p.nt - 1) / p.nt * p.num_slabs;
     if (p.num_items == 0) return cudaSuccess;
-    p.ystage_bytes = conv ? 0 : 4 * 2 * 2048;
+    p.ystage_bytes = 4 * 4096;     // per epilogue warp: two 2 KB boxes (GEMM) or one (conv)
     // shared memory: stages, output staging, barriers, index ring, and a copy of
     // kc_ptr when that costs no pipeline stage
     auto stages_for = [&](int64_t kc) {

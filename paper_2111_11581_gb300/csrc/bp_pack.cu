@@ -270,46 +270,178 @@ __global__ void plans_kernel(int64_t kc_total, uint8_t *__restrict__ meta_all) {
     }
 }
 
-// im2col: one thread per 8 consecutive columns n of one row k.
-__global__ void im2col_kernel(ConvShape cs, int64_t ldx, const uint16_t *__restrict__ in,
-                              uint16_t *__restrict__ xcol) {
-    const int64_t K = cs.C * cs.kh * cs.kw;
-    const int64_t N = cs.Nb * cs.Ho * cs.Wo;
-    const int64_t HoWo = cs.Ho * cs.Wo;
-    const int64_t units_per_row = (N + 7) / 8;
-    for (int64_t u = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; u < K * units_per_row;
-         u += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t k = u / units_per_row, n0 = (u % units_per_row) * 8;
-        const int64_t c = k / (cs.kh * cs.kw);
-        const int rs = (int)(k % (cs.kh * cs.kw));
-        const int i = rs / cs.kw, j = rs % cs.kw;
-        int64_t b = n0 / HoWo, hw = n0 % HoWo;
-        int oh = (int)(hw / cs.Wo), ow = (int)(hw % cs.Wo);
-        uint16_t v[8];
+// im2col of a 1x1, stride-1, unpadded convolution: row c of the im2col
+// matrix is the concatenation over images b of in[b, c, :, :].  One block per
+// (channel, image): a contiguous copy of H*W values, 16 bytes per thread when
+// source and destination are 16-byte aligned.
+__global__ void __launch_bounds__(256) im2col_copy_kernel(int64_t C, int64_t HW, int64_t ldx,
+                                                          const uint16_t *__restrict__ in,
+                                                          uint16_t *__restrict__ xcol) {
+    const int64_t c = blockIdx.x, b = blockIdx.y;
+    const uint16_t *src = in + (b * C + c) * HW;
+    uint16_t *dst = xcol + c * ldx + b * HW;
+    if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15u) == 0) {
+        const int64_t nv = HW / 8;
+        for (int64_t q = threadIdx.x; q < nv; q += blockDim.x)
+            reinterpret_cast<uint4 *>(dst)[q] = __ldg(reinterpret_cast<const uint4 *>(src) + q);
+        for (int64_t e = nv * 8 + threadIdx.x; e < HW; e += blockDim.x) dst[e] = src[e];
+    } else {
+        for (int64_t e = threadIdx.x; e < HW; e += blockDim.x) dst[e] = __ldg(src + e);
+    }
+}
+
+// im2col of a 1x1 convolution with stride or padding: row c of the im2col
+// matrix holds in[b, c, oh*sh - ph, ow*sw - pw] (zero outside) for every output
+// pixel.  One block per (channel, image); warps over output rows, lanes along
+// them (coalesced stores, strided loads).
+__global__ void __launch_bounds__(256) im2col_1x1_kernel(ConvShape cs, int64_t ldx,
+                                                         const uint16_t *__restrict__ in,
+                                                         uint16_t *__restrict__ xcol) {
+    const int H = (int)cs.H, W = (int)cs.W, Ho = (int)cs.Ho, Wo = (int)cs.Wo;
+    const int64_t c = blockIdx.x, b = blockIdx.y;
+    const uint16_t *src = in + (b * cs.C + c) * H * W;
+    uint16_t *dst = xcol + c * ldx + b * Ho * Wo;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+    for (int oh = warp; oh < Ho; oh += nwarps) {
+        const int ih = oh * cs.sh - cs.ph;
+        const bool row_in = (unsigned)ih < (unsigned)H;
+        for (int ow = lane; ow < Wo; ow += 32) {
+            const int iw = ow * cs.sw - cs.pw;
+            dst[oh * Wo + ow] =
+                (row_in && (unsigned)iw < (unsigned)W) ? __ldg(src + ih * W + iw) : (uint16_t)0;
+        }
+    }
+}
+
+// Writes the block's im2col rows from the staged planes: segments of 32*V
+// consecutive pixels of one channel per warp step, V pixels per lane.
+template <int V>
+__device__ __forceinline__ void im2col_emit(const uint16_t *plane, const int32_t *tab,
+                                            uint16_t *out, int64_t ldx, int PB, int ncg,
+                                            int chan_sz, int khw, int kh, int kw, int wp,
+                                            int lane, int warp, int nwarps) {
+    const int segs = (PB + 32 * V - 1) / (32 * V);
+    int cc = 0, sg = warp;
+    while (sg >= segs) { sg -= segs; ++cc; }
+    for (; cc < ncg;) {
+        const int p = (sg * 32 + lane) * V;
+        if (p < PB) {
+            const uint16_t *src[V];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            uint16_t x = 0;
-            if (n0 + e < N) {
-                const int ih = oh * cs.sh + i - cs.ph, iw = ow * cs.sw + j - cs.pw;
-                if ((unsigned)ih < (unsigned)cs.H && (unsigned)iw < (unsigned)cs.W)
-                    x = __ldg(in + ((b * cs.C + c) * cs.H + ih) * cs.W + iw);
-            }
-            v[e] = x;
-            if (++ow == cs.Wo) {
-                ow = 0;
-                if (++oh == cs.Ho) {
-                    oh = 0;
-                    ++b;
+            for (int e = 0; e < V; ++e) src[e] = plane + cc * chan_sz + tab[p + e];
+            uint16_t *dst = out + (int64_t)cc * khw * ldx + p;
+            for (int i = 0; i < kh; ++i) {
+                for (int j = 0; j < kw; ++j, dst += ldx) {
+                    const int o = i * wp + j;
+                    if (V == 1) {
+                        *dst = src[0][o];
+                    } else if (V == 2) {
+                        *reinterpret_cast<uint32_t *>(dst) =
+                            (uint32_t)src[0][o] | ((uint32_t)src[1][o] << 16);
+                    } else {
+                        *reinterpret_cast<uint2 *>(dst) =
+                            make_uint2((uint32_t)src[0][o] | ((uint32_t)src[1][o] << 16),
+                                       (uint32_t)src[2][o] | ((uint32_t)src[3][o] << 16));
+                    }
                 }
             }
         }
-        uint4 pk;
-        pk.x = v[0] | ((uint32_t)v[1] << 16);
-        pk.y = v[2] | ((uint32_t)v[3] << 16);
-        pk.z = v[4] | ((uint32_t)v[5] << 16);
-        pk.w = v[6] | ((uint32_t)v[7] << 16);
-        *reinterpret_cast<uint4 *>(xcol + k * ldx + n0) = pk;
+        sg += nwarps;
+        while (sg >= segs) { sg -= segs; ++cc; }
     }
+}
+
+// im2col, one block per (group of cg channels, group of ig images, band of
+// output rows; ig > 1 only when the band is the whole image).  The band's
+// input rows of each (channel, image) are staged in shared memory with pw zero
+// columns on either side (rows outside the image are zero too), so the window
+// reads need no bounds checks; a table gives each of the block's output pixels
+// (image-major: consecutive columns of the im2col matrix) its window's offset
+// in the staged planes.  Then each warp takes 32 consecutive output pixels of
+// one channel and writes them to the kh*kw rows that channel feeds:
+// conflict-free shared-memory reads, 64-byte coalesced stores, no division
+// per element.  Each input element is read from global memory once per band.
+__global__ void __launch_bounds__(256) im2col_kernel(ConvShape cs, int64_t ldx, int band_rows,
+                                                     int wp, int cg, int ig,
+                                                     const uint16_t *__restrict__ in,
+                                                     uint16_t *__restrict__ xcol) {
+    extern __shared__ __align__(16) uint8_t im2col_smem[];
+    const int C = (int)cs.C, H = (int)cs.H, W = (int)cs.W, Ho = (int)cs.Ho, Wo = (int)cs.Wo;
+    const int c0 = blockIdx.x * cg, b0 = blockIdx.y * ig;
+    const int ncg = min(cg, C - c0), nig = min(ig, (int)cs.Nb - b0);
+    const int oh0 = blockIdx.z * band_rows;
+    const int R = min(Ho, oh0 + band_rows) - oh0;
+    const int ih0 = oh0 * cs.sh - cs.ph;
+    const int rows = (R - 1) * cs.sh + cs.kh;
+    const int P = R * Wo;                      // the band's pixels per (channel, image)
+    const int PB = nig * P;                    // the block's pixels per channel
+    const int plane_sz = rows * wp;            // staged values per (channel, image)
+    int32_t *tab = reinterpret_cast<int32_t *>(im2col_smem);
+    uint16_t *plane = reinterpret_cast<uint16_t *>(im2col_smem + ((4 * ig * P + 15) & ~15));
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+    // stage: the staged rows (channel, image, row) are spread over the warps,
+    // `lpr` lanes per row (a power of two, 32 for rows longer than 32 values),
+    // so short rows still keep every lane busy; each lane walks its rows with
+    // increments only and keeps 4 loads in flight
+    {
+        int lpr = 32;
+        while (lpr > 1 && lpr / 2 >= wp) lpr >>= 1;
+        const int rpw = 32 / lpr;                       // rows per warp step
+        const int lr = lane / lpr, lx = lane - lr * lpr;
+        const int step = nwarps * rpw;                  // rows per block step
+        const int total = ncg * nig * rows;
+        int first = warp * rpw + lr;
+        // (cc, bb, r) of row index `first`, by division once
+        int r = first % rows, ci = first / rows;
+        int bb = ci % nig, cc = ci / nig;
+        const int dr = step % rows, dci = step / rows;
+        for (int row = first; row < total;) {
+            int rr[4], rb[4], rc[4];
+            bool ok[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                ok[q] = row < total;
+                rr[q] = r; rb[q] = bb; rc[q] = cc;
+                row += step;
+                r += dr;
+                int carry = dci;
+                if (r >= rows) { r -= rows; ++carry; }
+                bb += carry;
+                while (bb >= nig) { bb -= nig; ++cc; }
+            }
+            for (int x0 = lx; x0 < wp; x0 += lpr) {
+                uint16_t v[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int ih = ih0 + rr[q], iw = x0 - cs.pw;
+                    v[q] = (ok[q] && (unsigned)ih < (unsigned)H && (unsigned)iw < (unsigned)W)
+                               ? __ldg(in + (((int64_t)(b0 + rb[q]) * C + c0 + rc[q]) * H + ih) * W + iw)
+                               : (uint16_t)0;
+                }
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    if (ok[q]) plane[(rc[q] * ig + rb[q]) * plane_sz + rr[q] * wp + x0] = v[q];
+            }
+        }
+    }
+    // pixel table: warps over (image, output row), lanes along the row
+    for (int br = warp; br < nig * R; br += nwarps) {
+        const int bb = br / R, orow = br - bb * R;
+        const int base = bb * plane_sz + orow * cs.sh * wp;
+        for (int ow = lane; ow < Wo; ow += 32) tab[bb * P + orow * Wo + ow] = base + ow * cs.sw;
+    }
+    __syncthreads();
+    const int khw = cs.kh * cs.kw;
+    uint16_t *out = xcol + (int64_t)c0 * khw * ldx + (int64_t)b0 * Ho * Wo + (int64_t)oh0 * Wo;
+    const int64_t nbase = (int64_t)b0 * Ho * Wo + (int64_t)oh0 * Wo;
+    // V consecutive pixels per lane (one 2V-byte store per window offset) when
+    // the block's pixels start 2V-byte aligned in the im2col row
+    if (nbase % 4 == 0 && PB % 4 == 0 && ldx % 4 == 0)
+        im2col_emit<4>(plane, tab, out, ldx, PB, ncg, ig * plane_sz, khw, cs.kh, cs.kw, wp, lane, warp, nwarps);
+    else if (nbase % 2 == 0 && PB % 2 == 0)
+        im2col_emit<2>(plane, tab, out, ldx, PB, ncg, ig * plane_sz, khw, cs.kh, cs.kw, wp, lane, warp, nwarps);
+    else
+        im2col_emit<1>(plane, tab, out, ldx, PB, ncg, ig * plane_sz, khw, cs.kh, cs.kw, wp, lane, warp, nwarps);
 }
 
 }  // namespace
@@ -364,14 +496,59 @@ cudaError_t launch_pack(const bp_layout &lay, const void *W, const uint8_t *mask
     return cudaGetLastError();
 }
 
+int64_t im2col_row_width(const ConvShape &cs) {
+    // staged row: pw zeros, W values, pw zeros (window reads stay inside:
+    // (Wo - 1) * sw + kw - 1 <= W + 2 pw - 1)
+    return cs.W + 2 * cs.pw;
+}
+
 cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void *xcol,
                           cudaStream_t s) {
-    const int64_t K = cs.C * cs.kh * cs.kw, N = cs.Nb * cs.Ho * cs.Wo;
-    const int64_t units = K * ((N + 7) / 8);
-    int64_t blocks = (units + 255) / 256;
-    if (blocks > 152 * 64) blocks = 152 * 64;
-    im2col_kernel<<<(unsigned)blocks, 256, 0, s>>>(cs, ldx, static_cast<const uint16_t *>(in),
-                                                   static_cast<uint16_t *>(xcol));
+    if (cs.kh == 1 && cs.kw == 1 && cs.sh == 1 && cs.sw == 1 && cs.ph == 0 && cs.pw == 0) {
+        if (cs.C > 0x7fffffffLL || cs.Nb > 65535) return cudaErrorInvalidValue;
+        im2col_copy_kernel<<<dim3((unsigned)cs.C, (unsigned)cs.Nb), 256, 0, s>>>(
+            cs.C, cs.H * cs.W, ldx, static_cast<const uint16_t *>(in),
+            static_cast<uint16_t *>(xcol));
+        return cudaGetLastError();
+    }
+    if (cs.kh == 1 && cs.kw == 1) {
+        if (cs.C > 0x7fffffffLL || cs.Nb > 65535) return cudaErrorInvalidValue;
+        im2col_1x1_kernel<<<dim3((unsigned)cs.C, (unsigned)cs.Nb), 256, 0, s>>>(
+            cs, ldx, static_cast<const uint16_t *>(in), static_cast<uint16_t *>(xcol));
+        return cudaGetLastError();
+    }
+    constexpr int64_t kStage = 24 * 1024 / 2;     // staged values per block at most
+    constexpr int64_t kTab = 4096;                 // table entries (output pixels) per block at most
+    const int64_t wp = im2col_row_width(cs);
+    // output rows per block (the band): as many as fit, at least one
+    const int64_t max_rows = kStage / wp;
+    if (max_rows < cs.kh) return cudaErrorInvalidValue;
+    int64_t band = (max_rows - cs.kh) / cs.sh + 1;
+    if (band > cs.Ho) band = cs.Ho;
+    if (band * cs.Wo > kTab) band = kTab / cs.Wo > 0 ? kTab / cs.Wo : 1;
+    const int64_t rows = (band - 1) * cs.sh + cs.kh;
+    const int64_t nbands = (cs.Ho + band - 1) / band;
+    const int64_t pix = band * cs.Wo;
+    // images per block (whole images only): at least about 512 pixels per channel
+    int64_t ig = 1;
+    if (band == cs.Ho) {
+        ig = (512 + pix - 1) / pix;
+        if (ig > cs.Nb) ig = cs.Nb;
+        if (ig > kTab / pix) ig = kTab / pix;
+        if (ig > kStage / (rows * wp)) ig = kStage / (rows * wp);
+        if (ig < 1) ig = 1;
+    }
+    // channels per block: about 2048 output pixels, within the stage
+    int64_t cg = (2048 + ig * pix - 1) / (ig * pix);
+    if (cg > kStage / (ig * rows * wp)) cg = kStage / (ig * rows * wp);
+    if (cg > cs.C) cg = cs.C;
+    if (cg < 1) cg = 1;
+    const int64_t gx = (cs.C + cg - 1) / cg, gy = (cs.Nb + ig - 1) / ig;
+    if (gx > 0x7fffffffLL || gy > 65535 || nbands > 65535) return cudaErrorInvalidValue;
+    const size_t smem = (size_t)((4 * ig * pix + 15) & ~15) + (size_t)(cg * ig * rows * wp * 2);
+    im2col_kernel<<<dim3((unsigned)gx, (unsigned)gy, (unsigned)nbands), 256, smem, s>>>(
+        cs, ldx, (int)band, (int)wp, (int)cg, (int)ig, static_cast<const uint16_t *>(in),
+        static_cast<uint16_t *>(xcol));
     return cudaGetLastError();
 }
 
