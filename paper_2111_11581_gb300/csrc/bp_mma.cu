@@ -500,16 +500,11 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
         const bool vrow = row0 + lane < t.rows;
         const int64_t m = t.slab * kSlab + row0 + lane;
         const float bv = (p.bias && vrow) ? p.bias[m] : 0.f;
-        for (int c0 = 0; c0 < p.nt && t.n0 + c0 < p.N; c0 += 32) {
-            uint32_t r[32];
-            if (has) {
-                tmem_ld_32x32b_x32(tacc + c0, r);
-                tmem_ld_wait();
-            } else {
-#pragma unroll
-                for (int e = 0; e < 32; ++e) r[e] = 0u;
-            }
-            uint32_t pk[16];
+        // Column groups of 32: once group g's accumulators are converted (pk),
+        // the tensor-memory load of group g + 1 is issued into the same
+        // registers and runs while group g is stored.
+        // A warp whose 32 rows are all past the slab's real rows has nothing to write.
+        auto pack = [&](const uint32_t (&r)[32], uint32_t (&pk)[16]) {
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
                 float a = __uint_as_float(r[2 * e]) + bv, b = __uint_as_float(r[2 * e + 1]) + bv;
@@ -519,6 +514,8 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                 }
                 pk[e] = pack2(a, b, p.dtype);
             }
+        };
+        auto store = [&](const uint32_t (&pk)[16], int c0) {
             const int64_t n = t.n0 + c0;
             if (p.conv) {
                 // NCHW output, pixel n = b*HoWo + hw is element (b, m, hw): stage the
@@ -535,7 +532,7 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                             d4[ch] = make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2],
                                                 pk[4 * ch + 3]);
                     }
-                    continue;
+                    return;
                 }
                 uint8_t *box = s.ystage + (warp - kEpiWarp0) * 4096;
                 __syncwarp();                      // the previous box has been read
@@ -553,7 +550,7 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                     const uint16_t *src = reinterpret_cast<const uint16_t *>(box) + lane;
                     for (int r = 0; r < rmax; ++r) dst[r * p.HoWo] = src[r * 40];
                 }
-                continue;
+                return;
             }
             // GEMM: 32 x 32 box staged in shared memory (64-byte swizzle: 16-byte
             // chunk c of row r sits at chunk c ^ ((r >> 1) & 3)), then TMA-stored;
@@ -570,6 +567,24 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             if (lane == 0) {
                 tma_store_2d(&p.ymap, sb, (int32_t)n, (int32_t)(t.slab * kSlab + row0));
                 bulk_commit();
+            }
+                };
+        if (row0 < t.rows) {
+            const int64_t cols = min((int64_t)p.nt, p.N - t.n0);
+            const int G = (int)((cols + 31) / 32);
+            uint32_t r[32], pk[16];
+            if (has) {
+                tmem_ld_32x32b_x32(tacc, r);
+                tmem_ld_wait();
+            } else {
+#pragma unroll
+                for (int e = 0; e < 32; ++e) r[e] = 0u;
+            }
+            for (int g = 0; g < G; ++g) {
+                pack(r, pk);
+                if (has && g + 1 < G) tmem_ld_32x32b_x32(tacc + 32 * (g + 1), r);
+                store(pk, 32 * g);
+                if (has && g + 1 < G) tmem_ld_wait();
             }
         }
         if (has) {
