@@ -127,20 +127,28 @@ bool checked_mode() {
     return e && e[0] == '1';
 }
 
+static int64_t qmap_bytes(const bp_layout &lay) { return align_up(4 * lay.K, 16); }
+
+static void set_chunks(DevLayout &d, const bp_layout &lay, int64_t kc) {
+    d.kc_total = kc;
+    d.off_meta = d.off_tiles + kc * d.tile_bytes;
+    d.off_meta2 = d.off_meta + kc * kMetaBytes;
+    d.off_qmap = d.off_meta2 + kc * kMetaBytes;
+    d.bytes = d.off_qmap + qmap_bytes(lay);
+}
+
 DevLayout dev_layout(const bp_layout &lay, const int64_t *slab_chunks_host) {
     DevLayout d{};
     d.num_slabs = cdiv(lay.M, kSlab);
-    d.off_tiles = align_up(8 * (d.num_slabs + 1), 256);
+    d.off_tiles = align_up(8 * (d.num_slabs + 2), 256);
     d.tile_bytes = (int64_t)kSlab * kBK * 2;
     d.kc_total = -1;
-    d.off_meta = -1;
+    d.off_meta = d.off_meta2 = d.off_qmap = -1;
     d.bytes = -1;
     if (slab_chunks_host) {
         int64_t kc = 0;
         for (int64_t s = 0; s < d.num_slabs; ++s) kc += slab_chunks_host[s];
-        d.kc_total = kc;
-        d.off_meta = d.off_tiles + kc * d.tile_bytes;
-        d.bytes = d.off_meta + kc * kMetaBytes;
+        set_chunks(d, lay, kc);
     }
     return d;
 }
@@ -305,9 +313,9 @@ bp_status bp_pack(const bp_layout *lay, const void *W, const uint8_t *mask, bp_p
     if (out->dev_bytes != dl.bytes) return BP_ERR_INVALID_ARG;
     if (!out->dev || !aligned16(out->dev)) return BP_ERR_INVALID_ARG;
     out->lay = *lay;
-    std::vector<int64_t> kc(dl.num_slabs + 1, 0);
+    std::vector<int64_t> kc(dl.num_slabs + 2, 0);
     for (int64_t i = 0; i < dl.num_slabs; ++i) kc[i + 1] = kc[i] + sc[i];
-    e = cudaMemcpyAsync(out->dev, kc.data(), 8 * (dl.num_slabs + 1), cudaMemcpyHostToDevice, s);
+    e = cudaMemcpyAsync(out->dev, kc.data(), 8 * (dl.num_slabs + 2), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = launch_pack(*lay, W, mask, *out, dl, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     return cuda_status(e);
@@ -318,12 +326,10 @@ static bp_status check_packed(const bp_packed *P, DevLayout *dl) {
     if (P->num_rb != cdiv(P->lay.M, P->lay.bm)) return BP_ERR_INVALID_ARG;
     if (cdiv(P->lay.M, kSlab) > kMaxSlabs) return BP_ERR_UNSUPPORTED;
     *dl = dev_layout(P->lay, nullptr);
-    // the chunk count follows from the image size: tiles + list/plan records
-    const int64_t rest = P->dev_bytes - dl->off_tiles, per = dl->tile_bytes + kMetaBytes;
-    if (rest < 0 || rest % per) return BP_ERR_INVALID_ARG;
-    dl->kc_total = rest / per;
-    dl->off_meta = dl->off_tiles + dl->kc_total * dl->tile_bytes;
-    dl->bytes = P->dev_bytes;
+    // the chunk count follows from the image size: tiles + two record sets + qmap
+    const int64_t rest = P->dev_bytes - dl->off_tiles - qmap_bytes(P->lay);
+    if (rest < 0 || rest % kChunkBytes) return BP_ERR_INVALID_ARG;
+    set_chunks(*dl, P->lay, rest / kChunkBytes);
     return BP_OK;
 }
 
@@ -408,7 +414,9 @@ bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, i
     const int64_t ldx = align_up(N, 8);
     if (!ws || !aligned16(ws) || ws_bytes < (size_t)(P->lay.K * ldx * 2)) return BP_ERR_WORKSPACE;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    cudaError_t e = launch_im2col(cs, ldx, in, ws, s);
+    const int32_t *qmap =
+        reinterpret_cast<const int32_t *>(static_cast<const uint8_t *>(P->dev) + dl.off_qmap);
+    cudaError_t e = launch_im2col(cs, ldx, in, ws, qmap, s);
     if (e != cudaSuccess) return BP_ERR_CUDA;
     return finish_launch(launch_mma(*P, dl, ws, N, ldx, bias, relu, out, 0, &cs, s), s);
 }

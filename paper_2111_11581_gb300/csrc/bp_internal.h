@@ -32,6 +32,7 @@ constexpr int kMaxBoxes = 8;         // tile loads in a chunk's plan at most
 // where a row prunes them); the other union columns follow in ascending
 // order, 64 per k-chunk.  All offsets in bytes, C = total k-chunks:
 //   [0, 8*(S+1))                 int64 kc_ptr: first k-chunk of each slab
+//   [8*(S+1), 8*(S+2))           int64 Kc: number of columns any slab lists
 //   off_tiles + c*16384          k-chunk c's 128 x 64 16-bit weight tile in
 //                                K-major 128-byte-swizzled order
 //   off_meta + c*kMetaBytes      k-chunk c's record:
@@ -47,14 +48,25 @@ constexpr int kMaxBoxes = 8;         // tile loads in a chunk's plan at most
 //                                and each live entry of a load's range is its
 //                                first column plus its offset (repeats read
 //                                other rows, against zero weights).
+//   off_meta2 + c*kMetaBytes     the same record in compacted coordinates: list
+//                                entries replaced by their rank among the Kc
+//                                listed columns (qmap), plan built from those,
+//                                with no load reaching past row Kc - 1.  A
+//                                convolution writes only the Kc listed rows of
+//                                its im2col matrix, in that order.
+//   off_qmap + 4*k               int32 qmap[k]: rank of column k among the
+//                                listed columns, -1 if no slab lists it.
 struct DevLayout {
     int64_t num_slabs;
     int64_t kc_total;     // total k-chunks (-1 if unknown)
     int64_t off_tiles;
-    int64_t off_meta;     // (when kc_total is known)
+    int64_t off_meta;     // (this and the following when kc_total is known)
+    int64_t off_meta2;
+    int64_t off_qmap;
     int64_t tile_bytes;   // 128 * 64 * 2
     int64_t bytes;        // total image size (when kc_total is known)
 };
+constexpr int64_t kChunkBytes = 128 * kBK * 2 + 2 * kMetaBytes;   // per k-chunk, all parts
 
 // Image layout; slab_chunks_host = per-slab chunk counts (host) or nullptr.
 DevLayout dev_layout(const bp_layout &lay, const int64_t *slab_chunks_host);
@@ -95,12 +107,15 @@ struct ConvShape {
 };
 // im2col of an NCHW input: Xcol[k][n] (K x N row-major, leading dimension ldx),
 // k = c*kh*kw + i*kw + j, n = b*Ho*Wo + oh*Wo + ow, zero outside the image.
+// qmap: for row k of the full im2col matrix its row in xcol, or -1 to skip it
+// (nullptr: row k is row k).
 cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void *xcol,
-                          cudaStream_t s);
+                          const int32_t *qmap, cudaStream_t s);
 int64_t im2col_row_width(const ConvShape &cs);   // staged input row length (elements)
 // The block-sparse product on the tensor cores: Y = act(W_packed X + bias).
 // conv == nullptr: Y is M x N row-major (ldy).  Otherwise Y is the NCHW output
 // of the convolution and X its im2col matrix.
+// With conv, X holds only the listed rows (see DevLayout::off_meta2).
 cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, int64_t N,
                        int64_t ldx, const float *bias, int relu, void *Y, int64_t ldy,
                        const ConvShape *conv, cudaStream_t s);

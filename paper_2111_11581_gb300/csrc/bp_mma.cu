@@ -727,7 +727,8 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     p.tmem_cols = 2 * kNT;
     p.kc_ptr = reinterpret_cast<const int64_t *>(dev);
     p.tiles = dev + dl.off_tiles;
-    p.meta = dev + dl.off_meta;
+    // a convolution's X holds only the listed rows: use the compacted records
+    p.meta = dev + (conv ? dl.off_meta2 : dl.off_meta);
     p.X = static_cast<const uint16_t *>(X);
     p.ldx = ldx;
     p.Y = static_cast<uint16_t *>(Y);

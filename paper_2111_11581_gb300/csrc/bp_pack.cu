@@ -231,7 +231,10 @@ __global__ void tiles_kernel(int64_t M, int64_t K, const uint16_t *__restrict__ 
 // previous group's, or no live entry at all: padding, whose rows meet zero
 // weights) become loads of 64, 32, 16 or 8 rows; otherwise the plan is empty
 // and the kernel gathers the chunk's rows one by one.
-__global__ void plans_kernel(int64_t kc_total, uint8_t *__restrict__ meta_all) {
+// bound (device, or nullptr for none): no load may reach row *bound.
+__global__ void plans_kernel(int64_t kc_total, uint8_t *__restrict__ meta_all,
+                             const int64_t *__restrict__ bound) {
+    const int64_t lim = bound ? *bound : INT64_MAX;
     for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < kc_total;
          c += (int64_t)gridDim.x * blockDim.x) {
         uint8_t *meta = meta_all + c * kMetaBytes;
@@ -256,11 +259,16 @@ __global__ void plans_kernel(int64_t kc_total, uint8_t *__restrict__ meta_all) {
                                        l[8 * (g + run)] == l[8 * (g + run) - 1]))
                     ++run;
                 const int lg = run >= 8 ? 3 : run >= 4 ? 2 : run >= 2 ? 1 : 0;
+                if ((int64_t)first[g] + (8 << lg) > lim) {
+                    nb = 0;
+                    break;
+                }
                 w[1 + nb] = first[g];
                 desc[nb >> 2] |= (uint32_t)(g | (lg << 4)) << (8 * (nb & 3));
                 ++nb;
                 g += 1 << lg;
             }
+            if (nb == 0) desc[0] = desc[1] = 0u, w[1] = w[2] = w[3] = w[4] = w[5] = w[6] = w[7] = w[8] = 0;
             w[0] = nb;
             w[9] = (int32_t)desc[0];
             w[10] = (int32_t)desc[1];
@@ -270,16 +278,70 @@ __global__ void plans_kernel(int64_t kc_total, uint8_t *__restrict__ meta_all) {
     }
 }
 
+// Columns listed by any slab: qmap[k] = 1 for every list entry (qmap zeroed
+// first; equal values, so the racing writes agree).
+__global__ void mark_listed_kernel(int64_t entries, const uint8_t *__restrict__ meta,
+                                   int32_t *__restrict__ qmap) {
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < entries;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int32_t k = reinterpret_cast<const int32_t *>(meta + (e / kBK) * kMetaBytes)[e % kBK];
+        qmap[k] = 1;
+    }
+}
+
+// One block: marks -> ranks (exclusive scan in column order), -1 where
+// unmarked; *kc_out = number of listed columns.
+__global__ void __launch_bounds__(1024) qmap_scan_kernel(int64_t K, int32_t *__restrict__ qmap,
+                                                         int64_t *__restrict__ kc_out) {
+    __shared__ int32_t warp_sum[32];
+    __shared__ int32_t carry;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (threadIdx.x == 0) carry = 0;
+    __syncthreads();
+    for (int64_t k0 = 0; k0 < K; k0 += blockDim.x) {
+        const int64_t k = k0 + threadIdx.x;
+        const int32_t f = k < K ? qmap[k] : 0;
+        const unsigned bal = __ballot_sync(0xffffffffu, f != 0);
+        const int within = __popc(bal & ((1u << lane) - 1u));
+        if (lane == 0) warp_sum[warp] = __popc(bal);
+        __syncthreads();
+        int before = 0, total = 0;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+            if (w < warp) before += warp_sum[w];
+            total += warp_sum[w];
+        }
+        if (k < K) qmap[k] = f ? carry + before + within : -1;
+        __syncthreads();
+        if (threadIdx.x == 0) carry += total;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) *kc_out = carry;
+}
+
+// Records in compacted coordinates: each list entry replaced by its rank.
+__global__ void compact_lists_kernel(int64_t entries, const uint8_t *__restrict__ meta,
+                                     uint8_t *__restrict__ meta2, const int32_t *__restrict__ qmap) {
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < entries;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t c = e / kBK, i = e % kBK;
+        const int32_t k = reinterpret_cast<const int32_t *>(meta + c * kMetaBytes)[i];
+        reinterpret_cast<int32_t *>(meta2 + c * kMetaBytes)[i] = qmap[k];
+    }
+}
+
 // im2col of a 1x1, stride-1, unpadded convolution: row c of the im2col
 // matrix is the concatenation over images b of in[b, c, :, :].  One block per
 // (channel, image): a contiguous copy of H*W values, 16 bytes per thread when
 // source and destination are 16-byte aligned.
 __global__ void __launch_bounds__(256) im2col_copy_kernel(int64_t C, int64_t HW, int64_t ldx,
+                                                          const int32_t *__restrict__ qmap,
                                                           const uint16_t *__restrict__ in,
                                                           uint16_t *__restrict__ xcol) {
     const int64_t c = blockIdx.x, b = blockIdx.y;
+    const int64_t q = qmap ? qmap[c] : c;      // the row this channel becomes, or none
+    if (q < 0) return;
     const uint16_t *src = in + (b * C + c) * HW;
-    uint16_t *dst = xcol + c * ldx + b * HW;
+    uint16_t *dst = xcol + q * ldx + b * HW;
     if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15u) == 0) {
         const int64_t nv = HW / 8;
         for (int64_t q = threadIdx.x; q < nv; q += blockDim.x)
@@ -295,12 +357,15 @@ __global__ void __launch_bounds__(256) im2col_copy_kernel(int64_t C, int64_t HW,
 // pixel.  One block per (channel, image); warps over output rows, lanes along
 // them (coalesced stores, strided loads).
 __global__ void __launch_bounds__(256) im2col_1x1_kernel(ConvShape cs, int64_t ldx,
+                                                         const int32_t *__restrict__ qmap,
                                                          const uint16_t *__restrict__ in,
                                                          uint16_t *__restrict__ xcol) {
     const int H = (int)cs.H, W = (int)cs.W, Ho = (int)cs.Ho, Wo = (int)cs.Wo;
     const int64_t c = blockIdx.x, b = blockIdx.y;
+    const int64_t q = qmap ? qmap[c] : c;
+    if (q < 0) return;
     const uint16_t *src = in + (b * cs.C + c) * H * W;
-    uint16_t *dst = xcol + c * ldx + b * Ho * Wo;
+    uint16_t *dst = xcol + q * ldx + b * Ho * Wo;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     for (int oh = warp; oh < Ho; oh += nwarps) {
         const int ih = oh * cs.sh - cs.ph;
@@ -317,9 +382,9 @@ __global__ void __launch_bounds__(256) im2col_1x1_kernel(ConvShape cs, int64_t l
 // consecutive pixels of one channel per warp step, V pixels per lane.
 template <int V>
 __device__ __forceinline__ void im2col_emit(const uint16_t *plane, const int32_t *tab,
-                                            uint16_t *out, int64_t ldx, int PB, int ncg,
-                                            int chan_sz, int khw, int kh, int kw, int wp,
-                                            int lane, int warp, int nwarps) {
+                                            uint16_t *out, const int32_t *qrows, int64_t ldx,
+                                            int PB, int ncg, int chan_sz, int khw, int kh,
+                                            int kw, int wp, int lane, int warp, int nwarps) {
     const int segs = (PB + 32 * V - 1) / (32 * V);
     int cc = 0, sg = warp;
     while (sg >= segs) { sg -= segs; ++cc; }
@@ -329,9 +394,13 @@ __device__ __forceinline__ void im2col_emit(const uint16_t *plane, const int32_t
             const uint16_t *src[V];
 #pragma unroll
             for (int e = 0; e < V; ++e) src[e] = plane + cc * chan_sz + tab[p + e];
-            uint16_t *dst = out + (int64_t)cc * khw * ldx + p;
             for (int i = 0; i < kh; ++i) {
-                for (int j = 0; j < kw; ++j, dst += ldx) {
+                for (int j = 0; j < kw; ++j) {
+                    // row of the im2col matrix this (channel, i, j) becomes, or none
+                    const int kk = cc * khw + i * kw + j;
+                    const int64_t q = qrows ? (int64_t)__ldg(qrows + kk) : (int64_t)kk;
+                    if (q < 0) continue;
+                    uint16_t *dst = out + q * ldx + p;
                     const int o = i * wp + j;
                     if (V == 1) {
                         *dst = src[0][o];
@@ -363,6 +432,7 @@ __device__ __forceinline__ void im2col_emit(const uint16_t *plane, const int32_t
 // per element.  Each input element is read from global memory once per band.
 __global__ void __launch_bounds__(256) im2col_kernel(ConvShape cs, int64_t ldx, int band_rows,
                                                      int wp, int cg, int ig,
+                                                     const int32_t *__restrict__ qmap,
                                                      const uint16_t *__restrict__ in,
                                                      uint16_t *__restrict__ xcol) {
     extern __shared__ __align__(16) uint8_t im2col_smem[];
@@ -432,16 +502,19 @@ __global__ void __launch_bounds__(256) im2col_kernel(ConvShape cs, int64_t ldx, 
     }
     __syncthreads();
     const int khw = cs.kh * cs.kw;
-    uint16_t *out = xcol + (int64_t)c0 * khw * ldx + (int64_t)b0 * Ho * Wo + (int64_t)oh0 * Wo;
     const int64_t nbase = (int64_t)b0 * Ho * Wo + (int64_t)oh0 * Wo;
+    // rows: qmap[k] for k = c*kh*kw + i*kw + j (from this block's first channel),
+    // or k itself without a map
+    uint16_t *out = xcol + nbase + (qmap ? 0 : (int64_t)c0 * khw * ldx);
+    const int32_t *qrows = qmap ? qmap + (int64_t)c0 * khw : nullptr;
     // V consecutive pixels per lane (one 2V-byte store per window offset) when
     // the block's pixels start 2V-byte aligned in the im2col row
     if (nbase % 4 == 0 && PB % 4 == 0 && ldx % 4 == 0)
-        im2col_emit<4>(plane, tab, out, ldx, PB, ncg, ig * plane_sz, khw, cs.kh, cs.kw, wp, lane, warp, nwarps);
+        im2col_emit<4>(plane, tab, out, qrows, ldx, PB, ncg, ig * plane_sz, khw, cs.kh, cs.kw, wp, lane, warp, nwarps);
     else if (nbase % 2 == 0 && PB % 2 == 0)
-        im2col_emit<2>(plane, tab, out, ldx, PB, ncg, ig * plane_sz, khw, cs.kh, cs.kw, wp, lane, warp, nwarps);
+        im2col_emit<2>(plane, tab, out, qrows, ldx, PB, ncg, ig * plane_sz, khw, cs.kh, cs.kw, wp, lane, warp, nwarps);
     else
-        im2col_emit<1>(plane, tab, out, ldx, PB, ncg, ig * plane_sz, khw, cs.kh, cs.kw, wp, lane, warp, nwarps);
+        im2col_emit<1>(plane, tab, out, qrows, ldx, PB, ncg, ig * plane_sz, khw, cs.kh, cs.kw, wp, lane, warp, nwarps);
 }
 
 }  // namespace
@@ -476,18 +549,34 @@ cudaError_t launch_pack(const bp_layout &lay, const void *W, const uint8_t *mask
                                                static_cast<const uint16_t *>(W), P.rb_ptr,
                                                P.col_idx, static_cast<uint16_t *>(P.values));
     e = cudaGetLastError();
-    if (e != cudaSuccess || dl.kc_total == 0) return e;
+    if (e != cudaSuccess) return e;
     uint8_t *dev = static_cast<uint8_t *>(P.dev);
+    if (dl.kc_total == 0)   // nothing listed: no im2col row is needed
+        return cudaMemsetAsync(dev + dl.off_qmap, 0xff, 4 * lay.K, s);
     const int64_t *kc_ptr = reinterpret_cast<const int64_t *>(dev);
     uint8_t *tiles = dev + dl.off_tiles;
     uint8_t *meta = dev + dl.off_meta;
+    uint8_t *meta2 = dev + dl.off_meta2;
+    int32_t *qmap = reinterpret_cast<int32_t *>(dev + dl.off_qmap);
+    int64_t *kc_hdr = reinterpret_cast<int64_t *>(dev) + dl.num_slabs + 1;
     slab_lists_kernel<<<(unsigned)dl.num_slabs, 32, 0, s>>>(lay.M, lay.K, lay.bm, mask, kc_ptr,
                                                            meta);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
+    const int64_t entries = dl.kc_total * kBK;
+    int64_t eblocks = (entries + 255) / 256;
+    if (eblocks > 4096) eblocks = 4096;
+    e = cudaMemsetAsync(qmap, 0, 4 * lay.K, s);
+    if (e != cudaSuccess) return e;
+    mark_listed_kernel<<<(unsigned)eblocks, 256, 0, s>>>(entries, meta, qmap);
+    qmap_scan_kernel<<<1, 1024, 0, s>>>(lay.K, qmap, kc_hdr);
+    compact_lists_kernel<<<(unsigned)eblocks, 256, 0, s>>>(entries, meta, meta2, qmap);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
     int64_t pblocks = (dl.kc_total + 127) / 128;
     if (pblocks > 1024) pblocks = 1024;
-    plans_kernel<<<(unsigned)pblocks, 128, 0, s>>>(dl.kc_total, meta);
+    plans_kernel<<<(unsigned)pblocks, 128, 0, s>>>(dl.kc_total, meta, nullptr);
+    plans_kernel<<<(unsigned)pblocks, 128, 0, s>>>(dl.kc_total, meta2, kc_hdr);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     dim3 grid(16, (unsigned)dl.num_slabs);
@@ -503,18 +592,18 @@ int64_t im2col_row_width(const ConvShape &cs) {
 }
 
 cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void *xcol,
-                          cudaStream_t s) {
+                          const int32_t *qmap, cudaStream_t s) {
     if (cs.kh == 1 && cs.kw == 1 && cs.sh == 1 && cs.sw == 1 && cs.ph == 0 && cs.pw == 0) {
         if (cs.C > 0x7fffffffLL || cs.Nb > 65535) return cudaErrorInvalidValue;
         im2col_copy_kernel<<<dim3((unsigned)cs.C, (unsigned)cs.Nb), 256, 0, s>>>(
-            cs.C, cs.H * cs.W, ldx, static_cast<const uint16_t *>(in),
+            cs.C, cs.H * cs.W, ldx, qmap, static_cast<const uint16_t *>(in),
             static_cast<uint16_t *>(xcol));
         return cudaGetLastError();
     }
     if (cs.kh == 1 && cs.kw == 1) {
         if (cs.C > 0x7fffffffLL || cs.Nb > 65535) return cudaErrorInvalidValue;
         im2col_1x1_kernel<<<dim3((unsigned)cs.C, (unsigned)cs.Nb), 256, 0, s>>>(
-            cs, ldx, static_cast<const uint16_t *>(in), static_cast<uint16_t *>(xcol));
+            cs, ldx, qmap, static_cast<const uint16_t *>(in), static_cast<uint16_t *>(xcol));
         return cudaGetLastError();
     }
     constexpr int64_t kStage = 24 * 1024 / 2;     // staged values per block at most
@@ -547,7 +636,7 @@ cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void
     if (gx > 0x7fffffffLL || gy > 65535 || nbands > 65535) return cudaErrorInvalidValue;
     const size_t smem = (size_t)((4 * ig * pix + 15) & ~15) + (size_t)(cg * ig * rows * wp * 2);
     im2col_kernel<<<dim3((unsigned)gx, (unsigned)gy, (unsigned)nbands), 256, smem, s>>>(
-        cs, ldx, (int)band, (int)wp, (int)cg, (int)ig, static_cast<const uint16_t *>(in),
+        cs, ldx, (int)band, (int)wp, (int)cg, (int)ig, qmap, static_cast<const uint16_t *>(in),
         static_cast<uint16_t *>(xcol));
     return cudaGetLastError();
 }

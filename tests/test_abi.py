@@ -91,7 +91,7 @@ def test_rate_below_one_rejected_on_host(lib):
 
 def test_gemm_argument_checks_on_host(lib):
     lay = bp.layout(bp.BLOCK_BASED, bp.F16, 64, 64, 16, 16)
-    P = bp.Packed(lay, 4, 0, 0, 16, 16, 16, 256, 256 + 16384 + 320)
+    P = bp.Packed(lay, 4, 0, 0, 16, 16, 16, 256, 256 + 16384 + 640 + 4 * 64)   # kc_ptr, one chunk, qmap
     # ldx not a multiple of 8, misaligned X, N > ldx, null packed
     assert bp.bp_gemm(P, 256, 10, 10, None, 0, 256, 16, 0) == bp.ERR_INVALID_ARG
     assert bp.bp_gemm(P, 258, 8, 8, None, 0, 256, 8, 0) == bp.ERR_INVALID_ARG
@@ -109,7 +109,7 @@ def test_gemm_argument_checks_on_host(lib):
 
 def test_conv_argument_checks_on_host(lib):
     lay = bp.layout(bp.BLOCK_PUNCHED, bp.F16, 16, 8 * 9, 8, 4, 3, 3)
-    P = bp.Packed(lay, 2, 0, 0, 16, 16, 16, 256, 256 + 16384 + 320)
+    P = bp.Packed(lay, 2, 0, 0, 16, 16, 16, 256, 256 + 16384 + 640 + 4 * 72)   # kc_ptr, one chunk, qmap
     # C*kh*kw != K, negative pad, zero stride
     ws = 1 << 16
     assert bp.bp_conv2d(P, 256, 2, 7, 8, 8, 1, 1, 1, 1, None, 0, 256, ws, 1 << 20, 0) == \

@@ -59,7 +59,7 @@ def _sw128(row, k):
     return (row >> 3) * 1024 + (row & 7) * 128 + (((k >> 3) ^ (row & 7)) << 4) + (k & 7) * 2
 
 
-def _plan(l):
+def _plan(l, bound=None):
     """Expected load plan of a chunk list: tile loads of 8 << lg rows for runs of
     8-position groups whose live entries are consecutive columns (a group with
     no live entry, padding, continues any run)."""
@@ -77,6 +77,8 @@ def _plan(l):
         while g + run < 8 and (first[g + run] == first[g] + 8 * run or not live[8 * (g + run)]):
             run += 1
         lg = 3 if run >= 8 else 2 if run >= 4 else 1 if run >= 2 else 0
+        if bound is not None and int(first[g]) + (8 << lg) > bound:
+            return w                      # a load would pass the last listed row: gather
         boxes.append((int(first[g]), g | (lg << 4)))
         g += 1 << lg
     w[0] = len(boxes)
@@ -107,14 +109,20 @@ def _check_device_image(pw, mask, W, M, K):
     W where the row keeps the column (first occurrence of an index only)."""
     img = pw.dev.cpu().numpy()
     S = -(-M // 128)
-    kc_ptr = img[:8 * (S + 1)].view(np.int64)
-    off = (8 * (S + 1) + 255) // 256 * 256
+    hdr = img[:8 * (S + 2)].view(np.int64)
+    kc_ptr, Kc = hdr[:S + 1], int(hdr[S + 1])
+    off = (8 * (S + 2) + 255) // 256 * 256
     tile_bytes = 128 * 128
     C = int(kc_ptr[-1])
     meta_off = off + C * tile_bytes
+    meta2_off = meta_off + C * 320
+    qmap_off = meta2_off + C * 320
     assert kc_ptr[0] == 0
-    assert img.size == meta_off + C * 320
+    assert img.size == qmap_off + (4 * K + 15) // 16 * 16
+    qmap = img[qmap_off: qmap_off + 4 * K].view(np.int32)
     offs = _sw128(np.arange(128)[:, None], np.arange(64)[None, :])
+    listed = np.zeros(K, bool)
+    all_lists = []
     for s in range(S):
         r0, r1 = 128 * s, min(128 * s + 128, M)
         union = mask[r0:r1].any(axis=0)
@@ -132,6 +140,9 @@ def _check_device_image(pw, mask, W, M, K):
             l[:seg.size] = seg
             lists.append(l)
         assert kc_ptr[s + 1] - kc_ptr[s] == len(lists), s
+        for l in lists:
+            listed[l] = True
+        all_lists += [(int(kc_ptr[s]) + i, l) for i, l in enumerate(lists)]
         for i, l in enumerate(lists):
             c = int(kc_ptr[s]) + i
             base = off + c * tile_bytes
@@ -146,6 +157,15 @@ def _check_device_image(pw, mask, W, M, K):
             want[:r1 - r0] = np.where(keep, W[rows][:, l], 0)
             dec = img[base:base + tile_bytes].view(np.uint16)[offs // 2]
             assert (dec == want).all(), (s, i)
+    # compacted coordinates: rank of each listed column; records with ranked lists
+    want_q = np.where(listed, np.cumsum(listed) - 1, -1).astype(np.int32)
+    assert Kc == int(listed.sum())
+    assert (qmap == want_q).all()
+    for c, l in all_lists:
+        rec = meta2_off + c * 320
+        l2 = want_q[l]
+        assert (img[rec: rec + 256].view(np.int32) == l2).all(), c
+        assert (img[rec + 256: rec + 320].view(np.int32) == _plan(l2, bound=Kc)).all(), c
 
 
 def test_prune_ties_resolved_like_oracle():
