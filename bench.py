@@ -193,10 +193,15 @@ def run_ours(args):
         sets.append((c, dev, Xi, Yi))
     stream = torch.cuda.current_stream()
     sp = int(stream.cuda_stream)
+    # split-k workspace (partial tiles of the last wave), shared by the
+    # stream-ordered launches
+    ws = bp.gemm_workspace(pw, L.N)
+    ws_ptr, ws_bytes = (ws.data_ptr(), ws.numel()) if ws is not None else (None, 0)
 
     def step(i):
         c, _, Xi, Yi = sets[i % R]
-        st = bp.bp_gemm(c, Xi.data_ptr(), L.N, L.N, None, 0, Yi.data_ptr(), L.N, sp)
+        st = bp.bp_gemm(c, Xi.data_ptr(), L.N, L.N, None, 0, Yi.data_ptr(), L.N, ws_ptr, ws_bytes,
+                        sp)
         if st != bp.OK:
             raise bp.BpError(st, "bp_gemm")
 
@@ -272,13 +277,13 @@ def run_ours(args):
     pwe = bp.PackedWeight(c0, pw.rb_ptr, pw.col_idx, pw.values, sets[0][1])
     for i in range(2):
         Xe.copy_(Xh, non_blocking=True)
-        bp.gemm(pwe, Xe, out=Ye)
+        bp.gemm(pwe, Xe, out=Ye, ws=ws, split=ws is not None)
         Yh.copy_(Ye, non_blocking=True)
     torch.cuda.synchronize()
     ev0.record(stream)
     for i in range(ne):
         Xe.copy_(Xh, non_blocking=True)
-        bp.gemm(pwe, Xe, out=Ye)
+        bp.gemm(pwe, Xe, out=Ye, ws=ws, split=ws is not None)
         Yh.copy_(Ye, non_blocking=True)
     ev1.record(stream)
     torch.cuda.synchronize()
@@ -458,7 +463,13 @@ def _layer_step(layer, dtype, flush, reps=5):
             ours_fn = dense_fn
     else:
         dense_fn = lambda: torch.matmul(Wd, xd)  # noqa
-        ours_fn = (lambda: bp.gemm(pw, xd, bias=bd, relu=layer.relu)) if not dense else dense_fn
+        if not dense:
+            gws = bp.gemm_workspace(pw, xd.shape[1])
+            yg = bp.gemm(pw, xd, bias=bd, relu=layer.relu, ws=gws, split=gws is not None)
+            ours_fn = lambda: bp.gemm(pw, xd, bias=bd, relu=layer.relu, out=yg, ws=gws,  # noqa
+                                      split=gws is not None)
+        else:
+            ours_fn = dense_fn
     t_ours = timed(ours_fn)
     t_dense = timed(dense_fn)
     if bp.device_status() != bp.OK:

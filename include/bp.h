@@ -148,13 +148,25 @@ bp_status bp_pack(const bp_layout *lay, const void *W, const uint8_t *mask, bp_p
  *   bias  device fp32 [M] or NULL
  *   relu  0 / 1
  *   Y     device, M x N row-major (ldy >= N, multiple of 8)
+ *   ws    device workspace of bp_gemm_workspace_size() bytes (256-B aligned),
+ *         or NULL: with it, the work that would leave SMs idle in the last
+ *         wave (or when there is little work) is split along k and its fp32
+ *         partial sums are added in the workspace; without it nothing is
+ *         split (same result up to fp32 summation order).  Zero-fill a new
+ *         workspace (and again after a BP_ERR_TIMEOUT); the kernel leaves it
+ *         ready for the next call.  Calls that may overlap on the GPU need
+ *         separate workspaces.
  * Any bm: weights are processed in slabs of 128 rows (see bp_packed::dev).
  * X must be finite: rows of X that a slab lists may meet zero weights of rows
  * that prune them (0 * Inf is NaN).  The launch is a programmatic dependent
  * of the previous kernel in `stream` (its set-up overlaps that kernel's end;
  * it reads and writes nothing before that kernel has completed). */
 bp_status bp_gemm(const bp_packed *P, const void *X, int64_t N, int64_t ldx, const float *bias,
-                  int relu, void *Y, int64_t ldy, void *stream);
+                  int relu, void *Y, int64_t ldy, void *ws, size_t ws_bytes, void *stream);
+
+/* Workspace bytes bp_gemm may use for this packed weight and N (host output;
+ * 0 when nothing would be split). */
+bp_status bp_gemm_workspace_size(const bp_packed *P, int64_t N, size_t *bytes);
 
 /* Block-sparse convolution over the GEMM view of bp_layout (kept column
  * k = c*kh*kw + i*kw + j), NCHW input and output:
@@ -164,8 +176,10 @@ bp_status bp_gemm(const bp_packed *P, const void *X, int64_t N, int64_t ldx, con
  *   in    device, Nb x C x H x W;   out  device, Nb x M x Ho x Wo with
  *   Ho = (H + 2 pad_h - kh) / stride_h + 1, Wo likewise.
  *   ws    device workspace of at least bp_conv2d_workspace_size() bytes
- *         (16-B aligned): the input expanded to the K x (Nb*Ho*Wo) matrix
- *         (im2col), which the block-sparse product then reads.
+ *         (256-B aligned): the listed rows of the input expanded to the
+ *         K x (Nb*Ho*Wo) matrix (im2col), which the block-sparse product then
+ *         reads, and the partial sums of its split work (see bp_gemm: zero-fill
+ *         a new workspace).
  * Requires C*kh*kw == lay.K; dilation and groups are not supported.  The
  * input must be finite (see bp_gemm).  BP_ERR_UNSUPPORTED when kh input
  * rows padded to W + 2 pad_w exceed 12288 values, when Wo > 4096, Nb > 65535
@@ -176,7 +190,8 @@ bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, i
                     void *stream);
 
 /* Device workspace bytes bp_conv2d needs for this packed weight and input
- * shape (host output): 2 * K * (Nb*Ho*Wo rounded up to 8). */
+ * shape (host output): 2 * K * (Nb*Ho*Wo rounded up to 8), rounded up to 256,
+ * plus the split product's share (bp_gemm_workspace_size for N = Nb*Ho*Wo). */
 bp_status bp_conv2d_workspace_size(const bp_packed *P, int64_t Nb, int64_t C, int64_t H,
                                    int64_t W, int pad_h, int pad_w, int stride_h, int stride_w,
                                    size_t *bytes);

@@ -35,7 +35,8 @@ class Packed(ctypes.Structure):
 
 
 EXPORTS = ("bp_status_string", "bp_version", "bp_workspace_size", "bp_prune", "bp_pack_size",
-           "bp_pack", "bp_gemm", "bp_conv2d", "bp_conv2d_workspace_size", "bp_device_status", "bp_set_watchdog_ns",
+           "bp_pack", "bp_gemm", "bp_gemm_workspace_size", "bp_conv2d", "bp_conv2d_workspace_size",
+           "bp_device_status", "bp_set_watchdog_ns",
            "bp_debug_drop_stage", "bp_prune_noalloc")
 
 _lib = None
@@ -68,7 +69,8 @@ def load(path: str = LIB_PATH):
             "bp_prune": (i32, [P_L, vp, dbl, vp, vp, sz, vp]),
             "bp_pack_size": (i32, [P_L, vp, vp, P_i64, P_i64, P_i64, vp]),
             "bp_pack": (i32, [P_L, vp, vp, P_P, vp]),
-            "bp_gemm": (i32, [P_P, vp, i64, i64, vp, i32, vp, i64, vp]),
+            "bp_gemm": (i32, [P_P, vp, i64, i64, vp, i32, vp, i64, vp, sz, vp]),
+            "bp_gemm_workspace_size": (i32, [P_P, i64, ctypes.POINTER(sz)]),
             "bp_conv2d": (i32, [P_P, vp, i64, i64, i64, i64, i32, i32, i32, i32, vp, i32, vp,
                                 vp, sz, vp]),
             "bp_conv2d_workspace_size": (i32, [P_P, i64, i64, i64, i64, i32, i32, i32, i32,
@@ -122,8 +124,15 @@ def bp_pack(lay: Layout, W: int, mask: int, packed: Packed, stream: int = 0) -> 
 
 
 def bp_gemm(packed: Packed, X: int, N: int, ldx: int, bias: int | None, relu: int, Y: int,
-            ldy: int, stream: int = 0) -> int:
-    return load().bp_gemm(ctypes.byref(packed), X, N, ldx, bias, int(relu), Y, ldy, stream)
+            ldy: int, ws: int | None = None, ws_bytes: int = 0, stream: int = 0) -> int:
+    return load().bp_gemm(ctypes.byref(packed), X, N, ldx, bias, int(relu), Y, ldy, ws, ws_bytes,
+                          stream)
+
+
+def bp_gemm_workspace_size(packed: Packed, N: int):
+    n = ctypes.c_size_t()
+    st = load().bp_gemm_workspace_size(ctypes.byref(packed), N, ctypes.byref(n))
+    return st, n.value
 
 
 def bp_conv2d(packed: Packed, x: int, Nb: int, C: int, H: int, W: int, pad_h: int, pad_w: int,
@@ -220,15 +229,29 @@ def pack(lay: Layout, W, mask, stream=None) -> PackedWeight:
     return PackedWeight(c, rb_ptr, col_idx[:nc], values[:nv], devbuf)
 
 
-def gemm(pw: PackedWeight, X, bias=None, relu: bool = False, out=None, stream=None):
-    """Y = act(W_masked @ X + bias) through bp_gemm; X is K x N (device)."""
+def gemm_workspace(pw: PackedWeight, N: int, device="cuda"):
+    """Device workspace bp_gemm may use for N columns (None when it splits nothing)."""
+    torch = _torch()
+    st, n = bp_gemm_workspace_size(pw.c, N)
+    _chk(st, "bp_gemm_workspace_size")
+    return torch.zeros(n, dtype=torch.uint8, device=device) if n else None
+
+
+def gemm(pw: PackedWeight, X, bias=None, relu: bool = False, out=None, ws=None, stream=None,
+         split: bool = True):
+    """Y = act(W_masked @ X + bias) through bp_gemm; X is K x N (device).  `ws` from
+    gemm_workspace (allocated here when not given; split=False passes none)."""
     torch = _torch()
     K, N = X.shape
     if out is None:
         ldy = (N + 7) // 8 * 8
         out = torch.empty((pw.lay.M, ldy), dtype=X.dtype, device=X.device)[:, :N]
+    if ws is None and split:
+        ws = gemm_workspace(pw, N, X.device)
     st = bp_gemm(pw.c, X.data_ptr(), N, X.stride(0), None if bias is None else bias.data_ptr(),
-                 int(relu), out.data_ptr(), out.stride(0), _stream(stream))
+                 int(relu), out.data_ptr(), out.stride(0),
+                 None if ws is None else ws.data_ptr(),
+                 0 if ws is None else ws.numel() * ws.element_size(), _stream(stream))
     _chk(st, "bp_gemm")
     return out
 
@@ -239,7 +262,7 @@ def conv2d_workspace(pw: PackedWeight, shape, pad=(0, 0), stride=(1, 1), device=
     Nb, C, H, W = shape
     st, n = bp_conv2d_workspace_size(pw.c, Nb, C, H, W, pad[0], pad[1], stride[0], stride[1])
     _chk(st, "bp_conv2d_workspace_size")
-    return torch.empty(max(n, 16), dtype=torch.uint8, device=device)
+    return torch.zeros(max(n, 16), dtype=torch.uint8, device=device)
 
 
 def conv2d(pw: PackedWeight, x, pad=(0, 0), stride=(1, 1), bias=None, relu: bool = False,

@@ -189,7 +189,7 @@ const char *bp_status_string(int status) {
     }
 }
 
-int bp_version(void) { return (1 << 16) | 0; }
+int bp_version(void) { return (2 << 16) | 0; }
 
 bp_status bp_workspace_size(const bp_layout *lay, size_t *bytes) {
     if (!layout_ok(lay) || !bytes) return BP_ERR_INVALID_ARG;
@@ -339,17 +339,28 @@ static bp_status finish_launch(cudaError_t e, cudaStream_t s) {
     return BP_OK;
 }
 
+bp_status bp_gemm_workspace_size(const bp_packed *P, int64_t N, size_t *bytes) {
+    DevLayout dl;
+    if (!bytes || N < 0) return BP_ERR_INVALID_ARG;
+    const bp_status st = check_packed(P, &dl);
+    if (st != BP_OK) return st;
+    *bytes = N > 0 ? plan_split(dl, N, true).bytes : 0;
+    return BP_OK;
+}
+
 bp_status bp_gemm(const bp_packed *P, const void *X, int64_t N, int64_t ldx, const float *bias,
-                  int relu, void *Y, int64_t ldy, void *stream) {
+                  int relu, void *Y, int64_t ldy, void *ws, size_t ws_bytes, void *stream) {
     DevLayout dl;
     bp_status st = check_packed(P, &dl);
     if (st != BP_OK) return st;
     if (N < 0 || !X || !Y || ldx < N || ldy < N || ldx % 8 || ldy % 8) return BP_ERR_INVALID_ARG;
     if (!aligned16(X) || !aligned16(Y)) return BP_ERR_INVALID_ARG;
     if (bias && (reinterpret_cast<uintptr_t>(bias) & 3u)) return BP_ERR_INVALID_ARG;
+    if (ws && ((reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < plan_split(dl, N, true).bytes))
+        return BP_ERR_WORKSPACE;
     if (N == 0) return BP_OK;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    return finish_launch(launch_mma(*P, dl, X, N, ldx, bias, relu, Y, ldy, nullptr, s), s);
+    return finish_launch(launch_mma(*P, dl, X, N, ldx, bias, relu, Y, ldy, nullptr, ws, s), s);
 }
 
 static bp_status conv_shape(const bp_packed *P, int64_t Nb, int64_t C, int64_t H, int64_t W,
@@ -394,7 +405,7 @@ bp_status bp_conv2d_workspace_size(const bp_packed *P, int64_t Nb, int64_t C, in
     const bp_status st = conv_shape(P, Nb, C, H, W, pad_h, pad_w, stride_h, stride_w, &cs, &dl);
     if (st != BP_OK) return st;
     const int64_t N = Nb * cs.Ho * cs.Wo;
-    *bytes = (size_t)(P->lay.K * align_up(N, 8) * 2);
+    *bytes = (size_t)align_up(P->lay.K * align_up(N, 8) * 2, 256) + plan_split(dl, N, true).bytes;
     return BP_OK;
 }
 
@@ -412,13 +423,18 @@ bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, i
     const int64_t N = Nb * cs.Ho * cs.Wo;
     if (N == 0) return BP_OK;
     const int64_t ldx = align_up(N, 8);
-    if (!ws || !aligned16(ws) || ws_bytes < (size_t)(P->lay.K * ldx * 2)) return BP_ERR_WORKSPACE;
+    // workspace: the im2col matrix, then the split product's partial tiles
+    const size_t xbytes = (size_t)align_up(P->lay.K * ldx * 2, 256);
+    const size_t sbytes = plan_split(dl, N, true).bytes;
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < xbytes + sbytes)
+        return BP_ERR_WORKSPACE;
+    void *split_ws = sbytes ? static_cast<uint8_t *>(ws) + xbytes : nullptr;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const int32_t *qmap =
         reinterpret_cast<const int32_t *>(static_cast<const uint8_t *>(P->dev) + dl.off_qmap);
     cudaError_t e = launch_im2col(cs, ldx, in, ws, qmap, s);
     if (e != cudaSuccess) return BP_ERR_CUDA;
-    return finish_launch(launch_mma(*P, dl, ws, N, ldx, bias, relu, out, 0, &cs, s), s);
+    return finish_launch(launch_mma(*P, dl, ws, N, ldx, bias, relu, out, 0, &cs, split_ws, s), s);
 }
 
 bp_status bp_device_status(void *stream) {

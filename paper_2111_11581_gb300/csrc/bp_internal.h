@@ -115,9 +115,26 @@ int64_t im2col_row_width(const ConvShape &cs);   // staged input row length (ele
 // The block-sparse product on the tensor cores: Y = act(W_packed X + bias).
 // conv == nullptr: Y is M x N row-major (ldy).  Otherwise Y is the NCHW output
 // of the convolution and X its im2col matrix.
-// With conv, X holds only the listed rows (see DevLayout::off_meta2).
+// Split of the product into work units.  Persistent CTAs take (slab, column
+// tile) items in waves; when the last wave is partial (or there are fewer
+// items than SMs), its items are split along their k-chunks into `split`
+// units each, whose fp32 partial tiles meet in a workspace: the last unit of
+// an item to finish sums them and writes the output.
+struct SplitPlan {
+    int nt;             // activation columns per tile
+    int64_t items;      // (slab, column tile) items
+    int64_t full;       // items computed whole (the first `full`)
+    int split;          // units per remaining item (1: no split)
+    int64_t units;      // full + (items - full) * split
+    size_t bytes;       // workspace: partial tiles + arrival counters (0 if split == 1)
+};
+SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split);
+
+// With conv, X holds only the listed rows (see DevLayout::off_meta2).  ws:
+// at least plan_split(dl, N, true).bytes of 256-byte-aligned device memory,
+// or nullptr (no split).
 cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, int64_t N,
                        int64_t ldx, const float *bias, int relu, void *Y, int64_t ldy,
-                       const ConvShape *conv, cudaStream_t s);
+                       const ConvShape *conv, void *ws, cudaStream_t s);
 
 }  // namespace bp

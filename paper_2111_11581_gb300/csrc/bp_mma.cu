@@ -73,7 +73,12 @@ struct Params {
     int64_t N;              // tokens (GEMM) or Nb*Ho*Wo pixels (conv)
     int nt;                 // activation columns per tile: a multiple of 32, 64 .. 256
     int xboxes;             // 64-column TMA boxes per activation row: ceil(nt / 64)
-    int64_t num_items;
+    int64_t num_items;      // (slab, column tile) items
+    int64_t full_items;     // the first full_items items are single work units
+    int split;              // units per later item (k-chunk ranges)
+    int64_t num_units;      // full_items + (num_items - full_items) * split
+    float *part;            // split items: fp32 partial tiles, [item][unit][128][256]
+    int32_t *cnt;           // split items: arrivals per (item, row quadrant)
     int64_t stages;
     uint32_t tmem_cols, acc_cols, ystage_bytes;
     const int64_t *kc_ptr;
@@ -159,15 +164,37 @@ __device__ __forceinline__ void raise_timeout(const Params &p, const Smem &s) {
 
 struct Item {
     int64_t slab, n0, kc0, nkc, rows;   // rows = real rows of the slab
+    int64_t j;                          // split item index (-1: whole item)
+    int s, S;                           // unit s of S of the item
 };
 
-// Work unit u -> (slab, 256-column tile), slab fastest.
+// Work unit u -> (slab, column tile) item, slab fastest, and its k-chunk
+// range: the whole item for u < full_items, else unit s of `split` equal
+// shares of the item's chunks.
 __device__ __forceinline__ Item decode(const Params &p, const int64_t *kc, int64_t u) {
     Item t;
-    t.slab = u % p.num_slabs;
-    t.n0 = (u / p.num_slabs) * p.nt;
-    t.kc0 = kc[t.slab];
-    t.nkc = kc[t.slab + 1] - t.kc0;
+    int64_t it = u;
+    t.j = -1;
+    t.s = 0;
+    t.S = 1;
+    if (u >= p.full_items) {
+        const int64_t v = u - p.full_items;
+        t.j = v / p.split;
+        t.s = (int)(v - t.j * p.split);
+        t.S = p.split;
+        it = p.full_items + t.j;
+    }
+    t.slab = it % p.num_slabs;
+    t.n0 = (it / p.num_slabs) * p.nt;
+    const int64_t c0 = kc[t.slab], nc = kc[t.slab + 1] - c0;
+    if (t.S == 1) {
+        t.kc0 = c0;
+        t.nkc = nc;
+    } else {
+        const int64_t kb = nc * t.s / t.S, ke = nc * (t.s + 1) / t.S;
+        t.kc0 = c0 + kb;
+        t.nkc = ke - kb;
+    }
     t.rows = min((int64_t)kSlab, p.M - t.slab * kSlab);
     return t;
 }
@@ -180,7 +207,7 @@ struct Window {
     Item t;
     __device__ __forceinline__ void first(const Params &p, const int64_t *kcp) {
         k0 = 0;
-        for (it = blockIdx.x; it < p.num_items; it += gridDim.x) {
+        for (it = blockIdx.x; it < p.num_units; it += gridDim.x) {
             t = decode(p, kcp, it);
             if (t.nkc > 0) break;
         }
@@ -190,14 +217,14 @@ struct Window {
         k0 += kWin;
         if (k0 >= t.nkc) {
             k0 = 0;
-            for (it += gridDim.x; it < p.num_items; it += gridDim.x) {
+            for (it += gridDim.x; it < p.num_units; it += gridDim.x) {
                 t = decode(p, kcp, it);
                 if (t.nkc > 0) break;
             }
         }
         cnt = valid(p) ? min((int64_t)kWin, t.nkc - k0) : 0;
     }
-    __device__ __forceinline__ bool valid(const Params &p) const { return it < p.num_items; }
+    __device__ __forceinline__ bool valid(const Params &p) const { return it < p.num_units; }
 };
 
 // Load plan of a chunk record (see DevLayout): number of tile loads.
@@ -401,7 +428,7 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
     volatile int *abort_flag = s.abort_flag;
     const uint64_t wdog = p.watchdog_ns;
     const int nst = (int)p.stages;
-    const int64_t nitems = p.num_items;
+    const int64_t nitems = p.num_units;
     const uint32_t acc_cols = p.acc_cols;
     uint64_t *const wfull = s.wfull, *const full = s.full, *const empty = s.empty;
     const volatile uint32_t *const skind = s.skind;
@@ -474,6 +501,7 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
 }
 
 // ------------------------------------------------------------------ epilogue
+template <bool kSplit>
 __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
     const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
@@ -482,7 +510,7 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
     const uint32_t stg = smem_u32(s.ystage + (warp - kEpiWarp0) * 4096);
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int64_t it = blockIdx.x; it < p.num_items; it += gridDim.x) {
+    for (int64_t it = blockIdx.x; it < p.num_units; it += gridDim.x) {
         const Item t = decode(p, kcp, it);
         const bool has = t.nkc > 0;
         if (has) {
@@ -580,11 +608,70 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
 #pragma unroll
                 for (int e = 0; e < 32; ++e) r[e] = 0u;
             }
-            for (int g = 0; g < G; ++g) {
-                pack(r, pk);
-                if (has && g + 1 < G) tmem_ld_32x32b_x32(tacc + 32 * (g + 1), r);
-                store(pk, 32 * g);
-                if (has && g + 1 < G) tmem_ld_wait();
+            if (!kSplit || t.S == 1) {
+                for (int g = 0; g < G; ++g) {
+                    pack(r, pk);
+                    if (has && g + 1 < G) tmem_ld_32x32b_x32(tacc + 32 * (g + 1), r);
+                    store(pk, 32 * g);
+                    if (has && g + 1 < G) tmem_ld_wait();
+                }
+            } else {
+                // Split item: this unit's fp32 partial rows go to its slot; the
+                // unit whose arrival completes the (item, quadrant) count sums
+                // all slots and writes the output (no unit waits for another).
+                // Slot layout per quadrant: [group][8 float4][lane], so each
+                // warp access is 512 contiguous bytes.
+                constexpr int64_t kQuad = 8 * 8 * 32;            // float4 per (unit, quadrant)
+                float4 *slot = reinterpret_cast<float4 *>(p.part) +
+                               ((t.j * t.S + t.s) * 4 + q) * kQuad + lane;
+                for (int g = 0; g < G; ++g) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        __stcg(slot + (g * 8 + e) * 32,
+                               make_float4(__uint_as_float(r[4 * e]), __uint_as_float(r[4 * e + 1]),
+                                           __uint_as_float(r[4 * e + 2]), __uint_as_float(r[4 * e + 3])));
+                    if (has && g + 1 < G) {
+                        tmem_ld_32x32b_x32(tacc + 32 * (g + 1), r);
+                        tmem_ld_wait();
+                    }
+                }
+                __threadfence();
+                __syncwarp();
+                int last = 0;
+                if (lane == 0) last = atomicAdd(p.cnt + t.j * 4 + q, 1) == t.S - 1;
+                if (__shfl_sync(0xffffffffu, last, 0)) {
+                    __threadfence();
+                    if (lane == 0) p.cnt[t.j * 4 + q] = 0;     // zero again for the next launch
+                    const float4 *base = reinterpret_cast<const float4 *>(p.part) +
+                                         (t.j * t.S * 4 + q) * kQuad + lane;
+                    for (int g = 0; g < G; ++g) {
+                        float4 a[8];
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) a[e] = __ldcg(base + (g * 8 + e) * 32);
+                        for (int u = 1; u < t.S; ++u) {
+                            float4 v[8];
+#pragma unroll
+                            for (int e = 0; e < 8; ++e)
+                                v[e] = __ldcg(base + (int64_t)u * 4 * kQuad + (g * 8 + e) * 32);
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) {
+                                a[e].x += v[e].x;
+                                a[e].y += v[e].y;
+                                a[e].z += v[e].z;
+                                a[e].w += v[e].w;
+                            }
+                        }
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            r[4 * e] = __float_as_uint(a[e].x);
+                            r[4 * e + 1] = __float_as_uint(a[e].y);
+                            r[4 * e + 2] = __float_as_uint(a[e].z);
+                            r[4 * e + 3] = __float_as_uint(a[e].w);
+                        }
+                        pack(r, pk);
+                        store(pk, 32 * g);
+                    }
+                }
             }
         }
         if (has) {
@@ -599,6 +686,9 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
     if (!p.conv && lane == 0) bulk_wait_all();   // staged output fully written before exit
 }
 
+// kSplit: the launch has split items (a separate instantiation keeps the
+// common kernel free of the partial-tile code).
+template <bool kSplit>
 __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_constant__ Params p) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     const Smem s = carve(smem_raw, p);
@@ -649,7 +739,7 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
         if ((threadIdx.x & 31) == 0) mma_issuer(p, s, tmem);
         __syncwarp();
     } else {
-        epilogue(p, s, tmem);
+        epilogue<kSplit>(p, s, tmem);
     }
 
     tc_fence_before();
@@ -696,9 +786,40 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 }  // namespace
 
+SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split) {
+    SplitPlan sp{};
+    const int sms = num_sms();
+    sp.nt = pick_tile_width(N, dl.num_slabs, sms);
+    sp.items = (N + sp.nt - 1) / sp.nt * dl.num_slabs;
+    sp.full = sp.items;
+    sp.split = 1;
+    if (allow_split && sp.items < sms && dl.kc_total > 0) {
+        // Fewer items than SMs: split every item along its chunks so that the
+        // units fill the SMs, each unit keeping at least four chunks on
+        // average.  (Splitting only a partial last wave of a larger problem
+        // measured slower: the partial tiles' write, read and second epilogue
+        // cost more than the chunks they move.)
+        int64_t S = sms / sp.items;
+        const int64_t avg = dl.kc_total / dl.num_slabs;
+        if (S > avg / 4) S = avg / 4;
+        if (S > 32) S = 32;
+        if (S >= 2) {
+            sp.split = (int)S;
+            sp.full = 0;
+        }
+    }
+    sp.units = sp.full + (sp.items - sp.full) * sp.split;
+    if (sp.split > 1) {
+        const int64_t slots = (sp.items - sp.full) * sp.split;
+        sp.bytes = (size_t)((slots * kSlab * kNT * 4 + 255) / 256 * 256 +
+                            ((sp.items - sp.full) * 16 + 255) / 256 * 256);
+    }
+    return sp;
+}
+
 cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, int64_t N,
                        int64_t ldx, const float *bias, int relu, void *Y, int64_t ldy,
-                       const ConvShape *conv, cudaStream_t st) {
+                       const ConvShape *conv, void *ws, cudaStream_t st) {
     Params p{};
     const uint8_t *dev = static_cast<const uint8_t *>(P.dev);
     p.dtype = P.lay.dtype;
@@ -707,10 +828,23 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     p.M = P.lay.M;
     p.num_slabs = dl.num_slabs;
     p.N = N;
-    p.nt = pick_tile_width(N, p.num_slabs, num_sms());
+    const SplitPlan sp = plan_split(dl, N, ws != nullptr);
+    p.nt = sp.nt;
     p.xboxes = (p.nt + 63) / 64;
-    p.num_items = (N + p.nt - 1) / p.nt * p.num_slabs;
+    p.num_items = sp.items;
+    p.full_items = sp.full;
+    p.split = sp.split;
+    p.num_units = sp.units;
     if (p.num_items == 0) return cudaSuccess;
+    if (sp.split > 1) {
+        // partial tiles, then the arrival counters (zero on entry: the caller
+        // zero-fills a new workspace, and each item's last unit zeroes its
+        // counters again)
+        const int64_t slots = (sp.items - sp.full) * sp.split;
+        p.part = static_cast<float *>(ws);
+        p.cnt = reinterpret_cast<int32_t *>(static_cast<uint8_t *>(ws) +
+                                            (slots * kSlab * kNT * 4 + 255) / 256 * 256);
+    }
     p.ystage_bytes = 4 * 4096;     // per epilogue warp: two 2 KB boxes (GEMM) or one (conv)
     // shared memory: stages, output staging, barriers, index ring, and a copy of
     // kc_ptr when that costs no pipeline stage
@@ -768,11 +902,15 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [] {
-        attr_err = cudaFuncSetAttribute(bp_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        (int)kMaxSmem);
+        attr_err = cudaFuncSetAttribute(bp_mma_kernel<false>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxSmem);
+        if (attr_err == cudaSuccess)
+            attr_err = cudaFuncSetAttribute(bp_mma_kernel<true>,
+                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                            (int)kMaxSmem);
     });
     if (attr_err != cudaSuccess) return attr_err;
-    const int64_t grid = p.num_items < num_sms() ? p.num_items : num_sms();
+    const int64_t grid = p.num_units < num_sms() ? p.num_units : num_sms();
     // programmatic dependent launch: the kernel's set-up may overlap the tail of
     // the previous kernel in the stream (the kernel waits for it before any
     // global memory access)
@@ -786,7 +924,8 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, bp_mma_kernel, p);
+    return p.split > 1 ? cudaLaunchKernelEx(&cfg, bp_mma_kernel<true>, p)
+                       : cudaLaunchKernelEx(&cfg, bp_mma_kernel<false>, p);
 }
 
 }  // namespace bp

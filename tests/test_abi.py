@@ -58,7 +58,7 @@ def test_ctypes_structs_match_header(tmp_path):
 def test_status_strings_and_version(lib):
     assert bp.status_string(bp.OK) == "ok"
     assert bp.status_string(bp.ERR_TIMEOUT) == "kernel wait timed out"
-    assert bp.bp_version() >> 16 == 1
+    assert bp.bp_version() >> 16 == 2
 
 
 def test_workspace_size_is_host_only(lib):
@@ -96,7 +96,13 @@ def test_gemm_argument_checks_on_host(lib):
     assert bp.bp_gemm(P, 256, 10, 10, None, 0, 256, 16, 0) == bp.ERR_INVALID_ARG
     assert bp.bp_gemm(P, 258, 8, 8, None, 0, 256, 8, 0) == bp.ERR_INVALID_ARG
     assert bp.bp_gemm(P, 256, 16, 8, None, 0, 256, 16, 0) == bp.ERR_INVALID_ARG
-    assert bp.load().bp_gemm(None, 256, 8, 8, None, 0, 256, 8, None) == bp.ERR_INVALID_ARG
+    assert bp.load().bp_gemm(None, 256, 8, 8, None, 0, 256, 8, None, 0, None) == bp.ERR_INVALID_ARG
+    # a workspace must be 256-byte aligned and as large as bp_gemm_workspace_size says
+    st, n = bp.bp_gemm_workspace_size(P, 8)
+    assert st == bp.OK
+    assert bp.bp_gemm(P, 256, 8, 8, None, 0, 256, 8, 256 + 16, 1 << 30) == bp.ERR_WORKSPACE
+    if n:
+        assert bp.bp_gemm(P, 256, 8, 8, None, 0, 256, 8, 1 << 20, n - 1) == bp.ERR_WORKSPACE
     # an image size that is not kc_ptr + whole (tile, record) chunks
     Pbad = bp.Packed(lay, 4, 0, 0, 16, 16, 16, 256, 256 + 16384)
     assert bp.bp_gemm(Pbad, 256, 8, 8, None, 0, 256, 8, 0) == bp.ERR_INVALID_ARG

@@ -124,3 +124,30 @@ def test_sweep_full_size_sampled_rows(case):
     ref2 = (Wm @ Xd.float())
     err = (Y.float() - ref2).abs()
     assert bool((err <= 1e-2 * ref2.abs().clamp_min(1.0)).all())
+
+
+@pytest.mark.parametrize("case", [
+    # few items, many chunks: every item split along k (8 items x 8 units)
+    (512, 4096, 512, 128, 32, 4.0, bp.BF16, True, True),
+    # 4 slabs x 1 column tile, small bm: the union lists are long
+    (512, 2048, 200, 16, 8, 8.0, bp.F16, False, False),
+], ids=lambda c: f"{c[0]}x{c[1]}x{c[2]}_b{c[3]}x{c[4]}")
+def test_split_k_matches_oracle_and_unsplit(case):
+    """The k-split product (fp32 partial tiles summed in the workspace) and the
+    unsplit one both match the oracle."""
+    M, K, N, bm, bk, rate, dtype, has_bias, relu = case
+    W, X, b, mask, pw = _layer(M, K, N, bm, bk, rate, dtype, seed=7 * M + K, bias=has_bias,
+                               relu=relu)
+    Xd = dev16(X, dtype, pad_last_to=8)
+    bd = torch.from_numpy(b).cuda() if b is not None else None
+    ws = bp.gemm_workspace(pw, N)
+    assert ws is not None, "this shape should split"
+    Ys = bp.gemm(pw, Xd, bias=bd, relu=relu, ws=ws)
+    Yu = bp.gemm(pw, Xd, bias=bd, relu=relu, split=False)
+    Ys2 = bp.gemm(pw, Xd, bias=bd, relu=relu, ws=ws)     # counters were reset by the kernel
+    torch.cuda.synchronize()
+    assert bp.device_status() == bp.OK
+    ref = oracle.masked_gemm(W, mask, X, dtype, bias=b, relu=relu)
+    assert_close(host_bits(Ys), ref, dtype, "split")
+    assert_close(host_bits(Yu), ref, dtype, "unsplit")
+    assert torch.equal(Ys, Ys2), "split result not reproducible"
