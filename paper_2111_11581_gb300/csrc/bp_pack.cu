@@ -379,45 +379,72 @@ __global__ void __launch_bounds__(256) im2col_1x1_kernel(ConvShape cs, int64_t l
 }
 
 // Writes the block's im2col rows from the staged planes: segments of 32*V
-// consecutive pixels of one channel per warp step, V pixels per lane.
-template <int V>
+// consecutive pixels of one channel per warp step, V pixels per lane (one
+// 2V-byte store per window offset).  KH, KW > 0: the window's size at compile
+// time (loops unrolled); 0: taken from kh, kw.  qtab: the im2col row of each
+// (channel of the block, i, j), -1 for rows no slab lists.
+template <int V, int KH, int KW>
 __device__ __forceinline__ void im2col_emit(const uint16_t *plane, const int32_t *tab,
-                                            uint16_t *out, const int32_t *qrows, int64_t ldx,
-                                            int PB, int ncg, int chan_sz, int khw, int kh,
-                                            int kw, int wp, int lane, int warp, int nwarps) {
+                                            const int32_t *qtab, uint16_t *out, int64_t ldx,
+                                            int PB, int ncg, int chan_sz, int kh_rt, int kw_rt,
+                                            int wp, int lane, int warp, int nwarps) {
+    const int kh = KH > 0 ? KH : kh_rt, kw = KW > 0 ? KW : kw_rt;
+    const int khw = kh * kw;
     const int segs = (PB + 32 * V - 1) / (32 * V);
     int cc = 0, sg = warp;
     while (sg >= segs) { sg -= segs; ++cc; }
     for (; cc < ncg;) {
         const int p = (sg * 32 + lane) * V;
         if (p < PB) {
-            const uint16_t *src[V];
+            const uint16_t *pl = plane + cc * chan_sz;
+            int o0[V];
 #pragma unroll
-            for (int e = 0; e < V; ++e) src[e] = plane + cc * chan_sz + tab[p + e];
+            for (int e = 0; e < V; ++e) o0[e] = tab[p + e];
+            const int32_t *qc = qtab + cc * khw;
+            uint16_t *op = out + p;
+#pragma unroll (KH > 0 ? KH : 1)
             for (int i = 0; i < kh; ++i) {
+#pragma unroll (KW > 0 ? KW : 1)
                 for (int j = 0; j < kw; ++j) {
-                    // row of the im2col matrix this (channel, i, j) becomes, or none
-                    const int kk = cc * khw + i * kw + j;
-                    const int64_t q = qrows ? (int64_t)__ldg(qrows + kk) : (int64_t)kk;
+                    const int q = qc[i * kw + j];
                     if (q < 0) continue;
-                    uint16_t *dst = out + q * ldx + p;
                     const int o = i * wp + j;
-                    if (V == 1) {
-                        *dst = src[0][o];
-                    } else if (V == 2) {
-                        *reinterpret_cast<uint32_t *>(dst) =
-                            (uint32_t)src[0][o] | ((uint32_t)src[1][o] << 16);
-                    } else {
-                        *reinterpret_cast<uint2 *>(dst) =
-                            make_uint2((uint32_t)src[0][o] | ((uint32_t)src[1][o] << 16),
-                                       (uint32_t)src[2][o] | ((uint32_t)src[3][o] << 16));
+                    uint32_t v[(V + 1) / 2];
+#pragma unroll
+                    for (int e = 0; e < V; e += 2) {
+                        const uint32_t lo = pl[o0[e] + o];
+                        const uint32_t hi = e + 1 < V ? (uint32_t)pl[o0[e + 1] + o] : 0u;
+                        v[e / 2] = lo | (hi << 16);
                     }
+                    uint16_t *dst = op + (int64_t)q * ldx;
+                    if constexpr (V == 1) *dst = (uint16_t)v[0];
+                    else if constexpr (V == 2) *reinterpret_cast<uint32_t *>(dst) = v[0];
+                    else if constexpr (V == 4) *reinterpret_cast<uint2 *>(dst) = make_uint2(v[0], v[1]);
+                    else *reinterpret_cast<uint4 *>(dst) = make_uint4(v[0], v[1], v[2], v[3]);
                 }
             }
         }
         sg += nwarps;
         while (sg >= segs) { sg -= segs; ++cc; }
     }
+}
+
+// Picks the pixels per lane (alignment of the block's first im2col column and
+// pixel count) and the window specialisation.
+template <int KH, int KW>
+__device__ __forceinline__ void im2col_emit_any(int64_t nbase, const uint16_t *plane,
+                                                const int32_t *tab, const int32_t *qtab,
+                                                uint16_t *out, int64_t ldx, int PB, int ncg,
+                                                int chan_sz, int kh, int kw, int wp, int lane,
+                                                int warp, int nwarps) {
+    if (nbase % 8 == 0 && PB % 8 == 0)
+        im2col_emit<8, KH, KW>(plane, tab, qtab, out, ldx, PB, ncg, chan_sz, kh, kw, wp, lane, warp, nwarps);
+    else if (nbase % 4 == 0 && PB % 4 == 0)
+        im2col_emit<4, KH, KW>(plane, tab, qtab, out, ldx, PB, ncg, chan_sz, kh, kw, wp, lane, warp, nwarps);
+    else if (nbase % 2 == 0 && PB % 2 == 0)
+        im2col_emit<2, KH, KW>(plane, tab, qtab, out, ldx, PB, ncg, chan_sz, kh, kw, wp, lane, warp, nwarps);
+    else
+        im2col_emit<1, KH, KW>(plane, tab, qtab, out, ldx, PB, ncg, chan_sz, kh, kw, wp, lane, warp, nwarps);
 }
 
 // im2col, one block per (group of cg channels, group of ig images, band of
@@ -446,8 +473,11 @@ __global__ void __launch_bounds__(256) im2col_kernel(ConvShape cs, int64_t ldx, 
     const int P = R * Wo;                      // the band's pixels per (channel, image)
     const int PB = nig * P;                    // the block's pixels per channel
     const int plane_sz = rows * wp;            // staged values per (channel, image)
+    const int khw = cs.kh * cs.kw;
     int32_t *tab = reinterpret_cast<int32_t *>(im2col_smem);
-    uint16_t *plane = reinterpret_cast<uint16_t *>(im2col_smem + ((4 * ig * P + 15) & ~15));
+    int32_t *qtab = tab + ig * P;
+    uint16_t *plane =
+        reinterpret_cast<uint16_t *>(im2col_smem + ((4 * (ig * P + cg * khw) + 15) & ~15));
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     // stage: the staged rows (channel, image, row) are spread over the warps,
     // `lpr` lanes per row (a power of two, 32 for rows longer than 32 values),
@@ -500,21 +530,21 @@ __global__ void __launch_bounds__(256) im2col_kernel(ConvShape cs, int64_t ldx, 
         const int base = bb * plane_sz + orow * cs.sh * wp;
         for (int ow = lane; ow < Wo; ow += 32) tab[bb * P + orow * Wo + ow] = base + ow * cs.sw;
     }
+    // im2col row of each (channel, i, j) of the block: qmap[k], or k itself
+    for (int e = threadIdx.x; e < ncg * khw; e += blockDim.x) {
+        const int64_t k = (int64_t)c0 * khw + e;
+        qtab[e] = qmap ? qmap[k] : (int32_t)k;
+    }
     __syncthreads();
-    const int khw = cs.kh * cs.kw;
     const int64_t nbase = (int64_t)b0 * Ho * Wo + (int64_t)oh0 * Wo;
-    // rows: qmap[k] for k = c*kh*kw + i*kw + j (from this block's first channel),
-    // or k itself without a map
-    uint16_t *out = xcol + nbase + (qmap ? 0 : (int64_t)c0 * khw * ldx);
-    const int32_t *qrows = qmap ? qmap + (int64_t)c0 * khw : nullptr;
-    // V consecutive pixels per lane (one 2V-byte store per window offset) when
-    // the block's pixels start 2V-byte aligned in the im2col row
-    if (nbase % 4 == 0 && PB % 4 == 0 && ldx % 4 == 0)
-        im2col_emit<4>(plane, tab, out, qrows, ldx, PB, ncg, ig * plane_sz, khw, cs.kh, cs.kw, wp, lane, warp, nwarps);
-    else if (nbase % 2 == 0 && PB % 2 == 0)
-        im2col_emit<2>(plane, tab, out, qrows, ldx, PB, ncg, ig * plane_sz, khw, cs.kh, cs.kw, wp, lane, warp, nwarps);
+    uint16_t *out = xcol + nbase;
+    const int chan_sz = ig * plane_sz;
+    if (cs.kh == 3 && cs.kw == 3)
+        im2col_emit_any<3, 3>(nbase, plane, tab, qtab, out, ldx, PB, ncg, chan_sz, 3, 3, wp, lane,
+                              warp, nwarps);
     else
-        im2col_emit<1>(plane, tab, out, qrows, ldx, PB, ncg, ig * plane_sz, khw, cs.kh, cs.kw, wp, lane, warp, nwarps);
+        im2col_emit_any<0, 0>(nbase, plane, tab, qtab, out, ldx, PB, ncg, chan_sz, cs.kh, cs.kw, wp,
+                              lane, warp, nwarps);
 }
 
 }  // namespace
@@ -632,9 +662,15 @@ cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void
     if (cg > kStage / (ig * rows * wp)) cg = kStage / (ig * rows * wp);
     if (cg > cs.C) cg = cs.C;
     if (cg < 1) cg = 1;
+    auto smem_for = [&](int64_t g) {
+        return (size_t)((4 * (ig * pix + g * cs.kh * cs.kw) + 15) & ~15) +
+               (size_t)(g * ig * rows * wp * 2);
+    };
+    while (cg > 1 && smem_for(cg) > 48 * 1024) --cg;
+    if (smem_for(cg) > 48 * 1024) return cudaErrorInvalidValue;
     const int64_t gx = (cs.C + cg - 1) / cg, gy = (cs.Nb + ig - 1) / ig;
     if (gx > 0x7fffffffLL || gy > 65535 || nbands > 65535) return cudaErrorInvalidValue;
-    const size_t smem = (size_t)((4 * ig * pix + 15) & ~15) + (size_t)(cg * ig * rows * wp * 2);
+    const size_t smem = smem_for(cg);
     im2col_kernel<<<dim3((unsigned)gx, (unsigned)gy, (unsigned)nbands), 256, smem, s>>>(
         cs, ldx, (int)band, (int)wp, (int)cg, (int)ig, qmap, static_cast<const uint16_t *>(in),
         static_cast<uint16_t *>(xcol));
