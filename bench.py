@@ -489,6 +489,18 @@ def run_workload(args):
     bp.load()
     flush = torch.empty(256 * 2 ** 20 // 4, dtype=torch.float32, device="cuda")
     name = args.workload
+    if name == "blocksize":
+        # the rule-based block-size selection's latency model (Sec. 5.2), built
+        # with this library's kernels, and the block each setting gets at
+        # beta = 20 %
+        from paper_2111_11581_gb300 import latency_model as lm
+        settings = lm.default_settings()
+        model = lm.build_model(settings)
+        sel = {st.key(): lm.block_name(lm.select_block(model, st, 0.2)) for st in settings}
+        print(json.dumps({"workload": "blocksize", "beta": 0.2,
+                          "latency_unit": "seconds per dense MAC", "selected": sel,
+                          "model": model}), flush=True)
+        return
     if name == "fc512":
         layers, dtype = [inputs.fc512()], inputs.F16
     elif name == "conv3x3":
@@ -539,7 +551,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--workload", default=None,
                     help="fc512 | conv3x3 | vgg16 | resnet50 | sweep: per-layer timings "
-                         "of another workload (one JSON line), instead of the default step")
+                         "of another workload (one JSON line), instead of the default step; "
+                         "blocksize: the latency model and block-size selection")
     ap.add_argument("--sweep-subset", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
