@@ -213,6 +213,50 @@ int oracle_scores(int scheme, int dtype, int64_t M, int64_t K, int64_t kh, int64
     return OR_OK;
 }
 
+/* Reweighted group-Lasso regulariser of one layer (Eq. prob_block with
+ * Eq. column for block-based and Eq. punched for block-punched blocks) and
+ * its gradient with respect to W, the reweighting factors held fixed:
+ *   s_u     = ||W_u||_F^2 over the unit's weights (as oracle_scores),
+ *   alpha_u = 1 / (s_u + eps)                        (the reweighting rule),
+ *   R       = lambda * sum_u ||alpha_u o W_u||_F^2 = lambda * sum_u alpha_u^2 s_u,
+ *   dR/dW   = 2 lambda alpha_u^2 W  for every weight of unit u.
+ * Reading: alpha_u is a scalar per unit, so "alpha o W_u" scales the unit and
+ * its squared norm picks up alpha_u^2.  R is summed in unit order.  */
+int oracle_reweighted_penalty(int scheme, int dtype, int64_t M, int64_t K, int64_t kh,
+                              int64_t kw, int64_t bm, int64_t bk, const uint16_t *W, double eps,
+                              double lambda, double *alpha, double *R, double *grad)
+{
+    part_t p;
+    int st = make_part(&p, scheme, M, K, kh, kw, bm, bk);
+    if (st) return st;
+    if (!(eps > 0.0)) return OR_ERR_ARG;
+    st = oracle_scores(scheme, dtype, M, K, kh, kw, bm, bk, W, alpha);
+    if (st) return st;
+    double r = 0.0;
+    for (int64_t u = 0; u < p.U; ++u) {
+        double s = alpha[u];
+        alpha[u] = 1.0 / (s + eps);
+        r += alpha[u] * alpha[u] * s;
+    }
+    *R = lambda * r;
+#pragma omp parallel for schedule(static)
+    for (int64_t f = 0; f < M; ++f) {
+        int64_t rb = f / p.bm;
+        for (int64_t k = 0; k < K; ++k) {
+            int64_t u;
+            if (p.scheme == 0) {
+                u = rb * K + k;                                   /* (row-block, column) */
+            } else {
+                int64_t c = k / p.KK, pos = k % p.KK;               /* OIHW: k = c*KK + pos */
+                u = unit_index(&p, rb, c / p.bk, pos);
+            }
+            double a = alpha[u];
+            grad[f * K + k] = 2.0 * lambda * a * a * oracle_half_to_double(W[f * K + k], dtype);
+        }
+    }
+    return OR_OK;
+}
+
 /* Keep counts for a rate r >= 1 (Sec. 5.1 one-shot pruning at a set rate;
  * the rate is the parameter-reduction factor).  A block of P units keeps at
  * least base = floor(P / r); the layer keeps T = floor(sum P / r + 0.5) units

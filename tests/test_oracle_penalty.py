@@ -1,0 +1,88 @@
+"""Pins of the reweighted-regulariser oracle (Eq. prob_block with Eq. column /
+Eq. punched): autograd of an independent grouping of the same objective, a
+closed form, partial blocks by brute force.  CPU only."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2111_11581_gb300 import inputs
+
+F16, BF16 = 0, 1
+
+
+def _objective_grad(Wd, scheme, bm, bk, kh, kw, eps, lam):
+    """R and dR/dW by autograd, units formed by reshaping (full blocks only)."""
+    W = torch.tensor(Wd, dtype=torch.float64, requires_grad=True)
+    M, K = W.shape
+    if scheme == 0:
+        s = (W.reshape(M // bm, bm, K) ** 2).sum(1)                       # (RB, K)
+    else:
+        KK = kh * kw
+        C = K // KK
+        W5 = W.reshape(M // bm, bm, C // bk, bk, KK)
+        s = (W5 ** 2).sum((1, 3))                                           # (RB, CB, KK)
+    alpha = 1.0 / (s.detach() + eps)
+    R = lam * (alpha ** 2 * s).sum()
+    R.backward()
+    return alpha.reshape(-1).numpy(), R.item(), W.grad.numpy()
+
+
+@pytest.mark.parametrize("scheme,M,K,bm,bk,kh,kw,dtype", [
+    (0, 64, 96, 16, 8, 1, 1, F16),
+    (0, 32, 48, 32, 48, 1, 1, BF16),       # one block: structured
+    (0, 24, 40, 1, 1, 1, 1, F16),          # 1x1 blocks: unstructured
+    (1, 32, 16 * 9, 8, 4, 3, 3, BF16),
+    (1, 16, 8 * 25, 16, 8, 5, 5, F16),
+])
+def test_penalty_matches_autograd(scheme, M, K, bm, bk, kh, kw, dtype):
+    W = inputs.normal((M, K), 0.05, dtype, seed=M + K)
+    Wd = oracle.to_double(W, dtype)
+    eps, lam = 1e-3, 0.37
+    a, R, g = oracle.reweighted_penalty(W, dtype, scheme, bm, bk, eps, lam, kh, kw)
+    a2, R2, g2 = _objective_grad(Wd, scheme, bm, bk, kh, kw, eps, lam)
+    np.testing.assert_allclose(a, a2, rtol=1e-13)
+    assert R == pytest.approx(R2, rel=1e-12)
+    np.testing.assert_allclose(g, g2, rtol=1e-13, atol=0)
+
+
+def test_penalty_closed_form_single_unit():
+    # one column of 4 rows, values 1, 2, 2, 0 (exact in fp16): s = 9
+    W = oracle.round_to(np.array([[1.0], [2.0], [2.0], [0.0]]), F16)
+    eps, lam = 0.5, 2.0
+    a, R, g = oracle.reweighted_penalty(W, F16, 0, 4, 1, eps, lam)
+    assert a[0] == 1.0 / 9.5
+    assert R == pytest.approx(lam * 9.0 / 9.5 ** 2, rel=1e-15)
+    np.testing.assert_allclose(g[:, 0], 2 * lam / 9.5 ** 2 * np.array([1.0, 2.0, 2.0, 0.0]),
+                               rtol=1e-15)
+
+
+def test_penalty_partial_blocks_brute_force():
+    # M and C not multiples of the block: units of the last blocks are smaller
+    M, C, KK, bm, bk = 10, 7, 9, 4, 3
+    W = inputs.normal((M, C * KK), 0.1, BF16, seed=5)
+    Wd = oracle.to_double(W, BF16)
+    eps, lam = 1e-2, 1.0
+    a, R, g = oracle.reweighted_penalty(W, BF16, 1, bm, bk, eps, lam, 3, 3)
+    RB, CB = -(-M // bm), -(-C // bk)
+    want_g = np.zeros_like(Wd)
+    want_R = 0.0
+    for rb in range(RB):
+        for cb in range(CB):
+            for pos in range(KK):
+                idx = [(f, c * KK + pos) for f in range(rb * bm, min(M, rb * bm + bm))
+                       for c in range(cb * bk, min(C, cb * bk + bk))]
+                s = sum(Wd[i] ** 2 for i in idx)
+                al = 1.0 / (s + eps)
+                assert a[(rb * CB + cb) * KK + pos] == pytest.approx(al, rel=1e-15)
+                want_R += al * al * s
+                for i in idx:
+                    want_g[i] = 2 * lam * al * al * Wd[i]
+    assert R == pytest.approx(lam * want_R, rel=1e-13)
+    np.testing.assert_allclose(g, want_g, rtol=1e-14)
+
+
+def test_penalty_rejects_nonpositive_eps():
+    W = inputs.normal((8, 8), 0.1, F16, seed=1)
+    with pytest.raises(Exception):
+        oracle.reweighted_penalty(W, F16, 0, 4, 4, 0.0, 1.0)
