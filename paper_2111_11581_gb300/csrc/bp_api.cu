@@ -189,7 +189,7 @@ const char *bp_status_string(int status) {
     }
 }
 
-int bp_version(void) { return (2 << 16) | 0; }
+int bp_version(void) { return (2 << 16) | 1; }
 
 bp_status bp_workspace_size(const bp_layout *lay, size_t *bytes) {
     if (!layout_ok(lay) || !bytes) return BP_ERR_INVALID_ARG;
@@ -435,6 +435,43 @@ bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, i
     cudaError_t e = launch_im2col(cs, ldx, in, ws, qmap, s);
     if (e != cudaSuccess) return BP_ERR_CUDA;
     return finish_launch(launch_mma(*P, dl, ws, N, ldx, bias, relu, out, 0, &cs, split_ws, s), s);
+}
+
+bp_status bp_penalty_units(const bp_layout *lay, int64_t *units) {
+    if (!layout_ok(lay) || !units) return BP_ERR_INVALID_ARG;
+    const int64_t RB = cdiv(lay->M, lay->bm);
+    if (lay->scheme == BP_BLOCK_BASED) {
+        *units = RB * lay->K;
+    } else {
+        const int64_t KK = (int64_t)lay->kh * lay->kw;
+        *units = RB * cdiv(lay->K / KK, lay->bk) * KK;
+    }
+    return BP_OK;
+}
+
+bp_status bp_penalty_workspace_size(const bp_layout *lay, size_t *bytes) {
+    if (!layout_ok(lay) || !bytes) return BP_ERR_INVALID_ARG;
+    if (lay->M * lay->K >= INT32_MAX) return BP_ERR_UNSUPPORTED;
+    *bytes = penalty_workspace_bytes(*lay);
+    return BP_OK;
+}
+
+bp_status bp_reweighted_penalty(const bp_layout *lay, const void *W, double eps, double lambda,
+                                double *alpha, double *R, float *grad, void *ws,
+                                size_t ws_bytes, void *stream) {
+    if (!layout_ok(lay) || !W || !alpha || !R || !grad) return BP_ERR_INVALID_ARG;
+    if (!aligned16(W) || !aligned16(grad) || (reinterpret_cast<uintptr_t>(alpha) & 7u) ||
+        (reinterpret_cast<uintptr_t>(R) & 7u))
+        return BP_ERR_INVALID_ARG;
+    if (!(eps > 0.0) || !std::isfinite(eps) || !std::isfinite(lambda)) return BP_ERR_INVALID_ARG;
+    if (lay->M * lay->K >= INT32_MAX) return BP_ERR_UNSUPPORTED;
+    // the fp32 factors: eps and 1/eps representable, 2 |lambda| / eps^2 finite
+    if (eps < 0x1p-60 || eps > 0x1p60 || 2.0 * std::fabs(lambda) / (eps * eps) >= 0x1p127)
+        return BP_ERR_UNSUPPORTED;
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < penalty_workspace_bytes(*lay))
+        return BP_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    return cuda_status(launch_penalty(*lay, W, eps, lambda, alpha, R, grad, ws, s));
 }
 
 bp_status bp_device_status(void *stream) {

@@ -3,7 +3,9 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <cuda.h>
 #include <cuda_runtime.h>
+#include <cudaTypedefs.h>
 
 #include "bp.h"
 
@@ -76,6 +78,7 @@ uint64_t watchdog_ns();
 int64_t debug_drop_stage();     // -1 = no fault injection
 unsigned *device_status_ptr();   // device address of the status word
 int num_sms();
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder();   // nullptr if the driver lacks it
 bool checked_mode();
 
 // Launchers (return cudaError_t of the launch).
@@ -91,6 +94,14 @@ cudaError_t launch_threshold_select(int64_t U, const double *scores, uint8_t *ke
 cudaError_t launch_write_mask(const bp_layout &lay, const uint8_t *keep, uint8_t *mask,
                               cudaStream_t s);
 int64_t threshold_chunks(int64_t U);
+
+// Reweighted regulariser: per unit s = ||W_u||^2, alpha = 1/(s + eps),
+// R = lambda * sum alpha^2 s, grad = 2 lambda alpha^2 W (fp32).  The
+// workspace holds a completion counter (zero between calls) at offset 0 and
+// the per-block partial sums of R from offset 256.
+size_t penalty_workspace_bytes(const bp_layout &lay);
+cudaError_t launch_penalty(const bp_layout &lay, const void *W, double eps, double lambda,
+                           double *alpha, double *R, float *grad, void *ws, cudaStream_t s);
 
 cudaError_t launch_rb_counts(const bp_layout &lay, const uint8_t *mask, int64_t *rb_ptr,
                              int *bad, cudaStream_t s);

@@ -770,7 +770,9 @@ int pick_tile_width(int64_t N, int64_t slabs, int sms) {
     return best;
 }
 
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+}  // namespace
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     static std::once_flag once;
     std::call_once(once, [] {
@@ -783,8 +785,6 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     });
     return fn;
 }
-
-}  // namespace
 
 SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split) {
     SplitPlan sp{};
@@ -873,7 +873,7 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     p.drop_stage = debug_drop_stage();
     p.status = device_status_ptr();
 
-    PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
+    PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
     if (!enc) return cudaErrorNotSupported;
     const CUtensorMapDataType tdt =
         P.lay.dtype == BP_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;

@@ -58,7 +58,7 @@ def test_ctypes_structs_match_header(tmp_path):
 def test_status_strings_and_version(lib):
     assert bp.status_string(bp.OK) == "ok"
     assert bp.status_string(bp.ERR_TIMEOUT) == "kernel wait timed out"
-    assert bp.bp_version() >> 16 == 2
+    assert bp.bp_version() >> 16 == 2 and bp.bp_version() & 0xffff >= 1
 
 
 def test_workspace_size_is_host_only(lib):
@@ -135,3 +135,37 @@ def test_conv_argument_checks_on_host(lib):
         bp.ERR_WORKSPACE
     assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, 1, 1, 1, 1, None, 0, 256, ws + 8, 1 << 20, 0) == \
         bp.ERR_WORKSPACE
+
+
+def test_penalty_argument_checks_on_host(lib):
+    lay = bp.layout(bp.BLOCK_BASED, bp.BF16, 256, 512, 128, 32)
+    assert bp.bp_penalty_units(lay) == (bp.OK, 2 * 512)
+    play = bp.layout(bp.BLOCK_PUNCHED, bp.F16, 24, 5 * 9, 8, 2, 3, 3)
+    assert bp.bp_penalty_units(play) == (bp.OK, 3 * 3 * 9)      # 3 filter blocks x 3 channel blocks
+    # tiles of 128 rows x 64 columns (32 slices of 4 rows): 2 row-blocks x 8 tiles
+    assert bp.bp_penalty_workspace_size(lay) == (bp.OK, 256 + 8 * 16)
+    # one thread per unit: 81 units -> one block
+    assert bp.bp_penalty_workspace_size(play) == (bp.OK, 256 + 8)
+    a = 1 << 20
+    # eps must be positive and finite, lambda finite, W / grad 16-B aligned
+    for eps, lam in ((0.0, 1.0), (-1.0, 1.0), (float("inf"), 1.0), (1e-4, float("nan"))):
+        assert bp.bp_reweighted_penalty(lay, a, eps, lam, a, a, a, a, 1 << 16, 0) == \
+            bp.ERR_INVALID_ARG
+    assert bp.bp_reweighted_penalty(lay, a + 8, 1e-4, 1.0, a, a, a, a, 1 << 16, 0) == \
+        bp.ERR_INVALID_ARG
+    assert bp.bp_reweighted_penalty(lay, a, 1e-4, 1.0, a, a, a + 4, a, 1 << 16, 0) == \
+        bp.ERR_INVALID_ARG
+    # outside the fp32 range of the factors
+    for eps, lam in ((2.0 ** -61, 1.0), (2.0 ** 61, 1.0), (1e-18, 1e3)):
+        assert bp.bp_reweighted_penalty(lay, a, eps, lam, a, a, a, a, 1 << 16, 0) == \
+            bp.ERR_UNSUPPORTED
+    # missing, misaligned or short workspace
+    assert bp.bp_reweighted_penalty(lay, a, 1e-4, 1.0, a, a, a, None, 1 << 16, 0) == \
+        bp.ERR_WORKSPACE
+    assert bp.bp_reweighted_penalty(lay, a, 1e-4, 1.0, a, a, a, a + 16, 1 << 16, 0) == \
+        bp.ERR_WORKSPACE
+    assert bp.bp_reweighted_penalty(lay, a, 1e-4, 1.0, a, a, a, a, 256 + 8 * 16 - 1, 0) == \
+        bp.ERR_WORKSPACE
+    # M*K >= 2^31 is outside the kernels' 32-bit indexing
+    big = bp.layout(bp.BLOCK_BASED, bp.BF16, 1 << 16, 1 << 15, 128, 32)
+    assert bp.bp_penalty_workspace_size(big)[0] == bp.ERR_UNSUPPORTED
