@@ -77,8 +77,11 @@ def _load():
                                                  i64, i64, i64, i64, i64, vp, i32, vp, vp]
             lib.oracle_reweighted_penalty.argtypes = [i32, i32, i64, i64, i64, i64, i64, i64, vp,
                                                       dbl, dbl, vp, vp, vp]
+            lib.oracle_reweighted_penalty_rows.argtypes = [i32, i64, i64, i64, vp, dbl, dbl, vp,
+                                                           vp, vp]
             lib.oracle_max_threads.restype = i32
-            for f in ("oracle_scores", "oracle_reweighted_penalty", "oracle_counts", "oracle_prune",
+            for f in ("oracle_scores", "oracle_reweighted_penalty",
+                      "oracle_reweighted_penalty_rows", "oracle_counts", "oracle_prune",
                       "oracle_pack",
                       "oracle_unpack", "oracle_masked_gemm", "oracle_masked_conv2d"):
                 getattr(lib, f).restype = i32
@@ -145,11 +148,22 @@ def scores(W_bits, dtype, scheme, bm, bk, kh=1, kw=1) -> np.ndarray:
     return out
 
 
-def reweighted_penalty(W_bits, dtype, scheme, bm, bk, eps, lam, kh=1, kw=1):
+def reweighted_penalty(W_bits, dtype, scheme, bm, bk, eps, lam, kh=1, kw=1, groups="layout"):
     """Reweighted regulariser of one layer and its gradient (Eq. prob_block with
-    Eq. column / Eq. punched): returns (alpha[U], R, grad[M, K]) in fp64."""
+    Eq. column / Eq. punched, or with Eq. row when groups == "rows"): returns
+    (alpha[U], R, grad[M, K]) in fp64."""
     W = _u16(W_bits)
     M, K = W.shape
+    if groups == "rows":
+        if scheme != 0:
+            raise OracleError("row groups are defined for block-based layouts")
+        CB = (K + bk - 1) // bk
+        alpha = np.zeros(M * CB, np.float64)
+        R = np.zeros(1, np.float64)
+        grad = np.zeros((M, K), np.float64)
+        _check(_load().oracle_reweighted_penalty_rows(dtype, M, K, bk, _p(W), float(eps),
+                                                      float(lam), _p(alpha), _p(R), _p(grad)))
+        return alpha, float(R[0]), grad
     U = num_units(scheme, M, K, kh, kw, bm, bk)
     alpha = np.zeros(U, np.float64)
     R = np.zeros(1, np.float64)

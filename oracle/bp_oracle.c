@@ -257,6 +257,42 @@ int oracle_reweighted_penalty(int scheme, int dtype, int64_t M, int64_t K, int64
     return OR_OK;
 }
 
+/* The same regulariser with the row groups of block-based pruning (Sec. 4.2,
+ * Eq. row): the units are the rows of each bm x bk block, i.e. unit
+ * u = r * CB + cb holds W[r, cb*bk .. min(cb*bk + bk, K) - 1], summed with k
+ * ascending; alpha_u = 1 / (s_u + eps), R = lambda * sum_u alpha_u^2 s_u and
+ * grad = 2 lambda alpha_u^2 W.  bm does not enter (a block's rows are its
+ * groups); block-punched layouts have no row groups here (OR_ERR_ARG). */
+int oracle_reweighted_penalty_rows(int dtype, int64_t M, int64_t K, int64_t bk,
+                                   const uint16_t *W, double eps, double lambda, double *alpha,
+                                   double *R, double *grad)
+{
+    if (M < 1 || K < 1 || bk < 1 || !(eps > 0.0)) return OR_ERR_ARG;
+    const int64_t CB = (K + bk - 1) / bk;
+    for (int64_t r = 0; r < M; ++r)
+        for (int64_t cb = 0; cb < CB; ++cb) {
+            double s = 0.0;
+            for (int64_t k = cb * bk; k < K && k < cb * bk + bk; ++k) {
+                double w = oracle_half_to_double(W[r * K + k], dtype);
+                s += w * w;
+            }
+            alpha[r * CB + cb] = s;        /* the score; the factor below */
+        }
+    double sum = 0.0;
+    for (int64_t u = 0; u < M * CB; ++u) {
+        double s = alpha[u];
+        alpha[u] = 1.0 / (s + eps);
+        sum += alpha[u] * alpha[u] * s;
+    }
+    *R = lambda * sum;
+    for (int64_t r = 0; r < M; ++r)
+        for (int64_t k = 0; k < K; ++k) {
+            double a = alpha[r * CB + k / bk];
+            grad[r * K + k] = 2.0 * lambda * a * a * oracle_half_to_double(W[r * K + k], dtype);
+        }
+    return OR_OK;
+}
+
 /* Keep counts for a rate r >= 1 (Sec. 5.1 one-shot pruning at a set rate;
  * the rate is the parameter-reduction factor).  A block of P units keeps at
  * least base = floor(P / r); the layer keeps T = floor(sum P / r + 0.5) units

@@ -86,3 +86,53 @@ def test_penalty_rejects_nonpositive_eps():
     W = inputs.normal((8, 8), 0.1, F16, seed=1)
     with pytest.raises(Exception):
         oracle.reweighted_penalty(W, F16, 0, 4, 4, 0.0, 1.0)
+
+
+def _row_objective_grad(Wd, bk, eps, lam):
+    """Eq. row by autograd: the rows of each block (full column blocks)."""
+    W = torch.tensor(Wd, dtype=torch.float64, requires_grad=True)
+    M, K = W.shape
+    s = (W.reshape(M, K // bk, bk) ** 2).sum(2)                              # (M, CB)
+    alpha = 1.0 / (s.detach() + eps)
+    R = lam * (alpha ** 2 * s).sum()
+    R.backward()
+    return alpha.reshape(-1).numpy(), R.item(), W.grad.numpy()
+
+
+@pytest.mark.parametrize("M,K,bk,dtype", [(16, 64, 16, F16), (8, 48, 48, BF16), (12, 20, 1, F16)])
+def test_row_penalty_matches_autograd(M, K, bk, dtype):
+    W = inputs.normal((M, K), 0.05, dtype, seed=7 * M + K)
+    Wd = oracle.to_double(W, dtype)
+    eps, lam = 2e-3, 0.6
+    a, R, g = oracle.reweighted_penalty(W, dtype, 0, 4, bk, eps, lam, groups="rows")
+    a2, R2, g2 = _row_objective_grad(Wd, bk, eps, lam)
+    np.testing.assert_allclose(a, a2, rtol=1e-13)
+    assert R == pytest.approx(R2, rel=1e-12)
+    np.testing.assert_allclose(g, g2, rtol=1e-13, atol=0)
+
+
+def test_row_penalty_partial_block_and_transpose_duality():
+    # a partial last column block sums its real columns only; and the row
+    # groups of W are the column groups of W^T with bm = bk (whole-height
+    # column blocks of the transpose are its rows' segments)
+    M, K, bk = 6, 10, 4
+    W = inputs.normal((M, K), 0.05, F16, seed=3)
+    Wd = oracle.to_double(W, F16)
+    eps, lam = 1e-3, 1.5
+    a, R, g = oracle.reweighted_penalty(W, F16, 0, 1, bk, eps, lam, groups="rows")
+    CB = 3
+    s = np.array([[np.sum(Wd[r, cb * bk:min(K, cb * bk + bk)] ** 2) for cb in range(CB)]
+                  for r in range(M)])
+    np.testing.assert_allclose(a.reshape(M, CB), 1.0 / (s + eps), rtol=1e-14)
+    WT = np.ascontiguousarray(W.T)
+    aT, RT, gT = oracle.reweighted_penalty(WT, F16, 0, bk, 1, eps, lam)   # column groups of W^T
+    # W^T is K x M: row-blocks of bk rows, unit (rb, column r) = W[r, rb-block]
+    np.testing.assert_allclose(aT.reshape(CB, M).T.reshape(-1), a, rtol=1e-14)
+    assert RT == pytest.approx(R, rel=1e-14)
+    np.testing.assert_allclose(gT.T, g, rtol=1e-14)
+
+
+def test_row_penalty_rejects_punched():
+    W = inputs.normal((8, 18), 0.05, F16, seed=1)
+    with pytest.raises(oracle.OracleError):
+        oracle.reweighted_penalty(W, F16, 1, 4, 2, 1e-3, 1.0, 3, 3, groups="rows")
