@@ -503,31 +503,35 @@ def run_workload(args):
         return
     if name == "penalty":
         # the reweighted regulariser + gradient of the benchmark's 4096^2 weight
-        # (HBM-bound: W read, fp32 gradient and fp64 factors written)
+        # with the column groups (Eq. column) and the row groups (Eq. row) of
+        # its 128 x 32 blocks (HBM-bound: W read, fp32 gradient and the fp64
+        # factors written)
         M = K = 4096
         lay = bp.layout(bp.BLOCK_BASED, bp.BF16, M, K, 128, 32)
         Wd = inputs.as_torch(inputs.normal((M, K), 0.02, bp.BF16, 7), bp.BF16).cuda()
-        ws = bp.penalty_workspace(lay)
-        out = bp.penalty(lay, Wd, 1e-4, 1.0, ws=ws)
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
-        ts = []
-        for i in range(23):
-            # flush L2, then read the flush buffer back so that the lines left
-            # in L2 are clean (no write-back of the flush inside the timing)
-            flush.zero_()
-            flush.sum()
-            ev[0].record()
-            a, R, g = bp.penalty(lay, Wd, 1e-4, 1.0, ws=ws, out=out)
-            ev[1].record()
-            torch.cuda.synchronize()
-            if i >= 3:
-                ts.append(ev[0].elapsed_time(ev[1]) * 1e3)
-        us = statistics.median(ts)
-        U = a.numel()
-        alg = 2 * M * K + 4 * M * K + 8 * U
-        print(json.dumps({"workload": "penalty", "shape": [M, K], "bm": 128, "bk": 32,
-                          "us": round(us, 2), "algorithmic_bytes": alg,
-                          "achieved_gbs": round(alg / us / 1e3, 1),
+        res = {}
+        for gname, groups in (("columns", bp.GROUPS_LAYOUT), ("rows", bp.GROUPS_ROWS)):
+            ws = bp.penalty_workspace(lay, groups=groups)
+            out = bp.penalty(lay, Wd, 1e-4, 1.0, ws=ws, groups=groups)
+            ts = []
+            for i in range(23):
+                # flush L2, then read the flush buffer back so that the lines
+                # left in L2 are clean (no write-back of the flush inside the
+                # timing)
+                flush.zero_()
+                flush.sum()
+                ev[0].record()
+                a, R, g = bp.penalty(lay, Wd, 1e-4, 1.0, ws=ws, out=out, groups=groups)
+                ev[1].record()
+                torch.cuda.synchronize()
+                if i >= 3:
+                    ts.append(ev[0].elapsed_time(ev[1]) * 1e3)
+            us = statistics.median(ts)
+            alg = 2 * M * K + 4 * M * K + 8 * a.numel()
+            res[gname] = {"groups": a.numel(), "us": round(us, 2), "algorithmic_bytes": alg,
+                          "achieved_gbs": round(alg / us / 1e3, 1)}
+        print(json.dumps({"workload": "penalty", "shape": [M, K], "bm": 128, "bk": 32, **res,
                           "timing": "device time incl. launch, median of 20, L2 flushed "
                                     "and left clean"}),
               flush=True)

@@ -196,46 +196,56 @@ bp_status bp_conv2d_workspace_size(const bp_packed *P, int64_t Nb, int64_t C, in
                                    int64_t W, int pad_h, int pad_w, int stride_h, int stride_w,
                                    size_t *bytes);
 
-/* Number of pruning units of a layout (block-based: one per column of each
- * row-block; block-punched: one per kernel position of each filters x
- * channels block) -- the length of bp_reweighted_penalty's alpha. */
-bp_status bp_penalty_units(const bp_layout *lay, int64_t *units);
+/* Groups of the reweighted regulariser (Sec. 4.2).  BP_GROUPS_LAYOUT: the
+ * layout's pruning units -- the columns of each block for block-based layouts
+ * (Eq. column), the kernel positions of each filters x channels block for
+ * block-punched ones (Eq. punched).  BP_GROUPS_ROWS: the rows of each block of
+ * a block-based layout (Eq. row); unit u = r * ceil(K / bk) + cb is the
+ * segment W[r, cb*bk .. min(cb*bk + bk, K) - 1] (bm does not enter). */
+typedef enum { BP_GROUPS_LAYOUT = 0, BP_GROUPS_ROWS = 1 } bp_groups;
+
+/* Number of groups (host output) -- the length of bp_reweighted_penalty's
+ * alpha: ceil(M/bm) * K (block-based), ceil(M/bm) * ceil(C/bk) * kh*kw
+ * (block-punched), M * ceil(K/bk) (row groups).  BP_ERR_INVALID_ARG for row
+ * groups of a block-punched layout. */
+bp_status bp_penalty_units(const bp_layout *lay, int groups, int64_t *units);
 
 /* Reweighted group-Lasso regulariser of one layer and its gradient (Sec. 4.2:
- * Eq. prob_block with Eq. column for block-based and Eq. punched for
- * block-punched layouts; the reweighting of Candes et al. for the factors):
- *   s_u     = squared Frobenius norm of unit u's weights,
+ * Eq. prob_block with the groups above; the reweighting of Candes et al. for
+ * the factors):
+ *   s_u     = squared Frobenius norm of group u's weights,
  *   alpha_u = 1 / (s_u + eps),
  *   R       = lambda * sum_u ||alpha_u o W_u||_F^2 = lambda * sum_u alpha_u^2 s_u,
  *   grad    = dR/dW = 2 lambda alpha_u^2 W  (the factors held fixed, as in
  *             one reweighting step).
- *   W      device, M x K 16-bit weights (OIHW for convolutions), 16-B aligned
- *   eps    > 0 (see the range below), lambda finite
- *   alpha  device fp64 [bp_penalty_units] output
- *   R      device fp64 scalar output
- *   grad   device fp32 M x K output, 16-B aligned
- *   ws     device workspace of bp_penalty_workspace_size() bytes, 256-B
- *          aligned, zero-filled before its first use; every call leaves it
- *          zeroed again.  Calls that may run concurrently need separate
- *          workspaces.
+ *   groups  a bp_groups value
+ *   W       device, M x K 16-bit weights (OIHW for convolutions), 16-B aligned
+ *   eps     > 0 (see the range below), lambda finite
+ *   alpha   device fp64 [bp_penalty_units] output
+ *   R       device fp64 scalar output
+ *   grad    device fp32 M x K output, 16-B aligned
+ *   ws      device workspace of bp_penalty_workspace_size() bytes, 256-B
+ *           aligned, zero-filled before its first use; every call leaves it
+ *           zeroed again.  Calls that may run concurrently need separate
+ *           workspaces.
  * Precision (fp32, as in the paper's training): s_u is summed in fp32 (each
  * square of a 16-bit weight is exact in fp32; relative error at most
- * (n-1) 2^-24 for a unit of n weights); alpha_u, the unit's term alpha_u^2 s_u
- * and the factor 2 lambda alpha_u^2 are formed in fp32 from fp32(eps) and
- * fp32(2 lambda), and the gradient is that factor times each weight in fp32;
- * alpha is stored widened to fp64 and R is the fp64 sum of the fp32 terms
- * times lambda, in a fixed order (the same bits run to run on one GPU).
- * Non-finite weights, and units whose squared norm leaves the fp32 range
- * (|w| above about 1.8e19), give non-finite outputs.  Asynchronous.
+ * (n-1) 2^-24 for a group of n weights); alpha_u, the group's term
+ * alpha_u^2 s_u and the factor 2 lambda alpha_u^2 are formed in fp32 from
+ * fp32(eps) and fp32(2 lambda), and the gradient is that factor times each
+ * weight in fp32; alpha is stored widened to fp64 and R is the fp64 sum of the
+ * fp32 terms times lambda, in a fixed order (the same bits run to run on one
+ * GPU).  Non-finite weights, and groups whose squared norm leaves the fp32
+ * range (|w| above about 1.8e19), give non-finite outputs.  Asynchronous.
  * BP_ERR_UNSUPPORTED when M*K >= 2^31, or when eps is outside [2^-60, 2^60]
  * or 2 |lambda| / eps^2 >= 2^127 (the largest factor must be a finite fp32). */
-bp_status bp_reweighted_penalty(const bp_layout *lay, const void *W, double eps, double lambda,
-                                double *alpha, double *R, float *grad, void *ws,
+bp_status bp_reweighted_penalty(const bp_layout *lay, int groups, const void *W, double eps,
+                                double lambda, double *alpha, double *R, float *grad, void *ws,
                                 size_t ws_bytes, void *stream);
 
-/* Device workspace bytes bp_reweighted_penalty needs for `lay` (host output):
+/* Device workspace bytes bp_reweighted_penalty needs (host output):
  * 256 + 8 * (the number of blocks the launch uses, at most 2048). */
-bp_status bp_penalty_workspace_size(const bp_layout *lay, size_t *bytes);
+bp_status bp_penalty_workspace_size(const bp_layout *lay, int groups, size_t *bytes);
 
 /* Synchronizes `stream`, then returns BP_ERR_TIMEOUT if any kernel of this
  * library recorded an expired wait since the previous call (and clears the

@@ -75,9 +75,9 @@ def load(path: str = LIB_PATH):
                                 vp, sz, vp]),
             "bp_conv2d_workspace_size": (i32, [P_P, i64, i64, i64, i64, i32, i32, i32, i32,
                                                ctypes.POINTER(sz)]),
-            "bp_penalty_units": (i32, [P_L, P_i64]),
-            "bp_reweighted_penalty": (i32, [P_L, vp, dbl, dbl, vp, vp, vp, vp, sz, vp]),
-            "bp_penalty_workspace_size": (i32, [P_L, ctypes.POINTER(sz)]),
+            "bp_penalty_units": (i32, [P_L, i32, P_i64]),
+            "bp_reweighted_penalty": (i32, [P_L, i32, vp, dbl, dbl, vp, vp, vp, vp, sz, vp]),
+            "bp_penalty_workspace_size": (i32, [P_L, i32, ctypes.POINTER(sz)]),
             "bp_device_status": (i32, [vp]),
             "bp_set_watchdog_ns": (i32, [ctypes.c_uint64]),
             "bp_debug_drop_stage": (i32, [i64]),
@@ -153,22 +153,26 @@ def bp_conv2d_workspace_size(packed: Packed, Nb: int, C: int, H: int, W: int, pa
     return st, n.value
 
 
-def bp_penalty_units(lay: Layout):
+GROUPS_LAYOUT, GROUPS_ROWS = 0, 1
+
+
+def bp_penalty_units(lay: Layout, groups: int = GROUPS_LAYOUT):
     n = ctypes.c_int64()
-    st = load().bp_penalty_units(ctypes.byref(lay), ctypes.byref(n))
+    st = load().bp_penalty_units(ctypes.byref(lay), int(groups), ctypes.byref(n))
     return st, n.value
 
 
-def bp_penalty_workspace_size(lay: Layout):
+def bp_penalty_workspace_size(lay: Layout, groups: int = GROUPS_LAYOUT):
     n = ctypes.c_size_t()
-    st = load().bp_penalty_workspace_size(ctypes.byref(lay), ctypes.byref(n))
+    st = load().bp_penalty_workspace_size(ctypes.byref(lay), int(groups), ctypes.byref(n))
     return st, n.value
 
 
-def bp_reweighted_penalty(lay: Layout, W: int, eps: float, lam: float, alpha: int, R: int,
-                          grad: int, ws: int | None, ws_bytes: int, stream: int = 0) -> int:
-    return load().bp_reweighted_penalty(ctypes.byref(lay), W, float(eps), float(lam), alpha, R,
-                                        grad, ws, ws_bytes, stream)
+def bp_reweighted_penalty(lay: Layout, groups: int, W: int, eps: float, lam: float, alpha: int,
+                          R: int, grad: int, ws: int | None, ws_bytes: int,
+                          stream: int = 0) -> int:
+    return load().bp_reweighted_penalty(ctypes.byref(lay), int(groups), W, float(eps),
+                                        float(lam), alpha, R, grad, ws, ws_bytes, stream)
 
 
 def bp_device_status(stream: int = 0) -> int:
@@ -306,32 +310,33 @@ def conv2d(pw: PackedWeight, x, pad=(0, 0), stride=(1, 1), bias=None, relu: bool
     return out
 
 
-def penalty_workspace(lay: Layout, device="cuda"):
+def penalty_workspace(lay: Layout, device="cuda", groups: int = GROUPS_LAYOUT):
     """Zero-filled workspace for bp_reweighted_penalty (reusable: every call
     leaves it zeroed)."""
     torch = _torch()
-    st, n = bp_penalty_workspace_size(lay)
+    st, n = bp_penalty_workspace_size(lay, groups)
     _chk(st, "bp_penalty_workspace_size")
     return torch.zeros(n, dtype=torch.uint8, device=device)
 
 
-def penalty(lay: Layout, W, eps: float, lam: float, ws=None, out=None, stream=None):
+def penalty(lay: Layout, W, eps: float, lam: float, ws=None, out=None, stream=None,
+            groups: int = GROUPS_LAYOUT):
     """Reweighted regulariser of a layer (bp_reweighted_penalty): returns
-    (alpha fp64 [units], R fp64 [1], grad fp32 M x K) on W's device.  `out`
+    (alpha fp64 [groups], R fp64 [1], grad fp32 M x K) on W's device.  `out`
     may hold a previous result triple to write into."""
     torch = _torch()
     if out is None:
-        st, U = bp_penalty_units(lay)
+        st, U = bp_penalty_units(lay, groups)
         _chk(st, "bp_penalty_units")
         out = (torch.empty(U, dtype=torch.float64, device=W.device),
                torch.empty(1, dtype=torch.float64, device=W.device),
                torch.empty((lay.M, lay.K), dtype=torch.float32, device=W.device))
     alpha, R, grad = out
     if ws is None:
-        ws = penalty_workspace(lay, W.device)
-    st = load().bp_reweighted_penalty(ctypes.byref(lay), W.data_ptr(), float(eps), float(lam),
-                                      alpha.data_ptr(), R.data_ptr(), grad.data_ptr(),
-                                      ws.data_ptr(), ws.numel(), _stream(stream))
+        ws = penalty_workspace(lay, W.device, groups)
+    st = bp_reweighted_penalty(lay, groups, W.data_ptr(), eps, lam, alpha.data_ptr(),
+                               R.data_ptr(), grad.data_ptr(), ws.data_ptr(), ws.numel(),
+                               _stream(stream))
     _chk(st, "bp_reweighted_penalty")
     return alpha, R, grad
 

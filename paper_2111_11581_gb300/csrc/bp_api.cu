@@ -189,7 +189,7 @@ const char *bp_status_string(int status) {
     }
 }
 
-int bp_version(void) { return (2 << 16) | 1; }
+int bp_version(void) { return (2 << 16) | 2; }
 
 bp_status bp_workspace_size(const bp_layout *lay, size_t *bytes) {
     if (!layout_ok(lay) || !bytes) return BP_ERR_INVALID_ARG;
@@ -437,10 +437,17 @@ bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, i
     return finish_launch(launch_mma(*P, dl, ws, N, ldx, bias, relu, out, 0, &cs, split_ws, s), s);
 }
 
-bp_status bp_penalty_units(const bp_layout *lay, int64_t *units) {
-    if (!layout_ok(lay) || !units) return BP_ERR_INVALID_ARG;
+static bool groups_ok(const bp_layout *lay, int groups) {
+    if (groups == BP_GROUPS_LAYOUT) return true;
+    return groups == BP_GROUPS_ROWS && lay->scheme == BP_BLOCK_BASED;
+}
+
+bp_status bp_penalty_units(const bp_layout *lay, int groups, int64_t *units) {
+    if (!layout_ok(lay) || !units || !groups_ok(lay, groups)) return BP_ERR_INVALID_ARG;
     const int64_t RB = cdiv(lay->M, lay->bm);
-    if (lay->scheme == BP_BLOCK_BASED) {
+    if (groups == BP_GROUPS_ROWS) {
+        *units = lay->M * cdiv(lay->K, lay->bk);
+    } else if (lay->scheme == BP_BLOCK_BASED) {
         *units = RB * lay->K;
     } else {
         const int64_t KK = (int64_t)lay->kh * lay->kw;
@@ -449,17 +456,18 @@ bp_status bp_penalty_units(const bp_layout *lay, int64_t *units) {
     return BP_OK;
 }
 
-bp_status bp_penalty_workspace_size(const bp_layout *lay, size_t *bytes) {
-    if (!layout_ok(lay) || !bytes) return BP_ERR_INVALID_ARG;
+bp_status bp_penalty_workspace_size(const bp_layout *lay, int groups, size_t *bytes) {
+    if (!layout_ok(lay) || !bytes || !groups_ok(lay, groups)) return BP_ERR_INVALID_ARG;
     if (lay->M * lay->K >= INT32_MAX) return BP_ERR_UNSUPPORTED;
-    *bytes = penalty_workspace_bytes(*lay);
+    *bytes = penalty_workspace_bytes(*lay, groups);
     return BP_OK;
 }
 
-bp_status bp_reweighted_penalty(const bp_layout *lay, const void *W, double eps, double lambda,
-                                double *alpha, double *R, float *grad, void *ws,
+bp_status bp_reweighted_penalty(const bp_layout *lay, int groups, const void *W, double eps,
+                                double lambda, double *alpha, double *R, float *grad, void *ws,
                                 size_t ws_bytes, void *stream) {
-    if (!layout_ok(lay) || !W || !alpha || !R || !grad) return BP_ERR_INVALID_ARG;
+    if (!layout_ok(lay) || !W || !alpha || !R || !grad || !groups_ok(lay, groups))
+        return BP_ERR_INVALID_ARG;
     if (!aligned16(W) || !aligned16(grad) || (reinterpret_cast<uintptr_t>(alpha) & 7u) ||
         (reinterpret_cast<uintptr_t>(R) & 7u))
         return BP_ERR_INVALID_ARG;
@@ -468,10 +476,11 @@ bp_status bp_reweighted_penalty(const bp_layout *lay, const void *W, double eps,
     // the fp32 factors: eps and 1/eps representable, 2 |lambda| / eps^2 finite
     if (eps < 0x1p-60 || eps > 0x1p60 || 2.0 * std::fabs(lambda) / (eps * eps) >= 0x1p127)
         return BP_ERR_UNSUPPORTED;
-    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < penalty_workspace_bytes(*lay))
+    if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) ||
+        ws_bytes < penalty_workspace_bytes(*lay, groups))
         return BP_ERR_WORKSPACE;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    return cuda_status(launch_penalty(*lay, W, eps, lambda, alpha, R, grad, ws, s));
+    return cuda_status(launch_penalty(*lay, groups, W, eps, lambda, alpha, R, grad, ws, s));
 }
 
 bp_status bp_device_status(void *stream) {

@@ -99,9 +99,10 @@ int64_t threshold_chunks(int64_t U);
 // R = lambda * sum alpha^2 s, grad = 2 lambda alpha^2 W (fp32).  The
 // workspace holds a completion counter (zero between calls) at offset 0 and
 // the per-block partial sums of R from offset 256.
-size_t penalty_workspace_bytes(const bp_layout &lay);
-cudaError_t launch_penalty(const bp_layout &lay, const void *W, double eps, double lambda,
-                           double *alpha, double *R, float *grad, void *ws, cudaStream_t s);
+size_t penalty_workspace_bytes(const bp_layout &lay, int groups);
+cudaError_t launch_penalty(const bp_layout &lay, int groups, const void *W, double eps,
+                           double lambda, double *alpha, double *R, float *grad, void *ws,
+                           cudaStream_t s);
 
 cudaError_t launch_rb_counts(const bp_layout &lay, const uint8_t *mask, int64_t *rb_ptr,
                              int *bad, cudaStream_t s);

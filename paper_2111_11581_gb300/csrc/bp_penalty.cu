@@ -404,11 +404,121 @@ __global__ void __launch_bounds__(kThreads) penalty_unit_kernel(
     finish_R(rsum, lambda, part, count, R);
 }
 
-enum class Path { kTma, kLoop, kUnit };
+// Row groups of block-based layers (Eq. row): unit u = r * CB + cb is the
+// contiguous segment W[r, cb*bk .. min(cb*bk + bk, K) - 1]; one thread per
+// unit, so a warp reads 32 neighbouring segments of a row.  kVec: bk and K
+// multiples of 8, segments read and written 16 B at a time.
+template <bool kBF16, bool kVec>
+__global__ void __launch_bounds__(kThreads) penalty_rows_kernel(
+    Geo g, float eps, float lambda2, double lambda, const uint16_t *__restrict__ W,
+    double *__restrict__ alpha, float *__restrict__ grad, double *__restrict__ part,
+    unsigned *__restrict__ count, double *__restrict__ R) {
+    double rsum = 0.0;
+    for (int64_t uu = blockIdx.x * kThreads + threadIdx.x; uu < g.U;
+         uu += (int64_t)gridDim.x * kThreads) {
+        const int u = (int)uu;
+        const int r = u / g.CB, cb = u - r * g.CB;
+        const int k0 = cb * g.bk, n = min(g.bk, g.K - k0);
+        const size_t e0 = (size_t)r * g.K + k0;
+        float s = 0.f;
+        if constexpr (kVec) {
+            const uint4 *src = reinterpret_cast<const uint4 *>(W + e0);
+            for (int i = 0; i < n / 8; ++i) {
+                const uint4 v = __ldg(src + i);
+                const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float lo = to_f32<kBF16>(w4[j] & 0xffffu);
+                    const float hi = to_f32<kBF16>(w4[j] >> 16);
+                    s = fmaf(lo, lo, s);
+                    s = fmaf(hi, hi, s);
+                }
+            }
+        } else {
+            for (int i = 0; i < n; ++i) {
+                const float w = to_f32<kBF16>(__ldg(W + e0 + i));
+                s = fmaf(w, w, s);
+            }
+        }
+        const float k = finish_unit(s, eps, lambda2, alpha + u, rsum);
+        if constexpr (kVec) {
+            const uint4 *src = reinterpret_cast<const uint4 *>(W + e0);
+            float4 *dst = reinterpret_cast<float4 *>(grad + e0);
+            for (int i = 0; i < n / 8; ++i) {
+                const uint4 v = __ldg(src + i);
+                dst[2 * i] = make_float4(k * to_f32<kBF16>(v.x & 0xffffu), k * to_f32<kBF16>(v.x >> 16),
+                                         k * to_f32<kBF16>(v.y & 0xffffu), k * to_f32<kBF16>(v.y >> 16));
+                dst[2 * i + 1] =
+                    make_float4(k * to_f32<kBF16>(v.z & 0xffffu), k * to_f32<kBF16>(v.z >> 16),
+                                k * to_f32<kBF16>(v.w & 0xffffu), k * to_f32<kBF16>(v.w >> 16));
+            }
+        } else {
+            for (int i = 0; i < n; ++i) grad[e0 + i] = k * to_f32<kBF16>(__ldg(W + e0 + i));
+        }
+    }
+    finish_R(rsum, lambda, part, count, R);
+}
+
+// Row groups when bk is 8, 16, ..., 256 and divides K: the weight is one
+// stream of M K / bk whole segments, taken 256 weights per warp.  Lane l loads
+// weights 8l .. 8l + 7 (16 B; a warp load covers 512 contiguous bytes); the
+// L = bk / 8 lanes of a segment add their fp32 sums with a fixed butterfly,
+// the segment's first lane forms the factors, and the factor goes back to the
+// segment by a shuffle.  (Lanes store their 32 gradient bytes as two 16-B
+// halves; exchanging values between lanes so that each warp store covers
+// whole sectors, or 8-byte loads with that layout, measured slower.)
+template <bool kBF16>
+__global__ void __launch_bounds__(kThreads) penalty_rows_warp_kernel(
+    Geo g, float eps, float lambda2, double lambda, const uint16_t *__restrict__ W,
+    double *__restrict__ alpha, float *__restrict__ grad, double *__restrict__ part,
+    unsigned *__restrict__ count, double *__restrict__ R) {
+    const int lane = threadIdx.x & 31;
+    const int L = g.bk / 8;                        // lanes per segment (a power of two)
+    const int64_t total = (int64_t)g.M * g.K;      // a multiple of bk
+    const int64_t chunks = (total + 255) / 256;    // 256 weights per warp
+    const int64_t warps = (int64_t)gridDim.x * (kThreads / 32);
+    double rsum = 0.0;
+    for (int64_t c = blockIdx.x * (int64_t)(kThreads / 32) + threadIdx.x / 32; c < chunks;
+         c += warps) {
+        const int64_t e = c * 256 + lane * 8;
+        const bool in = e < total;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (in) v = __ldg(reinterpret_cast<const uint4 *>(W + e));
+        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+        float s = 0.f;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float lo = to_f32<kBF16>(w4[j] & 0xffffu);
+            const float hi = to_f32<kBF16>(w4[j] >> 16);
+            s = fmaf(lo, lo, s);
+            s = fmaf(hi, hi, s);
+        }
+        for (int m = 1; m < L; m *= 2) s += __shfl_xor_sync(0xffffffffu, s, m);
+        float k = 0.f;
+        if (in && (lane & (L - 1)) == 0)
+            k = finish_unit(s, eps, lambda2, alpha + e / g.bk, rsum);
+        k = __shfl_sync(0xffffffffu, k, lane & ~(L - 1));
+        if (in) {
+            float4 *d = reinterpret_cast<float4 *>(grad + e);
+            d[0] = make_float4(k * to_f32<kBF16>(v.x & 0xffffu), k * to_f32<kBF16>(v.x >> 16),
+                               k * to_f32<kBF16>(v.y & 0xffffu), k * to_f32<kBF16>(v.y >> 16));
+            d[1] = make_float4(k * to_f32<kBF16>(v.z & 0xffffu), k * to_f32<kBF16>(v.z >> 16),
+                               k * to_f32<kBF16>(v.w & 0xffffu), k * to_f32<kBF16>(v.w >> 16));
+        }
+    }
+    finish_R(rsum, lambda, part, count, R);
+}
+
+enum class Path { kTma, kLoop, kUnit, kRows, kRowsWarp };
 
 constexpr int kMaxBoxRows = 256;   // TMA box dimension limit
 
-Path path_of(const bp_layout &l) {
+Path path_of(const bp_layout &l, int groups) {
+    if (groups == BP_GROUPS_ROWS) {
+        const bool pow2 = (l.bk & (l.bk - 1)) == 0;
+        return l.bk % 8 == 0 && l.bk <= 256 && pow2 && l.K % l.bk == 0 ? Path::kRowsWarp
+                                                                     : Path::kRows;
+    }
     if (l.scheme != BP_BLOCK_BASED || l.K % 8 != 0) return Path::kUnit;
     return (l.bm < l.M ? l.bm : l.M) <= kMaxBoxRows ? Path::kTma : Path::kLoop;
 }
@@ -420,7 +530,7 @@ int box_width(int brows) {
     return bw;
 }
 
-Geo make_geo(const bp_layout &l) {
+Geo make_geo(const bp_layout &l, int groups) {
     Geo g{};
     g.M = (int)l.M;
     g.K = (int)l.K;
@@ -431,13 +541,13 @@ Geo make_geo(const bp_layout &l) {
     g.RB = (int)((l.M + l.bm - 1) / l.bm);
     if (l.scheme == BP_BLOCK_BASED) {
         g.CB = (g.K + l.bk - 1) / l.bk;
-        g.U = g.RB * g.K;
+        g.U = groups == BP_GROUPS_ROWS ? g.M * g.CB : g.RB * g.K;
     } else {
         g.CB = (g.C + l.bk - 1) / l.bk;
         g.U = g.RB * g.CB * g.KK;
     }
     const int brows = min(l.bm, g.M);
-    g.G = path_of(l) == Path::kTma ? box_width(brows) / 8 : 16;
+    g.G = path_of(l, groups) == Path::kTma ? box_width(brows) / 8 : 16;
     g.S = kThreads / g.G;
     g.TC = (g.K + 8 * g.G - 1) / (8 * g.G);
     g.tiles = g.RB * g.TC;
@@ -445,8 +555,12 @@ Geo make_geo(const bp_layout &l) {
 }
 
 // Upper bound of the grid (what the workspace is sized for).
-int max_grid(const bp_layout &l, const Geo &g) {
-    const int n = path_of(l) == Path::kUnit ? (g.U + kThreads - 1) / kThreads : g.tiles;
+int max_grid(const bp_layout &l, int groups, const Geo &g) {
+    const Path path = path_of(l, groups);
+    int n = g.tiles;
+    if (path == Path::kUnit || path == Path::kRows) n = (g.U + kThreads - 1) / kThreads;
+    if (path == Path::kRowsWarp)   // eight warps of 256 weights per block
+        n = (int)(((int64_t)g.M * g.K + 2047) / 2048);
     return max(1, min(n, kMaxBlocks));
 }
 
@@ -512,27 +626,40 @@ cudaError_t launch_tma(const bp_layout &lay, const Geo &g, const void *W, float 
         }
         per_sm = f->second;
     }
-    const int grid = max(1, min(max_grid(lay, g), per_sm * num_sms()));
+    const int grid = max(1, min(max_grid(lay, BP_GROUPS_LAYOUT, g), per_sm * num_sms()));
     k<<<grid, kThreads, smem, s>>>(a);
     return cudaGetLastError();
 }
 
 }  // namespace
 
-size_t penalty_workspace_bytes(const bp_layout &lay) {
-    return 256 + sizeof(double) * (size_t)max_grid(lay, make_geo(lay));
+size_t penalty_workspace_bytes(const bp_layout &lay, int groups) {
+    return 256 + sizeof(double) * (size_t)max_grid(lay, groups, make_geo(lay, groups));
 }
 
-cudaError_t launch_penalty(const bp_layout &lay, const void *W, double eps, double lambda,
-                           double *alpha, double *R, float *grad, void *ws, cudaStream_t s) {
-    const Geo g = make_geo(lay);
-    int grid = max_grid(lay, g);
+cudaError_t launch_penalty(const bp_layout &lay, int groups, const void *W, double eps,
+                           double lambda, double *alpha, double *R, float *grad, void *ws,
+                           cudaStream_t s) {
+    const Geo g = make_geo(lay, groups);
+    int grid = max_grid(lay, groups, g);
     unsigned *count = static_cast<unsigned *>(ws);
     double *part = reinterpret_cast<double *>(static_cast<char *>(ws) + 256);
     const uint16_t *w = static_cast<const uint16_t *>(W);
     const float eps_f = (float)eps, lambda2_f = (float)(2.0 * lambda);
     const bool bf = lay.dtype == BP_BF16;
-    switch (path_of(lay)) {
+    switch (path_of(lay, groups)) {
+    case Path::kRowsWarp: {
+        auto k = bf ? penalty_rows_warp_kernel<true> : penalty_rows_warp_kernel<false>;
+        k<<<grid, kThreads, 0, s>>>(g, eps_f, lambda2_f, lambda, w, alpha, grad, part, count, R);
+        break;
+    }
+    case Path::kRows: {
+        const bool vec = lay.bk % 8 == 0 && lay.K % 8 == 0;
+        auto k = bf ? (vec ? penalty_rows_kernel<true, true> : penalty_rows_kernel<true, false>)
+                    : (vec ? penalty_rows_kernel<false, true> : penalty_rows_kernel<false, false>);
+        k<<<grid, kThreads, 0, s>>>(g, eps_f, lambda2_f, lambda, w, alpha, grad, part, count, R);
+        break;
+    }
     case Path::kTma:
         return launch_tma(lay, g, W, eps_f, lambda2_f, lambda, alpha, grad, part, count, R, s);
     case Path::kLoop: {

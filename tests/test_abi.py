@@ -58,7 +58,7 @@ def test_ctypes_structs_match_header(tmp_path):
 def test_status_strings_and_version(lib):
     assert bp.status_string(bp.OK) == "ok"
     assert bp.status_string(bp.ERR_TIMEOUT) == "kernel wait timed out"
-    assert bp.bp_version() >> 16 == 2 and bp.bp_version() & 0xffff >= 1
+    assert bp.bp_version() >> 16 == 2 and bp.bp_version() & 0xffff >= 2
 
 
 def test_workspace_size_is_host_only(lib):
@@ -149,23 +149,34 @@ def test_penalty_argument_checks_on_host(lib):
     a = 1 << 20
     # eps must be positive and finite, lambda finite, W / grad 16-B aligned
     for eps, lam in ((0.0, 1.0), (-1.0, 1.0), (float("inf"), 1.0), (1e-4, float("nan"))):
-        assert bp.bp_reweighted_penalty(lay, a, eps, lam, a, a, a, a, 1 << 16, 0) == \
+        assert bp.bp_reweighted_penalty(lay, 0, a, eps, lam, a, a, a, a, 1 << 16, 0) == \
             bp.ERR_INVALID_ARG
-    assert bp.bp_reweighted_penalty(lay, a + 8, 1e-4, 1.0, a, a, a, a, 1 << 16, 0) == \
+    assert bp.bp_reweighted_penalty(lay, 0, a + 8, 1e-4, 1.0, a, a, a, a, 1 << 16, 0) == \
         bp.ERR_INVALID_ARG
-    assert bp.bp_reweighted_penalty(lay, a, 1e-4, 1.0, a, a, a + 4, a, 1 << 16, 0) == \
+    assert bp.bp_reweighted_penalty(lay, 0, a, 1e-4, 1.0, a, a, a + 4, a, 1 << 16, 0) == \
         bp.ERR_INVALID_ARG
     # outside the fp32 range of the factors
     for eps, lam in ((2.0 ** -61, 1.0), (2.0 ** 61, 1.0), (1e-18, 1e3)):
-        assert bp.bp_reweighted_penalty(lay, a, eps, lam, a, a, a, a, 1 << 16, 0) == \
+        assert bp.bp_reweighted_penalty(lay, 0, a, eps, lam, a, a, a, a, 1 << 16, 0) == \
             bp.ERR_UNSUPPORTED
     # missing, misaligned or short workspace
-    assert bp.bp_reweighted_penalty(lay, a, 1e-4, 1.0, a, a, a, None, 1 << 16, 0) == \
+    assert bp.bp_reweighted_penalty(lay, 0, a, 1e-4, 1.0, a, a, a, None, 1 << 16, 0) == \
         bp.ERR_WORKSPACE
-    assert bp.bp_reweighted_penalty(lay, a, 1e-4, 1.0, a, a, a, a + 16, 1 << 16, 0) == \
+    assert bp.bp_reweighted_penalty(lay, 0, a, 1e-4, 1.0, a, a, a, a + 16, 1 << 16, 0) == \
         bp.ERR_WORKSPACE
-    assert bp.bp_reweighted_penalty(lay, a, 1e-4, 1.0, a, a, a, a, 256 + 8 * 16 - 1, 0) == \
+    assert bp.bp_reweighted_penalty(lay, 0, a, 1e-4, 1.0, a, a, a, a, 256 + 8 * 16 - 1, 0) == \
         bp.ERR_WORKSPACE
+    # row groups (Eq. row): M x ceil(K / bk) segments; bk = 32 divides K: eight warps of
+    # 256 weights per block (64 blocks); bk = 7: one thread per segment (37 blocks)
+    assert bp.bp_penalty_units(lay, bp.GROUPS_ROWS) == (bp.OK, 256 * 16)
+    assert bp.bp_penalty_workspace_size(lay, bp.GROUPS_ROWS) == (bp.OK, 256 + 8 * 64)
+    lay7 = bp.layout(bp.BLOCK_BASED, bp.BF16, 128, 512, 128, 7)
+    assert bp.bp_penalty_units(lay7, bp.GROUPS_ROWS) == (bp.OK, 128 * 74)
+    assert bp.bp_penalty_workspace_size(lay7, bp.GROUPS_ROWS) == (bp.OK, 256 + 8 * 37)
+    assert bp.bp_penalty_units(play, bp.GROUPS_ROWS)[0] == bp.ERR_INVALID_ARG
+    assert bp.bp_penalty_units(lay, 2)[0] == bp.ERR_INVALID_ARG
+    assert bp.bp_reweighted_penalty(play, bp.GROUPS_ROWS, a, 1e-4, 1.0, a, a, a, a, 1 << 16, 0) \
+        == bp.ERR_INVALID_ARG
     # M*K >= 2^31 is outside the kernels' 32-bit indexing
     big = bp.layout(bp.BLOCK_BASED, bp.BF16, 1 << 16, 1 << 15, 128, 32)
     assert bp.bp_penalty_workspace_size(big)[0] == bp.ERR_UNSUPPORTED

@@ -34,24 +34,27 @@ CASES = [
 ]
 
 
-def unit_size(scheme, M, bm, bk):
+def unit_size(scheme, M, K, bm, bk, groups):
+    if groups == bp.GROUPS_ROWS:
+        return min(bk, K)
     return min(bm, M) * (1 if scheme == bp.BLOCK_BASED else bk)
 
 
-def check(case, W, eps, lam):
+def check(case, W, eps, lam, groups=bp.GROUPS_LAYOUT):
     scheme, dtype, M, K, kh, kw, bm, bk = case
     lay = bp.layout(scheme, dtype, M, K, bm, bk, kh, kw)
-    ws = bp.penalty_workspace(lay)
-    a, R, g = bp.penalty(lay, dev16(W, dtype), eps, lam, ws=ws)
+    ws = bp.penalty_workspace(lay, groups=groups)
+    a, R, g = bp.penalty(lay, dev16(W, dtype), eps, lam, ws=ws, groups=groups)
     torch.cuda.synchronize()
-    a0, R0, g0 = oracle.reweighted_penalty(W, dtype, scheme, bm, bk, eps, lam, kh, kw)
-    n = unit_size(scheme, M, bm, bk)
+    a0, R0, g0 = oracle.reweighted_penalty(W, dtype, scheme, bm, bk, eps, lam, kh, kw,
+                                           groups="rows" if groups == bp.GROUPS_ROWS else "layout")
+    n = unit_size(scheme, M, K, bm, bk, groups)
     np.testing.assert_allclose(a.cpu().numpy(), a0, rtol=(n + 2) * U32, atol=0)
     assert float(R.cpu()[0]) == pytest.approx(R0, rel=(n + 4) * U32, abs=0)
     np.testing.assert_allclose(g.cpu().numpy(), g0, rtol=(2 * n + 8) * U32, atol=1e-37)
     # the workspace comes back zeroed and the same call gives the same bits
     assert int(ws[:4].count_nonzero()) == 0
-    a2, R2, g2 = bp.penalty(lay, dev16(W, dtype), eps, lam, ws=ws)
+    a2, R2, g2 = bp.penalty(lay, dev16(W, dtype), eps, lam, ws=ws, groups=groups)
     assert torch.equal(a, a2) and torch.equal(R, R2) and torch.equal(g, g2)
     return a, R, g
 
@@ -80,3 +83,23 @@ def test_penalty_lambda_zero_and_negative():
     _, R, g = check(case, W, 1e-4, 0.0)
     assert float(R.cpu()[0]) == 0.0 and int(g.count_nonzero()) == 0
     check(case, W, 1e-4, -0.25)
+
+
+ROW_CASES = [
+    # dtype, M, K, bk
+    (bp.BF16, 256, 512, 16),
+    (bp.F16, 100, 200, 8),          # partial last column block (200 = 25 x 8, fine) and odd M
+    (bp.F16, 33, 70, 7),            # bk and K not multiples of 8: scalar path, partial block
+    (bp.BF16, 64, 4096, 4096),      # whole rows
+    (bp.F16, 40, 96, 40),           # partial last block of a vector-unfriendly width
+    (bp.BF16, 4096, 4096, 32),      # the benchmark's weight
+    (bp.BF16, 50, 512, 256),        # 32 lanes per segment
+    (bp.F16, 3, 40, 8),             # a partial warp chunk
+]
+
+
+@pytest.mark.parametrize("case", ROW_CASES, ids=lambda c: f"rows_{c[1]}x{c[2]}_bk{c[3]}")
+def test_row_penalty_matches_oracle(case):
+    dtype, M, K, bk = case
+    W = inputs.normal((M, K), 0.05, dtype, seed=5 * M + K)
+    check((bp.BLOCK_BASED, dtype, M, K, 1, 1, 4, bk), W, 1e-4, 0.75, groups=bp.GROUPS_ROWS)
