@@ -61,7 +61,13 @@ constexpr int kCtrlWarp = 8;
 constexpr int kMmaWarp = 9;
 constexpr int kEpiWarp0 = 10;
 constexpr int kThreads = (kEpiWarp0 + 4) * 32;
-constexpr uint32_t kGatherThreads = kGatherWarps * 32;
+// The gather warps form kGatherGroups groups that take turns: group g gathers
+// the chunks whose sequence number is g modulo kGatherGroups, so one group
+// issues copies while another waits for its next stage.
+constexpr int kGatherGroups = 2;
+constexpr int kGroupWarps = kGatherWarps / kGatherGroups;
+constexpr int kRowsPerWarp = 64 / kGroupWarps;      // list positions per warp and chunk
+constexpr uint32_t kGroupThreads = kGroupWarps * 32;
 
 struct Params {
     CUtensorMap ymap;       // GEMM output Y as a 2-D tensor, box 32 x 32, 64-byte swizzle
@@ -239,8 +245,7 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
     volatile int *abort_flag = s.abort_flag;
     Window win;
     win.first(p, kcp);
-    int stage = 0;
-    uint32_t phase = 0;
+    const int group = warp / kGroupWarps, gw = warp % kGroupWarps;
     int64_t count = 0, wseq = 0;
     bool ok = true;
     for (; win.valid(p) && ok; win.next(p, kcp), ++wseq) {
@@ -250,27 +255,38 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
                                               p.watchdog_ns, abort_flag));
         if (!ok) break;
         const uint8_t *recs = s.win + buf * kWinBytes;
-        for (int64_t j = 0; j < win.cnt; ++j) {
+        // the tile's token columns: 16 bytes (8 columns) per lane, lanes past
+        // the tile's width idle
+        const int64_t n = win.t.n0 + lane * 8;
+        const uint32_t nb =
+            (lane * 8 < p.nt && n < p.N) ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
+        const uint16_t *xcol = p.X + (nb ? n : 0);
+        // This warp's list positions of its next chunk are read from shared
+        // memory before the current chunk's copies are issued: the copies fill
+        // the load/store queue, and reads issued behind them would wait for it.
+        int32_t idx[kRowsPerWarp];
+        bool tma = false;
+        auto fetch = [&](int64_t j, int32_t (&ix)[kRowsPerWarp], bool &planned) {
             const uint8_t *rec = recs + j * kMetaBytes;
-            const bool tma = plan_loads(rec) > 0;
-            const int64_t seq = count++;
-            const bool drop = blockIdx.x == 0 && seq == p.drop_stage;
-            // source rows of this warp's 8 list positions, read before the stage is
-            // free: 16 bytes (8 columns) per lane, lanes past the tile's width idle
-            const uint16_t *src[kBK / kGatherWarps];
-            uint32_t nb = 0;
-            if (!tma) {
-                const int32_t *l = reinterpret_cast<const int32_t *>(rec);
-                const int64_t n = win.t.n0 + lane * 8;
-                nb = (lane * 8 < p.nt && n < p.N) ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
-                const uint16_t *xcol = p.X + (nb ? n : 0);
+            planned = plan_loads(rec) > 0;
+            const int32_t *l = reinterpret_cast<const int32_t *>(rec);
 #pragma unroll
-                for (int i = 0; i < kBK / kGatherWarps; ++i)
-                    src[i] = xcol + (int64_t)l[warp + kGatherWarps * i] * p.ldx;
-            }
+            for (int i = 0; i < kRowsPerWarp; ++i) ix[i] = l[gw + kGroupWarps * i];
+        };
+        const int64_t base = count;         // sequence number of the window's first chunk
+        int64_t j = (group - base % kGatherGroups + kGatherGroups) % kGatherGroups;
+        if (j < win.cnt) fetch(j, idx, tma);
+        for (; j < win.cnt; j += kGatherGroups) {
+            int32_t nidx[kRowsPerWarp];
+            bool ntma = false;
+            if (j + kGatherGroups < win.cnt) fetch(j + kGatherGroups, nidx, ntma);
+            const int64_t seq = base + j;
+            const int stage = (int)(seq % p.stages);
+            const uint32_t phase = (uint32_t)((seq / p.stages) & 1);
+            const bool drop = blockIdx.x == 0 && seq == p.drop_stage;
             // A planned chunk is loaded and signalled by the control thread; the
-            // warp still waits for its stage (lane 0 alone), which keeps it at most
-            // one phase of the stage barriers ahead of the tensor cores.
+            // group still waits for its stage (lane 0 alone), which keeps it at
+            // most one phase of the stage barriers ahead of the tensor cores.
             ok = __all_sync(0xffffffffu,
                             (!tma || lane == 0)
                                 ? mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)
@@ -282,9 +298,10 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
                 const int cn = lane >> 3, jj = lane & 7;
                 if (lane * 8 < p.nt) {
 #pragma unroll
-                    for (int i = 0; i < kBK / kGatherWarps; ++i) {
-                        const int r = warp + kGatherWarps * i;
-                        cp_async_16(xs + cn * 8192 + r * 128 + ((jj ^ (r & 7)) << 4), src[i], nb);
+                    for (int i = 0; i < kRowsPerWarp; ++i) {
+                        const int r = gw + kGroupWarps * i;
+                        cp_async_16(xs + cn * 8192 + r * 128 + ((jj ^ (r & 7)) << 4),
+                                    xcol + (int64_t)idx[i] * p.ldx, nb);
                     }
                 }
                 // Signal the stage once this thread's copies have landed, without
@@ -293,11 +310,11 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
                 // proxy fence after acquiring the barrier.
                 cp_async_arrive_noinc(&s.full[stage]);
             }
-            if (++stage == p.stages) {
-                stage = 0;
-                phase ^= 1u;
-            }
+#pragma unroll
+            for (int i = 0; i < kRowsPerWarp; ++i) idx[i] = nidx[i];
+            tma = ntma;
         }
+        count = base + win.cnt;
         if (!ok) break;
         __syncwarp();        // the lanes' reads of the window precede lane 0's release
         if (lane == 0) mbar_arrive(&s.pempty[buf]);
@@ -695,7 +712,7 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     const int warp = threadIdx.x >> 5;
     if (threadIdx.x == 0) {
         for (int i = 0; i < p.stages; ++i) {
-            mbar_init(&s.full[i], kGatherThreads);
+            mbar_init(&s.full[i], kGroupThreads);
             mbar_init(&s.wfull[i], 1);
             mbar_init(&s.empty[i], 1);
         }
