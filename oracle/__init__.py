@@ -79,9 +79,11 @@ def _load():
                                                       dbl, dbl, vp, vp, vp]
             lib.oracle_reweighted_penalty_rows.argtypes = [i32, i64, i64, i64, vp, dbl, dbl, vp,
                                                            vp, vp]
+            lib.oracle_prune_rows.argtypes = [i32, i64, i64, i64, i64, dbl, vp, vp, vp]
             lib.oracle_max_threads.restype = i32
             for f in ("oracle_scores", "oracle_reweighted_penalty",
                       "oracle_reweighted_penalty_rows", "oracle_counts", "oracle_prune",
+                      "oracle_prune_rows",
                       "oracle_pack",
                       "oracle_unpack", "oracle_masked_gemm", "oracle_masked_conv2d"):
                 getattr(lib, f).restype = i32
@@ -194,6 +196,20 @@ def prune(W_bits, dtype, scheme, bm, bk, rate, kh=1, kw=1, return_keep=False):
     _check(_load().oracle_prune(scheme, dtype, M, K, kh, kw, bm, bk, float(rate), _p(W),
                                 _p(keep), _p(mask)))
     return (mask, keep) if return_keep else mask
+
+
+def prune_rows(W_bits, dtype, bm, bk, rate, mask=None, return_keep=False):
+    """Row pruning of a block-based layer (rows of each bm x bk block), ANDed
+    into `mask` (all ones when None); returns the new M x K uint8 mask (and
+    the row-unit flags, numbered block-major then by row)."""
+    W = _u16(W_bits)
+    M, K = W.shape
+    CB = (K + bk - 1) // bk
+    m = (np.ones((M, K), np.uint8) if mask is None
+         else np.array(mask, dtype=np.uint8, copy=True).reshape(M, K))
+    keep = np.empty(M * CB, np.uint8)
+    _check(_load().oracle_prune_rows(dtype, M, K, bm, bk, float(rate), _p(W), _p(keep), _p(m)))
+    return (m, keep) if return_keep else m
 
 
 def pack(W_bits, mask, bm):

@@ -390,6 +390,76 @@ done:
     return st;
 }
 
+/* Row pruning of block-based layers (Sec. 4.1.1: rows and columns of each
+ * block are pruned independently; Eq. row names the row groups).  The units
+ * of block (rb, cb) are its rows r, i.e. the segments
+ * W[r, cb*bk .. min(cb*bk + bk, K) - 1], scored by their squared norm in
+ * fp64 with k ascending.  Counts as for column units: a block of P rows keeps
+ * floor(P / rate) units, the layer keeps T = floor(M*CB / rate + 0.5) units,
+ * and the T - sum(floor(P / rate)) extras go to the best remaining units of
+ * the whole layer.  Units are numbered block-major and then by row,
+ * g = rb*bm*CB + cb*rows_rb + (r - rb*bm) (rows_rb = real rows of rb), which is
+ * also the tie order.  The row keep is ANDed into mask: an element survives
+ * when its row unit survives and mask already held it (for example the column
+ * mask of oracle_prune).  keep (optional, M*CB) receives the row-unit flags. */
+int oracle_prune_rows(int dtype, int64_t M, int64_t K, int64_t bm, int64_t bk, double rate,
+                      const uint16_t *W, uint8_t *keep, uint8_t *mask)
+{
+    if (M < 1 || K < 1 || bm < 1 || bk < 1) return OR_ERR_ARG;
+    if (!(rate >= 1.0) || !isfinite(rate)) return OR_ERR_ARG;
+    const int64_t RB = (M + bm - 1) / bm, CB = (K + bk - 1) / bk, U = M * CB;
+    double *s = (double *)malloc((size_t)U * sizeof(double));
+    cand_t *blk = (cand_t *)malloc((size_t)bm * sizeof(cand_t));
+    cand_t *rest = (cand_t *)malloc((size_t)U * sizeof(cand_t));
+    uint8_t *kp = keep ? keep : (uint8_t *)malloc((size_t)U);
+    int st = OR_OK;
+    memset(kp, 0, (size_t)U);
+    int64_t nrest = 0, sum_base = 0;
+    for (int64_t rb = 0; rb < RB; ++rb) {
+        const int64_t r0 = rb * bm, rows = (r0 + bm <= M) ? bm : M - r0;
+        for (int64_t cb = 0; cb < CB; ++cb) {
+            const int64_t first = r0 * CB + cb * rows;
+            for (int64_t i = 0; i < rows; ++i) {
+                double acc = 0.0;
+                for (int64_t k = cb * bk; k < K && k < cb * bk + bk; ++k) {
+                    double w = oracle_half_to_double(W[(r0 + i) * K + k], dtype);
+                    if (!isfinite(w)) { st = OR_ERR_NONFINITE; goto done; }
+                    acc += w * w;
+                }
+                s[first + i] = acc;
+                blk[i].s = acc; blk[i].g = first + i;
+            }
+            const int64_t base = (int64_t)floor((double)rows / rate);
+            sum_base += base;
+            qsort(blk, (size_t)rows, sizeof(cand_t), cand_cmp);
+            for (int64_t i = 0; i < rows; ++i) {
+                if (i < base) kp[blk[i].g] = 1;
+                else rest[nrest++] = blk[i];
+            }
+        }
+    }
+    {
+        const int64_t T = (int64_t)floor((double)U / rate + 0.5);
+        const int64_t E = T - sum_base;
+        qsort(rest, (size_t)nrest, sizeof(cand_t), cand_cmp);
+        for (int64_t i = 0; i < E && i < nrest; ++i) kp[rest[i].g] = 1;
+    }
+    if (mask) {
+        for (int64_t r = 0; r < M; ++r) {
+            const int64_t rb = r / bm, r0 = rb * bm, rows = (r0 + bm <= M) ? bm : M - r0;
+            for (int64_t k = 0; k < K; ++k) {
+                const int64_t cb = k / bk;
+                const int64_t g = r0 * CB + cb * rows + (r - r0);
+                mask[r * K + k] = (uint8_t)(mask[r * K + k] && kp[g]);
+            }
+        }
+    }
+done:
+    free(s); free(blk); free(rest);
+    if (!keep) free(kp);
+    return st;
+}
+
 /* Compact storage (BCS, Sec. 4.3).  Because every row of a row-block keeps
  * the same columns, one column list serves the whole row-block (the
  * "occurrence" rows rb*bm .. rb*bm+bm_rb-1):
