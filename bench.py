@@ -544,6 +544,52 @@ def run_workload(args):
         layers, dtype = inputs.vgg16_cifar(), inputs.F16
     elif name == "resnet50":
         layers, dtype = inputs.resnet50_imagenet(), inputs.BF16
+    elif name == "rowcol":
+        # row + column pruning of the 4096^3 bf16 layer (128 x 32 blocks):
+        # columns at 2x and rows at 2x (independent, ~4x in weights), against
+        # columns alone at 4x and the dense layer
+        from paper_2111_11581_gb300 import bp
+        L = inputs.gemm_point(4096, 4096, 4096, 128, 32, 4.0, inputs.BF16)
+        W = inputs.layer_weight(L, inputs.BF16)
+        Wd = inputs.as_torch(W, inputs.BF16).cuda()
+        xd = inputs.as_torch(inputs.layer_input(L, inputs.BF16), inputs.BF16).cuda()
+        lay = bp.layout(bp.BLOCK_BASED, bp.BF16, 4096, 4096, 128, 32)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+
+        def timed(fn, reps=5):
+            ts = []
+            for _ in range(reps + 1):
+                flush.zero_()
+                ev[0].record()
+                fn()
+                ev[1].record()
+                torch.cuda.synchronize()
+                ts.append(ev[0].elapsed_time(ev[1]) * 1e3)
+            return statistics.median(ts[1:])
+
+        res = {}
+        for tag, mask, play in (
+                ("columns_4x", bp.prune(lay, Wd, 4.0), lay),
+                ("rows_2x_columns_2x", bp.prune_rows(lay, Wd, 2.0, bp.prune(lay, Wd, 2.0)),
+                 bp.layout(bp.BLOCK_BASED, bp.BF16, 4096, 4096, 1, 32))):
+            pw = bp.pack(play, Wd, mask)
+            y = bp.gemm(pw, xd)
+            us = timed(lambda: bp.gemm(pw, xd, out=y))
+            kept = int(pw.c.nnz_vals)
+            # k-chunks of 64 columns over the 32 slabs of 128 rows (kc_ptr[32])
+            chunks = int(pw.dev[8 * 32:8 * 33].view(torch.int64)[0])
+            res[tag] = {"kept_weights": kept, "us": round(us, 2),
+                        "effective_tflops": round(2.0 * kept * 4096 / us / 1e6, 1),
+                        "tensor_core_columns_per_slab": chunks * 64 // 32,
+                        "mma_tflops": round(2.0 * 128 * 64 * chunks * 4096 / us / 1e6, 1)}
+        res["dense_us"] = round(timed(lambda: torch.matmul(Wd, xd)), 2)
+        if bp.device_status() != bp.OK:
+            raise RuntimeError("kernel watchdog fired")
+        print(json.dumps({"workload": "rowcol", "shape": [4096, 4096, 4096], "bm": 128,
+                          "bk": 32, **res,
+                          "timing": "device time, median of 5, L2 flushed before each"}),
+              flush=True)
+        return
     elif name == "sweep":
         layers, dtype = [], None
         for dt in (inputs.BF16, inputs.F16):
@@ -587,7 +633,8 @@ def main():
     ap.add_argument("--workload", default=None,
                     help="fc512 | conv3x3 | vgg16 | resnet50 | sweep: per-layer timings "
                          "of another workload (one JSON line), instead of the default step; "
-                         "blocksize: the latency model and block-size selection")
+                         "blocksize: the latency model and block-size selection; penalty: "
+                         "the reweighted regulariser; rowcol: row + column pruning")
     ap.add_argument("--sweep-subset", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:

@@ -104,7 +104,8 @@ const char *bp_status_string(int status);
 /* Library ABI version: (major << 16) | minor. */
 int bp_version(void);
 
-/* Device workspace bytes bp_prune needs for `lay` (host output). */
+/* Device workspace bytes bp_prune needs for `lay` (host output); for
+ * block-based layouts the same workspace also serves bp_prune_rows. */
 bp_status bp_workspace_size(const bp_layout *lay, size_t *bytes);
 
 /* One-shot magnitude pruning by block (Sec. 5.1 with the block regularities
@@ -124,6 +125,22 @@ bp_status bp_workspace_size(const bp_layout *lay, size_t *bytes);
  * weight is Inf/NaN (mask then undefined). */
 bp_status bp_prune(const bp_layout *lay, const void *W, double rate, uint8_t *mask, void *ws,
                    size_t ws_bytes, void *stream);
+
+/* Row pruning of a block-based layer (Sec. 4.1.1: the rows and the columns of
+ * each block are pruned independently; the rows are the groups of Eq. row).
+ * The units of block (rb, cb) are its rows r -- the segments
+ * W[r, cb*bk .. min(cb*bk + bk, K) - 1] -- scored by their squared norm in fp64
+ * (columns ascending) and selected as bp_prune selects columns: floor(P_b / r)
+ * per block of P_b rows, plus the best remaining units of the layer up to
+ * T = floor(M * ceil(K/bk) / r + 0.5).  Units are ordered block-major (row-block,
+ * then column-block), then by row; ties prefer the lower.  The result is ANDed
+ * into `mask` (device, M x K uint8, in/out), so bp_prune followed by
+ * bp_prune_rows, both on the same W, gives independent row and column pruning.
+ * Rows of a row-block then keep different columns: pack such a mask with
+ * bm = 1 (every row its own list).  Same workspace, synchronisation and errors
+ * as bp_prune; BP_ERR_INVALID_ARG for block-punched layouts. */
+bp_status bp_prune_rows(const bp_layout *lay, const void *W, double rate, uint8_t *mask,
+                        void *ws, size_t ws_bytes, void *stream);
 
 /* First half of packing: checks that every row of each row-block keeps the
  * same columns as the row-block's first row (BP_ERR_INVALID_ARG otherwise)

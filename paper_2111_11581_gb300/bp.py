@@ -34,9 +34,10 @@ class Packed(ctypes.Structure):
                 ("dev", ctypes.c_void_p), ("dev_bytes", ctypes.c_int64)]
 
 
-EXPORTS = ("bp_status_string", "bp_version", "bp_workspace_size", "bp_prune", "bp_pack_size",
-           "bp_pack", "bp_gemm", "bp_gemm_workspace_size", "bp_conv2d", "bp_conv2d_workspace_size",
-           "bp_penalty_units", "bp_reweighted_penalty", "bp_penalty_workspace_size", "bp_device_status", "bp_set_watchdog_ns",
+EXPORTS = ("bp_status_string", "bp_version", "bp_workspace_size", "bp_prune", "bp_prune_rows",
+           "bp_pack_size", "bp_pack", "bp_gemm", "bp_gemm_workspace_size", "bp_conv2d",
+           "bp_conv2d_workspace_size", "bp_penalty_units", "bp_reweighted_penalty",
+           "bp_penalty_workspace_size", "bp_device_status", "bp_set_watchdog_ns",
            "bp_debug_drop_stage", "bp_prune_noalloc")
 
 _lib = None
@@ -67,6 +68,7 @@ def load(path: str = LIB_PATH):
             "bp_version": (i32, []),
             "bp_workspace_size": (i32, [P_L, ctypes.POINTER(sz)]),
             "bp_prune": (i32, [P_L, vp, dbl, vp, vp, sz, vp]),
+            "bp_prune_rows": (i32, [P_L, vp, dbl, vp, vp, sz, vp]),
             "bp_pack_size": (i32, [P_L, vp, vp, P_i64, P_i64, P_i64, vp]),
             "bp_pack": (i32, [P_L, vp, vp, P_P, vp]),
             "bp_gemm": (i32, [P_P, vp, i64, i64, vp, i32, vp, i64, vp, sz, vp]),
@@ -113,6 +115,11 @@ def bp_workspace_size(lay: Layout) -> int:
 def bp_prune(lay: Layout, W: int, rate: float, mask: int, ws: int, ws_bytes: int,
              stream: int = 0) -> int:
     return load().bp_prune(ctypes.byref(lay), W, float(rate), mask, ws, ws_bytes, stream)
+
+
+def bp_prune_rows(lay: Layout, W: int, rate: float, mask: int, ws: int, ws_bytes: int,
+                  stream: int = 0) -> int:
+    return load().bp_prune_rows(ctypes.byref(lay), W, float(rate), mask, ws, ws_bytes, stream)
 
 
 def bp_pack_size(lay: Layout, mask: int, rb_ptr: int, stream: int = 0):
@@ -221,6 +228,19 @@ def prune(lay: Layout, W, rate: float, stream=None):
     ws = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=W.device)
     _chk(bp_prune(lay, W.data_ptr(), rate, mask.data_ptr(), ws.data_ptr(), nbytes, _stream(stream)),
          "bp_prune")
+    return mask
+
+
+def prune_rows(lay: Layout, W, rate: float, mask=None, stream=None):
+    """Row pruning (bp_prune_rows) ANDed into `mask` (a new all-ones mask when
+    None); returns the mask."""
+    torch = _torch()
+    if mask is None:
+        mask = torch.ones((lay.M, lay.K), dtype=torch.uint8, device=W.device)
+    nbytes = bp_workspace_size(lay)
+    ws = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=W.device)
+    _chk(bp_prune_rows(lay, W.data_ptr(), rate, mask.data_ptr(), ws.data_ptr(), nbytes,
+                       _stream(stream)), "bp_prune_rows")
     return mask
 
 

@@ -61,6 +61,16 @@ Counts host_counts(const bp_layout &l, double rate) {
     const int64_t RB = cdiv(l.M, l.bm);
     const int64_t KK = (int64_t)l.kh * l.kw;
     int64_t per_rb_base = 0, per_rb_units = 0;
+    if (l.scheme == kSchemeRows) {
+        // row units: every block of row-block rb has rows_rb units
+        const int64_t CB = cdiv(l.K, l.bk), last = l.M - (RB - 1) * l.bm;
+        c.U = l.M * CB;
+        c.sum_base = CB * ((RB - 1) * (int64_t)std::floor((double)l.bm / rate) +
+                           (int64_t)std::floor((double)last / rate));
+        c.T = (int64_t)std::floor((double)c.U / rate + 0.5);
+        c.E = c.T - c.sum_base;
+        return c;
+    }
     if (l.scheme == BP_BLOCK_BASED) {
         const int64_t full = l.K / l.bk, tail = l.K % l.bk;
         per_rb_base = full * (int64_t)std::floor((double)l.bk / rate) +
@@ -85,7 +95,13 @@ struct PruneWs {
 int64_t align_up(int64_t v, int64_t a) { return (v + a - 1) / a * a; }
 
 PruneWs prune_ws(const bp_layout &l) {
-    const Counts c = host_counts(l, 1.0);
+    Counts c = host_counts(l, 1.0);
+    if (l.scheme == BP_BLOCK_BASED) {
+        // one workspace serves bp_prune and bp_prune_rows
+        bp_layout rows = l;
+        rows.scheme = (bp_scheme)kSchemeRows;
+        c.U = std::max(c.U, host_counts(rows, 1.0).U);
+    }
     PruneWs w;
     w.off_scores = 0;
     w.off_hist = align_up(c.U * 8, 256);
@@ -94,6 +110,53 @@ PruneWs prune_ws(const bp_layout &l) {
     w.off_keep = w.off_flag + 256;
     w.total = align_up(w.off_keep + c.U, 256);
     return w;
+}
+
+// The pruning pipeline over the units of `lay` (scheme may be kSchemeRows):
+// scores, per-block keep, layer-wide extras by radix select, mask.
+bp_status prune_units(const bp_layout &lay, const void *W, double rate, uint8_t *mask,
+                      void *ws, const PruneWs &w, cudaStream_t s) {
+    uint8_t *base = static_cast<uint8_t *>(ws);
+    double *scores = reinterpret_cast<double *>(base + w.off_scores);
+    unsigned *hist = reinterpret_cast<unsigned *>(base + w.off_hist);
+    int64_t *chunks = reinterpret_cast<int64_t *>(base + w.off_chunks);
+    int *flag = reinterpret_cast<int *>(base + w.off_flag);
+    uint8_t *keep = base + w.off_keep;
+    const Counts c = host_counts(lay, rate);
+
+    cudaError_t e = cudaMemsetAsync(flag, 0, sizeof(int), s);
+    if (e == cudaSuccess) e = launch_scores(lay, W, scores, flag, s);
+    if (e == cudaSuccess) e = launch_base_select(lay, scores, rate, keep, s);
+    int nonfinite = 0;
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&nonfinite, flag, sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return BP_ERR_CUDA;
+    if (nonfinite) return BP_ERR_NONFINITE;
+
+    if (c.E > 0) {
+        // most-significant-digit radix select of the E-th best remaining unit
+        uint64_t prefix = 0;
+        int64_t need = c.E;
+        unsigned h[256];
+        for (int shift = 56; shift >= 0; shift -= 8) {
+            e = cudaMemsetAsync(hist, 0, 256 * sizeof(unsigned), s);
+            if (e == cudaSuccess) e = launch_radix_hist(c.U, scores, keep, prefix, shift, hist, s);
+            if (e == cudaSuccess) e = cudaMemcpyAsync(h, hist, sizeof(h), cudaMemcpyDeviceToHost, s);
+            if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+            if (e != cudaSuccess) return BP_ERR_CUDA;
+            int d = 255;
+            for (; d > 0; --d) {
+                if ((int64_t)h[d] >= need) break;
+                need -= h[d];
+            }
+            prefix |= (uint64_t)d << shift;
+        }
+        e = launch_threshold_select(c.U, scores, keep, prefix, need, chunks, s);
+        if (e != cudaSuccess) return BP_ERR_CUDA;
+    }
+    e = launch_write_mask(lay, keep, mask, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    return cuda_status(e);
 }
 
 }  // namespace
@@ -189,7 +252,7 @@ const char *bp_status_string(int status) {
     }
 }
 
-int bp_version(void) { return (2 << 16) | 2; }
+int bp_version(void) { return (2 << 16) | 3; }
 
 bp_status bp_workspace_size(const bp_layout *lay, size_t *bytes) {
     if (!layout_ok(lay) || !bytes) return BP_ERR_INVALID_ARG;
@@ -204,48 +267,20 @@ bp_status bp_prune(const bp_layout *lay, const void *W, double rate, uint8_t *ma
     const PruneWs w = prune_ws(*lay);
     if (!ws || ws_bytes < (size_t)w.total || (reinterpret_cast<uintptr_t>(ws) & 255u))
         return BP_ERR_WORKSPACE;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    uint8_t *base = static_cast<uint8_t *>(ws);
-    double *scores = reinterpret_cast<double *>(base + w.off_scores);
-    unsigned *hist = reinterpret_cast<unsigned *>(base + w.off_hist);
-    int64_t *chunks = reinterpret_cast<int64_t *>(base + w.off_chunks);
-    int *flag = reinterpret_cast<int *>(base + w.off_flag);
-    uint8_t *keep = base + w.off_keep;
-    const Counts c = host_counts(*lay, rate);
+    return prune_units(*lay, W, rate, mask, ws, w, static_cast<cudaStream_t>(stream));
+}
 
-    cudaError_t e = cudaMemsetAsync(flag, 0, sizeof(int), s);
-    if (e == cudaSuccess) e = launch_scores(*lay, W, scores, flag, s);
-    if (e == cudaSuccess) e = launch_base_select(*lay, scores, rate, keep, s);
-    int nonfinite = 0;
-    if (e == cudaSuccess) e = cudaMemcpyAsync(&nonfinite, flag, sizeof(int), cudaMemcpyDeviceToHost, s);
-    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-    if (e != cudaSuccess) return BP_ERR_CUDA;
-    if (nonfinite) return BP_ERR_NONFINITE;
-
-    if (c.E > 0) {
-        // most-significant-digit radix select of the E-th best remaining unit
-        uint64_t prefix = 0;
-        int64_t need = c.E;
-        unsigned h[256];
-        for (int shift = 56; shift >= 0; shift -= 8) {
-            e = cudaMemsetAsync(hist, 0, 256 * sizeof(unsigned), s);
-            if (e == cudaSuccess) e = launch_radix_hist(c.U, scores, keep, prefix, shift, hist, s);
-            if (e == cudaSuccess) e = cudaMemcpyAsync(h, hist, sizeof(h), cudaMemcpyDeviceToHost, s);
-            if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-            if (e != cudaSuccess) return BP_ERR_CUDA;
-            int d = 255;
-            for (; d > 0; --d) {
-                if ((int64_t)h[d] >= need) break;
-                need -= h[d];
-            }
-            prefix |= (uint64_t)d << shift;
-        }
-        e = launch_threshold_select(c.U, scores, keep, prefix, need, chunks, s);
-        if (e != cudaSuccess) return BP_ERR_CUDA;
-    }
-    e = launch_write_mask(*lay, keep, mask, s);
-    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-    return cuda_status(e);
+bp_status bp_prune_rows(const bp_layout *lay, const void *W, double rate, uint8_t *mask,
+                        void *ws, size_t ws_bytes, void *stream) {
+    if (!layout_ok(lay) || !W || !mask || lay->scheme != BP_BLOCK_BASED)
+        return BP_ERR_INVALID_ARG;
+    if (!(rate >= 1.0) || !std::isfinite(rate)) return BP_ERR_INVALID_ARG;
+    const PruneWs w = prune_ws(*lay);
+    if (!ws || ws_bytes < (size_t)w.total || (reinterpret_cast<uintptr_t>(ws) & 255u))
+        return BP_ERR_WORKSPACE;
+    bp_layout rows = *lay;
+    rows.scheme = (bp_scheme)kSchemeRows;
+    return prune_units(rows, W, rate, mask, ws, w, static_cast<cudaStream_t>(stream));
 }
 
 bp_status bp_pack_size(const bp_layout *lay, const uint8_t *mask, int64_t *rb_ptr,

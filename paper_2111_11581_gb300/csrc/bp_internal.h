@@ -11,6 +11,10 @@
 
 namespace bp {
 
+// Internal scheme value of the prune kernels: the row units of a block-based
+// layout (rows of each bm x bk block; written into the mask with AND).
+constexpr int kSchemeRows = 2;
+
 // Device status bits recorded by kernels (read by bp_device_status).
 constexpr unsigned kDevTimeout = 1u;
 

@@ -3,8 +3,12 @@
 // the remaining best units (a most-significant-digit radix select on the
 // fp64 score bits, ties to the lower unit index), then the element mask.
 //
-// Units are numbered g = (rb*CB + cb)*P + u for block-punched layers and
-// g = rb*K + column for block-based ones, which is also the tie order.
+// Units are numbered g = (rb*CB + cb)*P + u for block-punched layers,
+// g = rb*K + column for block-based ones, and, for the row units of
+// block-based layers, g = rb*bm*CB + cb*rows_rb + (r - rb*bm) (rows_rb = real
+// rows of row-block rb: block-major, then row); the numbering is also the tie
+// order.
+
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -31,11 +35,31 @@ Part make_part(const bp_layout &l) {
     if (l.scheme == BP_BLOCK_BASED) {
         p.CB = (l.K + l.bk - 1) / l.bk;
         p.U = p.RB * l.K;
+    } else if (l.scheme == kSchemeRows) {
+        p.CB = (l.K + l.bk - 1) / l.bk;
+        p.U = l.M * p.CB;
     } else {
         p.CB = (p.C + l.bk - 1) / l.bk;
         p.U = p.RB * p.CB * p.KK;
     }
     return p;
+}
+
+// Row unit g of a block-based layer -> (row, column-block), and the first
+// unit and size of its block.
+struct RowUnit {
+    int64_t r, cb, first, P;
+};
+__device__ __forceinline__ RowUnit row_unit(const Part &p, int64_t g) {
+    const int64_t rb = g / (p.bm * p.CB), r0 = rb * p.bm;
+    const int64_t rows = min(p.bm, p.M - r0);
+    const int64_t rem = g - r0 * p.CB, cb = rem / rows;
+    RowUnit u;
+    u.r = r0 + (rem - cb * rows);
+    u.cb = cb;
+    u.first = r0 * p.CB + cb * rows;
+    u.P = rows;
+    return u;
 }
 
 __device__ __forceinline__ float ld_half(const uint16_t *w, int64_t i, int dtype) {
@@ -57,6 +81,16 @@ __global__ void scores_kernel(Part p, int dtype, const uint16_t *__restrict__ W,
             const int64_t r0 = rb * p.bm, r1 = min(r0 + p.bm, p.M);
             for (int64_t r = r0; r < r1; ++r) {
                 const float f = ld_half(W, r * p.K + j, dtype);
+                bad |= !isfinite(f);
+                const double w = (double)f;
+                s += w * w;
+            }
+        } else if (p.scheme == kSchemeRows) {
+            // the row's segment in its column-block, columns ascending
+            const RowUnit u = row_unit(p, g);
+            const int64_t k0 = u.cb * p.bk, k1 = min(k0 + p.bk, p.K);
+            for (int64_t k = k0; k < k1; ++k) {
+                const float f = ld_half(W, u.r * p.K + k, dtype);
                 bad |= !isfinite(f);
                 const double w = (double)f;
                 s += w * w;
@@ -90,6 +124,10 @@ __global__ void base_select_kernel(Part p, double rate, const double *__restrict
             const int64_t rb = g / p.K, j = g % p.K, cb = j / p.bk;
             first = rb * p.K + cb * p.bk;
             P = min(p.bk, p.K - cb * p.bk);
+        } else if (p.scheme == kSchemeRows) {
+            const RowUnit u = row_unit(p, g);
+            first = u.first;
+            P = u.P;
         } else {
             first = (g / p.KK) * p.KK;
             P = p.KK;
@@ -218,6 +256,12 @@ __global__ void write_mask_kernel(Part p, const uint8_t *__restrict__ keep,
         int64_t g;
         if (p.scheme == BP_BLOCK_BASED) {
             g = rb * p.K + k;
+        } else if (p.scheme == kSchemeRows) {
+            // row units are ANDed into the mask already there
+            const int64_t r0 = rb * p.bm, rows = min(p.bm, p.M - r0), cb = k / p.bk;
+            g = r0 * p.CB + cb * rows + (r - r0);
+            if (!keep[g]) mask[i] = 0;
+            continue;
         } else {
             const int64_t c = k / p.KK, pos = k % p.KK;
             g = (rb * p.CB + c / p.bk) * p.KK + pos;

@@ -58,7 +58,7 @@ def test_ctypes_structs_match_header(tmp_path):
 def test_status_strings_and_version(lib):
     assert bp.status_string(bp.OK) == "ok"
     assert bp.status_string(bp.ERR_TIMEOUT) == "kernel wait timed out"
-    assert bp.bp_version() >> 16 == 2 and bp.bp_version() & 0xffff >= 2
+    assert bp.bp_version() >> 16 == 2 and bp.bp_version() & 0xffff >= 3
 
 
 def test_workspace_size_is_host_only(lib):
@@ -180,3 +180,16 @@ def test_penalty_argument_checks_on_host(lib):
     # M*K >= 2^31 is outside the kernels' 32-bit indexing
     big = bp.layout(bp.BLOCK_BASED, bp.BF16, 1 << 16, 1 << 15, 128, 32)
     assert bp.bp_penalty_workspace_size(big)[0] == bp.ERR_UNSUPPORTED
+
+
+def test_prune_rows_argument_checks_on_host(lib):
+    lay = bp.layout(bp.BLOCK_BASED, bp.F16, 256, 64, 128, 8)
+    # one workspace serves both: row units (256 x 8 = 2048) outnumber column units (2 x 64)
+    n = bp.bp_workspace_size(lay)
+    lay_cols_only = bp.layout(bp.BLOCK_BASED, bp.F16, 256, 64, 128, 128)
+    assert n >= 2048 * 8 + 2048 and n > bp.bp_workspace_size(lay_cols_only)
+    a = 1 << 20
+    assert bp.bp_prune_rows(lay, a, 0.5, a, a, n, 0) == bp.ERR_INVALID_ARG
+    assert bp.bp_prune_rows(lay, a, 2.0, a, a, n - 1, 0) == bp.ERR_WORKSPACE
+    play = bp.layout(bp.BLOCK_PUNCHED, bp.F16, 16, 8 * 9, 8, 4, 3, 3)
+    assert bp.bp_prune_rows(play, a, 2.0, a, a, 1 << 20, 0) == bp.ERR_INVALID_ARG
