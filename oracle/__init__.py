@@ -80,10 +80,11 @@ def _load():
             lib.oracle_reweighted_penalty_rows.argtypes = [i32, i64, i64, i64, vp, dbl, dbl, vp,
                                                            vp, vp]
             lib.oracle_prune_rows.argtypes = [i32, i64, i64, i64, i64, dbl, vp, vp, vp]
+            lib.oracle_prune_pattern.argtypes = [i32, i64, i64, vp, i32, dbl, vp, vp, vp]
             lib.oracle_max_threads.restype = i32
             for f in ("oracle_scores", "oracle_reweighted_penalty",
                       "oracle_reweighted_penalty_rows", "oracle_counts", "oracle_prune",
-                      "oracle_prune_rows",
+                      "oracle_prune_rows", "oracle_prune_pattern",
                       "oracle_pack",
                       "oracle_unpack", "oracle_masked_gemm", "oracle_masked_conv2d"):
                 getattr(lib, f).restype = i32
@@ -210,6 +211,37 @@ def prune_rows(W_bits, dtype, bm, bk, rate, mask=None, return_keep=False):
     keep = np.empty(M * CB, np.uint8)
     _check(_load().oracle_prune_rows(dtype, M, K, bm, bk, float(rate), _p(W), _p(keep), _p(m)))
     return (m, keep) if return_keep else m
+
+
+# The 4-entry 3x3 kernel patterns used by default (positions pos = 3i + j):
+# the centre with three of its edge neighbours (four "T" shapes) and the
+# centre with two adjacent edge neighbours and the corner between them (four
+# 2 x 2 squares).
+DEFAULT_PATTERNS = np.array([
+    (1 << 1) | (1 << 3) | (1 << 4) | (1 << 5),
+    (1 << 1) | (1 << 4) | (1 << 5) | (1 << 7),
+    (1 << 3) | (1 << 4) | (1 << 5) | (1 << 7),
+    (1 << 1) | (1 << 3) | (1 << 4) | (1 << 7),
+    (1 << 0) | (1 << 1) | (1 << 3) | (1 << 4),
+    (1 << 1) | (1 << 2) | (1 << 4) | (1 << 5),
+    (1 << 3) | (1 << 4) | (1 << 6) | (1 << 7),
+    (1 << 4) | (1 << 5) | (1 << 7) | (1 << 8),
+], np.uint16)
+
+
+def prune_pattern(W_bits, dtype, rate, patterns=DEFAULT_PATTERNS, return_patterns=False):
+    """Pattern-based pruning of an F x C x 3 x 3 weight (kernel patterns +
+    connectivity pruning at `rate` >= 9/4): F x 9C uint8 mask (and the chosen
+    pattern index of each kernel)."""
+    W = _u16(W_bits)
+    F = W.shape[0]
+    C = W.size // (F * 9)
+    pats = np.ascontiguousarray(patterns, np.uint16)
+    pat = np.empty(F * C, np.uint8)
+    mask = np.empty((F, 9 * C), np.uint8)
+    _check(_load().oracle_prune_pattern(dtype, F, C, _p(pats), len(pats), float(rate), _p(W),
+                                        _p(pat), _p(mask)))
+    return (mask, pat) if return_patterns else mask
 
 
 def pack(W_bits, mask, bm):

@@ -460,6 +460,70 @@ done:
     return st;
 }
 
+/* Pattern-based pruning of 3x3 CONV layers (Sec. 2, pattern-based pruning:
+ * kernel pattern pruning plus connectivity pruning), on the OIHW weight
+ * (F filters, C channels, positions pos = 3i + j):
+ *  - kernel pattern pruning: kernel (f, c) keeps the 4 positions of the
+ *    pattern, among the npat given 9-bit masks (each with 4 bits set), whose
+ *    kept squared norm (fp64, positions ascending) is largest; ties go to the
+ *    lower pattern index;
+ *  - connectivity pruning: of the F*C kernels, the T = floor(9 F C / (4 rate)
+ *    + 0.5) with the largest kept norm survive (ties to the lower kernel index
+ *    f*C + c), the others are removed whole; rate >= 9/4 is the
+ *    parameter-reduction factor (9/4 keeps every kernel).
+ * mask (F x 9C uint8) receives the element mask, pattern (optional, F*C) the
+ * chosen pattern index of each kernel. */
+int oracle_prune_pattern(int dtype, int64_t F, int64_t C, const uint16_t *patterns, int npat,
+                         double rate, const uint16_t *W, uint8_t *pattern, uint8_t *mask)
+{
+    if (F < 1 || C < 1 || npat < 1 || npat > 255 || !(rate >= 2.25) || !isfinite(rate))
+        return OR_ERR_ARG;
+    for (int q = 0; q < npat; ++q) {
+        int bits = 0;
+        for (int b = 0; b < 9; ++b) bits += (patterns[q] >> b) & 1;
+        if (bits != 4 || (patterns[q] >> 9)) return OR_ERR_ARG;
+    }
+    const int64_t U = F * C, K = 9 * C;
+    cand_t *all = (cand_t *)malloc((size_t)U * sizeof(cand_t));
+    uint8_t *pat = pattern ? pattern : (uint8_t *)malloc((size_t)U);
+    int st = OR_OK;
+    for (int64_t f = 0; f < F; ++f)
+        for (int64_t c = 0; c < C; ++c) {
+            double sq[9];
+            for (int pos = 0; pos < 9; ++pos) {
+                double w = oracle_half_to_double(W[f * K + c * 9 + pos], dtype);
+                if (!isfinite(w)) { st = OR_ERR_NONFINITE; goto done; }
+                sq[pos] = w * w;
+            }
+            double best = -1.0;
+            int bq = 0;
+            for (int q = 0; q < npat; ++q) {
+                double e = 0.0;
+                for (int pos = 0; pos < 9; ++pos)
+                    if ((patterns[q] >> pos) & 1) e += sq[pos];
+                if (e > best) { best = e; bq = q; }
+            }
+            pat[f * C + c] = (uint8_t)bq;
+            all[f * C + c].s = best;
+            all[f * C + c].g = f * C + c;
+        }
+    {
+        const int64_t T = (int64_t)floor(9.0 * (double)U / (4.0 * rate) + 0.5);
+        qsort(all, (size_t)U, sizeof(cand_t), cand_cmp);
+        memset(mask, 0, (size_t)(F * K));
+        for (int64_t i = 0; i < T && i < U; ++i) {
+            const int64_t g = all[i].g, f = g / C, c = g % C;
+            const uint16_t m = patterns[pat[g]];
+            for (int pos = 0; pos < 9; ++pos)
+                if ((m >> pos) & 1) mask[f * K + c * 9 + pos] = 1;
+        }
+    }
+done:
+    free(all);
+    if (!pattern) free(pat);
+    return st;
+}
+
 /* Compact storage (BCS, Sec. 4.3).  Because every row of a row-block keeps
  * the same columns, one column list serves the whole row-block (the
  * "occurrence" rows rb*bm .. rb*bm+bm_rb-1):
