@@ -590,6 +590,63 @@ def run_workload(args):
                           "timing": "device time, median of 5, L2 flushed before each"}),
               flush=True)
         return
+    elif name == "e4":
+        # 3x3 CONV, 28 x 28 feature map, 128 input / output channels (the
+        # paper's pattern vs block-punched latency comparison), fp16, batch 1
+        # and 32: pattern-based pruning (kernel patterns + connectivity) and
+        # block-punched pruning with 8x16, 16x32 and 128x32 blocks at the same
+        # weight rates, against dense cuDNN
+        from paper_2111_11581_gb300 import bp
+        C = F = 128
+        H = 28
+        Wb = inputs.normal((F, C, 3, 3), inputs.kaiming_std(C * 9), inputs.F16, 9100)
+        Wd = inputs.as_torch(Wb.reshape(F, -1), inputs.F16).cuda()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+
+        def timed(fn, reps=9):
+            ts = []
+            for _ in range(reps + 1):
+                flush.zero_()
+                ev[0].record()
+                fn()
+                ev[1].record()
+                torch.cuda.synchronize()
+                ts.append(ev[0].elapsed_time(ev[1]) * 1e3)
+            return statistics.median(ts[1:])
+
+        out = {"workload": "e4", "layer": "conv3x3 28x28 C=F=128 fp16", "points": []}
+        for nb in (1, 32):
+            x = inputs.as_torch(inputs.normal((nb, C, H, H), 1.0, inputs.F16, 9101),
+                                inputs.F16).cuda()
+            wc = Wd.reshape(F, C, 3, 3)
+            dense_us = timed(lambda: torch.nn.functional.conv2d(x, wc, padding=1))
+            for rate in (4.0, 8.0, 12.0):
+                for scheme in ("pattern", "punched8x16", "punched16x32", "punched128x32"):
+                    if scheme == "pattern":
+                        mask = bp.prune_pattern(bp.layout(bp.BLOCK_PUNCHED, bp.F16, F, C * 9, 8,
+                                                          4, 3, 3), Wd, rate)
+                        play = bp.layout(bp.BLOCK_PUNCHED, bp.F16, F, C * 9, 1, 1, 3, 3)
+                    else:
+                        bmk = scheme[len("punched"):].split("x")
+                        play = bp.layout(bp.BLOCK_PUNCHED, bp.F16, F, C * 9, int(bmk[0]),
+                                         int(bmk[1]), 3, 3)
+                        mask = bp.prune(play, Wd, rate)
+                    pw = bp.pack(play, Wd, mask)
+                    ws = bp.conv2d_workspace(pw, tuple(x.shape), (1, 1))
+                    y = bp.conv2d(pw, x, pad=(1, 1), ws=ws)
+                    us = timed(lambda: bp.conv2d(pw, x, pad=(1, 1), out=y, ws=ws))
+                    chunks = int(pw.dev[8:16].view(torch.int64)[0])      # kc_ptr[1]: one slab
+                    out["points"].append({"batch": nb, "rate": rate, "scheme": scheme,
+                                          "kept_weights": int(pw.c.nnz_vals),
+                                          "tensor_core_columns": chunks * 64,
+                                          "us": round(us, 2), "dense_us": round(dense_us, 2)})
+                    print(f"# b{nb} r{rate:g} {scheme:14s} {us:8.2f} us (dense {dense_us:.2f})"
+                          f" cols {chunks * 64}", file=sys.stderr, flush=True)
+        if bp.device_status() != bp.OK:
+            raise RuntimeError("kernel watchdog fired")
+        out["timing"] = "device time of bp_conv2d (im2col + product), median of 9, L2 flushed"
+        print(json.dumps(out), flush=True)
+        return
     elif name == "sweep":
         layers, dtype = [], None
         for dt in (inputs.BF16, inputs.F16):
@@ -634,7 +691,8 @@ def main():
                     help="fc512 | conv3x3 | vgg16 | resnet50 | sweep: per-layer timings "
                          "of another workload (one JSON line), instead of the default step; "
                          "blocksize: the latency model and block-size selection; penalty: "
-                         "the reweighted regulariser; rowcol: row + column pruning")
+                         "the reweighted regulariser; rowcol: row + column pruning; e4: "
+                         "pattern vs block-punched 3x3 latency")
     ap.add_argument("--sweep-subset", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:

@@ -105,7 +105,8 @@ const char *bp_status_string(int status);
 int bp_version(void);
 
 /* Device workspace bytes bp_prune needs for `lay` (host output); for
- * block-based layouts the same workspace also serves bp_prune_rows. */
+ * block-based layouts the same workspace also serves bp_prune_rows, for
+ * block-punched 3x3 layouts bp_prune_pattern. */
 bp_status bp_workspace_size(const bp_layout *lay, size_t *bytes);
 
 /* One-shot magnitude pruning by block (Sec. 5.1 with the block regularities
@@ -141,6 +142,22 @@ bp_status bp_prune(const bp_layout *lay, const void *W, double rate, uint8_t *ma
  * as bp_prune; BP_ERR_INVALID_ARG for block-punched layouts. */
 bp_status bp_prune_rows(const bp_layout *lay, const void *W, double rate, uint8_t *mask,
                         void *ws, size_t ws_bytes, void *stream);
+
+/* Pattern-based pruning of a 3x3 CONV layer (Sec. 2: kernel pattern pruning
+ * plus connectivity pruning), the alternative the paper maps to 3x3 layers
+ * for large datasets.  lay: block-punched, kh = kw = 3 (bm, bk unused).
+ * Kernel (f, c) keeps the 4 positions (pos = 3i + j) of the pattern, among
+ * `patterns` (host, npatterns 9-bit masks with 4 bits set, 1..16 of them),
+ * whose kept squared norm (fp64, positions ascending) is largest, ties to the
+ * lower pattern index; then the T = floor(9 F C / (4 rate) + 0.5) kernels
+ * with the largest kept norms survive (connectivity pruning, ties to the
+ * lower kernel index f*C + c) and the rest are removed.  rate >= 9/4 is the
+ * parameter-reduction factor.  Filters then keep different columns: pack the
+ * mask with bm = bk = 1.  Same workspace (bp_workspace_size of the layout),
+ * synchronisation and errors as bp_prune. */
+bp_status bp_prune_pattern(const bp_layout *lay, const void *W, double rate,
+                           const uint16_t *patterns, int npatterns, uint8_t *mask, void *ws,
+                           size_t ws_bytes, void *stream);
 
 /* First half of packing: checks that every row of each row-block keeps the
  * same columns as the row-block's first row (BP_ERR_INVALID_ARG otherwise)

@@ -35,6 +35,7 @@ class Packed(ctypes.Structure):
 
 
 EXPORTS = ("bp_status_string", "bp_version", "bp_workspace_size", "bp_prune", "bp_prune_rows",
+           "bp_prune_pattern",
            "bp_pack_size", "bp_pack", "bp_gemm", "bp_gemm_workspace_size", "bp_conv2d",
            "bp_conv2d_workspace_size", "bp_penalty_units", "bp_reweighted_penalty",
            "bp_penalty_workspace_size", "bp_device_status", "bp_set_watchdog_ns",
@@ -69,6 +70,7 @@ def load(path: str = LIB_PATH):
             "bp_workspace_size": (i32, [P_L, ctypes.POINTER(sz)]),
             "bp_prune": (i32, [P_L, vp, dbl, vp, vp, sz, vp]),
             "bp_prune_rows": (i32, [P_L, vp, dbl, vp, vp, sz, vp]),
+            "bp_prune_pattern": (i32, [P_L, vp, dbl, vp, i32, vp, vp, sz, vp]),
             "bp_pack_size": (i32, [P_L, vp, vp, P_i64, P_i64, P_i64, vp]),
             "bp_pack": (i32, [P_L, vp, vp, P_P, vp]),
             "bp_gemm": (i32, [P_P, vp, i64, i64, vp, i32, vp, i64, vp, sz, vp]),
@@ -120,6 +122,13 @@ def bp_prune(lay: Layout, W: int, rate: float, mask: int, ws: int, ws_bytes: int
 def bp_prune_rows(lay: Layout, W: int, rate: float, mask: int, ws: int, ws_bytes: int,
                   stream: int = 0) -> int:
     return load().bp_prune_rows(ctypes.byref(lay), W, float(rate), mask, ws, ws_bytes, stream)
+
+
+def bp_prune_pattern(lay: Layout, W: int, rate: float, patterns, mask: int, ws: int,
+                     ws_bytes: int, stream: int = 0) -> int:
+    pats = (ctypes.c_uint16 * len(patterns))(*[int(p) for p in patterns])
+    return load().bp_prune_pattern(ctypes.byref(lay), W, float(rate), pats, len(patterns), mask,
+                                   ws, ws_bytes, stream)
 
 
 def bp_pack_size(lay: Layout, mask: int, rb_ptr: int, stream: int = 0):
@@ -241,6 +250,24 @@ def prune_rows(lay: Layout, W, rate: float, mask=None, stream=None):
     ws = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=W.device)
     _chk(bp_prune_rows(lay, W.data_ptr(), rate, mask.data_ptr(), ws.data_ptr(), nbytes,
                        _stream(stream)), "bp_prune_rows")
+    return mask
+
+
+# 4-entry 3x3 kernel patterns (pos = 3i + j): the centre with three edge
+# neighbours (four T shapes) and the centre with two adjacent edge neighbours
+# and the corner between them (four 2 x 2 squares).
+DEFAULT_PATTERNS = (0b000111010, 0b010110010, 0b010111000, 0b010011010,
+                    0b000011011, 0b000110110, 0b011011000, 0b110110000)
+
+
+def prune_pattern(lay: Layout, W, rate: float, patterns=DEFAULT_PATTERNS, stream=None):
+    """Mask (uint8 M x K, device) of bp_prune_pattern on a 3x3 weight."""
+    torch = _torch()
+    mask = torch.empty((lay.M, lay.K), dtype=torch.uint8, device=W.device)
+    nbytes = bp_workspace_size(lay)
+    ws = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=W.device)
+    _chk(bp_prune_pattern(lay, W.data_ptr(), rate, patterns, mask.data_ptr(), ws.data_ptr(),
+                          nbytes, _stream(stream)), "bp_prune_pattern")
     return mask
 
 

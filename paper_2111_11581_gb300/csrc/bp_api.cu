@@ -61,6 +61,15 @@ Counts host_counts(const bp_layout &l, double rate) {
     const int64_t RB = cdiv(l.M, l.bm);
     const int64_t KK = (int64_t)l.kh * l.kw;
     int64_t per_rb_base = 0, per_rb_units = 0;
+    if (l.scheme == kSchemePattern) {
+        // one unit per kernel, each a block of its own, kept at the kernel
+        // rate 4 r / 9 (r = the weight rate): T = floor(9 F C / (4 r) + 0.5)
+        c.U = l.M * (l.K / 9);
+        c.sum_base = c.U * (int64_t)std::floor(1.0 / (4.0 * rate / 9.0));
+        c.T = (int64_t)std::floor(9.0 * (double)c.U / (4.0 * rate) + 0.5);
+        c.E = c.T - c.sum_base;
+        return c;
+    }
     if (l.scheme == kSchemeRows) {
         // row units: every block of row-block rb has rows_rb units
         const int64_t CB = cdiv(l.K, l.bk), last = l.M - (RB - 1) * l.bm;
@@ -89,7 +98,7 @@ Counts host_counts(const bp_layout &l, double rate) {
 }
 
 struct PruneWs {
-    int64_t off_scores, off_hist, off_chunks, off_flag, off_keep, total;
+    int64_t off_scores, off_hist, off_chunks, off_flag, off_keep, off_patsel, total;
 };
 
 int64_t align_up(int64_t v, int64_t a) { return (v + a - 1) / a * a; }
@@ -102,20 +111,24 @@ PruneWs prune_ws(const bp_layout &l) {
         rows.scheme = (bp_scheme)kSchemeRows;
         c.U = std::max(c.U, host_counts(rows, 1.0).U);
     }
+    const bool k3 = l.scheme == BP_BLOCK_PUNCHED && l.kh == 3 && l.kw == 3;
+    if (k3) c.U = std::max(c.U, l.M * (l.K / 9));   // ... and bp_prune_pattern
     PruneWs w;
     w.off_scores = 0;
     w.off_hist = align_up(c.U * 8, 256);
     w.off_chunks = w.off_hist + 1024;
     w.off_flag = align_up(w.off_chunks + 8 * threshold_chunks(c.U), 256);
     w.off_keep = w.off_flag + 256;
-    w.total = align_up(w.off_keep + c.U, 256);
+    w.off_patsel = align_up(w.off_keep + c.U, 256);
+    w.total = k3 ? align_up(w.off_patsel + c.U, 256) : w.off_patsel;
     return w;
 }
 
 // The pruning pipeline over the units of `lay` (scheme may be kSchemeRows):
 // scores, per-block keep, layer-wide extras by radix select, mask.
 bp_status prune_units(const bp_layout &lay, const void *W, double rate, uint8_t *mask,
-                      void *ws, const PruneWs &w, cudaStream_t s) {
+                      void *ws, const PruneWs &w, cudaStream_t s,
+                      const PatternSet *ps = nullptr) {
     uint8_t *base = static_cast<uint8_t *>(ws);
     double *scores = reinterpret_cast<double *>(base + w.off_scores);
     unsigned *hist = reinterpret_cast<unsigned *>(base + w.off_hist);
@@ -124,9 +137,13 @@ bp_status prune_units(const bp_layout &lay, const void *W, double rate, uint8_t 
     uint8_t *keep = base + w.off_keep;
     const Counts c = host_counts(lay, rate);
 
+    uint8_t *patsel = base + w.off_patsel;
     cudaError_t e = cudaMemsetAsync(flag, 0, sizeof(int), s);
-    if (e == cudaSuccess) e = launch_scores(lay, W, scores, flag, s);
-    if (e == cudaSuccess) e = launch_base_select(lay, scores, rate, keep, s);
+    if (e == cudaSuccess)
+        e = ps ? launch_pattern_scores(lay, W, *ps, scores, patsel, flag, s)
+               : launch_scores(lay, W, scores, flag, s);
+    // pattern units are blocks of one kernel: floor(1 / (4 r / 9)) of each
+    if (e == cudaSuccess) e = launch_base_select(lay, scores, ps ? 4.0 * rate / 9.0 : rate, keep, s);
     int nonfinite = 0;
     if (e == cudaSuccess) e = cudaMemcpyAsync(&nonfinite, flag, sizeof(int), cudaMemcpyDeviceToHost, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
@@ -154,7 +171,8 @@ bp_status prune_units(const bp_layout &lay, const void *W, double rate, uint8_t 
         e = launch_threshold_select(c.U, scores, keep, prefix, need, chunks, s);
         if (e != cudaSuccess) return BP_ERR_CUDA;
     }
-    e = launch_write_mask(lay, keep, mask, s);
+    e = ps ? launch_pattern_mask(lay, keep, patsel, *ps, mask, s)
+           : launch_write_mask(lay, keep, mask, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     return cuda_status(e);
 }
@@ -252,7 +270,7 @@ const char *bp_status_string(int status) {
     }
 }
 
-int bp_version(void) { return (2 << 16) | 3; }
+int bp_version(void) { return (2 << 16) | 4; }
 
 bp_status bp_workspace_size(const bp_layout *lay, size_t *bytes) {
     if (!layout_ok(lay) || !bytes) return BP_ERR_INVALID_ARG;
@@ -268,6 +286,28 @@ bp_status bp_prune(const bp_layout *lay, const void *W, double rate, uint8_t *ma
     if (!ws || ws_bytes < (size_t)w.total || (reinterpret_cast<uintptr_t>(ws) & 255u))
         return BP_ERR_WORKSPACE;
     return prune_units(*lay, W, rate, mask, ws, w, static_cast<cudaStream_t>(stream));
+}
+
+bp_status bp_prune_pattern(const bp_layout *lay, const void *W, double rate,
+                           const uint16_t *patterns, int npatterns, uint8_t *mask, void *ws,
+                           size_t ws_bytes, void *stream) {
+    if (!layout_ok(lay) || !W || !mask || !patterns) return BP_ERR_INVALID_ARG;
+    if (lay->scheme != BP_BLOCK_PUNCHED || lay->kh != 3 || lay->kw != 3)
+        return BP_ERR_INVALID_ARG;
+    if (!(rate >= 2.25) || !std::isfinite(rate)) return BP_ERR_INVALID_ARG;
+    if (npatterns < 1 || npatterns > kMaxPatterns) return BP_ERR_INVALID_ARG;
+    PatternSet ps{};
+    ps.n = npatterns;
+    for (int q = 0; q < npatterns; ++q) {
+        if ((patterns[q] >> 9) || __builtin_popcount(patterns[q]) != 4) return BP_ERR_INVALID_ARG;
+        ps.m[q] = patterns[q];
+    }
+    const PruneWs w = prune_ws(*lay);
+    if (!ws || ws_bytes < (size_t)w.total || (reinterpret_cast<uintptr_t>(ws) & 255u))
+        return BP_ERR_WORKSPACE;
+    bp_layout pl = *lay;
+    pl.scheme = (bp_scheme)kSchemePattern;
+    return prune_units(pl, W, rate, mask, ws, w, static_cast<cudaStream_t>(stream), &ps);
 }
 
 bp_status bp_prune_rows(const bp_layout *lay, const void *W, double rate, uint8_t *mask,

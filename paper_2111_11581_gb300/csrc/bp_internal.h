@@ -14,6 +14,14 @@ namespace bp {
 // Internal scheme value of the prune kernels: the row units of a block-based
 // layout (rows of each bm x bk block; written into the mask with AND).
 constexpr int kSchemeRows = 2;
+// ... and the kernels of a 3x3 layer for pattern-based pruning (one unit per
+// (filter, channel) kernel, scored by its best pattern's kept norm).
+constexpr int kSchemePattern = 3;
+constexpr int kMaxPatterns = 16;
+struct PatternSet {
+    uint16_t m[kMaxPatterns];   // 9-bit masks, 4 bits set, pos = 3i + j
+    int n;
+};
 
 // Device status bits recorded by kernels (read by bp_device_status).
 constexpr unsigned kDevTimeout = 1u;
@@ -95,6 +103,11 @@ cudaError_t launch_radix_hist(int64_t U, const double *scores, const uint8_t *ke
 cudaError_t launch_threshold_select(int64_t U, const double *scores, uint8_t *keep,
                                     uint64_t thr, int64_t need, int64_t *chunk_cnt,
                                     cudaStream_t s);
+cudaError_t launch_pattern_scores(const bp_layout &lay, const void *W, const PatternSet &ps,
+                                  double *scores, uint8_t *patsel, int *nonfinite,
+                                  cudaStream_t s);
+cudaError_t launch_pattern_mask(const bp_layout &lay, const uint8_t *keep, const uint8_t *patsel,
+                                const PatternSet &ps, uint8_t *mask, cudaStream_t s);
 cudaError_t launch_write_mask(const bp_layout &lay, const uint8_t *keep, uint8_t *mask,
                               cudaStream_t s);
 int64_t threshold_chunks(int64_t U);

@@ -38,6 +38,9 @@ Part make_part(const bp_layout &l) {
     } else if (l.scheme == kSchemeRows) {
         p.CB = (l.K + l.bk - 1) / l.bk;
         p.U = l.M * p.CB;
+    } else if (l.scheme == kSchemePattern) {
+        p.CB = p.C;
+        p.U = l.M * p.C;
     } else {
         p.CB = (p.C + l.bk - 1) / l.bk;
         p.U = p.RB * p.CB * p.KK;
@@ -128,6 +131,9 @@ __global__ void base_select_kernel(Part p, double rate, const double *__restrict
             const RowUnit u = row_unit(p, g);
             first = u.first;
             P = u.P;
+        } else if (p.scheme == kSchemePattern) {
+            first = g;            // each kernel is a block of one unit
+            P = 1;
         } else {
             first = (g / p.KK) * p.KK;
             P = p.KK;
@@ -270,6 +276,57 @@ __global__ void write_mask_kernel(Part p, const uint8_t *__restrict__ keep,
     }
 }
 
+// Pattern units: kernel g = f*C + c.  Its squared weights (fp64), the kept
+// norm of every pattern (positions ascending), the best pattern (ties to the
+// lower index) into patsel and its norm into scores.
+__global__ void pattern_scores_kernel(Part p, int dtype, const uint16_t *__restrict__ W,
+                                      PatternSet ps, double *__restrict__ scores,
+                                      uint8_t *__restrict__ patsel, int *__restrict__ nonfinite) {
+    for (int64_t g = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; g < p.U;
+         g += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t f = g / p.C, c = g - f * p.C;
+        const uint16_t *k = W + f * p.K + c * 9;
+        double sq[9];
+        bool bad = false;
+#pragma unroll
+        for (int pos = 0; pos < 9; ++pos) {
+            const float v = ld_half(k, pos, dtype);
+            bad |= !isfinite(v);
+            const double w = (double)v;
+            sq[pos] = w * w;
+        }
+        double best = -1.0;
+        int bq = 0;
+        for (int q = 0; q < ps.n; ++q) {
+            double e = 0.0;
+#pragma unroll
+            for (int pos = 0; pos < 9; ++pos)
+                if ((ps.m[q] >> pos) & 1u) e += sq[pos];
+            if (e > best) {
+                best = e;
+                bq = q;
+            }
+        }
+        scores[g] = best;
+        patsel[g] = (uint8_t)bq;
+        if (bad) atomicExch(nonfinite, 1);
+    }
+}
+
+// Element (f, 9c + pos) survives when kernel (f, c) survives and pos is in
+// its pattern.
+__global__ void pattern_mask_kernel(Part p, const uint8_t *__restrict__ keep,
+                                    const uint8_t *__restrict__ patsel, PatternSet ps,
+                                    uint8_t *__restrict__ mask) {
+    const int64_t total = p.M * p.K;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t f = i / p.K, k = i - f * p.K, c = k / 9, pos = k - c * 9;
+        const int64_t g = f * p.C + c;
+        mask[i] = (keep[g] && ((ps.m[patsel[g]] >> pos) & 1u)) ? 1 : 0;
+    }
+}
+
 int grid_for(int64_t n, int threads) {
     int64_t b = (n + threads - 1) / threads;
     const int64_t cap = (int64_t)num_sms() * 16;
@@ -316,6 +373,22 @@ cudaError_t launch_threshold_select(int64_t U, const double *scores, uint8_t *ke
     if (need > 0)
         threshold_ties_kernel<<<(unsigned)nch, kSelThreads, 0, s>>>(U, scores, keep, thr, need,
                                                                    chunk_cnt);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_pattern_scores(const bp_layout &lay, const void *W, const PatternSet &ps,
+                                  double *scores, uint8_t *patsel, int *nonfinite,
+                                  cudaStream_t s) {
+    const Part p = make_part(lay);
+    pattern_scores_kernel<<<grid_for(p.U, 256), 256, 0, s>>>(
+        p, lay.dtype, static_cast<const uint16_t *>(W), ps, scores, patsel, nonfinite);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_pattern_mask(const bp_layout &lay, const uint8_t *keep, const uint8_t *patsel,
+                                const PatternSet &ps, uint8_t *mask, cudaStream_t s) {
+    const Part p = make_part(lay);
+    pattern_mask_kernel<<<grid_for(p.M * p.K, 256), 256, 0, s>>>(p, keep, patsel, ps, mask);
     return cudaGetLastError();
 }
 

@@ -58,7 +58,7 @@ def test_ctypes_structs_match_header(tmp_path):
 def test_status_strings_and_version(lib):
     assert bp.status_string(bp.OK) == "ok"
     assert bp.status_string(bp.ERR_TIMEOUT) == "kernel wait timed out"
-    assert bp.bp_version() >> 16 == 2 and bp.bp_version() & 0xffff >= 3
+    assert bp.bp_version() >> 16 == 2 and bp.bp_version() & 0xffff >= 4
 
 
 def test_workspace_size_is_host_only(lib):
@@ -193,3 +193,20 @@ def test_prune_rows_argument_checks_on_host(lib):
     assert bp.bp_prune_rows(lay, a, 2.0, a, a, n - 1, 0) == bp.ERR_WORKSPACE
     play = bp.layout(bp.BLOCK_PUNCHED, bp.F16, 16, 8 * 9, 8, 4, 3, 3)
     assert bp.bp_prune_rows(play, a, 2.0, a, a, 1 << 20, 0) == bp.ERR_INVALID_ARG
+
+
+def test_prune_pattern_argument_checks_on_host(lib):
+    lay = bp.layout(bp.BLOCK_PUNCHED, bp.F16, 64, 32 * 9, 8, 4, 3, 3)
+    n = bp.bp_workspace_size(lay)
+    a = 1 << 20
+    pats = list(bp.DEFAULT_PATTERNS)
+    assert bp.bp_prune_pattern(lay, a, 2.0, pats, a, a, n, 0) == bp.ERR_INVALID_ARG      # rate < 9/4
+    assert bp.bp_prune_pattern(lay, a, 4.0, [0b111], a, a, n, 0) == bp.ERR_INVALID_ARG   # 3 entries
+    assert bp.bp_prune_pattern(lay, a, 4.0, [1 << 9 | 0b111], a, a, n, 0) == bp.ERR_INVALID_ARG
+    assert bp.bp_prune_pattern(lay, a, 4.0, pats * 3, a, a, n, 0) == bp.ERR_INVALID_ARG  # 24 > 16
+    assert bp.bp_prune_pattern(lay, a, 4.0, pats, a, a, n - 1, 0) == bp.ERR_WORKSPACE
+    for other in (bp.layout(bp.BLOCK_PUNCHED, bp.F16, 64, 32 * 25, 8, 4, 5, 5),
+                  bp.layout(bp.BLOCK_BASED, bp.F16, 64, 288, 8, 4)):
+        assert bp.bp_prune_pattern(other, a, 4.0, pats, a, a, 1 << 22, 0) == bp.ERR_INVALID_ARG
+    # the workspace covers one unit per kernel (64 x 32) plus its pattern byte
+    assert n >= 64 * 32 * (8 + 1 + 1)
