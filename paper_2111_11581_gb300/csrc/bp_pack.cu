@@ -378,6 +378,80 @@ __global__ void __launch_bounds__(256) im2col_1x1_kernel(ConvShape cs, int64_t l
     }
 }
 
+// im2col of a 3x3, stride-1, padding-1 convolution whose image has H*W a
+// multiple of 8 and fits in shared memory with its zero border: one block per
+// (channel, image).  The block stages the padded plane ((H+2) x (W+2)) once,
+// collects the channel's listed window positions, then writes each listed row
+// 8 pixels (16 bytes) per thread, consecutive threads on consecutive pixels
+// (512 contiguous bytes per warp store).  A pixel group's 8 window offsets are
+// computed once and reused for every listed position.
+__global__ void __launch_bounds__(256) im2col_3x3_plane_kernel(ConvShape cs, int64_t ldx,
+                                                               const int32_t *__restrict__ qmap,
+                                                               const uint16_t *__restrict__ in,
+                                                               uint16_t *__restrict__ xcol) {
+    extern __shared__ __align__(16) uint8_t plane_smem[];
+    uint16_t *plane = reinterpret_cast<uint16_t *>(plane_smem);
+    __shared__ int32_t qrow[9], qoff[9];
+    __shared__ int nlisted;
+    const int H = (int)cs.H, W = (int)cs.W, wp = W + 2, HW = H * W;
+    const int64_t c = blockIdx.x, b = blockIdx.y;
+    if (threadIdx.x == 0) {
+        int n = 0;
+        for (int pos = 0; pos < 9; ++pos) {
+            const int64_t k = c * 9 + pos;
+            const int32_t q = qmap ? qmap[k] : (int32_t)k;
+            if (q >= 0) {
+                qrow[n] = q;
+                qoff[n] = (pos / 3) * wp + pos % 3;
+                ++n;
+            }
+        }
+        nlisted = n;
+    }
+    // zero border + the plane (16-byte loads: H*W is a multiple of 8 and the
+    // plane starts 16-byte aligned when the input does)
+    for (int e = threadIdx.x; e < (H + 2) * wp; e += blockDim.x) plane[e] = 0;
+    __syncthreads();
+    const uint16_t *src = in + (b * cs.C + c) * (int64_t)HW;
+    for (int v = threadIdx.x; v < HW / 8; v += blockDim.x) {
+        const uint4 q = __ldg(reinterpret_cast<const uint4 *>(src) + v);
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+        int p = v * 8, ih = p / W, iw = p - ih * W;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            plane[(ih + 1) * wp + iw + 1] = (uint16_t)(w[e >> 1] >> (16 * (e & 1)));
+            if (++iw == W) {
+                iw = 0;
+                ++ih;
+            }
+        }
+    }
+    __syncthreads();
+    const int L = nlisted, G = HW / 8;
+    uint16_t *dst = xcol + b * (int64_t)HW;
+    for (int g = threadIdx.x; g < G; g += blockDim.x) {
+        int off[8];
+        int p = g * 8, oh = p / W, ow = p - oh * W;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            off[e] = oh * wp + ow;
+            if (++ow == W) {
+                ow = 0;
+                ++oh;
+            }
+        }
+        for (int l = 0; l < L; ++l) {
+            const uint16_t *pl = plane + qoff[l];
+            uint32_t v[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                v[e] = (uint32_t)pl[off[2 * e]] | ((uint32_t)pl[off[2 * e + 1]] << 16);
+            *reinterpret_cast<uint4 *>(dst + (int64_t)qrow[l] * ldx + 8 * g) =
+                make_uint4(v[0], v[1], v[2], v[3]);
+        }
+    }
+}
+
 // Writes the block's im2col rows from the staged planes: segments of 32*V
 // consecutive pixels of one channel per warp step, V pixels per lane (one
 // 2V-byte store per window offset).  KH, KW > 0: the window's size at compile
@@ -633,6 +707,15 @@ cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void
     if (cs.kh == 1 && cs.kw == 1) {
         if (cs.C > 0x7fffffffLL || cs.Nb > 65535) return cudaErrorInvalidValue;
         im2col_1x1_kernel<<<dim3((unsigned)cs.C, (unsigned)cs.Nb), 256, 0, s>>>(
+            cs, ldx, qmap, static_cast<const uint16_t *>(in), static_cast<uint16_t *>(xcol));
+        return cudaGetLastError();
+    }
+    if (cs.kh == 3 && cs.kw == 3 && cs.sh == 1 && cs.sw == 1 && cs.ph == 1 && cs.pw == 1 &&
+        (cs.H * cs.W) % 8 == 0 && (cs.H + 2) * (cs.W + 2) * 2 <= 48 * 1024 && ldx % 8 == 0 &&
+        (reinterpret_cast<uintptr_t>(in) & 15u) == 0 && (reinterpret_cast<uintptr_t>(xcol) & 15u) == 0 &&
+        cs.C <= 0x7fffffffLL && cs.Nb <= 65535) {
+        const size_t smem = (size_t)(cs.H + 2) * (cs.W + 2) * 2;
+        im2col_3x3_plane_kernel<<<dim3((unsigned)cs.C, (unsigned)cs.Nb), 256, smem, s>>>(
             cs, ldx, qmap, static_cast<const uint16_t *>(in), static_cast<uint16_t *>(xcol));
         return cudaGetLastError();
     }
