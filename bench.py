@@ -440,7 +440,10 @@ def _layer_step(layer, dtype, flush, reps=5):
     def timed(fn):
         ts = []
         for _ in range(reps + 1):
+            # flush L2, then read the flush buffer back so that L2 holds clean
+            # lines (no write-back of the flush inside the timing)
             flush.zero_()
+            flush.sum()
             ev[0].record()
             fn()
             ev[1].record()
@@ -674,7 +677,8 @@ def run_workload(args):
     out = {"metric": METRIC, "value": round(fl / t / 1e6, 2), "unit": UNIT, "n_gpus": 1,
            "workload": name, "pruned_layers": len(pr), "sum_us": round(t, 2),
            "dense_sum_us": round(td, 2), "speedup_vs_dense": round(td / t, 3),
-           "timing": "per-layer device time, median of 5, L2 flushed (256 MiB write) before each launch",
+           "timing": "per-layer device time, median of 5, L2 flushed (256 MiB write, read back) "
+                     "before each launch",
            "layers": rows}
     print(json.dumps(out), flush=True)
 

@@ -379,47 +379,55 @@ __global__ void __launch_bounds__(256) im2col_1x1_kernel(ConvShape cs, int64_t l
 }
 
 // im2col of a 3x3, stride-1, padding-1 convolution whose image has H*W a
-// multiple of 8 and fits in shared memory with its zero border: one block per
-// (channel, image).  The block stages the padded plane ((H+2) x (W+2)) once,
-// collects the channel's listed window positions, then writes each listed row
-// 8 pixels (16 bytes) per thread, consecutive threads on consecutive pixels
-// (512 contiguous bytes per warp store).  A pixel group's 8 window offsets are
-// computed once and reused for every listed position.
-__global__ void __launch_bounds__(256) im2col_3x3_plane_kernel(ConvShape cs, int64_t ldx,
+// multiple of 8: one block per (group of ppb channels, image).  The block
+// stages the channels' padded planes ((H+2) x (W+2) each) once, collects each
+// channel's listed window positions, then writes each listed row 8 pixels
+// (16 bytes) per thread, consecutive threads on consecutive pixels (512
+// contiguous bytes per warp store).  A pixel group's 8 window offsets are
+// computed once and reused for every listed position.  Small images take
+// several channels per block so that every thread has a pixel group.
+constexpr int kPlaneMaxChannels = 128;
+constexpr int64_t kPlaneSmem = 40 * 1024;   // dynamic shared memory (the tables take ~7 KB)
+__global__ void __launch_bounds__(256) im2col_3x3_plane_kernel(ConvShape cs, int64_t ldx, int ppb,
                                                                const int32_t *__restrict__ qmap,
                                                                const uint16_t *__restrict__ in,
                                                                uint16_t *__restrict__ xcol) {
     extern __shared__ __align__(16) uint8_t plane_smem[];
-    uint16_t *plane = reinterpret_cast<uint16_t *>(plane_smem);
-    __shared__ int32_t qrow[9], qoff[9];
-    __shared__ int nlisted;
-    const int H = (int)cs.H, W = (int)cs.W, wp = W + 2, HW = H * W;
-    const int64_t c = blockIdx.x, b = blockIdx.y;
-    if (threadIdx.x == 0) {
+    __shared__ int32_t qrow[kPlaneMaxChannels][9];
+    __shared__ int16_t qoff[kPlaneMaxChannels][9];
+    __shared__ int8_t nlisted[kPlaneMaxChannels];
+    const int H = (int)cs.H, W = (int)cs.W, wp = W + 2, HW = H * W, psz = (H + 2) * wp;
+    const int64_t c0 = (int64_t)blockIdx.x * ppb, b = blockIdx.y;
+    const int np = (int)min((int64_t)ppb, cs.C - c0);
+    uint16_t *planes = reinterpret_cast<uint16_t *>(plane_smem);
+    for (int ci = threadIdx.x; ci < np; ci += blockDim.x) {
         int n = 0;
         for (int pos = 0; pos < 9; ++pos) {
-            const int64_t k = c * 9 + pos;
+            const int64_t k = (c0 + ci) * 9 + pos;
             const int32_t q = qmap ? qmap[k] : (int32_t)k;
             if (q >= 0) {
-                qrow[n] = q;
-                qoff[n] = (pos / 3) * wp + pos % 3;
+                qrow[ci][n] = q;
+                qoff[ci][n] = (int16_t)((pos / 3) * wp + pos % 3);
                 ++n;
             }
         }
-        nlisted = n;
+        nlisted[ci] = (int8_t)n;
     }
-    // zero border + the plane (16-byte loads: H*W is a multiple of 8 and the
-    // plane starts 16-byte aligned when the input does)
-    for (int e = threadIdx.x; e < (H + 2) * wp; e += blockDim.x) plane[e] = 0;
+    // zero borders, then the planes (16-byte loads: H*W is a multiple of 8 and
+    // each plane starts 16-byte aligned when the input does)
+    for (int e = threadIdx.x; e < np * psz; e += blockDim.x) planes[e] = 0;
     __syncthreads();
-    const uint16_t *src = in + (b * cs.C + c) * (int64_t)HW;
-    for (int v = threadIdx.x; v < HW / 8; v += blockDim.x) {
-        const uint4 q = __ldg(reinterpret_cast<const uint4 *>(src) + v);
+    const int G = HW / 8;
+    const uint4 *src = reinterpret_cast<const uint4 *>(in + (b * cs.C + c0) * (int64_t)HW);
+    for (int t = threadIdx.x; t < np * G; t += blockDim.x) {
+        const int ci = t / G, v = t - ci * G;
+        const uint4 q = __ldg(src + (int64_t)ci * G + v);
         const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+        uint16_t *pl = planes + ci * psz;
         int p = v * 8, ih = p / W, iw = p - ih * W;
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-            plane[(ih + 1) * wp + iw + 1] = (uint16_t)(w[e >> 1] >> (16 * (e & 1)));
+            pl[(ih + 1) * wp + iw + 1] = (uint16_t)(w[e >> 1] >> (16 * (e & 1)));
             if (++iw == W) {
                 iw = 0;
                 ++ih;
@@ -427,9 +435,9 @@ __global__ void __launch_bounds__(256) im2col_3x3_plane_kernel(ConvShape cs, int
         }
     }
     __syncthreads();
-    const int L = nlisted, G = HW / 8;
     uint16_t *dst = xcol + b * (int64_t)HW;
-    for (int g = threadIdx.x; g < G; g += blockDim.x) {
+    for (int t = threadIdx.x; t < np * G; t += blockDim.x) {
+        const int ci = t / G, g = t - ci * G;
         int off[8];
         int p = g * 8, oh = p / W, ow = p - oh * W;
 #pragma unroll
@@ -440,13 +448,15 @@ __global__ void __launch_bounds__(256) im2col_3x3_plane_kernel(ConvShape cs, int
                 ++oh;
             }
         }
+        const uint16_t *pl0 = planes + ci * psz;
+        const int L = nlisted[ci];
         for (int l = 0; l < L; ++l) {
-            const uint16_t *pl = plane + qoff[l];
+            const uint16_t *pl = pl0 + qoff[ci][l];
             uint32_t v[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e)
                 v[e] = (uint32_t)pl[off[2 * e]] | ((uint32_t)pl[off[2 * e + 1]] << 16);
-            *reinterpret_cast<uint4 *>(dst + (int64_t)qrow[l] * ldx + 8 * g) =
+            *reinterpret_cast<uint4 *>(dst + (int64_t)qrow[ci][l] * ldx + 8 * g) =
                 make_uint4(v[0], v[1], v[2], v[3]);
         }
     }
@@ -711,13 +721,24 @@ cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void
         return cudaGetLastError();
     }
     if (cs.kh == 3 && cs.kw == 3 && cs.sh == 1 && cs.sw == 1 && cs.ph == 1 && cs.pw == 1 &&
-        (cs.H * cs.W) % 8 == 0 && (cs.H + 2) * (cs.W + 2) * 2 <= 48 * 1024 && ldx % 8 == 0 &&
-        (reinterpret_cast<uintptr_t>(in) & 15u) == 0 && (reinterpret_cast<uintptr_t>(xcol) & 15u) == 0 &&
-        cs.C <= 0x7fffffffLL && cs.Nb <= 65535) {
-        const size_t smem = (size_t)(cs.H + 2) * (cs.W + 2) * 2;
-        im2col_3x3_plane_kernel<<<dim3((unsigned)cs.C, (unsigned)cs.Nb), 256, smem, s>>>(
-            cs, ldx, qmap, static_cast<const uint16_t *>(in), static_cast<uint16_t *>(xcol));
-        return cudaGetLastError();
+        (cs.H * cs.W) % 8 == 0 && (cs.H + 2) * (cs.W + 2) * 2 <= kPlaneSmem && ldx % 8 == 0 &&
+        cs.H * cs.W <= 32767 && (reinterpret_cast<uintptr_t>(in) & 15u) == 0 &&
+        (reinterpret_cast<uintptr_t>(xcol) & 15u) == 0 && cs.Nb <= 65535) {
+        // channels per block: enough pixel groups for the 256 threads, within
+        // the shared memory and the per-block channel tables
+        const int64_t G = cs.H * cs.W / 8, psz = (cs.H + 2) * (cs.W + 2) * 2;
+        int64_t ppb = (256 + G - 1) / G;
+        if (ppb > kPlaneMaxChannels) ppb = kPlaneMaxChannels;
+        if (ppb > kPlaneSmem / psz) ppb = kPlaneSmem / psz;
+        if (ppb > cs.C) ppb = cs.C;
+        const int64_t gx = (cs.C + ppb - 1) / ppb;
+        if (gx <= 0x7fffffffLL) {
+            im2col_3x3_plane_kernel<<<dim3((unsigned)gx, (unsigned)cs.Nb), 256,
+                                      (size_t)(ppb * psz), s>>>(
+                cs, ldx, (int)ppb, qmap, static_cast<const uint16_t *>(in),
+                static_cast<uint16_t *>(xcol));
+            return cudaGetLastError();
+        }
     }
     constexpr int64_t kStage = 24 * 1024 / 2;     // staged values per block at most
     constexpr int64_t kTab = 4096;                 // table entries (output pixels) per block at most
