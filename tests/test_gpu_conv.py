@@ -44,6 +44,11 @@ CASES = [
     (20, 8, 3, 3, 1, 5, 6, 2, 1, BB, 4, 16, 2.0, bp.F16),        # block-based on a 3x3 view
     (128, 16, 3, 3, 2, 9, 9, 1, 1, BPU, 128, 4, 3.0, bp.BF16),   # bm = 128 filters
     (8, 8, 3, 3, 4, 4, 4, 1, 1, BPU, 8, 4, 9.0, bp.F16),         # keep 1 of 9
+    # plane-staged 3x3 im2col: several channels per block with a partial last
+    # group (4x4: 128 channels per block, 200 = 128 + 72; 8x8: 32 per block)
+    (32, 200, 3, 3, 3, 4, 4, 1, 1, BPU, 8, 4, 4.0, bp.BF16),
+    (24, 40, 3, 3, 2, 8, 8, 1, 1, BPU, 8, 8, 3.0, bp.F16),
+    (16, 12, 3, 3, 2, 28, 28, 1, 1, BPU, 8, 4, 2.0, bp.F16),     # pixel groups cross rows
 ]
 
 
