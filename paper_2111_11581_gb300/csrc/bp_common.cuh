@@ -129,6 +129,16 @@ __device__ __forceinline__ void tma_store_2d(const void *tmap, uint32_t src, int
                  "r"(src), "r"(x), "r"(y)
                  : "memory");
 }
+// 3-D tile store shared -> global through a tensor map (out-of-range parts of
+// the box are not written); tracked by the issuing thread's bulk groups.
+__device__ __forceinline__ void tma_store_3d(const void *tmap, uint32_t src, int32_t x, int32_t y,
+                                             int32_t z) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+            tmap),
+        "r"(src), "r"(x), "r"(y), "r"(z)
+        : "memory");
+}
 // 2-D tile load global -> shared through a tensor map; completion counted in
 // bytes on `bar`, out-of-range elements of the box read as zero.  x (the
 // innermost coordinate) times the element size must be a multiple of 16.

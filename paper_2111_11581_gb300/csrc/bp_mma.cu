@@ -70,11 +70,13 @@ constexpr int kRowsPerWarp = 64 / kGroupWarps;      // list positions per warp a
 constexpr uint32_t kGroupThreads = kGroupWarps * 32;
 
 struct Params {
-    CUtensorMap ymap;       // GEMM output Y as a 2-D tensor, box 32 x 32, 64-byte swizzle
+    CUtensorMap ymap;       // output, box 32 x 32 (x 1), 64-byte swizzle: GEMM Y as a 2-D
+                            // tensor (N, M); NCHW output as a 3-D tensor (Ho*Wo, M, Nb)
     CUtensorMap xmap[4];    // activations X (N inner, K rows), boxes 64 x (8 << i), 128-byte swizzle
     int dtype;
     int relu;
     int conv;               // 1: Y is the NCHW output of a convolution
+    int ytma;               // 1: output boxes are written with TMA stores through ymap
     int64_t M, num_slabs;
     int64_t N;              // tokens (GEMM) or Nb*Ho*Wo pixels (conv)
     int nt;                 // activation columns per tile: a multiple of 32, 64 .. 256
@@ -518,13 +520,14 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
 }
 
 // ------------------------------------------------------------------ epilogue
-template <bool kSplit>
+template <bool kSplit, bool kConv>
 __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
     const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int q = warp & 3;                  // tensor-memory lane quadrant this warp may read
     const uint32_t stg = smem_u32(s.ystage + (warp - kEpiWarp0) * 4096);
+    uint32_t yseq = 0;                       // TMA box stores issued by this warp
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int64_t it = blockIdx.x; it < p.num_units; it += gridDim.x) {
@@ -562,24 +565,40 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
         };
         auto store = [&](const uint32_t (&pk)[16], int c0) {
             const int64_t n = t.n0 + c0;
-            if (p.conv) {
-                // NCHW output, pixel n = b*HoWo + hw is element (b, m, hw): stage the
-                // 32 x 32 box (lane = channel row, 80-byte rows), then write it with
-                // lanes along the pixels, one coalesced 64-byte store per channel
-                if ((p.HoWo & 7) == 0 && (n % p.HoWo) + 32 <= p.HoWo && n + 32 <= p.N) {
-                    // the 32 pixels are consecutive in one image, 16-byte aligned:
-                    // each lane stores its channel's 64-byte row segment directly
-                    if (vrow) {
-                        const int64_t bb = n / p.HoWo, hw = n - bb * p.HoWo;
-                        uint4 *d4 = reinterpret_cast<uint4 *>(p.Y + (bb * p.M + m) * p.HoWo + hw);
+            if (kConv) {
+                // NCHW output, pixel n = b*HoWo + hw is element (b, m, hw)
+                const uint32_t bb = (uint32_t)n / (uint32_t)p.HoWo;
+                const uint32_t hw = (uint32_t)n - bb * (uint32_t)p.HoWo;
+                if (p.ytma && hw + 32 <= (uint32_t)p.HoWo) {
+                    // the 32 pixels lie in one image: stage the box like a GEMM
+                    // box (below) and store it at (hw, m, b) of the 3-D output
+                    // map (Ho*Wo is a multiple of 8, so hw is 16-byte aligned)
+                    const uint32_t sb = stg + (yseq & 1u) * 2048;
+                    ++yseq;
+                    if (lane == 0) bulk_wait_read<1>();
+                    __syncwarp();
 #pragma unroll
-                        for (int ch = 0; ch < 4; ++ch)
-                            d4[ch] = make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2],
-                                                pk[4 * ch + 3]);
+                    for (int ch = 0; ch < 4; ++ch)
+                        st_shared_v4(sb + lane * 64 + ((ch ^ ((lane >> 1) & 3)) << 4),
+                                     make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2],
+                                                pk[4 * ch + 3]));
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_3d(&p.ymap, sb, (int32_t)hw, (int32_t)(t.slab * kSlab + row0),
+                                     (int32_t)bb);
+                        bulk_commit();
                     }
                     return;
                 }
+                // Ho*Wo not a multiple of 8, or the 32 pixels cross an image
+                // boundary: stage the 32 x 32 box (lane = channel row, 80-byte
+                // rows), then write it with lanes along the pixels, one
+                // coalesced 64-byte store per channel
                 uint8_t *box = s.ystage + (warp - kEpiWarp0) * 4096;
+                // the box overlaps both TMA staging boxes: their stores must
+                // have read them
+                if (p.ytma && lane == 0) bulk_wait_read<0>();
                 __syncwarp();                      // the previous box has been read
 #pragma unroll
                 for (int ch = 0; ch < 4; ++ch)
@@ -600,8 +619,12 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             // GEMM: 32 x 32 box staged in shared memory (64-byte swizzle: 16-byte
             // chunk c of row r sits at chunk c ^ ((r >> 1) & 3)), then TMA-stored;
             // rows past M and columns past N of the box are not written
-            const uint32_t sb = stg + ((c0 >> 5) & 1) * 2048;
-            if (lane == 0) bulk_wait_read<1>();     // the store that used this buffer is done
+            // the two boxes alternate over the warp's stores, across items (an
+            // item may have an odd number of groups): the box about to be written
+            // was used by the store before last
+            const uint32_t sb = stg + (yseq & 1u) * 2048;
+            ++yseq;
+            if (lane == 0) bulk_wait_read<1>();     // the store that used this box is done
             __syncwarp();
 #pragma unroll
             for (int ch = 0; ch < 4; ++ch)
@@ -700,12 +723,13 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             }
         }
     }
-    if (!p.conv && lane == 0) bulk_wait_all();   // staged output fully written before exit
+    if (p.ytma && lane == 0) bulk_wait_all();    // staged output fully written before exit
 }
 
 // kSplit: the launch has split items (a separate instantiation keeps the
-// common kernel free of the partial-tile code).
-template <bool kSplit>
+// common kernel free of the partial-tile code); kConv: the output is the NCHW
+// tensor of a convolution (GEMM launches compile no convolution store code).
+template <bool kSplit, bool kConv>
 __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_constant__ Params p) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     const Smem s = carve(smem_raw, p);
@@ -756,7 +780,7 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
         if ((threadIdx.x & 31) == 0) mma_issuer(p, s, tmem);
         __syncwarp();
     } else {
-        epilogue<kSplit>(p, s, tmem);
+        epilogue<kSplit, kConv>(p, s, tmem);
     }
 
     tc_fence_before();
@@ -915,16 +939,32 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
                 CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
+        p.ytma = 1;
+    } else if (p.HoWo % 8 == 0) {
+        // NCHW output as (Ho*Wo, M, Nb): 32-pixel x 32-channel boxes of one
+        // image (the image stride, Ho*Wo*2 bytes, must be a multiple of 16)
+        const cuuint64_t gdim[3] = {(cuuint64_t)p.HoWo, (cuuint64_t)P.lay.M,
+                                    (cuuint64_t)conv->Nb};
+        const cuuint64_t gstride[2] = {(cuuint64_t)p.HoWo * 2, (cuuint64_t)(P.lay.M * p.HoWo * 2)};
+        const cuuint32_t box[3] = {32, 32, 1};
+        const cuuint32_t estride[3] = {1, 1, 1};
+        if (enc(&p.ymap, tdt, 3, Y, gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+        p.ytma = 1;
     }
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [] {
-        attr_err = cudaFuncSetAttribute(bp_mma_kernel<false>,
-                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxSmem);
-        if (attr_err == cudaSuccess)
-            attr_err = cudaFuncSetAttribute(bp_mma_kernel<true>,
-                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                            (int)kMaxSmem);
+        const void *fns[4] = {(const void *)bp_mma_kernel<false, false>,
+                              (const void *)bp_mma_kernel<true, false>,
+                              (const void *)bp_mma_kernel<false, true>,
+                              (const void *)bp_mma_kernel<true, true>};
+        for (const void *f : fns)
+            if (attr_err == cudaSuccess)
+                attr_err = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                (int)kMaxSmem);
     });
     if (attr_err != cudaSuccess) return attr_err;
     const int64_t grid = p.num_units < num_sms() ? p.num_units : num_sms();
@@ -941,8 +981,11 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return p.split > 1 ? cudaLaunchKernelEx(&cfg, bp_mma_kernel<true>, p)
-                       : cudaLaunchKernelEx(&cfg, bp_mma_kernel<false>, p);
+    if (conv)
+        return p.split > 1 ? cudaLaunchKernelEx(&cfg, bp_mma_kernel<true, true>, p)
+                           : cudaLaunchKernelEx(&cfg, bp_mma_kernel<false, true>, p);
+    return p.split > 1 ? cudaLaunchKernelEx(&cfg, bp_mma_kernel<true, false>, p)
+                       : cudaLaunchKernelEx(&cfg, bp_mma_kernel<false, false>, p);
 }
 
 }  // namespace bp

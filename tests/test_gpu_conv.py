@@ -49,6 +49,10 @@ CASES = [
     (32, 200, 3, 3, 3, 4, 4, 1, 1, BPU, 8, 4, 4.0, bp.BF16),
     (24, 40, 3, 3, 2, 8, 8, 1, 1, BPU, 8, 8, 3.0, bp.F16),
     (16, 12, 3, 3, 2, 28, 28, 1, 1, BPU, 8, 4, 2.0, bp.F16),     # pixel groups cross rows
+    # TMA box stores of the NCHW output: two filter slabs, the second partial
+    # (boxes clipped at F); 28x28 = 784 pixels, some 32-pixel groups cross images
+    (200, 16, 3, 3, 3, 8, 8, 1, 1, BPU, 8, 4, 3.0, bp.BF16),
+    (96, 64, 1, 1, 2, 28, 28, 0, 1, BB, 32, 32, 2.0, bp.BF16),
 ]
 
 
