@@ -517,12 +517,32 @@ def _layer_step(layer, dtype, flush, reps=5):
             ours_fn = dense_fn
     t_ours = timed(ours_fn)
     t_dense = timed(dense_fn)
+
+    # the same calls replayed from a CUDA graph (one graph launch per layer):
+    # what a serving loop that captures its layers pays, without the host
+    # path of each call (argument checks, tensor-map encoding, the launch)
+    def graphed(fn):
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            fn()
+        torch.cuda.current_stream().wait_stream(side)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            fn()
+        return g
+
+    g_ours, g_dense = graphed(ours_fn), graphed(dense_fn)
+    t_ours_g = timed(g_ours.replay)
+    t_dense_g = timed(g_dense.replay)
+    del g_ours, g_dense
     if bp.device_status() != bp.OK:
         raise RuntimeError("kernel watchdog fired")
     n = layer.gemm_n
     return {"layer": layer.name, "kind": layer.kind, "M": layer.M, "K": layer.K, "N": n,
             "bm": layer.bm, "bk": layer.bk, "rate": layer.rate, "pruned": not dense,
-            "kept_flop": 2.0 * kept * n, "us": round(t_ours, 2), "dense_us": round(t_dense, 2)}
+            "kept_flop": 2.0 * kept * n, "us": round(t_ours, 2), "dense_us": round(t_dense, 2),
+            "us_graph": round(t_ours_g, 2), "dense_us_graph": round(t_dense_g, 2)}
 
 
 def run_workload(args):
@@ -711,16 +731,21 @@ def run_workload(args):
         rows.append(_layer_step(layer, dt, flush))
         r = rows[-1]
         print(f"# {r['layer']:40s} {r['us']:9.2f} us (dense {r['dense_us']:9.2f})"
+              f"  graph {r['us_graph']:9.2f} (dense {r['dense_us_graph']:9.2f})"
               f"  {r['kept_flop'] / r['us'] / 1e6:8.1f} TFLOP/s", file=sys.stderr, flush=True)
     pr = [r for r in rows if r["pruned"]]
     t = sum(r["us"] for r in pr)
     fl = sum(r["kept_flop"] for r in pr)
     td = sum(r["dense_us"] for r in pr)
+    tg = sum(r["us_graph"] for r in pr)
+    tdg = sum(r["dense_us_graph"] for r in pr)
     out = {"metric": METRIC, "value": round(fl / t / 1e6, 2), "unit": UNIT, "n_gpus": 1,
            "workload": name, "pruned_layers": len(pr), "sum_us": round(t, 2),
            "dense_sum_us": round(td, 2), "speedup_vs_dense": round(td / t, 3),
+           "graph": {"value": round(fl / tg / 1e6, 2), "sum_us": round(tg, 2),
+                     "dense_sum_us": round(tdg, 2), "speedup_vs_dense": round(tdg / tg, 3)},
            "timing": "per-layer device time, median of 5, L2 flushed (256 MiB write, read back) "
-                     "before each launch",
+                     "before each launch; 'graph': the same calls replayed from a CUDA graph",
            "layers": rows}
     print(json.dumps(out), flush=True)
 
