@@ -378,6 +378,51 @@ __global__ void __launch_bounds__(256) im2col_1x1_kernel(ConvShape cs, int64_t l
     }
 }
 
+// im2col of a 1x1 convolution (any stride and padding) for small or
+// unaligned planes: row q = qmap[c] of the im2col matrix, column
+// e = b*Ho*Wo + oh*Wo + ow, holds in[b, c, oh*sh - ph, ow*sw - pw] (zero
+// outside).  Grid (column groups, channels): each thread writes 8 consecutive
+// columns with one 16-byte store (ldx is a multiple of 8, so the group stays
+// inside the row's ldx columns; columns past N get zeros), walking (b, oh, ow)
+// incrementally from its first column.  A warp covers 256 consecutive columns
+// of one row, whatever the plane size.
+__global__ void __launch_bounds__(256) im2col_1x1_rows_kernel(ConvShape cs, int64_t ldx,
+                                                              const int32_t *__restrict__ qmap,
+                                                              const uint16_t *__restrict__ in,
+                                                              uint16_t *__restrict__ xcol) {
+    const int64_t c = blockIdx.y;
+    const int64_t q = qmap ? qmap[c] : c;
+    if (q < 0) return;
+    const uint32_t Wo = (uint32_t)cs.Wo, HoWo = (uint32_t)(cs.Ho * cs.Wo);
+    const uint32_t N = (uint32_t)cs.Nb * HoWo;                  // < 2^31 (checked on the host)
+    const uint32_t e0 = (blockIdx.x * 256u + threadIdx.x) * 8u;
+    if (e0 >= N) return;
+    uint32_t b = e0 / HoWo, r = e0 - b * HoWo;
+    uint32_t oh = r / Wo, ow = r - oh * Wo;
+    uint32_t w[4];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        uint16_t v = 0;
+        if (e0 + j < N) {
+            const int ih = (int)(oh * cs.sh) - cs.ph, iw = (int)(ow * cs.sw) - cs.pw;
+            if ((unsigned)ih < (unsigned)cs.H && (unsigned)iw < (unsigned)cs.W)
+                v = __ldg(in + (((int64_t)b * cs.C + c) * cs.H + ih) * cs.W + iw);
+            if (++ow == Wo) {
+                ow = 0;
+                if (++oh == (uint32_t)cs.Ho) {
+                    oh = 0;
+                    ++b;
+                }
+            }
+        }
+        if (j & 1)
+            w[j >> 1] |= (uint32_t)v << 16;
+        else
+            w[j >> 1] = v;
+    }
+    *reinterpret_cast<uint4 *>(xcol + q * ldx + e0) = make_uint4(w[0], w[1], w[2], w[3]);
+}
+
 // im2col of a 3x3, stride-1, padding-1 convolution whose image has H*W a
 // multiple of 8: one block per (group of ppb channels, image).  The block
 // stages the channels' padded planes ((H+2) x (W+2) each) once, collects each
@@ -707,11 +752,22 @@ int64_t im2col_row_width(const ConvShape &cs) {
 
 cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void *xcol,
                           const int32_t *qmap, cudaStream_t s) {
-    if (cs.kh == 1 && cs.kw == 1 && cs.sh == 1 && cs.sw == 1 && cs.ph == 0 && cs.pw == 0) {
+    if (cs.kh == 1 && cs.kw == 1 && cs.sh == 1 && cs.sw == 1 && cs.ph == 0 && cs.pw == 0 &&
+        (cs.H * cs.W) % 8 == 0 && cs.H * cs.W >= 256) {
+        // large planes of 16-byte multiples: one block copies one plane
         if (cs.C > 0x7fffffffLL || cs.Nb > 65535) return cudaErrorInvalidValue;
         im2col_copy_kernel<<<dim3((unsigned)cs.C, (unsigned)cs.Nb), 256, 0, s>>>(
             cs.C, cs.H * cs.W, ldx, qmap, static_cast<const uint16_t *>(in),
             static_cast<uint16_t *>(xcol));
+        return cudaGetLastError();
+    }
+    if (cs.kh == 1 && cs.kw == 1 && ldx % 8 == 0 && (reinterpret_cast<uintptr_t>(xcol) & 15u) == 0) {
+        // small or unaligned planes, strided or padded 1x1: threads along the rows
+        const int64_t N = cs.Nb * cs.Ho * cs.Wo;
+        const int64_t gx = (N + 2047) / 2048;
+        if (cs.C > 65535 || N > 0x7fffffffLL - 8 || gx > 0x7fffffffLL) return cudaErrorInvalidValue;
+        im2col_1x1_rows_kernel<<<dim3((unsigned)gx, (unsigned)cs.C), 256, 0, s>>>(
+            cs, ldx, qmap, static_cast<const uint16_t *>(in), static_cast<uint16_t *>(xcol));
         return cudaGetLastError();
     }
     if (cs.kh == 1 && cs.kw == 1) {
