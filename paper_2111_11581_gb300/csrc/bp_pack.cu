@@ -378,21 +378,33 @@ __global__ void __launch_bounds__(256) im2col_1x1_kernel(ConvShape cs, int64_t l
     }
 }
 
-// im2col of a 1x1 convolution (any stride and padding) for small or
-// unaligned planes: row q = qmap[c] of the im2col matrix, column
-// e = b*Ho*Wo + oh*Wo + ow, holds in[b, c, oh*sh - ph, ow*sw - pw] (zero
-// outside).  Grid (column groups, channels): each thread writes 8 consecutive
-// columns with one 16-byte store (ldx is a multiple of 8, so the group stays
-// inside the row's ldx columns; columns past N get zeros), walking (b, oh, ow)
-// incrementally from its first column.  A warp covers 256 consecutive columns
-// of one row, whatever the plane size.
-__global__ void __launch_bounds__(256) im2col_1x1_rows_kernel(ConvShape cs, int64_t ldx,
-                                                              const int32_t *__restrict__ qmap,
-                                                              const uint16_t *__restrict__ in,
-                                                              uint16_t *__restrict__ xcol) {
-    const int64_t c = blockIdx.y;
-    const int64_t q = qmap ? qmap[c] : c;
+// im2col with threads along the rows (any kernel size, stride and
+// padding; small or unaligned planes): row q = qmap[k] of the im2col matrix,
+// k = c*kh*kw + i*kw + j, column e = b*Ho*Wo + oh*Wo + ow, holds
+// in[b, c, oh*sh - ph + i, ow*sw - pw + j] (zero outside).  Grid (column
+// groups, K): each thread writes 8 consecutive columns with one 16-byte store
+// (ldx is a multiple of 8, so the group stays inside the row's ldx columns;
+// columns past N get zeros), walking (b, oh, ow) incrementally from its first
+// column.  A warp covers 256 consecutive columns of one row whatever the plane
+// size; the rows of one channel read the same input pixels, from L2.
+// k1: a 1x1 kernel (row k is channel k).
+template <bool k1>
+__global__ void __launch_bounds__(256) im2col_rows_kernel(ConvShape cs, int64_t ldx,
+                                                          const int32_t *__restrict__ qmap,
+                                                          const uint16_t *__restrict__ in,
+                                                          uint16_t *__restrict__ xcol) {
+    const int64_t k = blockIdx.y;
+    const int64_t q = qmap ? qmap[k] : k;
     if (q < 0) return;
+    uint32_t c = (uint32_t)k;                                   // k < 65536 (grid y)
+    int di = -cs.ph, dj = -cs.pw;
+    if (!k1) {
+        const uint32_t kk = (uint32_t)(cs.kh * cs.kw);
+        c = (uint32_t)k / kk;
+        const int pos = (int)((uint32_t)k - c * kk);
+        di += pos / cs.kw;
+        dj += pos % cs.kw;
+    }
     const uint32_t Wo = (uint32_t)cs.Wo, HoWo = (uint32_t)(cs.Ho * cs.Wo);
     const uint32_t N = (uint32_t)cs.Nb * HoWo;                  // < 2^31 (checked on the host)
     const uint32_t e0 = (blockIdx.x * 256u + threadIdx.x) * 8u;
@@ -401,10 +413,10 @@ __global__ void __launch_bounds__(256) im2col_1x1_rows_kernel(ConvShape cs, int6
     uint32_t oh = r / Wo, ow = r - oh * Wo;
     uint32_t w[4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int t = 0; t < 8; ++t) {
         uint16_t v = 0;
-        if (e0 + j < N) {
-            const int ih = (int)(oh * cs.sh) - cs.ph, iw = (int)(ow * cs.sw) - cs.pw;
+        if (e0 + t < N) {
+            const int ih = (int)(oh * cs.sh) + di, iw = (int)(ow * cs.sw) + dj;
             if ((unsigned)ih < (unsigned)cs.H && (unsigned)iw < (unsigned)cs.W)
                 v = __ldg(in + (((int64_t)b * cs.C + c) * cs.H + ih) * cs.W + iw);
             if (++ow == Wo) {
@@ -415,10 +427,10 @@ __global__ void __launch_bounds__(256) im2col_1x1_rows_kernel(ConvShape cs, int6
                 }
             }
         }
-        if (j & 1)
-            w[j >> 1] |= (uint32_t)v << 16;
+        if (t & 1)
+            w[t >> 1] |= (uint32_t)v << 16;
         else
-            w[j >> 1] = v;
+            w[t >> 1] = v;
     }
     *reinterpret_cast<uint4 *>(xcol + q * ldx + e0) = make_uint4(w[0], w[1], w[2], w[3]);
 }
@@ -750,6 +762,26 @@ int64_t im2col_row_width(const ConvShape &cs) {
     return cs.W + 2 * cs.pw;
 }
 
+static bool rows_kernel_ok(const ConvShape &cs, int64_t ldx, const void *xcol) {
+    return ldx % 8 == 0 && (reinterpret_cast<uintptr_t>(xcol) & 15u) == 0 &&
+           cs.C * cs.kh * cs.kw <= 65535 && cs.Nb * cs.Ho * cs.Wo <= 0x7fffffffLL - 8;
+}
+
+static cudaError_t launch_im2col_rows(const ConvShape &cs, int64_t ldx, const void *in, void *xcol,
+                                      const int32_t *qmap, cudaStream_t s) {
+    const int64_t gx = (cs.Nb * cs.Ho * cs.Wo + 2047) / 2048;
+    const dim3 grid((unsigned)gx, (unsigned)(cs.C * cs.kh * cs.kw));
+    if (cs.kh == 1 && cs.kw == 1)
+        im2col_rows_kernel<true><<<grid, 256, 0, s>>>(cs, ldx, qmap,
+                                                      static_cast<const uint16_t *>(in),
+                                                      static_cast<uint16_t *>(xcol));
+    else
+        im2col_rows_kernel<false><<<grid, 256, 0, s>>>(cs, ldx, qmap,
+                                                       static_cast<const uint16_t *>(in),
+                                                       static_cast<uint16_t *>(xcol));
+    return cudaGetLastError();
+}
+
 cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void *xcol,
                           const int32_t *qmap, cudaStream_t s) {
     if (cs.kh == 1 && cs.kw == 1 && cs.sh == 1 && cs.sw == 1 && cs.ph == 0 && cs.pw == 0 &&
@@ -761,14 +793,9 @@ cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void
             static_cast<uint16_t *>(xcol));
         return cudaGetLastError();
     }
-    if (cs.kh == 1 && cs.kw == 1 && ldx % 8 == 0 && (reinterpret_cast<uintptr_t>(xcol) & 15u) == 0) {
+    if (cs.kh == 1 && cs.kw == 1 && rows_kernel_ok(cs, ldx, xcol)) {
         // small or unaligned planes, strided or padded 1x1: threads along the rows
-        const int64_t N = cs.Nb * cs.Ho * cs.Wo;
-        const int64_t gx = (N + 2047) / 2048;
-        if (cs.C > 65535 || N > 0x7fffffffLL - 8 || gx > 0x7fffffffLL) return cudaErrorInvalidValue;
-        im2col_1x1_rows_kernel<<<dim3((unsigned)gx, (unsigned)cs.C), 256, 0, s>>>(
-            cs, ldx, qmap, static_cast<const uint16_t *>(in), static_cast<uint16_t *>(xcol));
-        return cudaGetLastError();
+        return launch_im2col_rows(cs, ldx, in, xcol, qmap, s);
     }
     if (cs.kh == 1 && cs.kw == 1) {
         if (cs.C > 0x7fffffffLL || cs.Nb > 65535) return cudaErrorInvalidValue;
@@ -796,6 +823,12 @@ cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void
             return cudaGetLastError();
         }
     }
+    // strided convolutions and planes of fewer than 32 output pixels: threads
+    // along the rows (measured faster there: ResNet-50's stride-2 3x3 layers,
+    // VGG-16's 2x2 layers); stride-1 layers on larger planes stage the input
+    // rows of a band in shared memory once for all kernel positions
+    if ((cs.sh != 1 || cs.sw != 1 || cs.Ho * cs.Wo < 32) && rows_kernel_ok(cs, ldx, xcol))
+        return launch_im2col_rows(cs, ldx, in, xcol, qmap, s);
     constexpr int64_t kStage = 24 * 1024 / 2;     // staged values per block at most
     constexpr int64_t kTab = 4096;                 // table entries (output pixels) per block at most
     const int64_t wp = im2col_row_width(cs);

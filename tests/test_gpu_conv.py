@@ -53,6 +53,9 @@ CASES = [
     # (boxes clipped at F); 28x28 = 784 pixels, some 32-pixel groups cross images
     (200, 16, 3, 3, 3, 8, 8, 1, 1, BPU, 8, 4, 3.0, bp.BF16),
     (96, 64, 1, 1, 2, 28, 28, 0, 1, BB, 32, 32, 2.0, bp.BF16),
+    # im2col with threads along the rows: stride-1 planes under 32 pixels
+    (16, 8, 3, 3, 3, 5, 5, 1, 1, BPU, 8, 4, 3.0, bp.F16),
+    (32, 16, 3, 3, 5, 2, 2, 1, 1, BPU, 8, 4, 8.0, bp.BF16),
 ]
 
 
