@@ -173,6 +173,13 @@ __device__ __forceinline__ void cp_async_16(uint32_t dst, const void *src, uint3
                  "r"(src_bytes)
                  : "memory");
 }
+// The same copy of a full 16 bytes, without the zero-fill operand: the
+// activation gather of full tiles measured ~2 % faster with it (the L2
+// access-size hint measured neutral: none, 128 and 256 bytes alike).
+__device__ __forceinline__ void cp_async_16_full(uint32_t dst, const void *src) {
+    asm volatile("cp.async.cg.shared.global.L2::128B [%0], [%1], 16;" ::"r"(dst), "l"(src)
+                 : "memory");
+}
 // Arrive on `bar` once every cp.async this thread issued so far has landed
 // (the arrival is not pre-counted: the barrier's expected count includes it).
 __device__ __forceinline__ void cp_async_arrive_noinc(uint64_t *bar) {

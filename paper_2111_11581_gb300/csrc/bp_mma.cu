@@ -299,11 +299,22 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
                 const uint32_t xs = smem_u32(s.x + stage * kXTileBytes);
                 const int cn = lane >> 3, jj = lane & 7;
                 if (lane * 8 < p.nt) {
+                    // lanes whose 8 columns are all inside N copy without the
+                    // zero-fill operand
+                    if (nb == 16u) {
 #pragma unroll
-                    for (int i = 0; i < kRowsPerWarp; ++i) {
-                        const int r = gw + kGroupWarps * i;
-                        cp_async_16(xs + cn * 8192 + r * 128 + ((jj ^ (r & 7)) << 4),
-                                    xcol + (int64_t)idx[i] * p.ldx, nb);
+                        for (int i = 0; i < kRowsPerWarp; ++i) {
+                            const int r = gw + kGroupWarps * i;
+                            cp_async_16_full(xs + cn * 8192 + r * 128 + ((jj ^ (r & 7)) << 4),
+                                             xcol + (int64_t)idx[i] * p.ldx);
+                        }
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < kRowsPerWarp; ++i) {
+                            const int r = gw + kGroupWarps * i;
+                            cp_async_16(xs + cn * 8192 + r * 128 + ((jj ^ (r & 7)) << 4),
+                                        xcol + (int64_t)idx[i] * p.ldx, nb);
+                        }
                     }
                 }
                 // Signal the stage once this thread's copies have landed, without
