@@ -56,6 +56,10 @@ CASES = [
     # im2col with threads along the rows: stride-1 planes under 32 pixels
     (16, 8, 3, 3, 3, 5, 5, 1, 1, BPU, 8, 4, 3.0, bp.F16),
     (32, 16, 3, 3, 5, 2, 2, 1, 1, BPU, 8, 4, 8.0, bp.BF16),
+    # planes of 32-127 pixels, H*W not a multiple of 8: image groups staged in
+    # shared memory, 8-column groups spanning two images, a partial last group
+    (24, 16, 3, 3, 11, 7, 7, 1, 1, BPU, 8, 4, 3.0, bp.BF16),
+    (16, 24, 3, 3, 10, 6, 6, 1, 1, BPU, 8, 4, 3.0, bp.F16),
 ]
 
 
