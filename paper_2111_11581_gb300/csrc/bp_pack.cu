@@ -523,7 +523,8 @@ __global__ void __launch_bounds__(256) im2col_3x3_plane_kernel(ConvShape cs, int
 // multiple of 8: one block per (group of ppb channels, group of ig images),
 // ig * H*W a multiple of 8 so that every block's columns start 16-byte
 // aligned.  The block stages the zero-bordered planes [channel][image] in
-// shared memory (2-byte loads: planes are not 16-byte aligned), then each
+// shared memory (one warp per plane, 2-byte loads: planes are not 16-byte
+// aligned), then each
 // thread writes 8 consecutive columns of a channel's listed rows with one
 // 16-byte store; the 8 columns may span two images of the group.  Columns of
 // the last group past N are written as zeros (inside the row's ldx).
@@ -556,13 +557,28 @@ __global__ void __launch_bounds__(256) im2col_3x3_images_kernel(ConvShape cs, in
     }
     for (int e = threadIdx.x; e < np * ig * psz; e += blockDim.x) planes[e] = 0;
     __syncthreads();
-    // interiors: element (ci, bi, p) of the block's input
+    // interiors: one warp per (channel, image) plane, lanes along its pixels;
+    // (ih, iw) advance by 32 pixels per step (one conditional carry: the
+    // column step 32 mod W is below W)
     const int per_ch = ni * HW;
-    for (int t = threadIdx.x; t < np * per_ch; t += blockDim.x) {
-        const int ci = t / per_ch, r = t - ci * per_ch, bi = r / HW, p = r - bi * HW;
-        const int ih = p / W, iw = p - ih * W;
-        planes[(ci * ig + bi) * psz + (ih + 1) * wp + iw + 1] =
-            __ldg(in + ((b0 + bi) * cs.C + c0 + ci) * (int64_t)HW + p);
+    {
+        const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+        const int dq = 32 / W, dr = 32 - dq * W, lq = lane / W, lr = lane - lq * W;
+        for (int pl = warp; pl < np * ni; pl += nw) {
+            const int ci = pl / ni, bi = pl - ci * ni;
+            const uint16_t *src = in + ((b0 + bi) * cs.C + c0 + ci) * (int64_t)HW;
+            uint16_t *pd = planes + (ci * ig + bi) * psz + wp + 1;
+            int ih = lq, iw = lr;
+            for (int p = lane; p < HW; p += 32) {
+                pd[ih * wp + iw] = __ldg(src + p);
+                ih += dq;
+                iw += dr;
+                if (iw >= W) {
+                    iw -= W;
+                    ++ih;
+                }
+            }
+        }
     }
     __syncthreads();
     const int G = (per_ch + 7) / 8;                  // 8-column groups per channel row
@@ -903,11 +919,12 @@ cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void
         }
     }
     if (cs.kh == 3 && cs.kw == 3 && cs.sh == 1 && cs.sw == 1 && cs.ph == 1 && cs.pw == 1 &&
-        (cs.H * cs.W) % 8 != 0 && cs.H * cs.W >= 32 && cs.H * cs.W < 128 && ldx % 8 == 0 &&
+        (cs.H * cs.W) % 8 != 0 && cs.H * cs.W >= 32 && cs.H * cs.W < 256 && ldx % 8 == 0 &&
         (reinterpret_cast<uintptr_t>(xcol) & 15u) == 0) {
-        // H*W not a multiple of 8, 32 to 127 pixels (measured: 7x7 planes
-        // 62.3 -> 53.5 us on ResNet-50 s4b2_3x3; 14x14 planes stay faster with
-        // the banded kernel, planes under 32 pixels with the rows kernel):
+        // H*W not a multiple of 8, 32 to 255 pixels (measured on ResNet-50:
+        // 7x7 planes 62.3 -> 51.5 us on s4b2_3x3, 14x14 planes even with the
+        // banded kernel at 51.5 us; planes under 32 pixels stay faster with the
+        // rows kernel):
         // image groups with ig * H*W a multiple of 8, at least ~256 columns
         // per channel row, planes within the stage
         const int64_t HW = cs.H * cs.W, psz = (cs.H + 2) * (cs.W + 2) * 2;
