@@ -725,6 +725,11 @@ def run_workload(args):
                      [l for l in layers if l[0].bk == 32 and l[0].M != 4096 and l[1] == inputs.BF16]
     else:
         raise SystemExit(f"unknown workload {name}")
+    if args.layers:
+        keep = set(args.layers.split(","))
+        layers = [l for l in layers if (l[0] if isinstance(l, tuple) else l).name in keep]
+        if not layers:
+            raise SystemExit(f"no layer of {name} is named in --layers {args.layers}")
     rows = []
     for item in layers:
         layer, dt = item if isinstance(item, tuple) else (item, dtype)
@@ -734,6 +739,8 @@ def run_workload(args):
               f"  graph {r['us_graph']:9.2f} (dense {r['dense_us_graph']:9.2f})"
               f"  {r['kept_flop'] / r['us'] / 1e6:8.1f} TFLOP/s", file=sys.stderr, flush=True)
     pr = [r for r in rows if r["pruned"]]
+    if not pr:
+        raise SystemExit(f"the selected layers of {name} are all dense")
     t = sum(r["us"] for r in pr)
     fl = sum(r["kept_flop"] for r in pr)
     td = sum(r["dense_us"] for r in pr)
@@ -765,6 +772,8 @@ def main():
                          "the reweighted regulariser; rowcol: row + column pruning; e4: "
                          "pattern vs block-punched 3x3 latency")
     ap.add_argument("--sweep-subset", action="store_true")
+    ap.add_argument("--layers", default=None,
+                    help="comma-separated layer names: time only these layers of the workload")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
