@@ -116,6 +116,13 @@ def max_threads() -> int:
     return int(_load().oracle_max_threads())
 
 
+def set_threads(n: int) -> None:
+    """Threads of the oracle's parallel loops from now on (results do not depend on it)."""
+    lib = _load()
+    lib.oracle_set_threads.argtypes = [ctypes.c_int]
+    lib.oracle_set_threads(int(n))
+
+
 # ---------------------------------------------------------------- conversions
 def to_double(bits, dtype: int) -> np.ndarray:
     """Exact value of each fp16/bf16 bit pattern as float64."""

@@ -691,3 +691,16 @@ int oracle_max_threads(void)
     return 1;
 #endif
 }
+
+/* Threads of the parallel loops from now on (timing only: every loop's
+ * result is the same for any thread count, each output element being
+ * computed by one thread in a fixed order). */
+void oracle_set_threads(int n)
+{
+#ifdef _OPENMP
+    extern void omp_set_num_threads(int);
+    if (n >= 1) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}

@@ -408,3 +408,30 @@ def test_masked_conv2d_1x1_is_gemm_per_image():
     for b in range(Nb):
         _, g = oracle.masked_gemm(W, mask, x[b].reshape(C, H * Wd), F16, return_acc=True)
         assert np.abs(acc[b].reshape(F, -1) - g).max() == 0.0
+
+
+def test_oracle_results_do_not_depend_on_thread_count():
+    """The parallel loops compute each output in one thread in a fixed order,
+    so masks and outputs are identical with one thread and with all."""
+    dt = inputs.BF16
+    W = inputs.normal((96, 160), 0.05, dt, 41)
+    X = inputs.uniform((160, 24), -1.0, 1.0, dt, 42)
+    Wc = inputs.normal((12, 6, 3, 3), 0.2, dt, 43)
+    x = inputs.normal((2, 6, 9, 7), 1.0, dt, 44)
+    n = oracle.max_threads()
+
+    def run():
+        m = oracle.prune(W, dt, BB, 32, 16, 3.0)
+        y = oracle.masked_gemm(W, m, X, dt)
+        mc = oracle.prune(Wc.reshape(12, -1), dt, BP, 4, 2, 3.0, 3, 3)
+        yc = oracle.masked_conv2d(Wc, mc, x, dt, pad=(1, 1), stride=(2, 1))
+        return m, y, mc, yc
+
+    many = run()
+    oracle.set_threads(1)
+    try:
+        one = run()
+    finally:
+        oracle.set_threads(n)
+    for a, b in zip(many, one):
+        assert np.array_equal(a, b)
