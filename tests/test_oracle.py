@@ -231,6 +231,62 @@ def test_prune_is_the_unique_energy_optimum(scheme, M, K, kh, kw, bm, bk, rate):
     assert abs(sum(s[keep == 1]) - best) < 1e-9
 
 
+def _random_layouts(n, seed):
+    rng = np.random.default_rng(seed)
+    out = []
+    for _ in range(n):
+        if rng.random() < 0.5:
+            M, K = int(rng.integers(1, 200)), int(rng.integers(1, 300))
+            bm = int(rng.choice([1, 2, 3, 8, 16, 32, 64, 128]))
+            bk = int(rng.choice([1, 4, 7, 8, 16, 32]))
+            rate = float(rng.choice([1.0, 1.5, 2.0, 3.0, 8.0 / 3.0, 4.0, 6.0, 16.0]))
+            out.append((BB, M, K, 1, 1, bm, bk, rate))
+        else:
+            kh, kw = [(1, 1), (3, 3), (2, 3)][int(rng.integers(0, 3))]
+            M, C = int(rng.integers(1, 70)), int(rng.integers(1, 40))
+            bm = int(rng.choice([1, 4, 8, 16]))
+            bk = int(rng.choice([1, 2, 4, 8]))
+            rate = float(rng.choice([1.0, 2.0, 3.0, 4.5, 8.0, 9.0]))
+            out.append((BP, M, C * kh * kw, kh, kw, bm, bk, rate))
+    return out
+
+
+@pytest.mark.parametrize("scheme,M,K,kh,kw,bm,bk,rate", _random_layouts(40, 2024))
+def test_prune_satisfies_the_exchange_optimality_conditions(scheme, M, K, kh, kw, bm, bk, rate):
+    """Kept energy is maximal over all unit sets of size T = floor(sum P_b / r + 0.5)
+    with at least floor(P_b / r) units per block iff (1) every block keeps its
+    highest-scoring units and (2) no unit left out scores above a kept unit of
+    another block that holds more than its floor (block energies are concave in
+    the count, so single transfers certify the optimum).  Checked on random
+    layouts with partial blocks, both schemes and non-integer rates, from the
+    scores and the kept set alone."""
+    dt = F16 if (M + K) % 2 else BF16
+    W = inputs.normal((M, K), 0.05, dt, seed=M * 1000 + K)
+    s = oracle.scores(W, dt, scheme, bm, bk, kh, kw)
+    _, keep = oracle.prune(W, dt, scheme, bm, bk, rate, kh, kw, return_keep=True)
+    blocks = _units_of_blocks(scheme, M, K, kh, kw, bm, bk)
+    sizes = [len(b) for b in blocks]
+    T = int(np.floor(sum(sizes) / rate + 0.5))
+    assert int(keep.sum()) == T
+    slack_min = []                                   # (lowest kept score, block) of blocks above floor
+    for i, b in enumerate(blocks):
+        kb = keep[b] == 1
+        base = int(np.floor(len(b) / rate))
+        assert kb.sum() >= base
+        if kb.any() and (~kb).any():
+            assert s[b][kb].min() >= s[b][~kb].max()          # condition (1)
+        if kb.sum() > base:
+            slack_min.append((s[b][kb].min(), i))
+    slack_min.sort()
+    for i, b in enumerate(blocks):
+        out = s[b][keep[b] == 0]
+        if out.size == 0:
+            continue
+        others = [m for m, j in slack_min[:2] if j != i]
+        if others:
+            assert out.max() <= others[0]                     # condition (2)
+
+
 def test_prune_ties_go_to_lower_index():
     W = oracle.round_to(np.ones((4, 8)), F16)     # every score equal
     mask, keep = oracle.prune(W, F16, BB, 2, 4, 8.0 / 3.0, return_keep=True)
