@@ -109,3 +109,49 @@ def test_rows_rejects_bad_rate():
     W = inputs.normal((8, 8), 0.05, F16, seed=1)
     with pytest.raises(oracle.OracleError):
         oracle.prune_rows(W, F16, 4, 4, 0.5)
+
+
+def _row_layouts(n, seed):
+    rng = np.random.default_rng(seed)
+    return [(int(rng.integers(1, 150)), int(rng.integers(1, 200)),
+             int(rng.choice([1, 2, 5, 8, 16, 32])), int(rng.choice([1, 3, 8, 16, 32])),
+             float(rng.choice([1.0, 1.5, 2.0, 8.0 / 3.0, 4.0, 7.0])), int(rng.integers(0, 2)))
+            for _ in range(n)]
+
+
+@pytest.mark.parametrize("M,K,bm,bk,rate,dtype", _row_layouts(30, 77))
+def test_rows_satisfy_the_exchange_optimality_conditions(M, K, bm, bk, rate, dtype):
+    """The row units (one row of one bm x bk block each, scored by the squared
+    norm of its bk weights, computed here from the weights) are selected like
+    column units: T = floor(sum P_b / r + 0.5) in total, at least floor(P_b / r)
+    per block, maximal kept energy.  Certified by the exchange conditions:
+    each block keeps its top rows, and no left-out row outscores a kept row of
+    another block above its floor."""
+    W = inputs.normal((M, K), 0.05, dtype, seed=M * 31 + K)
+    s2 = _row_scores(oracle.to_double(W, dtype), bm, bk)       # [row, column block]
+    _, keep = oracle.prune_rows(W, dtype, bm, bk, rate, return_keep=True)
+    CB = -(-K // bk)
+    blocks, g = [], 0
+    for rb in range(-(-M // bm)):
+        rows = range(rb * bm, min(M, rb * bm + bm))
+        for cb in range(CB):
+            blocks.append((list(range(g, g + len(rows))), np.array([s2[r, cb] for r in rows])))
+            g += len(rows)
+    assert g == keep.size
+    T = int(np.floor(sum(len(u) for u, _ in blocks) / rate + 0.5))
+    assert int(keep.sum()) == T
+    slack = []
+    for i, (u, sc) in enumerate(blocks):
+        kb = keep[u] == 1
+        base = int(np.floor(len(u) / rate))
+        assert kb.sum() >= base
+        if kb.any() and (~kb).any():
+            assert sc[kb].min() >= sc[~kb].max()
+        if kb.sum() > base:
+            slack.append((sc[kb].min(), i))
+    slack.sort()
+    for i, (u, sc) in enumerate(blocks):
+        out = sc[keep[u] == 0]
+        others = [m for m, j in slack[:2] if j != i]
+        if out.size and others:
+            assert out.max() <= others[0]
