@@ -524,10 +524,10 @@ __global__ void __launch_bounds__(256) im2col_3x3_plane_kernel(ConvShape cs, int
 // ig * H*W a multiple of 8 so that every block's columns start 16-byte
 // aligned.  The block stages the zero-bordered planes [channel][image] in
 // shared memory (one warp per plane, 2-byte loads: planes are not 16-byte
-// aligned), then each
-// thread writes 8 consecutive columns of a channel's listed rows with one
-// 16-byte store; the 8 columns may span two images of the group.  Columns of
-// the last group past N are written as zeros (inside the row's ldx).
+// aligned), then each thread writes 8 consecutive columns of a channel's
+// listed rows with one 16-byte store; the 8 columns may span two images of
+// the group.  Columns of the last group past N are written as zeros (inside
+// the row's ldx).
 __global__ void __launch_bounds__(256) im2col_3x3_images_kernel(ConvShape cs, int64_t ldx, int ppb,
                                                                 int ig,
                                                                 const int32_t *__restrict__ qmap,
