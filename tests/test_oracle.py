@@ -401,6 +401,26 @@ def test_pack_roundtrip(scheme, M, K, kh, kw, bm, bk, rate):
         assert mask[rb * bm:(rb + 1) * bm].sum() == rows.shape[0] * kp
 
 
+@pytest.mark.parametrize("scheme,M,K,kh,kw,bm,bk,rate", _random_layouts(30, 91))
+def test_pack_roundtrip_random_layouts(scheme, M, K, kh, kw, bm, bk, rate):
+    """The compact storage of random layouts unpacks to the mask and the
+    masked weight exactly; each row-block's list is ascending and its values
+    are the row-block's rows at those columns."""
+    W = inputs.normal((M, K), 1.0, BF16, seed=M + 7 * K)
+    mask = oracle.prune(W, BF16, scheme, bm, bk, rate, kh, kw)
+    rb_ptr, col_idx, values = oracle.pack(W, mask, bm)
+    W2, mask2 = oracle.unpack(M, K, bm, rb_ptr, col_idx, values)
+    assert (mask2 == mask).all()
+    assert (W2 == np.where(mask == 1, W, 0)).all()
+    assert rb_ptr[0] == 0 and rb_ptr[-1] == col_idx.size and len(rb_ptr) == -(-M // bm) + 1
+    for rb in range(len(rb_ptr) - 1):
+        seg = col_idx[rb_ptr[rb]:rb_ptr[rb + 1]]
+        assert (np.diff(seg) > 0).all()
+        rows = W[rb * bm:(rb + 1) * bm]
+        blk = values[bm * rb_ptr[rb]: bm * rb_ptr[rb] + rows.shape[0] * seg.size]
+        assert (blk.reshape(rows.shape[0], seg.size) == rows[:, seg]).all()
+
+
 def test_pack_rejects_inconsistent_rows():
     W = oracle.round_to(np.ones((4, 4)), F16)
     mask = np.eye(4, dtype=np.uint8)
@@ -452,6 +472,40 @@ def test_masked_conv2d_matches_torch(stride, pad, kh, kw):
     assert acc.shape == ref.shape
     assert np.abs(acc - ref).max() < 1e-12
     assert (out == oracle.round_to(acc, BF16)).all()
+
+
+def _conv_cases(n, seed):
+    rng = np.random.default_rng(seed)
+    out = []
+    for _ in range(n):
+        kh, kw = int(rng.integers(1, 6)), int(rng.integers(1, 6))
+        sh, sw = int(rng.integers(1, 4)), int(rng.integers(1, 4))
+        ph, pw = int(rng.integers(0, 4)), int(rng.integers(0, 4))
+        H = int(rng.integers(max(1, kh - 2 * ph), 14))
+        W = int(rng.integers(max(1, kw - 2 * pw), 14))
+        out.append((int(rng.integers(1, 7)), int(rng.integers(1, 6)), int(rng.integers(1, 3)),
+                    H, W, kh, kw, sh, sw, ph, pw))
+    return out
+
+
+@pytest.mark.parametrize("F,C,Nb,H,W,kh,kw,sh,sw,ph,pw", _conv_cases(30, 5))
+def test_masked_conv2d_random_shapes_match_torch(F, C, Nb, H, W, kh, kw, sh, sw, ph, pw):
+    """Random kernel sizes, unequal strides and paddings, non-square images:
+    the fp64 accumulation equals torch's fp64 convolution of the masked weight."""
+    rng = np.random.default_rng(F * 1000 + C * 100 + H * 10 + W)
+    Wt = oracle.round_to(rng.normal(0, 0.3, (F, C, kh, kw)), F16)
+    x = oracle.round_to(rng.normal(0, 1, (Nb, C, H, W)), F16)
+    mask = (rng.random((F, C * kh * kw)) < 0.6).astype(np.uint8)
+    bias = rng.normal(0, 0.1, F).astype(np.float32)
+    out, acc = oracle.masked_conv2d(Wt, mask, x, F16, pad=(ph, pw), stride=(sh, sw), bias=bias,
+                                    return_acc=True)
+    wt = torch.from_numpy(oracle.to_double(Wt, F16) * mask.reshape(F, C, kh, kw))
+    ref = torch.nn.functional.conv2d(torch.from_numpy(oracle.to_double(x, F16)), wt,
+                                     torch.from_numpy(bias.astype(np.float64)),
+                                     stride=(sh, sw), padding=(ph, pw)).numpy()
+    assert acc.shape == ref.shape
+    assert np.abs(acc - ref).max() < 1e-12
+    assert (out == oracle.round_to(acc, F16)).all()
 
 
 def test_masked_conv2d_1x1_is_gemm_per_image():
