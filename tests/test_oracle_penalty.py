@@ -46,6 +46,36 @@ def test_penalty_matches_autograd(scheme, M, K, bm, bk, kh, kw, dtype):
     np.testing.assert_allclose(g, g2, rtol=1e-13, atol=0)
 
 
+def _full_block_layouts(n, seed):
+    rng = np.random.default_rng(seed)
+    out = []
+    for _ in range(n):
+        bm = int(rng.choice([1, 2, 4, 8, 16]))
+        if rng.random() < 0.5:
+            bk = int(rng.choice([1, 3, 8, 16]))
+            out.append((0, bm * int(rng.integers(1, 6)), bk * int(rng.integers(1, 8)), bm, bk,
+                        1, 1, int(rng.integers(0, 2))))
+        else:
+            kh, kw = [(1, 1), (3, 3), (2, 5)][int(rng.integers(0, 3))]
+            bk = int(rng.choice([1, 2, 4]))
+            out.append((1, bm * int(rng.integers(1, 5)), bk * int(rng.integers(1, 6)) * kh * kw,
+                        bm, bk, kh, kw, int(rng.integers(0, 2))))
+    return out
+
+
+@pytest.mark.parametrize("scheme,M,K,bm,bk,kh,kw,dtype", _full_block_layouts(25, 13))
+def test_penalty_matches_autograd_random_layouts(scheme, M, K, bm, bk, kh, kw, dtype):
+    """alpha, R and dR/dW of random full-block layouts (both schemes) equal the
+    autograd of the objective with its groups formed by reshaping."""
+    W = inputs.normal((M, K), 0.05, dtype, seed=3 * M + K)
+    eps, lam = 10.0 ** -int(2 + (M + K) % 4), 0.5 + (M % 3)
+    a, R, g = oracle.reweighted_penalty(W, dtype, scheme, bm, bk, eps, lam, kh, kw)
+    a2, R2, g2 = _objective_grad(oracle.to_double(W, dtype), scheme, bm, bk, kh, kw, eps, lam)
+    np.testing.assert_allclose(a, a2, rtol=1e-13)
+    assert R == pytest.approx(R2, rel=1e-12)
+    np.testing.assert_allclose(g, g2, rtol=1e-13, atol=0)
+
+
 def test_penalty_closed_form_single_unit():
     # one column of 4 rows, values 1, 2, 2, 0 (exact in fp16): s = 9
     W = oracle.round_to(np.array([[1.0], [2.0], [2.0], [0.0]]), F16)
