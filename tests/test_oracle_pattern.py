@@ -50,6 +50,40 @@ def test_pattern_choice_and_connectivity(F, C, rate, dtype):
     assert mask.sum() == 4 * T
 
 
+def _random_pattern_cases(n, seed):
+    rng = np.random.default_rng(seed)
+    all4 = [sum(1 << b for b in comb) for comb in itertools.combinations(range(9), 4)]
+    out = []
+    for _ in range(n):
+        k = int(rng.integers(1, 17))
+        pats = tuple(int(p) for p in rng.choice(all4, size=k, replace=False))
+        out.append((int(rng.integers(1, 40)), int(rng.integers(1, 30)),
+                    float(rng.choice([2.25, 3.0, 4.5, 6.0, 8.0, 9.0])), int(rng.integers(0, 2)),
+                    pats))
+    return out
+
+
+@pytest.mark.parametrize("F,C,rate,dtype,pats", _random_pattern_cases(25, 8))
+def test_pattern_choice_and_connectivity_random_sets(F, C, rate, dtype, pats):
+    """Random layers and random pattern sets (1 to 16 distinct 4-entry masks):
+    each kernel takes its highest kept-energy pattern (ties to the lower
+    index), and the T = floor(9FC / (4r) + 0.5) kernels of highest kept energy
+    survive (ties to the lower kernel index)."""
+    W = inputs.normal((F, C, 3, 3), 0.05, dtype, seed=F * 100 + C)
+    P = np.array(pats, np.uint16)
+    mask, pat = oracle.prune_pattern(W, dtype, rate, patterns=P, return_patterns=True)
+    e = _energies(oracle.to_double(W, dtype), P)
+    np.testing.assert_array_equal(pat.reshape(F, C), np.argmax(e, axis=2))
+    best = e.max(axis=2).reshape(-1)
+    T = int(np.floor(9 * F * C / (4 * rate) + 0.5))
+    kept = np.zeros(F * C, bool)
+    kept[np.lexsort((np.arange(F * C), -best))[:T]] = True
+    ref = np.zeros((F * C, 9), np.uint8)
+    for g in np.flatnonzero(kept):
+        ref[g] = [(int(P[pat[g]]) >> b) & 1 for b in range(9)]
+    np.testing.assert_array_equal(mask, ref.reshape(F, C, 9).reshape(F, 9 * C))
+
+
 def test_all_patterns_keep_the_four_largest_weights():
     # with every 4-entry pattern allowed, a kernel keeps its 4 largest magnitudes
     pats = np.array([sum(1 << b for b in comb) for comb in itertools.combinations(range(9), 4)],
