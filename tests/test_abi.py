@@ -89,6 +89,16 @@ def test_rate_below_one_rejected_on_host(lib):
     assert bp.bp_prune(lay, 16, 2.0, 16, 256, 16, 0) == bp.ERR_WORKSPACE
 
 
+def test_noalloc_checks_on_host(lib):
+    # rejected before any device call: a layout whose workspace exceeds the
+    # library's 8 MiB scratch array, and an invalid layout
+    big = bp.layout(bp.BLOCK_BASED, bp.BF16, 8192, 8192, 1, 1)
+    assert bp.bp_workspace_size(big) > 8 << 20
+    assert bp.bp_prune_noalloc(big, 16, 2.0, 16, 0) == bp.ERR_WORKSPACE
+    bad = bp.Layout(0, 1, 64, 64, 1, 1, 0, 16)                        # bm = 0
+    assert bp.bp_prune_noalloc(bad, 16, 2.0, 16, 0) == bp.ERR_INVALID_ARG
+
+
 def test_gemm_argument_checks_on_host(lib):
     lay = bp.layout(bp.BLOCK_BASED, bp.F16, 64, 64, 16, 16)
     P = bp.Packed(lay, 4, 0, 0, 16, 16, 16, 256, 256 + 16384 + 640 + 4 * 64)   # kc_ptr, one chunk, qmap
