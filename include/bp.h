@@ -299,10 +299,10 @@ bp_status bp_set_watchdog_ns(uint64_t ns);
  * fixed 8 MiB array inside the library's device memory (held on every GPU
  * that loads the library until it is unloaded).  Layouts whose
  * bp_workspace_size() exceeds 8 MiB are rejected with BP_ERR_WORKSPACE before
- * anything is launched.  The array's address is looked up on the first call
- * made on each device (make that call before any stream capture).  All calls
- * share the array: calls that may overlap on the GPU race and must be
- * serialised by the caller.  Allocates nothing. */
+ * anything is launched.  Like bp_prune it synchronises `stream` (the
+ * selection reads counts back), so it cannot run inside a stream capture.
+ * All calls share the array: calls that may overlap on the GPU race and must
+ * be serialised by the caller.  Allocates nothing. */
 bp_status bp_prune_noalloc(const bp_layout *lay, const void *W, double rate, uint8_t *mask,
                            void *stream);
 

@@ -25,7 +25,6 @@ uint64_t g_watchdog_ns = kDefaultWatchdogNs;
 int64_t g_drop_stage = -1;
 std::mutex g_mu;            // guards the per-device caches and g_pack_bad
 constexpr int kMaxDev = 64;
-unsigned *g_status_ptr[kMaxDev];
 int g_sms[kMaxDev];
 
 int cur_dev() {
@@ -182,15 +181,12 @@ bp_status prune_units(const bp_layout &lay, const void *W, double rate, uint8_t 
 uint64_t watchdog_ns() { return g_watchdog_ns; }
 int64_t debug_drop_stage() { return g_drop_stage; }
 
+// Looked up on every call (a host-side lookup, no allocation): an address
+// cached across calls would go stale when the device's context is reset.
 unsigned *device_status_ptr() {
-    std::lock_guard<std::mutex> lk(g_mu);
-    const int d = cur_dev();
-    if (!g_status_ptr[d]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_dev_status) == cudaSuccess)
-            g_status_ptr[d] = static_cast<unsigned *>(p);
-    }
-    return g_status_ptr[d];
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_dev_status) != cudaSuccess) return nullptr;
+    return static_cast<unsigned *>(p);
 }
 
 int num_sms() {

@@ -9,15 +9,16 @@
 // fixed array in the library's own device memory, declared below.
 //
 // The array costs kNoAllocScratchBytes of device memory on every GPU that
-// loads the library, for as long as the library stays loaded.  Its address
-// is looked up once per device, on the first call made with that device
-// current; make that first call before any stream capture.  Every call uses
-// the same array: calls that can overlap on the GPU (different streams,
-// different host threads) race on it and must be serialised by the caller.
-// The array keeps whatever the previous call left; bp_prune clears every
-// table it reads before use, so no state carries over between calls.
-#include <mutex>
-
+// loads the library, for as long as the library stays loaded.  Its device
+// address is looked up on every call, with the caller's device current (a
+// host-side lookup that allocates nothing), so no address outlives a reset
+// of the device's context.  Like bp_prune, the call synchronises its stream
+// (the selection reads counts back), so it cannot be used inside a stream
+// capture.  Every call uses the same array: calls that can overlap on the GPU
+// (different streams, different host threads) race on it and must be
+// serialised by the caller.  The array keeps whatever the previous call left;
+// bp_prune clears every table it reads before use, so no state carries over
+// between calls.
 #include "bp_common.cuh"
 
 namespace bp {
@@ -27,21 +28,13 @@ constexpr size_t kNoAllocScratchBytes = 8u << 20;   // 8 MiB
 
 static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_noalloc_mu;
-void *g_noalloc_ptr[kMaxDevices];
-
-// Device address of the scratch array for the current device (looked up once).
+// Device address of the scratch array in the current device's context.  In
+// host code g_noalloc_scratch names a host-side stand-in, never the device
+// array, so the address must come from the runtime.
 bp_status scratch_for_current_device(void **out) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return BP_ERR_CUDA;
-    std::lock_guard<std::mutex> lk(g_noalloc_mu);
-    if (!g_noalloc_ptr[dev]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return BP_ERR_CUDA;
-        g_noalloc_ptr[dev] = p;
-    }
-    *out = g_noalloc_ptr[dev];
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return BP_ERR_CUDA;
+    *out = p;
     return BP_OK;
 }
 

@@ -2,8 +2,10 @@
 (it uses a fixed scratch array inside the library instead of a caller-provided
 workspace).  Its masks must equal those of bp_prune with a workspace, on two
 calls in a row (the second call reuses the scratch array the first one left
-behind), and a layout whose workspace exceeds the array is rejected up front.
-This file is collected last on purpose."""
+behind), on a layout whose workspace fills nearly all of the array, and a
+layout whose workspace exceeds the array is rejected up front.  Once the
+array's module is loaded, a call changes neither the device's free memory nor
+torch's allocations.  This file is collected last on purpose."""
 import ctypes
 
 import numpy as np
@@ -45,3 +47,34 @@ def test_noalloc_rejects_layout_beyond_its_scratch():
     mask = torch.zeros(16, dtype=torch.uint8, device="cuda")
     st = bp.bp_prune_noalloc(lay, W.data_ptr(), 2.0, mask.data_ptr(), 0)
     assert st == bp.ERR_WORKSPACE
+
+
+# 768 filters x 1088 channels, 3x3, blocks of 4 x 4: bp_workspace_size is
+# 8,358,912 bytes, 99.6 % of the 8 MiB array, so the array's tail is used.
+BIG = (bp.BLOCK_PUNCHED, bp.BF16, 768, 1088 * 9, 3, 3, 4, 4, 3.0)
+
+
+def test_noalloc_near_its_limit_allocates_nothing():
+    scheme, dtype, M, K, kh, kw, bm, bk, rate = BIG
+    lay = bp.layout(scheme, dtype, M, K, bm, bk, kh, kw)
+    need = bp.bp_workspace_size(lay)
+    assert (8 << 20) * 0.99 < need <= 8 << 20
+    stream = int(torch.cuda.current_stream().cuda_stream)
+    W = _dev(inputs.normal((M, K), 0.05, dtype, seed=977), dtype)
+    ref = bp.prune(lay, W, rate)
+    got = torch.full((M, K), 7, dtype=torch.uint8, device="cuda")
+    # warm-up call: loads the array's module (its device memory is claimed then)
+    assert bp.bp_prune_noalloc(lay, W.data_ptr(), rate, got.data_ptr(), stream) == bp.OK
+    torch.cuda.synchronize()
+    assert torch.equal(got, ref)
+    got.fill_(7)
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    alloc0 = torch.cuda.memory_allocated()
+    st = bp.bp_prune_noalloc(lay, W.data_ptr(), rate, got.data_ptr(), stream)
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert st == bp.OK, bp.status_string(st)
+    assert torch.cuda.memory_allocated() == alloc0
+    assert free1 == free0, f"free device memory changed by {free0 - free1} bytes"
+    assert torch.equal(got, ref), f"masks differ in {int((got != ref).sum())} bytes"
