@@ -166,6 +166,32 @@ __device__ __forceinline__ void bulk_wait_all() {
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 
+// ---------------------------------------------------------------- flags between CTAs
+__device__ __forceinline__ void st_release_gpu(int32_t *p, int32_t v) {
+    asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ int32_t ld_acquire_gpu(const int32_t *p) {
+    int32_t v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+// Bounded wait for a flag another CTA raises (to a nonzero value) with
+// st_release_gpu; false once `limit_ns` have passed or `*abort` is raised.
+__device__ __forceinline__ bool wait_flag_gpu(const int32_t *f, uint64_t limit_ns,
+                                              volatile int *abort) {
+    uint64_t deadline = 0;
+    for (uint32_t it = 1;; ++it) {
+        if (ld_acquire_gpu(f) != 0) return true;
+        __nanosleep(64);
+        if ((it & 15u) == 0u) {
+            if (abort != nullptr && *abort) return false;
+            const uint64_t now = globaltimer_ns();
+            if (deadline == 0) deadline = now + limit_ns;
+            else if (now > deadline) return false;
+        }
+    }
+}
+
 // ---------------------------------------------------------------- cp.async (16 B)
 // src_bytes < 16 zero-fills the rest of the 16-byte destination.
 __device__ __forceinline__ void cp_async_16(uint32_t dst, const void *src, uint32_t src_bytes) {

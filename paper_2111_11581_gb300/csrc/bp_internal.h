@@ -149,13 +149,19 @@ int64_t im2col_row_width(const ConvShape &cs);   // staged input row length (ele
 // items than SMs), its items are split along their k-chunks into `split`
 // units each, whose fp32 partial tiles meet in a workspace: the last unit of
 // an item to finish sums them and writes the output.
+// Balanced launches (enough items for every SM, but a last wave that would
+// leave many SMs idle): the chunks of all items are cut into one equal range
+// per CTA; an item cut by a range boundary meets its parts through fp32
+// partial tiles, one per CTA, and per-(CTA, quadrant) flags in the workspace.
 struct SplitPlan {
     int nt;             // activation columns per tile
     int64_t items;      // (slab, column tile) items
     int64_t full;       // items computed whole (the first `full`)
     int split;          // units per remaining item (1: no split)
-    int64_t units;      // full + (items - full) * split
-    size_t bytes;       // workspace: partial tiles + arrival counters (0 if split == 1)
+    int64_t units;      // full + (items - full) * split; balanced: the CTA count
+    bool balanced;      // balanced launch
+    int64_t total;      // balanced: chunks of all items
+    size_t bytes;       // workspace: partial tiles + counters / flags (0 if none)
 };
 SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split);
 

@@ -41,6 +41,34 @@
 
 #include "bp_common.cuh"
 
+// BP_TRACE (off by default; a build for measurement only): CTA 0 records
+// clock64() at fixed points of each of its first kTraceChunks pipeline stages,
+// read back with bp_debug_trace_read().  Events per stage: 0 control thread
+// found the stage free, 1 gather group found it free, 2 gather group issued
+// its copies, 3 MMA thread saw the weight tile, 4 MMA thread saw the gathered
+// rows, 5 MMA thread committed the stage, 6 and 7 control thread before /
+// after issuing the weight copy.  Per window w (entries 256 + w): 0 control
+// thread at the window, 1 after copying the next window, 2 saw this window, 3
+// gather warp 0 saw it; per item i (entries 384 + i): 4 MMA thread holds a
+// free accumulator.  Entries 448 .. hold the global-timer start and end of
+// each of the first 256 CTAs.
+#ifdef BP_TRACE
+namespace bp {
+constexpr int kTraceChunks = 512;
+constexpr int kTraceEvents = 8;
+__device__ unsigned long long g_trace[kTraceChunks * kTraceEvents];
+}  // namespace bp
+#define BP_TR(seq, ev)                                                                   \
+    do {                                                                                 \
+        if (blockIdx.x == 0 && (seq) < bp::kTraceChunks)                                 \
+            bp::g_trace[(seq) * bp::kTraceEvents + (ev)] = clock64();                    \
+    } while (0)
+#else
+#define BP_TR(seq, ev) \
+    do {               \
+    } while (0)
+#endif
+
 namespace bp {
 namespace {
 
@@ -61,12 +89,21 @@ constexpr int kCtrlWarp = 8;
 constexpr int kMmaWarp = 9;
 constexpr int kEpiWarp0 = 10;
 constexpr int kThreads = (kEpiWarp0 + 4) * 32;
-// The gather warps form kGatherGroups groups that take turns: group g gathers
-// the chunks whose sequence number is g modulo kGatherGroups, so one group
-// issues copies while another waits for its next stage.
+// The gather warps form kGatherGroups groups.  By default the groups take
+// turns: group g gathers the chunks whose sequence number is g modulo
+// kGatherGroups, so one group issues copies while another waits for its next
+// stage.  With BP_GATHER_HALVES group h gathers rows 32h .. 32h+31 of every
+// chunk instead, each half signalling a barrier of its own, and the tensor
+// cores start on the first half while the second is still landing.
 constexpr int kGatherGroups = 2;
 constexpr int kGroupWarps = kGatherWarps / kGatherGroups;
+#ifdef BP_GATHER_HALVES
+constexpr int kRowsPerWarp = 32 / kGroupWarps;      // list positions per warp and chunk
+constexpr int kFullPerStage = 2;
+#else
 constexpr int kRowsPerWarp = 64 / kGroupWarps;      // list positions per warp and chunk
+constexpr int kFullPerStage = 1;
+#endif
 constexpr uint32_t kGroupThreads = kGroupWarps * 32;
 
 struct Params {
@@ -85,8 +122,15 @@ struct Params {
     int64_t full_items;     // the first full_items items are single work units
     int split;              // units per later item (k-chunk ranges)
     int64_t num_units;      // full_items + (num_items - full_items) * split
-    float *part;            // split items: fp32 partial tiles, [item][unit][128][256]
-    int32_t *cnt;           // split items: arrivals per (item, row quadrant)
+    float *part;            // split items: fp32 partial tiles, [item][unit][128][256];
+                            // balanced launches: one tile per CTA
+    int32_t *cnt;           // split items: arrivals per (item, row quadrant); balanced
+                            // launches: per (CTA, row quadrant) "partial written" flags
+    int sk;                 // 1: balanced launch (whole items in full waves, then each CTA
+                            // one equal range of the remaining items' chunks)
+    int64_t sk_i0;          // balanced launch: first item of the ranges
+    int64_t sk_total;       // balanced launch: chunks of all items (tiles x kc_total)
+    int64_t kc_total;       // chunks of one column tile (all slabs)
     int64_t stages;
     uint32_t tmem_cols, acc_cols, ystage_bytes;
     const int64_t *kc_ptr;
@@ -124,11 +168,14 @@ struct Smem {
     uint64_t *tfull;     // [2] accumulator ready for the epilogue
     uint64_t *tempty;    // [2] accumulator drained
     uint64_t *drain;     // [1]
+    uint64_t *fixbar;    // [4] balanced launch: a partial tile's quadrant landed (per epilogue warp)
     uint64_t *pfull;     // [kWinBufs] a window of chunk records landed (TMA byte count)
     uint64_t *pempty;    // [kWinBufs] the gather warps and the control thread are done with it
     uint32_t *skind;     // [stages] 1: the stage's activations come from TMA tile loads
     uint32_t *tmem_base;
     int *abort_flag;
+    int64_t *skv;        // [4] balanced launch: chunk position of item sk_i0, chunks from
+                         // there on, this CTA's range [lo, hi) (set in the prologue)
     uint8_t *win;        // [kWinBufs][kWinBytes] chunk records of the current windows
     int64_t *kc;         // [kc_cached] copy of kc_ptr, or nullptr
 };
@@ -142,18 +189,21 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
     s.ystage = s.x + p.stages * kXTileBytes;
     uint8_t *b = s.ystage + p.ystage_bytes;
     s.full = reinterpret_cast<uint64_t *>(b);
-    s.wfull = s.full + p.stages;
+    s.wfull = s.full + kFullPerStage * p.stages;
     s.empty = s.wfull + p.stages;
     s.tfull = s.empty + p.stages;
     s.tempty = s.tfull + 2;
     s.drain = s.tempty + 2;
-    s.pfull = s.drain + 1;
+    s.fixbar = s.drain + 1;
+    s.pfull = s.fixbar + 4;
     s.pempty = s.pfull + kWinBufs;
     s.skind = reinterpret_cast<uint32_t *>(s.pempty + kWinBufs);
     s.tmem_base = s.skind + p.stages;
     s.abort_flag = reinterpret_cast<int *>(s.tmem_base + 1);
+    s.skv = reinterpret_cast<int64_t *>(
+        (reinterpret_cast<uintptr_t>(s.abort_flag + 1) + 7) & ~static_cast<uintptr_t>(7));
     // TMA bulk copies need a 16-byte-aligned destination: round up to 128 bytes
-    const uintptr_t after = reinterpret_cast<uintptr_t>(s.abort_flag + 1);
+    const uintptr_t after = reinterpret_cast<uintptr_t>(s.skv + 4);
     s.win = reinterpret_cast<uint8_t *>((after + 127) & ~static_cast<uintptr_t>(127));
     s.kc = p.kc_cached ? reinterpret_cast<int64_t *>(s.win + kWinBufs * kWinBytes) : nullptr;
     return s;
@@ -161,7 +211,7 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
 
 size_t smem_bytes(int64_t stages, uint32_t ystage_bytes, int64_t kc_cached) {
     return 1024 + (size_t)stages * (kWTileBytes + kXTileBytes) + ystage_bytes +
-           (3 * (size_t)stages + 5 + 2 * kWinBufs) * 8 + 4 * (size_t)stages + 8 + 128 +
+           ((2 + kFullPerStage) * (size_t)stages + 9 + 2 * kWinBufs) * 8 + 4 * (size_t)stages + 8 + 8 + 32 + 128 +
            (size_t)kWinBufs * kWinBytes + 8 * (size_t)kc_cached;
 }
 
@@ -174,26 +224,39 @@ struct Item {
     int64_t slab, n0, kc0, nkc, rows;   // rows = real rows of the slab
     int64_t j;                          // split item index (-1: whole item)
     int s, S;                           // unit s of S of the item
+    // balanced launches: 0 the whole item, 1 its first chunks (this CTA adds
+    // the partial tiles of the CTAs that own the rest and writes the output),
+    // 2 a later range of its chunks (this CTA writes a partial tile)
+    int role;
+    int64_t gpos, nitem;                // first chunk of the item (global position), its chunks
 };
 
 // Work unit u -> (slab, column tile) item, slab fastest, and its k-chunk
 // range: the whole item for u < full_items, else unit s of `split` equal
-// shares of the item's chunks.
+// shares of the item's chunks.  Unit, item and slab counts are below 2^31
+// (checked at launch), so the divisions are 32-bit: 64-bit divisions by a
+// runtime value cost hundreds of cycles, and the control thread decodes units
+// on its issue path.
 __device__ __forceinline__ Item decode(const Params &p, const int64_t *kc, int64_t u) {
     Item t;
-    int64_t it = u;
+    uint32_t it = (uint32_t)u;
+    t.role = 0;
+    t.gpos = 0;
     t.j = -1;
     t.s = 0;
     t.S = 1;
     if (u >= p.full_items) {
-        const int64_t v = u - p.full_items;
-        t.j = v / p.split;
-        t.s = (int)(v - t.j * p.split);
+        const uint32_t v = (uint32_t)(u - p.full_items), sp = (uint32_t)p.split;
+        const uint32_t jj = v / sp;
+        t.j = jj;
+        t.s = (int)(v - jj * sp);
         t.S = p.split;
-        it = p.full_items + t.j;
+        it = (uint32_t)p.full_items + jj;
     }
-    t.slab = it % p.num_slabs;
-    t.n0 = (it / p.num_slabs) * p.nt;
+    const uint32_t ns = (uint32_t)p.num_slabs;
+    const uint32_t tile = it / ns;
+    t.slab = it - tile * ns;
+    t.n0 = (int64_t)tile * p.nt;
     const int64_t c0 = kc[t.slab], nc = kc[t.slab + 1] - c0;
     if (t.S == 1) {
         t.kc0 = c0;
@@ -204,19 +267,105 @@ __device__ __forceinline__ Item decode(const Params &p, const int64_t *kc, int64
         t.nkc = ke - kb;
     }
     t.rows = min((int64_t)kSlab, p.M - t.slab * kSlab);
+    t.nitem = t.nkc;
     return t;
 }
+
+// Balanced launches: CTA c first runs whole items c, c + gridDim.x, ... below
+// item sk_i0 (full waves: the same count for every CTA), then the chunks of
+// items sk_i0 .. in item order (column tile, then slab) are cut into
+// gridDim.x equal ranges, CTA c taking the c-th.  An item cut by a range
+// boundary is finished by the CTA that computes its first chunks (the last
+// thing that CTA does); the CTAs that compute its later chunks do so first
+// thing in their range and leave fp32 partial tiles.  Every CTA thus runs the
+// same number of chunks, instead of a last wave that leaves most SMs idle, and
+// the whole-item waves keep the working set of the first waves as small as a
+// plain launch's (a few column tiles at a time).
+// first chunk position (relative to the ranges' start) of CTA c's range; T =
+// chunks of the ranges
+__device__ __forceinline__ int64_t sk_lo(int64_t T, int64_t c) { return c * T / gridDim.x; }
+// the CTA whose range holds chunk position g (absolute); skv as in Smem
+__device__ __forceinline__ int64_t sk_owner(const int64_t *skv, int64_t g) {
+    const int64_t T = skv[1], r = g - skv[0];
+    const int64_t G = gridDim.x;
+    int64_t c = r * G / T;
+    while (c + 1 < G && sk_lo(T, c + 1) <= r) ++c;
+    while (c > 0 && sk_lo(T, c) > r) --c;
+    return c;
+}
+// The part of the item holding chunk position u that lies in [u, end).
+__device__ __forceinline__ Item sk_decode(const Params &p, const int64_t *kc, int64_t u,
+                                          int64_t end) {
+    Item t;
+    t.j = -1;
+    t.s = 0;
+    t.S = 1;
+    const uint32_t kct = (uint32_t)p.kc_total;
+    const uint32_t tile = (uint32_t)u / kct;      // positions are below 2^31 (checked at launch)
+    const int64_t o = u - (int64_t)tile * kct;
+    // the slab whose chunks hold o: the last s with kc[s] <= o (o < kc[num_slabs])
+    int64_t lo = 0, hi = p.num_slabs;
+    while (hi - lo > 1) {
+        const int64_t mid = (lo + hi) >> 1;
+        if (kc[mid] <= o) lo = mid;
+        else hi = mid;
+    }
+    t.slab = lo;
+    t.n0 = (int64_t)tile * p.nt;
+    const int64_t klo = o - kc[lo];
+    t.nitem = kc[lo + 1] - kc[lo];
+    const int64_t khi = min(t.nitem, klo + (end - u));
+    t.kc0 = kc[lo] + klo;
+    t.nkc = khi - klo;
+    t.gpos = u - klo;
+    t.role = klo > 0 ? 2 : (khi < t.nitem ? 1 : 0);
+    t.rows = min((int64_t)kSlab, p.M - t.slab * kSlab);
+    return t;
+}
+
+// This CTA's work units in order: items (or split units) blockIdx.x, + gridDim.x,
+// ...; in balanced launches those below sk_i0, then the item parts of its
+// chunk range.
+struct UnitIter {
+    int64_t u, end;
+    bool ranged;         // in the chunk range of a balanced launch
+    const int64_t *skv;
+    __device__ __forceinline__ void enter_range() {
+        ranged = true;
+        u = skv[2];
+        end = skv[3];
+    }
+    __device__ __forceinline__ void init(const Params &p, const int64_t *skv_) {
+        skv = skv_;
+        ranged = false;
+        u = blockIdx.x;
+        end = p.sk ? p.sk_i0 : p.num_units;
+        if (p.sk && u >= end) enter_range();
+    }
+    __device__ __forceinline__ bool valid() const { return u < end; }
+    __device__ __forceinline__ Item get(const Params &p, const int64_t *kc) const {
+        return ranged ? sk_decode(p, kc, u, end) : decode(p, kc, u);
+    }
+    __device__ __forceinline__ void step(const Params &p, const Item &t) {
+        if (ranged) {
+            u += t.nkc;
+        } else {
+            u += gridDim.x;
+            if (p.sk && u >= end) enter_range();
+        }
+    }
+};
 
 // Walks this CTA's windows: runs of up to kWin consecutive k-chunks of one
 // work unit, in the order the CTA processes them (units with no chunk skipped).
 struct Window {
-    int64_t it;          // work unit
+    UnitIter ui;         // work unit
     int64_t k0, cnt;     // first chunk of the window within the unit, chunks in it
     Item t;
-    __device__ __forceinline__ void first(const Params &p, const int64_t *kcp) {
+    __device__ __forceinline__ void first(const Params &p, const int64_t *kcp, const int64_t *skv) {
         k0 = 0;
-        for (it = blockIdx.x; it < p.num_units; it += gridDim.x) {
-            t = decode(p, kcp, it);
+        for (ui.init(p, skv); ui.valid(); ui.step(p, t)) {
+            t = ui.get(p, kcp);
             if (t.nkc > 0) break;
         }
         cnt = valid(p) ? min((int64_t)kWin, t.nkc) : 0;
@@ -225,14 +374,14 @@ struct Window {
         k0 += kWin;
         if (k0 >= t.nkc) {
             k0 = 0;
-            for (it += gridDim.x; it < p.num_units; it += gridDim.x) {
-                t = decode(p, kcp, it);
+            for (ui.step(p, t); ui.valid(); ui.step(p, t)) {
+                t = ui.get(p, kcp);
                 if (t.nkc > 0) break;
             }
         }
         cnt = valid(p) ? min((int64_t)kWin, t.nkc - k0) : 0;
     }
-    __device__ __forceinline__ bool valid(const Params &p) const { return it < p.num_units; }
+    __device__ __forceinline__ bool valid(const Params &) const { return ui.valid(); }
 };
 
 // Load plan of a chunk record (see DevLayout): number of tile loads.
@@ -246,8 +395,19 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
     const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
     Window win;
-    win.first(p, kcp);
+    win.first(p, kcp, s.skv);
     const int group = warp / kGroupWarps, gw = warp % kGroupWarps;
+    const int nst = (int)p.stages;
+#ifdef BP_GATHER_HALVES
+    constexpr int kStep = 1;    // every chunk
+    const int rbase = 32 * group;
+    int gst = 0;
+#else
+    constexpr int kStep = kGatherGroups;
+    constexpr int rbase = 0;
+    int gst = group;            // stage of this group's next chunk (sequence number group + 2i)
+#endif
+    uint32_t gph = 0;
     int64_t count = 0, wseq = 0;
     bool ok = true;
     for (; win.valid(p) && ok; win.next(p, kcp), ++wseq) {
@@ -256,6 +416,7 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
         ok = __all_sync(0xffffffffu, mbar_wait(&s.pfull[buf], (uint32_t)((wseq / kWinBufs) & 1),
                                               p.watchdog_ns, abort_flag));
         if (!ok) break;
+        if (warp == 0 && lane == 0) BP_TR(256 + wseq, 3);
         const uint8_t *recs = s.win + buf * kWinBytes;
         // the tile's token columns: 16 bytes (8 columns) per lane, lanes past
         // the tile's width idle
@@ -273,18 +434,29 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
             planned = plan_loads(rec) > 0;
             const int32_t *l = reinterpret_cast<const int32_t *>(rec);
 #pragma unroll
-            for (int i = 0; i < kRowsPerWarp; ++i) ix[i] = l[gw + kGroupWarps * i];
+            for (int i = 0; i < kRowsPerWarp; ++i) ix[i] = l[rbase + gw + kGroupWarps * i];
         };
         const int64_t base = count;         // sequence number of the window's first chunk
+#ifdef BP_GATHER_HALVES
+        int64_t j = 0;
+#else
         int64_t j = (group - base % kGatherGroups + kGatherGroups) % kGatherGroups;
+#endif
         if (j < win.cnt) fetch(j, idx, tma);
-        for (; j < win.cnt; j += kGatherGroups) {
+        for (; j < win.cnt; j += kStep) {
             int32_t nidx[kRowsPerWarp];
             bool ntma = false;
-            if (j + kGatherGroups < win.cnt) fetch(j + kGatherGroups, nidx, ntma);
+            if (j + kStep < win.cnt) fetch(j + kStep, nidx, ntma);
             const int64_t seq = base + j;
-            const int stage = (int)(seq % p.stages);
-            const uint32_t phase = (uint32_t)((seq / p.stages) & 1);
+            // stage = seq mod stages, phase = its ring pass parity (kept
+            // incrementally: a 64-bit division per chunk sits on the issue path)
+            const int stage = gst;
+            const uint32_t phase = gph;
+            gst += kStep;
+            if (gst >= nst) {
+                gst -= nst;
+                gph ^= 1u;
+            }
             const bool drop = blockIdx.x == 0 && seq == p.drop_stage;
             // A planned chunk is loaded and signalled by the control thread; the
             // group still waits for its stage (lane 0 alone), which keeps it at
@@ -294,6 +466,7 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
                                 ? mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)
                                 : true);
             if (!ok) break;
+            if (gw == 0 && lane == 0) BP_TR(seq, 1);
             if (!tma && !drop) {
                 // 64 rows x nt columns: one warp instruction per row segment
                 const uint32_t xs = smem_u32(s.x + stage * kXTileBytes);
@@ -304,14 +477,14 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
                     if (nb == 16u) {
 #pragma unroll
                         for (int i = 0; i < kRowsPerWarp; ++i) {
-                            const int r = gw + kGroupWarps * i;
+                            const int r = rbase + gw + kGroupWarps * i;
                             cp_async_16_full(xs + cn * 8192 + r * 128 + ((jj ^ (r & 7)) << 4),
                                              xcol + (int64_t)idx[i] * p.ldx);
                         }
                     } else {
 #pragma unroll
                         for (int i = 0; i < kRowsPerWarp; ++i) {
-                            const int r = gw + kGroupWarps * i;
+                            const int r = rbase + gw + kGroupWarps * i;
                             cp_async_16(xs + cn * 8192 + r * 128 + ((jj ^ (r & 7)) << 4),
                                         xcol + (int64_t)idx[i] * p.ldx, nb);
                         }
@@ -321,7 +494,8 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
                 // blocking.  The tile was written through the generic proxy; the
                 // tensor-core thread orders it before its async-proxy reads with a
                 // proxy fence after acquiring the barrier.
-                cp_async_arrive_noinc(&s.full[stage]);
+                cp_async_arrive_noinc(&s.full[kFullPerStage * stage + (kFullPerStage - 1) * group]);
+                if (gw == 0 && lane == 0) BP_TR(seq, 2);
             }
 #pragma unroll
             for (int i = 0; i < kRowsPerWarp; ++i) idx[i] = nidx[i];
@@ -362,7 +536,7 @@ __device__ void control_thread(const Params &p, const Smem &s) {
     const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
     Window win;
-    win.first(p, kcp);
+    win.first(p, kcp, s.skv);
     WindowFiller wf;
     wf.ahead = win;
     wf.filled = 0;
@@ -373,6 +547,7 @@ __device__ void control_thread(const Params &p, const Smem &s) {
     int64_t count = 0, wseq = 0;
     for (; win.valid(p) && ok; win.next(p, kcp), ++wseq) {
         const int buf = (int)(wseq % kWinBufs);
+        BP_TR(256 + wseq, 0);
         // copy the next window into the buffer released by window wseq - 2
         if (wf.ahead.valid(p)) {
             const int64_t prev = wf.filled - kWinBufs;
@@ -384,11 +559,13 @@ __device__ void control_thread(const Params &p, const Smem &s) {
             }
             wf.fill(p, s, kcp);
         }
+        BP_TR(256 + wseq, 1);
         if (!mbar_wait(&s.pfull[buf], (uint32_t)((wseq / kWinBufs) & 1), p.watchdog_ns,
                        abort_flag)) {
             ok = false;
             break;
         }
+        BP_TR(256 + wseq, 2);
         const uint8_t *recs = s.win + buf * kWinBytes;
         for (int64_t j = 0; j < win.cnt; ++j) {
             const int64_t seq = count;
@@ -396,6 +573,7 @@ __device__ void control_thread(const Params &p, const Smem &s) {
                 ok = false;
                 break;
             }
+            BP_TR(seq, 0);
             // the plan: words 0..11 in three 16-byte loads
             const uint4 *pv = reinterpret_cast<const uint4 *>(recs + j * kMetaBytes + kListBytes);
             const uint4 q0 = pv[0], q1 = pv[1], q2 = pv[2];
@@ -406,9 +584,11 @@ __device__ void control_thread(const Params &p, const Smem &s) {
                 s.skind[stage] = tma ? 1u : 0u;    // read by the MMA thread after wfull
                 mbar_arrive_expect_tx(&s.wfull[stage],
                                       kWTileBytes + (tma ? (uint32_t)p.xboxes * (kBK * 128) : 0u));
+                BP_TR(seq, 6);
                 bulk_g2s(smem_u32(s.w + stage * kWTileBytes),
                          p.tiles + (win.t.kc0 + win.k0 + j) * (int64_t)kWTileBytes, kWTileBytes,
                          &s.wfull[stage]);
+                BP_TR(seq, 7);
                 if (tma) {
                     // load b: rows y[b] .. + (8 << lg) - 1 of X into list positions
                     // 8g ..; x = a multiple of 64 tokens (16-byte aligned), and
@@ -458,7 +638,6 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
     volatile int *abort_flag = s.abort_flag;
     const uint64_t wdog = p.watchdog_ns;
     const int nst = (int)p.stages;
-    const int64_t nitems = p.num_units;
     const uint32_t acc_cols = p.acc_cols;
     uint64_t *const wfull = s.wfull, *const full = s.full, *const empty = s.empty;
     const volatile uint32_t *const skind = s.skind;
@@ -469,17 +648,28 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
     const uint64_t xdesc0 = make_sdesc_sw128(smem_u32(s.x), 8192, 1024);
     int stage = 0;
     uint32_t phase = 0;
-    uint32_t gphase = 0;     // per stage: parity of the next gathered fill (bit = stage)
+    uint32_t gphase = 0;     // per gather barrier: parity of its next fill (bit = barrier)
     int acc = 0;
     uint32_t acc_phase = 0;
     bool ok = true;
-    for (int64_t it = blockIdx.x; it < nitems && ok; it += gridDim.x) {
-        const Item t = decode(p, kcp, it);
+#ifdef BP_TRACE
+    int64_t tseq = 0, titem = 0;
+#else
+    constexpr int64_t tseq = 0;
+#endif
+    UnitIter ui;
+    Item t;
+    for (ui.init(p, s.skv); ui.valid() && ok; ui.step(p, t)) {
+        t = ui.get(p, kcp);
         if (t.nkc == 0) continue;
         if (!mbar_wait(&s.tempty[acc], acc_phase ^ 1u, wdog, abort_flag)) {
             raise_timeout(p, s);
             break;
         }
+#ifdef BP_TRACE
+        BP_TR(384 + titem, 4);
+        ++titem;
+#endif
         tc_fence_after();
         const uint32_t d = tmem + acc * acc_cols;
         bool ready = mbar_test_wait(&wfull[stage], phase);
@@ -489,17 +679,21 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
                 ok = false;
                 break;
             }
-            if (skind[stage] == 0u) {
-                // gathered rows: wait for them, then order their generic-proxy
-                // (cp.async) writes, acquired through the barrier, before the tensor
-                // core's async-proxy reads
-                if (!mbar_wait(&full[stage], (gphase >> stage) & 1u, wdog, abort_flag)) {
+            BP_TR(tseq, 3);
+            const bool gathered = skind[stage] == 0u;
+            // gathered rows: wait for them, then order their generic-proxy
+            // (cp.async) writes, acquired through the barrier, before the tensor
+            // core's async-proxy reads
+            const uint32_t fb = kFullPerStage * stage;
+            if (gathered) {
+                if (!mbar_wait(&full[fb], (gphase >> fb) & 1u, wdog, abort_flag)) {
                     raise_timeout(p, s);
                     ok = false;
                     break;
                 }
-                gphase ^= 1u << stage;
+                gphase ^= 1u << fb;
                 fence_proxy_async_smem();
+                BP_TR(tseq, 4);
             }
             // order the MMAs below after the barrier waits above
             tc_fence_after();
@@ -510,11 +704,35 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
             // probe the next chunk's barrier now: the answer is needed only after
             // the MMAs below have been issued
             ready = kc + 1 < t.nkc && mbar_test_wait(&wfull[nstage], nphase);
+#ifdef BP_GATHER_HALVES
+#pragma unroll
+            for (int kk = 0; kk < 2; ++kk)
+                umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * (2048 >> 4), idesc,
+                            (kc > 0 || kk > 0) ? 1u : 0u);
+            if (gathered) {
+                if (!mbar_wait(&full[fb + 1], (gphase >> (fb + 1)) & 1u, wdog, abort_flag)) {
+                    raise_timeout(p, s);
+                    ok = false;
+                    break;
+                }
+                gphase ^= 1u << (fb + 1);
+                fence_proxy_async_smem();
+                tc_fence_after();
+            }
+#pragma unroll
+            for (int kk = 2; kk < 4; ++kk)
+                umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * (2048 >> 4), idesc, 1u);
+#else
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk)
                 umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * (2048 >> 4), idesc,
                             (kc > 0 || kk > 0) ? 1u : 0u);
+#endif
             umma_commit(&empty[stage]);
+            BP_TR(tseq, 5);
+#ifdef BP_TRACE
+            ++tseq;
+#endif
             stage = nstage;
             phase = nphase;
         }
@@ -541,8 +759,10 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
     uint32_t yseq = 0;                       // TMA box stores issued by this warp
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int64_t it = blockIdx.x; it < p.num_units; it += gridDim.x) {
-        const Item t = decode(p, kcp, it);
+    UnitIter ui;
+    Item t;
+    for (ui.init(p, s.skv); ui.valid(); ui.step(p, t)) {
+        t = ui.get(p, kcp);
         const bool has = t.nkc > 0;
         if (has) {
             // warp-uniform outcome: tcgen05.ld below is a warp-collective instruction
@@ -659,7 +879,86 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
 #pragma unroll
                 for (int e = 0; e < 32; ++e) r[e] = 0u;
             }
-            if (!kSplit || t.S == 1) {
+            constexpr int64_t kQuad = 8 * 8 * 32;            // float4 per (tile, quadrant)
+            if (kSplit && t.role == 2) {
+                // Balanced launch, a later range of the item's chunks: this CTA's
+                // fp32 partial rows go to its own tile of the workspace, then the
+                // quadrant's flag is raised for the CTA that finishes the item.
+                float4 *slot = reinterpret_cast<float4 *>(p.part) +
+                               ((int64_t)blockIdx.x * 4 + q) * kQuad + lane;
+                for (int g = 0; g < G; ++g) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        __stcg(slot + (g * 8 + e) * 32,
+                               make_float4(__uint_as_float(r[4 * e]), __uint_as_float(r[4 * e + 1]),
+                                           __uint_as_float(r[4 * e + 2]), __uint_as_float(r[4 * e + 3])));
+                    if (g + 1 < G) {
+                        tmem_ld_32x32b_x32(tacc + 32 * (g + 1), r);
+                        tmem_ld_wait();
+                    }
+                }
+                __threadfence();
+                __syncwarp();
+                if (lane == 0) st_release_gpu(p.cnt + (int64_t)blockIdx.x * 4 + q, 1);
+            } else if (kSplit && t.role == 1) {
+                // Balanced launch, the item's first chunks: add the partial rows of
+                // the CTAs that own the rest of its chunks (each raised its flag
+                // first thing in its range), then the usual epilogue.  This is the
+                // CTA's last unit, so its pipeline stages are idle: the first
+                // partial's quadrant (32 KB) comes in with one TMA bulk copy into
+                // the stage area (a latency-bound load loop over eight column
+                // groups measured several microseconds); further partials (items
+                // spread over three or more ranges) are read directly.
+                const int64_t c0 = sk_owner(s.skv, t.gpos + t.nkc);
+                const int64_t c1 = sk_owner(s.skv, t.gpos + t.nitem - 1);
+                const float4 *part4 = reinterpret_cast<const float4 *>(p.part);
+                uint8_t *fbuf = s.w + q * (kQuad * 16);
+                bool okw = true;
+                if (lane == 0) {
+                    for (int64_t c = c0; c <= c1 && okw; ++c)
+                        okw = wait_flag_gpu(p.cnt + c * 4 + q, p.watchdog_ns, abort_flag);
+                    if (okw) {
+                        mbar_arrive_expect_tx(&s.fixbar[q], (uint32_t)(kQuad * 16));
+                        bulk_g2s(smem_u32(fbuf), part4 + (c0 * 4 + q) * kQuad,
+                                 (uint32_t)(kQuad * 16), &s.fixbar[q]);
+                        okw = mbar_wait(&s.fixbar[q], 0, p.watchdog_ns, abort_flag);
+                    }
+                }
+                okw = __shfl_sync(0xffffffffu, okw ? 1 : 0, 0) != 0;
+                if (!okw) raise_timeout(p, s);
+                const float4 *sm4 = reinterpret_cast<const float4 *>(fbuf) + lane;
+                for (int g = 0; g < G && okw; ++g) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float4 v = sm4[(g * 8 + e) * 32];
+                        r[4 * e] = __float_as_uint(__uint_as_float(r[4 * e]) + v.x);
+                        r[4 * e + 1] = __float_as_uint(__uint_as_float(r[4 * e + 1]) + v.y);
+                        r[4 * e + 2] = __float_as_uint(__uint_as_float(r[4 * e + 2]) + v.z);
+                        r[4 * e + 3] = __float_as_uint(__uint_as_float(r[4 * e + 3]) + v.w);
+                    }
+                    for (int64_t c = c0 + 1; c <= c1; ++c) {
+                        const float4 *src = part4 + (c * 4 + q) * kQuad + lane + g * 8 * 32;
+                        float4 v[8];
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) v[e] = __ldcg(src + e * 32);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            r[4 * e] = __float_as_uint(__uint_as_float(r[4 * e]) + v[e].x);
+                            r[4 * e + 1] = __float_as_uint(__uint_as_float(r[4 * e + 1]) + v[e].y);
+                            r[4 * e + 2] = __float_as_uint(__uint_as_float(r[4 * e + 2]) + v[e].z);
+                            r[4 * e + 3] = __float_as_uint(__uint_as_float(r[4 * e + 3]) + v[e].w);
+                        }
+                    }
+                    pack(r, pk);
+                    if (g + 1 < G) tmem_ld_32x32b_x32(tacc + 32 * (g + 1), r);
+                    store(pk, 32 * g);
+                    if (g + 1 < G) tmem_ld_wait();
+                }
+                // zero the flags again for the next launch (read, and only written
+                // again, after this launch: launches on one stream are ordered)
+                if (lane == 0 && okw)
+                    for (int64_t c = c0; c <= c1; ++c) p.cnt[c * 4 + q] = 0;
+            } else if (!kSplit || t.S == 1) {
                 for (int g = 0; g < G; ++g) {
                     pack(r, pk);
                     if (has && g + 1 < G) tmem_ld_32x32b_x32(tacc + 32 * (g + 1), r);
@@ -672,7 +971,6 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                 // all slots and writes the output (no unit waits for another).
                 // Slot layout per quadrant: [group][8 float4][lane], so each
                 // warp access is 512 contiguous bytes.
-                constexpr int64_t kQuad = 8 * 8 * 32;            // float4 per (unit, quadrant)
                 float4 *slot = reinterpret_cast<float4 *>(p.part) +
                                ((t.j * t.S + t.s) * 4 + q) * kQuad + lane;
                 for (int g = 0; g < G; ++g) {
@@ -747,7 +1045,7 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     const int warp = threadIdx.x >> 5;
     if (threadIdx.x == 0) {
         for (int i = 0; i < p.stages; ++i) {
-            mbar_init(&s.full[i], kGroupThreads);
+            for (int h = 0; h < kFullPerStage; ++h) mbar_init(&s.full[kFullPerStage * i + h], kGroupThreads);
             mbar_init(&s.wfull[i], 1);
             mbar_init(&s.empty[i], 1);
         }
@@ -756,6 +1054,7 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
             mbar_init(&s.tempty[i], 128);
         }
         mbar_init(s.drain, 1);
+        for (int i = 0; i < 4; ++i) mbar_init(&s.fixbar[i], 1);
         for (int i = 0; i < kWinBufs; ++i) {
             mbar_init(&s.pfull[i], 1);
             mbar_init(&s.pempty[i], kGatherWarps + 1);
@@ -775,8 +1074,21 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     // let the next kernel start its own set-up as SMs come free.
     grid_dependency_wait();
     grid_launch_dependents();
+#ifdef BP_TRACE
+    if (threadIdx.x == 0 && blockIdx.x < 256) g_trace[448 * kTraceEvents + 2 * blockIdx.x] = globaltimer_ns();
+#endif
     if (s.kc)
         for (int64_t i = threadIdx.x; i < p.kc_cached; i += kThreads) s.kc[i] = p.kc_ptr[i];
+    if (p.sk && threadIdx.x == 0) {
+        // the balanced launch's constants, once per CTA (64-bit divisions)
+        const int64_t tile = p.sk_i0 / p.num_slabs;
+        const int64_t p0 = tile * p.kc_total + p.kc_ptr[p.sk_i0 - tile * p.num_slabs];
+        const int64_t T = p.sk_total - p0;
+        s.skv[0] = p0;
+        s.skv[1] = T;
+        s.skv[2] = p0 + (int64_t)blockIdx.x * T / gridDim.x;
+        s.skv[3] = p0 + ((int64_t)blockIdx.x + 1) * T / gridDim.x;
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -797,6 +1109,9 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+#ifdef BP_TRACE
+    if (threadIdx.x == 0 && blockIdx.x < 256) g_trace[448 * kTraceEvents + 2 * blockIdx.x + 1] = globaltimer_ns();
+#endif
     if (warp == kMmaWarp) tmem_dealloc(tmem, p.tmem_cols);
 }
 
@@ -860,6 +1175,37 @@ SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split) {
             sp.full = 0;
         }
     }
+#ifdef BP_BALANCE
+    // Balanced launches are built only with BP_BALANCE: on this kernel they
+    // measured slower than whole items in waves on the 4096^3 layer at 1/4
+    // (46.5 against 41.7 us) and the BERT 3072 x 768 layer (32.6 against 25.4
+    // us), faster only on long dense-union items (4096^3, 8 x 64 blocks at
+    // 1/2: 136.5 against 147.9 us).
+    if (allow_split && sp.items >= sms && dl.kc_total > 0) {
+        // Whole items run in waves of `sms`; when the last wave is partial
+        // the busiest SMs run ceil(items / sms) items against items / sms on
+        // average.  Cut the chunks into equal ranges instead (widest tile:
+        // waves no longer matter) when that wins at least 10 % and every CTA
+        // keeps at least 8 chunks.
+        const int nt = (int)std::max<int64_t>(64, std::min<int64_t>(kNT, (N + 31) / 32 * 32));
+        const int64_t items = (N + nt - 1) / nt * dl.num_slabs;
+        const int64_t total = (N + nt - 1) / nt * dl.kc_total;
+        const double waves = (double)((items + sms - 1) / sms), avg = (double)items / sms;
+        if (waves > 1.1 * avg && total / sms >= 8 && total < INT32_MAX) {
+            sp.nt = nt;
+            sp.items = items;
+            // whole items for all but the last full wave; the ranges then cover
+            // between one and two waves of items
+            sp.full = (items / sms - 1) * sms;
+            sp.balanced = true;
+            sp.total = total;
+            sp.units = sms;
+            sp.bytes = (size_t)((int64_t)sms * kSlab * kNT * 4 + (int64_t)sms * 16);
+            sp.bytes = (sp.bytes + 255) / 256 * 256;
+            return sp;
+        }
+    }
+#endif
     sp.units = sp.full + (sp.items - sp.full) * sp.split;
     if (sp.split > 1) {
         const int64_t slots = (sp.items - sp.full) * sp.split;
@@ -888,6 +1234,19 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     p.split = sp.split;
     p.num_units = sp.units;
     if (p.num_items == 0) return cudaSuccess;
+    if (p.num_units >= INT32_MAX) return cudaErrorInvalidValue;   // 32-bit unit decoding
+    if (sp.balanced) {
+        // one partial tile per CTA, then the per-(CTA, quadrant) flags (zero
+        // on entry: the caller zero-fills a new workspace, and the CTA that
+        // reads a flag zeroes it again)
+        p.sk = 1;
+        p.sk_i0 = sp.full;
+        p.sk_total = sp.total;
+        p.kc_total = dl.kc_total;
+        p.part = static_cast<float *>(ws);
+        p.cnt = reinterpret_cast<int32_t *>(static_cast<uint8_t *>(ws) +
+                                            (int64_t)sp.units * kSlab * kNT * 4);
+    }
     if (sp.split > 1) {
         // partial tiles, then the arrival counters (zero on entry: the caller
         // zero-fills a new workspace, and each item's last unit zeroes its
@@ -992,11 +1351,24 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    const bool parts = p.split > 1 || p.sk;
     if (conv)
-        return p.split > 1 ? cudaLaunchKernelEx(&cfg, bp_mma_kernel<true, true>, p)
-                           : cudaLaunchKernelEx(&cfg, bp_mma_kernel<false, true>, p);
-    return p.split > 1 ? cudaLaunchKernelEx(&cfg, bp_mma_kernel<true, false>, p)
-                       : cudaLaunchKernelEx(&cfg, bp_mma_kernel<false, false>, p);
+        return parts ? cudaLaunchKernelEx(&cfg, bp_mma_kernel<true, true>, p)
+                     : cudaLaunchKernelEx(&cfg, bp_mma_kernel<false, true>, p);
+    return parts ? cudaLaunchKernelEx(&cfg, bp_mma_kernel<true, false>, p)
+                 : cudaLaunchKernelEx(&cfg, bp_mma_kernel<false, false>, p);
 }
 
 }  // namespace bp
+
+#ifdef BP_TRACE
+// Copies the trace (kTraceChunks x kTraceEvents clock64 values) to host memory.
+extern "C" int bp_debug_trace_read(unsigned long long *host, int n) {
+    if (n > bp::kTraceChunks * bp::kTraceEvents) n = bp::kTraceChunks * bp::kTraceEvents;
+    return cudaMemcpyFromSymbol(host, bp::g_trace, n * sizeof(unsigned long long)) == cudaSuccess ? n : -1;
+}
+extern "C" int bp_debug_trace_clear(void) {
+    static unsigned long long zero[bp::kTraceChunks * bp::kTraceEvents];
+    return cudaMemcpyToSymbol(bp::g_trace, zero, sizeof(zero)) == cudaSuccess ? 0 : -1;
+}
+#endif
