@@ -642,7 +642,10 @@ def run_workload(args):
         def timed(fn, reps=5):
             ts = []
             for _ in range(reps + 1):
+                # flush L2 and read the flush buffer back: the lines left in L2
+                # are clean, so no write-back of the flush lands in the timing
                 flush.zero_()
+                flush.sum()
                 ev[0].record()
                 fn()
                 ev[1].record()
@@ -689,7 +692,10 @@ def run_workload(args):
         def timed(fn, reps=9):
             ts = []
             for _ in range(reps + 1):
+                # flush L2 and read the flush buffer back: the lines left in L2
+                # are clean, so no write-back of the flush lands in the timing
                 flush.zero_()
+                flush.sum()
                 ev[0].record()
                 fn()
                 ev[1].record()
@@ -775,6 +781,64 @@ def run_workload(args):
     print(json.dumps(out), flush=True)
 
 
+def _free_port() -> int:
+    import socket
+    with socket.socket() as sk:
+        sk.bind(("127.0.0.1", 0))
+        return sk.getsockname()[1]
+
+
+def torchrun_cmd(n: int, argv, port: int):
+    """The one-process-per-GPU launch the benchmark contract uses, for N ranks."""
+    return [sys.executable, "-m", "torch.distributed.run", "--nnodes=1",
+            f"--nproc-per-node={n}", "--master-addr=127.0.0.1", f"--master-port={port}",
+            os.path.abspath(__file__), *argv]
+
+
+def launch_ranks(n: int, argv) -> int:
+    """`--gpus N` (N > 1) started without torchrun: start N ranks through
+    torch.distributed.run on this node and return the launcher's exit code."""
+    import subprocess
+    return subprocess.call(torchrun_cmd(n, argv, _free_port()))
+
+
+def run_dry(args):
+    """The multi-rank skeleton without GPU work (gloo on CPU): every rank joins
+    the process group, times a fixed amount of host work between two barriers,
+    and rank 0 prints the whole-job line the same way the GPU arm does."""
+    import torch
+    import torch.distributed as dist
+    world, rank, _ = dist_setup()
+    if world > 1:
+        dist.init_process_group("gloo")
+    units_per_step = 1.0e6 * (rank + 1)
+    if world > 1:
+        dist.barrier()
+    t0 = time.perf_counter()
+    acc = 0.0
+    for i in range(args.steps):
+        acc += float(torch.ones(256).sum())
+    local_s = time.perf_counter() - t0
+    if world > 1:
+        dist.barrier()
+
+        def red(v, op):
+            t = torch.tensor([v], dtype=torch.float64)
+            dist.all_reduce(t, op=op)
+            return float(t.item())
+        rmax = lambda v: red(v, dist.ReduceOp.MAX)  # noqa: E731
+        rsum = lambda v: red(v, dist.ReduceOp.SUM)  # noqa: E731
+    else:
+        rmax = rsum = (lambda v: v)
+    value, tmax = aggregate(local_s, units_per_step * args.steps, world, rmax, rsum)
+    units = rsum(units_per_step * args.steps)
+    if rank == 0:
+        print(json.dumps({"dry_run": True, "n_gpus": world, "steps": args.steps,
+                          "value": value, "seconds_max": tmax, "units": units}), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -792,9 +856,22 @@ def main():
     ap.add_argument("--sweep-subset", action="store_true")
     ap.add_argument("--layers", default=None,
                     help="comma-separated layer names: time only these layers of the workload")
+    ap.add_argument("--dry-run", action="store_true",
+                    help="the multi-rank skeleton on CPU (gloo), no GPU work: for testing "
+                         "the launch and aggregation")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
+    world = os.environ.get("WORLD_SIZE")
+    if world is None and args.gpus > 1:
+        # one process per GPU, as the benchmark contract launches them
+        sys.exit(launch_ranks(args.gpus, sys.argv[1:]))
+    if world is not None and int(world) != args.gpus:
+        print(f"bench.py: --gpus {args.gpus} but WORLD_SIZE={world}", file=sys.stderr)
+        sys.exit(2)
+    if args.dry_run:
+        run_dry(args)
+        return
     if args.workload:
         run_workload(args)
     elif args.impl == "reference":

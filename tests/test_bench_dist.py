@@ -1,8 +1,12 @@
 """Host logic of the multi-rank benchmark on CPU: world_size-2 gloo ranks
 combine their local times and work the way bench.py does (whole-job units
-over the slowest rank's time), and only rank 0 of the reference arm runs."""
+over the slowest rank's time), only rank 0 of the reference arm runs, and
+`bench.py --gpus 2` started without torchrun launches two ranks itself."""
+import json
 import os
 import socket
+import subprocess
+import sys
 
 import pytest
 import torch
@@ -67,3 +71,34 @@ def test_reference_arm_other_ranks_do_nothing(monkeypatch, capsys):
         steps, warmup = 3, 3
     bench.run_reference(A())
     assert capsys.readouterr().out == ""
+
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def test_gpus_flag_launches_that_many_ranks():
+    """--gpus 2 without a torchrun environment: bench.py starts two ranks through
+    torch.distributed.run (gloo in the dry run) and rank 0 prints one line for
+    the whole job."""
+    env = {k: v for k, v in os.environ.items()
+           if k not in ("WORLD_SIZE", "RANK", "LOCAL_RANK", "MASTER_ADDR", "MASTER_PORT")}
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--gpus", "2",
+                        "--dry-run", "--steps", "5"], capture_output=True, text=True,
+                       timeout=300, env=env, cwd=ROOT)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, r.stdout
+    out = json.loads(lines[0])
+    assert out["n_gpus"] == 2 and out["dry_run"]
+    # rank r does (r + 1) * 1e6 units per step: 3e6 per step in total
+    assert out["units"] == pytest.approx(3.0e6 * 5)
+    assert out["value"] == pytest.approx(out["units"] / out["seconds_max"])
+
+
+def test_gpus_flag_must_match_the_launch(monkeypatch):
+    env = dict(os.environ, WORLD_SIZE="1", RANK="0", LOCAL_RANK="0")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--gpus", "2",
+                        "--dry-run"], capture_output=True, text=True, timeout=120, env=env,
+                       cwd=ROOT)
+    assert r.returncode != 0
+    assert "WORLD_SIZE" in r.stderr
