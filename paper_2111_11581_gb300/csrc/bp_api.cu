@@ -206,12 +206,34 @@ bool checked_mode() {
 
 static int64_t qmap_bytes(const bp_layout &lay) { return align_up(4 * lay.K, 16); }
 
+int64_t kgroups(const bp_layout &lay) {
+    if ((int64_t)lay.kh * lay.kw <= 1) return 0;
+    const int64_t C = lay.K / ((int64_t)lay.kh * lay.kw);
+    return cdiv(C, 64) * lay.kh * lay.kw;
+}
+
+static int64_t sec3_chunks(const bp_layout &lay) {
+    return cdiv(lay.M, kSlab) * kgroups(lay);
+}
+
+int64_t sec3_bytes(const bp_layout &lay) {
+    const int64_t c3 = sec3_chunks(lay);
+    if (c3 == 0) return 0;
+    return align_up(8 * (cdiv(lay.M, kSlab) + 1), 256) + c3 * ((int64_t)kSlab * kBK * 2 + kMetaBytes);
+}
+
 static void set_chunks(DevLayout &d, const bp_layout &lay, int64_t kc) {
     d.kc_total = kc;
     d.off_meta = d.off_tiles + kc * d.tile_bytes;
     d.off_meta2 = d.off_meta + kc * kMetaBytes;
     d.off_qmap = d.off_meta2 + kc * kMetaBytes;
     d.bytes = d.off_qmap + qmap_bytes(lay);
+    if (d.c3max > 0) {
+        d.off_sec3 = align_up(d.bytes, 256);
+        d.off_tiles3 = d.off_sec3 + align_up(8 * (d.num_slabs + 1), 256);
+        d.off_meta3 = d.off_tiles3 + d.c3max * d.tile_bytes;
+        d.bytes = d.off_sec3 + sec3_bytes(lay);
+    }
 }
 
 DevLayout dev_layout(const bp_layout &lay, const int64_t *slab_chunks_host) {
@@ -221,6 +243,8 @@ DevLayout dev_layout(const bp_layout &lay, const int64_t *slab_chunks_host) {
     d.tile_bytes = (int64_t)kSlab * kBK * 2;
     d.kc_total = -1;
     d.off_meta = d.off_meta2 = d.off_qmap = -1;
+    d.c3max = sec3_chunks(lay);
+    d.off_sec3 = d.off_tiles3 = d.off_meta3 = -1;
     d.bytes = -1;
     if (slab_chunks_host) {
         int64_t kc = 0;
@@ -245,6 +269,53 @@ static bp_status slab_chunk_counts(const bp_layout &lay, const uint8_t *mask, cu
     chunks.resize(S);
     for (int64_t i = 0; i < S; ++i) chunks[i] = h[2 * i] + cdiv(h[2 * i + 1], kBK);
     return BP_OK;
+}
+
+ImplicitTiles implicit_tiles(const ConvShape &cs) {
+    ImplicitTiles t{};
+    t.ok = false;
+    if (cs.Wo < 1 || cs.Ho < 1 || cs.Wo > 256 || cs.W > 256 || cs.Nb < 1) return t;
+    const int64_t HoWo = cs.Ho * cs.Wo;
+    int64_t px;
+    if (HoWo <= 256) {
+        // tiles of whole images (box: 64 channels x Wo x Ho x ipt)
+        t.ipt = std::min<int64_t>(256 / HoWo, cs.Nb);
+        t.rpt = cs.Ho;
+        t.tpi = 1;
+        t.tiles = cdiv(cs.Nb, t.ipt);
+        px = t.ipt * HoWo;
+    } else {
+        // tiles of rpt whole rows of one image (box: 64 channels x Wo x rpt x 1);
+        // rpt * Wo a multiple of 8 where possible, so that every tile starts
+        // 16-byte aligned in the NCHW output (its TMA box stores need that)
+        t.ipt = 0;
+        t.rpt = 256 / cs.Wo;
+        for (int64_t r = t.rpt; r >= 1; --r)
+            if ((r * cs.Wo) % 8 == 0) {
+                t.rpt = r;
+                break;
+            }
+        t.tpi = cdiv(cs.Ho, t.rpt);
+        t.tiles = cs.Nb * t.tpi;
+        px = t.rpt * cs.Wo;
+    }
+    t.nt = (int)align_up(px, 32);
+    t.ok = t.nt <= 256 && t.tiles < INT32_MAX;
+    return t;
+}
+
+// The implicit convolution serves stride-1 layers with a kh x kw > 1 window
+// (the image's section 3); strided and 1 x 1 layers take the im2col path.
+bool implicit_conv_ok(const bp_packed &P, const ConvShape &cs) {
+    if ((int64_t)cs.kh * cs.kw <= 1 || cs.sh != 1 || cs.sw != 1) return false;
+    if (sec3_bytes(P.lay) == 0) return false;
+    if (cs.ph > 255 || cs.pw > 255 || cs.kh > 255 || cs.kw > 255) return false;
+    if ((cs.C + 63) / 64 > 32767) return false;
+    return implicit_tiles(cs).ok;
+}
+
+size_t nhwc8_bytes(const ConvShape &cs) {
+    return (size_t)align_up(cs.Nb * cs.H * cs.W * align_up(cs.C, 8) * 2, 256);
 }
 
 }  // namespace bp
@@ -388,6 +459,11 @@ bp_status bp_pack(const bp_layout *lay, const void *W, const uint8_t *mask, bp_p
     for (int64_t i = 0; i < dl.num_slabs; ++i) kc[i + 1] = kc[i] + sc[i];
     e = cudaMemcpyAsync(out->dev, kc.data(), 8 * (dl.num_slabs + 2), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = launch_pack(*lay, W, mask, *out, dl, s);
+    if (e == cudaSuccess && dl.c3max > 0) {
+        int64_t *scratch = nullptr;   // the slab-count words (under g_mu)
+        e = cudaGetSymbolAddress(reinterpret_cast<void **>(&scratch), g_slab_info);
+        if (e == cudaSuccess) e = launch_pack_sec3(*lay, W, mask, *out, dl, scratch, s);
+    }
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     return cuda_status(e);
 }
@@ -398,10 +474,15 @@ static bp_status check_packed(const bp_packed *P, DevLayout *dl) {
     if (cdiv(P->lay.M, kSlab) > kMaxSlabs) return BP_ERR_UNSUPPORTED;
     *dl = dev_layout(P->lay, nullptr);
     // the chunk count follows from the image size: tiles + two record sets + qmap
-    const int64_t rest = P->dev_bytes - dl->off_tiles - qmap_bytes(P->lay);
-    if (rest < 0 || rest % kChunkBytes) return BP_ERR_INVALID_ARG;
-    set_chunks(*dl, P->lay, rest / kChunkBytes);
-    return BP_OK;
+    // (+ section 3, whose size the layout fixes; it starts 256-byte aligned)
+    const int64_t s3 = sec3_bytes(P->lay);
+    for (int64_t pad = 0; pad < (s3 ? 256 : 1); pad += 16) {
+        const int64_t rest = P->dev_bytes - s3 - pad - dl->off_tiles - qmap_bytes(P->lay);
+        if (rest < 0 || rest % kChunkBytes) continue;
+        set_chunks(*dl, P->lay, rest / kChunkBytes);
+        if (dl->bytes == P->dev_bytes) return BP_OK;
+    }
+    return BP_ERR_INVALID_ARG;
 }
 
 static bp_status finish_launch(cudaError_t e, cudaStream_t s) {
@@ -476,6 +557,11 @@ bp_status bp_conv2d_workspace_size(const bp_packed *P, int64_t Nb, int64_t C, in
     const bp_status st = conv_shape(P, Nb, C, H, W, pad_h, pad_w, stride_h, stride_w, &cs, &dl);
     if (st != BP_OK) return st;
     const int64_t N = Nb * cs.Ho * cs.Wo;
+    if (implicit_conv_ok(*P, cs)) {
+        const ImplicitTiles it = implicit_tiles(cs);
+        *bytes = nhwc8_bytes(cs) + plan_split(dl, N, true, &it).bytes;
+        return BP_OK;
+    }
     *bytes = (size_t)align_up(P->lay.K * align_up(N, 8) * 2, 256) + plan_split(dl, N, true).bytes;
     return BP_OK;
 }
@@ -493,6 +579,21 @@ bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, i
     if (bias && (reinterpret_cast<uintptr_t>(bias) & 3u)) return BP_ERR_INVALID_ARG;
     const int64_t N = Nb * cs.Ho * cs.Wo;
     if (N == 0) return BP_OK;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (implicit_conv_ok(*P, cs)) {
+        // implicit GEMM: the input goes to NHWC (channels padded to 8) in the
+        // workspace; the product loads its B operand from it with TMA boxes
+        const ImplicitTiles it = implicit_tiles(cs);
+        const size_t xb = nhwc8_bytes(cs);
+        const size_t sb = plan_split(dl, N, true, &it).bytes;
+        if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < xb + sb)
+            return BP_ERR_WORKSPACE;
+        void *split_ws = sb ? static_cast<uint8_t *>(ws) + xb : nullptr;
+        cudaError_t e = launch_nhwc8(cs, in, ws, s);
+        if (e != cudaSuccess) return BP_ERR_CUDA;
+        return finish_launch(
+            launch_mma(*P, dl, ws, N, 0, bias, relu, out, 0, &cs, split_ws, s, true), s);
+    }
     const int64_t ldx = align_up(N, 8);
     // workspace: the im2col matrix, then the split product's partial tiles
     const size_t xbytes = (size_t)align_up(P->lay.K * ldx * 2, 256);
@@ -500,7 +601,6 @@ bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, i
     if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < xbytes + sbytes)
         return BP_ERR_WORKSPACE;
     void *split_ws = sbytes ? static_cast<uint8_t *>(ws) + xbytes : nullptr;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
     const int32_t *qmap =
         reinterpret_cast<const int32_t *>(static_cast<const uint8_t *>(P->dev) + dl.off_qmap);
     cudaError_t e = launch_im2col(cs, ldx, in, ws, qmap, s);

@@ -70,6 +70,22 @@ constexpr int kMaxBoxes = 8;         // tile loads in a chunk's plan at most
 //                                its im2col matrix, in that order.
 //   off_qmap + 4*k               int32 qmap[k]: rank of column k among the
 //                                listed columns, -1 if no slab lists it.
+//
+//
+// Layers with kh * kw > 1 carry a third section, the same slabs in the form
+// the implicit convolution streams.  There a chunk is one K-group: 64
+// consecutive input channels at one kernel position, (c64, i, j), i.e. the
+// GEMM-view columns (64 c64 + u) kh kw + i kw + j, u < 64 (channels past C
+// have zero weights).  Per slab, the K-groups any of its rows keeps are listed
+// position-major ((i, j), then c64).  The section is sized for every K-group
+// listed (c3max chunks), so its size follows from the layout:
+//   off_sec3                     int64 kc3_ptr[S+1]: first chunk of each slab
+//   off_tiles3 + c*16384         chunk c's 128 x 64 weight tile, K-major with
+//                                the 128-byte swizzle; column u = channel
+//                                64 c64 + u
+//   off_meta3 + c*kMetaBytes     chunk c's record: int32 word [0] its K-group
+//                                (c64 << 16 | i << 8 | j), [64] = 1 (every
+//                                chunk is loaded with TMA)
 struct DevLayout {
     int64_t num_slabs;
     int64_t kc_total;     // total k-chunks (-1 if unknown)
@@ -78,8 +94,15 @@ struct DevLayout {
     int64_t off_meta2;
     int64_t off_qmap;
     int64_t tile_bytes;   // 128 * 64 * 2
+    int64_t c3max;        // section 3: chunks it has room for (0: no section)
+    int64_t off_sec3;     // (these three when kc_total is known and c3max > 0)
+    int64_t off_tiles3;
+    int64_t off_meta3;
     int64_t bytes;        // total image size (when kc_total is known)
 };
+// K-groups of a layout's section 3, and the section's size
+int64_t kgroups(const bp_layout &lay);
+int64_t sec3_bytes(const bp_layout &lay);
 constexpr int64_t kChunkBytes = 128 * kBK * 2 + 2 * kMetaBytes;   // per k-chunk, all parts
 
 // Image layout; slab_chunks_host = per-slab chunk counts (host) or nullptr.
@@ -129,6 +152,11 @@ cudaError_t launch_slab_counts(const bp_layout &lay, const uint8_t *mask, int64_
                                cudaStream_t s);
 cudaError_t launch_pack(const bp_layout &lay, const void *W, const uint8_t *mask,
                         const bp_packed &P, const DevLayout &dl, cudaStream_t s);
+// Section 3 of the device image (see DevLayout); scratch: 8 * (S + 1) bytes of
+// device memory for the per-slab counts.
+cudaError_t launch_pack_sec3(const bp_layout &lay, const void *W, const uint8_t *mask,
+                             const bp_packed &P, const DevLayout &dl, int64_t *scratch,
+                             cudaStream_t s);
 
 struct ConvShape {
     int64_t Nb, C, H, W, Ho, Wo;
@@ -141,6 +169,19 @@ struct ConvShape {
 cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void *xcol,
                           const int32_t *qmap, cudaStream_t s);
 int64_t im2col_row_width(const ConvShape &cs);   // staged input row length (elements)
+// NCHW input -> NHWC with the channels padded to a multiple of 8 (zeros):
+// out[b][h][w][c], C8 = roundup(C, 8) channels per pixel.
+cudaError_t launch_nhwc8(const ConvShape &cs, const void *in, void *out, cudaStream_t s);
+// Implicit convolution (stride 1, kh * kw > 1): output tiles of whole output
+// rows.  ipt > 0: tiles of ipt whole images; else tiles of rpt rows of one
+// image (tpi tiles per image).  nt = the tile's pixels rounded up to 32.
+struct ImplicitTiles {
+    int64_t ipt, rpt, tpi, tiles;
+    int nt;
+    bool ok;
+};
+ImplicitTiles implicit_tiles(const ConvShape &cs);
+bool implicit_conv_ok(const bp_packed &P, const ConvShape &cs);
 // The block-sparse product on the tensor cores: Y = act(W_packed X + bias).
 // conv == nullptr: Y is M x N row-major (ldy).  Otherwise Y is the NCHW output
 // of the convolution and X its im2col matrix.
@@ -163,13 +204,16 @@ struct SplitPlan {
     int64_t total;      // balanced: chunks of all items
     size_t bytes;       // workspace: partial tiles + counters / flags (0 if none)
 };
-SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split);
+// it: the implicit convolution's tiles (nullptr: tiles of nt consecutive columns)
+SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split,
+                     const ImplicitTiles *it = nullptr);
 
 // With conv, X holds only the listed rows (see DevLayout::off_meta2).  ws:
 // at least plan_split(dl, N, true).bytes of 256-byte-aligned device memory,
 // or nullptr (no split).
 cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, int64_t N,
                        int64_t ldx, const float *bias, int relu, void *Y, int64_t ldy,
-                       const ConvShape *conv, void *ws, cudaStream_t s);
+                       const ConvShape *conv, void *ws, cudaStream_t s,
+                       bool implicit = false);
 
 }  // namespace bp

@@ -126,6 +126,15 @@ struct Params {
                             // balanced launches: one tile per CTA
     int32_t *cnt;           // split items: arrivals per (item, row quadrant); balanced
                             // launches: per (CTA, row quadrant) "partial written" flags
+    // implicit convolution (stride 1): X is the NHWC input with channels padded
+    // to 8 (imap: 4-D (C8, W, H, Nb), boxes of 64 channels x Wo x hbox x nbox);
+    // a chunk's B operand is one box: per output pixel a K-major row of 64
+    // channels at one kernel position (128-byte swizzle)
+    int impl;
+    CUtensorMap imap;
+    int64_t i_ipt, i_rpt, i_tpi, i_HoWo, i_Wo, i_Ho, i_Nb;
+    int i_ph, i_pw;
+    uint32_t i_box_bytes;
     int sk;                 // 1: balanced launch (whole items in full waves, then each CTA
                             // one equal range of the remaining items' chunks)
     int64_t sk_i0;          // balanced launch: first item of the ranges
@@ -229,6 +238,8 @@ struct Item {
     // 2 a later range of its chunks (this CTA writes a partial tile)
     int role;
     int64_t gpos, nitem;                // first chunk of the item (global position), its chunks
+    int64_t ncols;                      // output columns (pixels) of the tile
+    int64_t img0, h0;                   // implicit convolution: first image and row of the tile
 };
 
 // Work unit u -> (slab, column tile) item, slab fastest, and its k-chunk
@@ -257,6 +268,23 @@ __device__ __forceinline__ Item decode(const Params &p, const int64_t *kc, int64
     const uint32_t tile = it / ns;
     t.slab = it - tile * ns;
     t.n0 = (int64_t)tile * p.nt;
+    t.ncols = min((int64_t)p.nt, p.N - t.n0);
+    t.img0 = t.h0 = 0;
+    if (p.impl) {
+        // tiles of whole output rows: ipt images, or rpt rows of one image
+        if (p.i_ipt > 0) {
+            t.img0 = (int64_t)tile * p.i_ipt;
+            t.n0 = t.img0 * p.i_HoWo;
+            t.ncols = min(p.i_ipt, p.i_Nb - t.img0) * p.i_HoWo;
+        } else {
+            const uint32_t tpi = (uint32_t)p.i_tpi;
+            const uint32_t img = tile / tpi;
+            t.img0 = img;
+            t.h0 = (int64_t)(tile - img * tpi) * p.i_rpt;
+            t.n0 = t.img0 * p.i_HoWo + t.h0 * p.i_Wo;
+            t.ncols = min(p.i_rpt, p.i_Ho - t.h0) * p.i_Wo;
+        }
+    }
     const int64_t c0 = kc[t.slab], nc = kc[t.slab + 1] - c0;
     if (t.S == 1) {
         t.kc0 = c0;
@@ -320,6 +348,8 @@ __device__ __forceinline__ Item sk_decode(const Params &p, const int64_t *kc, in
     t.gpos = u - klo;
     t.role = klo > 0 ? 2 : (khi < t.nitem ? 1 : 0);
     t.rows = min((int64_t)kSlab, p.M - t.slab * kSlab);
+    t.ncols = min((int64_t)p.nt, p.N - t.n0);
+    t.img0 = t.h0 = 0;
     return t;
 }
 
@@ -580,7 +610,20 @@ __device__ void control_thread(const Params &p, const Smem &s) {
             const int nb = (int)q0.x;
             const bool tma = nb > 0;
             ++count;
-            if (!(blockIdx.x == 0 && seq == p.drop_stage)) {
+            if (p.impl && !(blockIdx.x == 0 && seq == p.drop_stage)) {
+                // implicit convolution: the weight tile and one box of 64
+                // channels at kernel position (i, j) for the tile's pixels (the
+                // padding and channels past C read as zeros)
+                const int32_t d = *reinterpret_cast<const int32_t *>(recs + j * kMetaBytes);
+                s.skind[stage] = 1u;
+                mbar_arrive_expect_tx(&s.wfull[stage], kWTileBytes + p.i_box_bytes);
+                bulk_g2s(smem_u32(s.w + stage * kWTileBytes),
+                         p.tiles + (win.t.kc0 + win.k0 + j) * (int64_t)kWTileBytes, kWTileBytes,
+                         &s.wfull[stage]);
+                tma_load_4d(smem_u32(s.x + stage * kXTileBytes), &p.imap, (d >> 16) * 64,
+                            (d & 0xff) - p.i_pw, (int32_t)win.t.h0 + ((d >> 8) & 0xff) - p.i_ph,
+                            (int32_t)win.t.img0, &s.wfull[stage]);
+            } else if (!(blockIdx.x == 0 && seq == p.drop_stage)) {
                 s.skind[stage] = tma ? 1u : 0u;    // read by the MMA thread after wfull
                 mbar_arrive_expect_tx(&s.wfull[stage],
                                       kWTileBytes + (tma ? (uint32_t)p.xboxes * (kBK * 128) : 0u));
@@ -641,11 +684,17 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
     const uint32_t acc_cols = p.acc_cols;
     uint64_t *const wfull = s.wfull, *const full = s.full, *const empty = s.empty;
     const volatile uint32_t *const skind = s.skind;
-    const uint32_t idesc = make_idesc(p.dtype == BP_BF16, false, true, kSlab, p.nt);
+    // B: MN-major activation rows, or for the implicit convolution K-major
+    // pixel rows (both with the 128-byte swizzle)
+    const uint32_t idesc = make_idesc(p.dtype == BP_BF16, false, !p.impl, kSlab, p.nt);
     // descriptors of stage 0; a stage / K=16 step adds its byte offset / 16 to
     // the start-address field (shared addresses stay below 256 KB: no carry)
     const uint64_t wdesc0 = make_sdesc_sw128(smem_u32(s.w), 16, 1024);
-    const uint64_t xdesc0 = make_sdesc_sw128(smem_u32(s.x), 8192, 1024);
+    const uint64_t xdesc0 = p.impl ? make_sdesc_sw128(smem_u32(s.x), 16, 1024)
+                                   : make_sdesc_sw128(smem_u32(s.x), 8192, 1024);
+    // one K=16 step: 16 activation rows (MN-major) or 32 bytes of every pixel
+    // row (implicit: K-major pixel rows of 64 channels)
+    const uint32_t xkstep = p.impl ? 32u >> 4 : 2048u >> 4;
     int stage = 0;
     uint32_t phase = 0;
     uint32_t gphase = 0;     // per gather barrier: parity of its next fill (bit = barrier)
@@ -707,7 +756,7 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
 #ifdef BP_GATHER_HALVES
 #pragma unroll
             for (int kk = 0; kk < 2; ++kk)
-                umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * (2048 >> 4), idesc,
+                umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * xkstep, idesc,
                             (kc > 0 || kk > 0) ? 1u : 0u);
             if (gathered) {
                 if (!mbar_wait(&full[fb + 1], (gphase >> (fb + 1)) & 1u, wdog, abort_flag)) {
@@ -721,11 +770,11 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
             }
 #pragma unroll
             for (int kk = 2; kk < 4; ++kk)
-                umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * (2048 >> 4), idesc, 1u);
+                umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * xkstep, idesc, 1u);
 #else
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk)
-                umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * (2048 >> 4), idesc,
+                umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * xkstep, idesc,
                             (kc > 0 || kk > 0) ? 1u : 0u);
 #endif
             umma_commit(&empty[stage]);
@@ -800,10 +849,10 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                 // NCHW output, pixel n = b*HoWo + hw is element (b, m, hw)
                 const uint32_t bb = (uint32_t)n / (uint32_t)p.HoWo;
                 const uint32_t hw = (uint32_t)n - bb * (uint32_t)p.HoWo;
-                if (p.ytma && hw + 32 <= (uint32_t)p.HoWo) {
-                    // the 32 pixels lie in one image: stage the box like a GEMM
-                    // box (below) and store it at (hw, m, b) of the 3-D output
-                    // map (Ho*Wo is a multiple of 8, so hw is 16-byte aligned)
+                if (p.ytma && hw + 32 <= (uint32_t)p.HoWo && c0 + 32 <= t.ncols && (hw & 7u) == 0) {
+                    // the 32 pixels lie in one image and in the tile: stage the box
+                    // like a GEMM box (below) and store it at (hw, m, b) of the
+                    // 3-D output map (a TMA store needs hw 16-byte aligned)
                     const uint32_t sb = stg + (yseq & 1u) * 2048;
                     ++yseq;
                     if (lane == 0) bulk_wait_read<1>();
@@ -822,8 +871,8 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                     }
                     return;
                 }
-                // Ho*Wo not a multiple of 8, or the 32 pixels cross an image
-                // boundary: stage the 32 x 32 box (lane = channel row, 80-byte
+                // Ho*Wo not a multiple of 8, the 32 pixels cross an image
+                // boundary or the tile's end: stage the 32 x 32 box (lane = channel row, 80-byte
                 // rows), then write it with lanes along the pixels, one
                 // coalesced 64-byte store per channel
                 uint8_t *box = s.ystage + (warp - kEpiWarp0) * 4096;
@@ -838,7 +887,9 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                 __syncwarp();
                 const int64_t nn = n + lane;
                 const int rmax = (int)min((int64_t)32, t.rows - row0);
-                if (nn < p.N && rmax > 0) {
+                // only the tile's own pixels: an implicit convolution's tile
+                // holds fewer pixels than the MMA's N
+                if (nn < t.n0 + t.ncols && rmax > 0) {
                     const uint32_t bb = (uint32_t)nn / (uint32_t)p.HoWo;
                     const uint32_t hw = (uint32_t)nn - bb * (uint32_t)p.HoWo;
                     uint16_t *dst = p.Y + ((int64_t)bb * p.M + t.slab * kSlab + row0) * p.HoWo + hw;
@@ -869,7 +920,7 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             }
                 };
         if (row0 < t.rows) {
-            const int64_t cols = min((int64_t)p.nt, p.N - t.n0);
+            const int64_t cols = t.ncols;
             const int G = (int)((cols + 31) / 32);
             uint32_t r[32], pk[16];
             if (has) {
@@ -1153,21 +1204,23 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
     return fn;
 }
 
-SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split) {
+SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split, const ImplicitTiles *it) {
     SplitPlan sp{};
     const int sms = num_sms();
-    sp.nt = pick_tile_width(N, dl.num_slabs, sms);
-    sp.items = (N + sp.nt - 1) / sp.nt * dl.num_slabs;
+    sp.nt = it ? it->nt : pick_tile_width(N, dl.num_slabs, sms);
+    sp.items = (it ? it->tiles : (N + sp.nt - 1) / sp.nt) * dl.num_slabs;
     sp.full = sp.items;
     sp.split = 1;
-    if (allow_split && sp.items < sms && dl.kc_total > 0) {
+    // chunks of all slabs (the implicit convolution's section: its capacity)
+    const int64_t kct = it ? dl.c3max : dl.kc_total;
+    if (allow_split && sp.items < sms && kct > 0) {
         // Fewer items than SMs: split every item along its chunks so that the
         // units fill the SMs, each unit keeping at least four chunks on
         // average.  (Splitting only a partial last wave of a larger problem
         // measured slower: the partial tiles' write, read and second epilogue
         // cost more than the chunks they move.)
         int64_t S = sms / sp.items;
-        const int64_t avg = dl.kc_total / dl.num_slabs;
+        const int64_t avg = kct / dl.num_slabs;
         if (S > avg / 4) S = avg / 4;
         if (S > 32) S = 32;
         if (S >= 2) {
@@ -1176,6 +1229,7 @@ SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split) {
         }
     }
 #ifdef BP_BALANCE
+    if (!it)
     // Balanced launches are built only with BP_BALANCE: on this kernel they
     // measured slower than whole items in waves on the 4096^3 layer at 1/4
     // (46.5 against 41.7 us) and the BERT 3072 x 768 layer (32.6 against 25.4
@@ -1217,7 +1271,7 @@ SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split) {
 
 cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, int64_t N,
                        int64_t ldx, const float *bias, int relu, void *Y, int64_t ldy,
-                       const ConvShape *conv, void *ws, cudaStream_t st) {
+                       const ConvShape *conv, void *ws, cudaStream_t st, bool implicit) {
     Params p{};
     const uint8_t *dev = static_cast<const uint8_t *>(P.dev);
     p.dtype = P.lay.dtype;
@@ -1226,7 +1280,10 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     p.M = P.lay.M;
     p.num_slabs = dl.num_slabs;
     p.N = N;
-    const SplitPlan sp = plan_split(dl, N, ws != nullptr);
+    if (implicit && (!conv || dl.c3max == 0)) return cudaErrorInvalidValue;
+    const ImplicitTiles itl = implicit ? implicit_tiles(*conv) : ImplicitTiles{};
+    if (implicit && !itl.ok) return cudaErrorInvalidValue;
+    const SplitPlan sp = plan_split(dl, N, ws != nullptr, implicit ? &itl : nullptr);
     p.nt = sp.nt;
     p.xboxes = (p.nt + 63) / 64;
     p.num_items = sp.items;
@@ -1274,6 +1331,22 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     p.tiles = dev + dl.off_tiles;
     // a convolution's X holds only the listed rows: use the compacted records
     p.meta = dev + (conv ? dl.off_meta2 : dl.off_meta);
+    if (implicit) {
+        // section 3 of the image: K-group chunks
+        p.impl = 1;
+        p.kc_ptr = reinterpret_cast<const int64_t *>(dev + dl.off_sec3);
+        p.tiles = dev + dl.off_tiles3;
+        p.meta = dev + dl.off_meta3;
+        p.i_ipt = itl.ipt;
+        p.i_rpt = itl.rpt;
+        p.i_tpi = itl.tpi;
+        p.i_HoWo = conv->Ho * conv->Wo;
+        p.i_Wo = conv->Wo;
+        p.i_Ho = conv->Ho;
+        p.i_Nb = conv->Nb;
+        p.i_ph = conv->ph;
+        p.i_pw = conv->pw;
+    }
     p.X = static_cast<const uint16_t *>(X);
     p.ldx = ldx;
     p.Y = static_cast<uint16_t *>(Y);
@@ -1288,7 +1361,27 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     if (!enc) return cudaErrorNotSupported;
     const CUtensorMapDataType tdt =
         P.lay.dtype == BP_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
-    for (int i = 0; i < 4; ++i) {
+    if (implicit) {
+        // NHWC input, channels padded to C8: boxes of 64 channels x Wo x hbox x
+        // nbox (channels past C8 read as zero), written as K-major 128-byte rows
+        // with the 128-byte swizzle
+        const int64_t C8 = (conv->C + 7) / 8 * 8;
+        const cuuint64_t gdim[4] = {(cuuint64_t)C8, (cuuint64_t)conv->W, (cuuint64_t)conv->H,
+                                    (cuuint64_t)conv->Nb};
+        const cuuint64_t gstride[3] = {(cuuint64_t)(C8 * 2), (cuuint64_t)(conv->W * C8 * 2),
+                                       (cuuint64_t)(conv->H * conv->W * C8 * 2)};
+        const cuuint32_t hbox = (cuuint32_t)(itl.ipt > 0 ? conv->Ho : itl.rpt);
+        const cuuint32_t nbox = (cuuint32_t)(itl.ipt > 0 ? itl.ipt : 1);
+        const cuuint32_t box[4] = {64, (cuuint32_t)conv->Wo, hbox, nbox};
+        const cuuint32_t estride[4] = {1, 1, 1, 1};
+        p.i_box_bytes = 128u * box[1] * hbox * nbox;
+        if (p.i_box_bytes > 128u * (uint32_t)p.nt) return cudaErrorInvalidValue;
+        if (enc(&p.imap, tdt, 4, const_cast<void *>(X), gdim, gstride, box, estride,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    for (int i = 0; i < 4 && !implicit; ++i) {
         // X (N inner, K rows): 64-token x (8 << i)-row boxes for runs of consecutive columns
         const cuuint64_t gdim[2] = {(cuuint64_t)N, (cuuint64_t)P.lay.K};
         const cuuint64_t gstride[1] = {(cuuint64_t)ldx * 2};

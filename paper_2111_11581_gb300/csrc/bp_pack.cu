@@ -804,6 +804,201 @@ cudaError_t launch_slab_counts(const bp_layout &lay, const uint8_t *mask, int64_
     return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------- section 3
+// K-group q of a layer (list order: q = pos * C64 + c64, pos = i * kw + j):
+// does any row of slab s keep any of its 64 columns?  (The first row of each
+// row-block the slab touches decides: rows of a row-block are identical.)
+__device__ __forceinline__ bool kg_listed(const uint8_t *__restrict__ mask, int64_t M, int64_t K,
+                                          int64_t bm, int khw, int64_t C, int64_t C64, int64_t s,
+                                          int64_t q) {
+    const int64_t pos = q / C64, c64 = q - pos * C64;
+    const int64_t r0 = s * kSlab, r1 = min(r0 + kSlab, M);
+    const int64_t ce = min(C, 64 * c64 + 64);
+    for (int64_t rb = r0 / bm; rb * bm < r1; ++rb) {
+        const uint8_t *row = mask + rb * bm * K;
+        for (int64_t c = 64 * c64; c < ce; ++c)
+            if (row[c * khw + pos]) return true;
+    }
+    return false;
+}
+
+// One block per slab: its chunk count (listed K-groups).
+__global__ void kg_counts_kernel(int64_t M, int64_t K, int64_t bm, int khw, int64_t C,
+                                 int64_t C64, const uint8_t *__restrict__ mask,
+                                 int64_t *__restrict__ counts) {
+    const int64_t s = blockIdx.x, KG = C64 * khw;
+    int n = 0;
+    for (int64_t q = threadIdx.x; q < KG; q += blockDim.x)
+        n += kg_listed(mask, M, K, bm, khw, C, C64, s, q) ? 1 : 0;
+    __shared__ int tot;
+    if (threadIdx.x == 0) tot = 0;
+    __syncthreads();
+    atomicAdd(&tot, n);
+    __syncthreads();
+    if (threadIdx.x == 0) counts[s] = tot;
+}
+
+// One block (256 threads) per slab: the records of its chunks, the listed
+// K-groups in list order (block-wide ordered compaction).
+__global__ void __launch_bounds__(256) kg_lists_kernel(int64_t M, int64_t K, int64_t bm, int khw,
+                                                       int kw, int64_t C, int64_t C64,
+                                                       const uint8_t *__restrict__ mask,
+                                                       const int64_t *__restrict__ kc3,
+                                                       uint8_t *__restrict__ meta3) {
+    const int64_t s = blockIdx.x, KG = C64 * khw;
+    const int64_t c0 = kc3[s];
+    if (kc3[s + 1] == c0) return;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    __shared__ int wsum[8];
+    int64_t running = 0;
+    for (int64_t q0 = 0; q0 < KG; q0 += 256) {
+        const int64_t q = q0 + threadIdx.x;
+        const bool f = q < KG && kg_listed(mask, M, K, bm, khw, C, C64, s, q);
+        const unsigned b = __ballot_sync(0xffffffffu, f);
+        if (lane == 0) wsum[warp] = __popc(b);
+        __syncthreads();
+        int before = 0, total = 0;
+        for (int w = 0; w < 8; ++w) {
+            if (w < warp) before += wsum[w];
+            total += wsum[w];
+        }
+        if (f) {
+            const int64_t pos = q / C64, c64 = q - pos * C64;
+            const int64_t e = running + before + __popc(b & ((1u << lane) - 1u));
+            int32_t *r = reinterpret_cast<int32_t *>(meta3 + (c0 + e) * kMetaBytes);
+            r[0] = (int32_t)((c64 << 16) | ((pos / kw) << 8) | (pos % kw));
+            r[kListBytes / 4] = 1;
+        }
+        running += total;
+        __syncthreads();
+    }
+}
+
+// One thread per 16-byte unit (row, 8 channels) of a chunk's weight tile.
+__global__ void kg_tiles_kernel(int64_t M, int64_t K, int khw, int kw, int64_t C,
+                                const uint16_t *__restrict__ W, const uint8_t *__restrict__ mask,
+                                const int64_t *__restrict__ kc3, uint8_t *__restrict__ tiles3,
+                                const uint8_t *__restrict__ meta3) {
+    const int64_t s = blockIdx.y;
+    const int64_t c0 = kc3[s], nkc = kc3[s + 1] - c0;
+    const int64_t units = nkc * kSlab * 8;
+    for (int64_t u = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; u < units;
+         u += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t kc = u / (kSlab * 8);
+        const int64_t rem = u - kc * (kSlab * 8);
+        const uint32_t row = (uint32_t)(rem >> 3), ch = (uint32_t)(rem & 7);
+        const int32_t d = reinterpret_cast<const int32_t *>(meta3 + (c0 + kc) * kMetaBytes)[0];
+        const int64_t c64 = d >> 16, pos = ((d >> 8) & 0xff) * kw + (d & 0xff);
+        const int64_t r = s * kSlab + row;
+        uint16_t v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int64_t c = 64 * c64 + 8 * ch + e;
+            const int64_t k = c * khw + pos;
+            v[e] = (r < M && c < C && mask[r * K + k]) ? W[r * K + k] : (uint16_t)0;
+        }
+        uint4 pk;
+        pk.x = v[0] | ((uint32_t)v[1] << 16);
+        pk.y = v[2] | ((uint32_t)v[3] << 16);
+        pk.z = v[4] | ((uint32_t)v[5] << 16);
+        pk.w = v[6] | ((uint32_t)v[7] << 16);
+        *reinterpret_cast<uint4 *>(tiles3 + (c0 + kc) * (int64_t)(kSlab * kBK * 2) +
+                                   sw128_kmajor_offset(row, ch * 8)) = pk;
+    }
+}
+
+// NCHW -> NHWC with channels padded to a multiple of 8 (zeros): one block per
+// (image, 64 consecutive pixels, 64 channels).  Each channel's 64 pixels are
+// 128 contiguous bytes of the input, each pixel's 64 channels 128 contiguous
+// bytes of the output; the transposition goes through shared memory.
+__global__ void __launch_bounds__(256) nhwc8_kernel(ConvShape cs, const uint16_t *__restrict__ in,
+                                                    uint16_t *__restrict__ out) {
+    const int64_t HW = cs.H * cs.W, C8 = (cs.C + 7) / 8 * 8;
+    const int64_t b = blockIdx.z, p0 = (int64_t)blockIdx.x * 64, c0 = (int64_t)blockIdx.y * 64;
+    __shared__ uint16_t tile[64][66];           // [channel][pixel] (+2 against bank conflicts)
+    const int np = (int)min((int64_t)64, HW - p0), nc = (int)min((int64_t)64, C8 - c0);
+    const bool vec = HW % 8 == 0;               // channel planes start 16-byte aligned
+    // 64 channels x 64 pixels, 8 pixels per thread and pass
+    for (int e = threadIdx.x; e < 64 * 8; e += blockDim.x) {
+        const int cc = e >> 3, q = (e & 7) * 8;
+        const int64_t c = c0 + cc;
+        uint16_t v[8];
+        if (c < cs.C && q < np) {
+            const uint16_t *src = in + (b * cs.C + c) * HW + p0 + q;
+            if (vec && q + 8 <= np) {
+                const uint4 w = *reinterpret_cast<const uint4 *>(src);
+                v[0] = (uint16_t)w.x; v[1] = (uint16_t)(w.x >> 16);
+                v[2] = (uint16_t)w.y; v[3] = (uint16_t)(w.y >> 16);
+                v[4] = (uint16_t)w.z; v[5] = (uint16_t)(w.z >> 16);
+                v[6] = (uint16_t)w.w; v[7] = (uint16_t)(w.w >> 16);
+            } else {
+#pragma unroll
+                for (int u = 0; u < 8; ++u) v[u] = q + u < np ? src[u] : (uint16_t)0;
+            }
+        } else {
+#pragma unroll
+            for (int u = 0; u < 8; ++u) v[u] = 0;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) tile[cc][q + u] = v[u];
+    }
+    __syncthreads();
+    // each pixel's channels c0 .. c0 + nc - 1, 8 per 16-byte store
+    const int ng = nc / 8;
+    for (int e = threadIdx.x; e < np * ng; e += blockDim.x) {
+        const int px = e / ng, g = e - px * ng;
+        uint16_t v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[u] = tile[g * 8 + u][px];
+        uint4 pk;
+        pk.x = v[0] | ((uint32_t)v[1] << 16);
+        pk.y = v[2] | ((uint32_t)v[3] << 16);
+        pk.z = v[4] | ((uint32_t)v[5] << 16);
+        pk.w = v[6] | ((uint32_t)v[7] << 16);
+        *reinterpret_cast<uint4 *>(out + (b * HW + p0 + px) * C8 + c0 + g * 8) = pk;
+    }
+}
+
+cudaError_t launch_pack_sec3(const bp_layout &lay, const void *W, const uint8_t *mask,
+                             const bp_packed &P, const DevLayout &dl, int64_t *scratch,
+                             cudaStream_t s) {
+    if (dl.c3max == 0) return cudaSuccess;
+    const int khw = lay.kh * lay.kw;
+    const int64_t C = lay.K / khw, C64 = (C + 63) / 64;
+    const int64_t S = dl.num_slabs;
+    uint8_t *dev = static_cast<uint8_t *>(P.dev);
+    int64_t *kc3 = reinterpret_cast<int64_t *>(dev + dl.off_sec3);
+    cudaError_t e = cudaMemsetAsync(scratch, 0, 8 * (S + 1), s);
+    if (e != cudaSuccess) return e;
+    kg_counts_kernel<<<(unsigned)S, 256, 0, s>>>(lay.M, lay.K, lay.bm, khw, C, C64, mask, scratch);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    exclusive_scan_kernel<<<1, kScanThreads, 0, s>>>(S + 1, scratch);
+    e = cudaGetLastError();
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(kc3, scratch, 8 * (S + 1), cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return e;
+    uint8_t *meta3 = dev + dl.off_meta3;
+    kg_lists_kernel<<<(unsigned)S, 256, 0, s>>>(lay.M, lay.K, lay.bm, khw, lay.kw, C, C64, mask,
+                                                 kc3, meta3);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    dim3 grid(16, (unsigned)S);
+    kg_tiles_kernel<<<grid, 256, 0, s>>>(lay.M, lay.K, khw, lay.kw, C,
+                                         static_cast<const uint16_t *>(W), mask, kc3,
+                                         dev + dl.off_tiles3, meta3);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_nhwc8(const ConvShape &cs, const void *in, void *out, cudaStream_t s) {
+    const int64_t HW = cs.H * cs.W, C8 = (cs.C + 7) / 8 * 8;
+    if (cs.Nb * HW == 0) return cudaSuccess;
+    const dim3 grid((unsigned)((HW + 63) / 64), (unsigned)((C8 + 63) / 64), (unsigned)cs.Nb);
+    nhwc8_kernel<<<grid, 256, 0, s>>>(cs, static_cast<const uint16_t *>(in),
+                                      static_cast<uint16_t *>(out));
+    return cudaGetLastError();
+}
+
 cudaError_t launch_pack(const bp_layout &lay, const void *W, const uint8_t *mask,
                         const bp_packed &P, const DevLayout &dl, cudaStream_t s) {
     const int64_t RB = P.num_rb;

@@ -125,7 +125,11 @@ def test_gemm_argument_checks_on_host(lib):
 
 def test_conv_argument_checks_on_host(lib):
     lay = bp.layout(bp.BLOCK_PUNCHED, bp.F16, 16, 8 * 9, 8, 4, 3, 3)
-    P = bp.Packed(lay, 2, 0, 0, 16, 16, 16, 256, 256 + 16384 + 640 + 4 * 72)   # kc_ptr, one chunk, qmap
+    # kc_ptr, one chunk, qmap; then (256-byte aligned) the implicit convolution's
+    # section, sized for all 9 K-groups (64 channels at each of 9 positions)
+    head = 256 + 16384 + 640 + 4 * 72
+    sec3 = 256 + 9 * (16384 + 320)
+    P = bp.Packed(lay, 2, 0, 0, 16, 16, 16, 256, (head + 255) // 256 * 256 + sec3)
     # C*kh*kw != K, negative pad, zero stride
     ws = 1 << 16
     assert bp.bp_conv2d(P, 256, 2, 7, 8, 8, 1, 1, 1, 1, None, 0, 256, ws, 1 << 20, 0) == \
@@ -134,12 +138,16 @@ def test_conv_argument_checks_on_host(lib):
         bp.ERR_INVALID_ARG
     assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, 1, 1, 0, 1, None, 0, 256, ws, 1 << 20, 0) == \
         bp.ERR_INVALID_ARG
-    # the im2col workspace: K x roundup8(Nb*Ho*Wo) 16-bit values = 72 x 128 x 2 bytes
-    assert bp.bp_conv2d_workspace_size(P, 2, 8, 8, 8, 1, 1, 1, 1) == (bp.OK, 72 * 128 * 2)
+    # stride 1: the implicit convolution's workspace, the input in NHWC with the
+    # channels padded to 8: 2 x 8 x 8 x 8 16-bit values
+    assert bp.bp_conv2d_workspace_size(P, 2, 8, 8, 8, 1, 1, 1, 1) == (bp.OK, 2 * 8 * 8 * 8 * 2)
+    # strided: the im2col workspace, K x roundup8(Nb*Ho*Wo) 16-bit values
     assert bp.bp_conv2d_workspace_size(P, 3, 8, 7, 5, 0, 0, 2, 1) == (bp.OK, 72 * 32 * 2)
     assert bp.bp_conv2d_workspace_size(P, 2, 7, 8, 8, 1, 1, 1, 1)[0] == bp.ERR_INVALID_ARG
     # too small, missing or misaligned workspace
-    assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, 1, 1, 1, 1, None, 0, 256, ws, 72 * 128 * 2 - 1, 0) \
+    assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, 1, 1, 1, 1, None, 0, 256, ws, 2 * 8 * 8 * 8 * 2 - 1,
+                        0) == bp.ERR_WORKSPACE
+    assert bp.bp_conv2d(P, 256, 3, 8, 7, 5, 0, 0, 2, 1, None, 0, 256, ws, 72 * 32 * 2 - 1, 0) \
         == bp.ERR_WORKSPACE
     assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, 1, 1, 1, 1, None, 0, 256, None, 1 << 20, 0) == \
         bp.ERR_WORKSPACE

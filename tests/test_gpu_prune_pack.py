@@ -100,6 +100,45 @@ def _plan(l, bound=None):
     return w
 
 
+def _check_section3(img, off, pw, mask, W, M, K):
+    """The implicit convolution's section, from the mask and weights alone: per
+    slab, the K-groups (64 channels c64*64 .. at kernel position (i, j)) any row
+    keeps, listed position-major, one per chunk; records (c64 << 16 | i << 8 |
+    j, TMA word); weight tiles K-major 128-byte swizzled with column u =
+    channel 64 c64 + u (zero for channels past C and pruned weights)."""
+    kh, kw = pw.lay.kh, pw.lay.kw
+    khw = kh * kw
+    C = K // khw
+    C64 = -(-C // 64)
+    S = -(-M // 128)
+    cmax = S * C64 * khw
+    tiles = off + (8 * (S + 1) + 255) // 256 * 256
+    meta = tiles + cmax * 16384
+    assert img.size == meta + cmax * 320
+    kc3 = img[off: off + 8 * (S + 1)].view(np.int64)
+    assert kc3[0] == 0
+    offs = _sw128(np.arange(128)[:, None], np.arange(64)[None, :])
+    for s in range(S):
+        r0, r1 = 128 * s, min(128 * s + 128, M)
+        keep = mask[r0:r1].reshape(r1 - r0, C, khw)
+        groups = [(c64, pos // kw, pos % kw) for pos in range(khw) for c64 in range(C64)
+                  if keep[:, 64 * c64: 64 * c64 + 64, pos].any()]
+        assert kc3[s + 1] - kc3[s] == len(groups), (s, kc3[s + 1] - kc3[s], len(groups))
+        rows = np.arange(r0, r1)
+        for c, (c64, i, j) in enumerate(groups):
+            rec = img[meta + (kc3[s] + c) * 320: meta + (kc3[s] + c + 1) * 320].view(np.int32)
+            assert rec[0] == (c64 << 16) | (i << 8) | j and rec[64] == 1, (s, c)
+            tw = np.zeros((128, 64), np.uint16)
+            for u in range(64):
+                ch = 64 * c64 + u
+                if ch < C:
+                    k = ch * khw + i * kw + j
+                    tw[:r1 - r0, u] = np.where(mask[rows, k], W[rows, k], 0)
+            base = tiles + (kc3[s] + c) * 16384
+            dec = img[base: base + 16384].view(np.uint16)[offs // 2]
+            assert (dec == tw).all(), (s, c)
+
+
 def _check_device_image(pw, mask, W, M, K):
     """Decode the device image on the host, from the mask and weights alone:
     per 128-row slab, aligned 64-column blocks whose union of kept columns has
@@ -118,7 +157,12 @@ def _check_device_image(pw, mask, W, M, K):
     meta2_off = meta_off + C * 320
     qmap_off = meta2_off + C * 320
     assert kc_ptr[0] == 0
-    assert img.size == qmap_off + (4 * K + 15) // 16 * 16
+    end = qmap_off + (4 * K + 15) // 16 * 16
+    kh, kw = pw.lay.kh, pw.lay.kw
+    if kh * kw > 1:
+        _check_section3(img, (end + 255) // 256 * 256, pw, mask, W, M, K)
+    else:
+        assert img.size == end
     qmap = img[qmap_off: qmap_off + 4 * K].view(np.int32)
     offs = _sw128(np.arange(128)[:, None], np.arange(64)[None, :])
     listed = np.zeros(K, bool)
