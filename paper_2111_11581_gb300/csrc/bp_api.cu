@@ -512,6 +512,11 @@ bp_status bp_gemm(const bp_packed *P, const void *X, int64_t N, int64_t ldx, con
         return BP_ERR_WORKSPACE;
     if (N == 0) return BP_OK;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (small_path_ok(*P, N)) {
+        if ((P->nnz_cols > 0 && !P->col_idx) || (P->nnz_vals > 0 && !P->values) || !P->rb_ptr)
+            return BP_ERR_INVALID_ARG;
+        return finish_launch(launch_small(*P, X, N, ldx, bias, relu, Y, ldy, s), s);
+    }
     return finish_launch(launch_mma(*P, dl, X, N, ldx, bias, relu, Y, ldy, nullptr, ws, s), s);
 }
 

@@ -204,6 +204,12 @@ struct SplitPlan {
     int64_t total;      // balanced: chunks of all items
     size_t bytes;       // workspace: partial tiles + counters / flags (0 if none)
 };
+// Short path of bp_gemm (small layers with row-blocks of at most 64 rows): one
+// CTA per (row-block, 64 tokens) on the compact storage, CUDA-core fp32.
+bool small_path_ok(const bp_packed &P, int64_t N);
+cudaError_t launch_small(const bp_packed &P, const void *X, int64_t N, int64_t ldx,
+                         const float *bias, int relu, void *Y, int64_t ldy, cudaStream_t s);
+
 // it: the implicit convolution's tiles (nullptr: tiles of nt consecutive columns)
 SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split,
                      const ImplicitTiles *it = nullptr);
