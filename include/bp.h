@@ -8,7 +8,8 @@
  *                                                       Eq. punched, Sec. 5.1)
  *   bp_pack      dense weight + mask -> compact per-row-block storage (Sec. 4.3)
  *   bp_gemm      block-sparse GEMM  Y = (W o mask) X, fused bias/ReLU/cast
- *   bp_conv2d    block-sparse convolution (im2col + the same product), same epilogue
+ *   bp_conv2d    block-sparse convolution (implicit GEMM for stride-1 k x k layers,
+ *                im2col + the same product otherwise), same epilogue
  *
  * Conventions shared by every call:
  *   - All tensor pointers are DEVICE pointers allocated by the caller; the
@@ -84,8 +85,11 @@ typedef struct {
  *                      slabs of 128 rows, each with the union of its rows'
  *                      kept columns in chunks of 64 (pre-swizzled tiles, zero
  *                      weights where a row prunes a column), their index lists
- *                      and load plans; opaque to callers, its size fixed by
- *                      the layout and the mask (bp_pack_size). */
+ *                      and load plans, and for layers with kh * kw > 1 a
+ *                      second set of the slabs' tiles for the implicit
+ *                      convolution (chunks of 64 channels at one kernel
+ *                      position); opaque to callers, its size fixed by the
+ *                      layout and the mask (bp_pack_size). */
 typedef struct {
     bp_layout lay;
     int64_t num_rb;
@@ -191,10 +195,16 @@ bp_status bp_pack(const bp_layout *lay, const void *W, const uint8_t *mask, bp_p
  *         ready for the next call.  Calls that may overlap on the GPU need
  *         separate workspaces.
  * Any bm: weights are processed in slabs of 128 rows (see bp_packed::dev).
+ * Small layers with row-blocks of at most 32 rows (nnz_vals * N <= 2^24) take
+ * a short path instead: one CTA per (row-block, 32 tokens) on the compact
+ * arrays (rb_ptr, col_idx, values), fp32 accumulation on the CUDA cores; `ws`
+ * is not used there.
  * X must be finite: rows of X that a slab lists may meet zero weights of rows
  * that prune them (0 * Inf is NaN).  The launch is a programmatic dependent
  * of the previous kernel in `stream` (its set-up overlaps that kernel's end;
- * it reads and writes nothing before that kernel has completed). */
+ * it reads X and writes Y only after that kernel has completed; the short
+ * path reads the packed weights before, so they must not be written by that
+ * kernel -- bp_pack synchronises its stream). */
 bp_status bp_gemm(const bp_packed *P, const void *X, int64_t N, int64_t ldx, const float *bias,
                   int relu, void *Y, int64_t ldy, void *ws, size_t ws_bytes, void *stream);
 
@@ -210,10 +220,15 @@ bp_status bp_gemm_workspace_size(const bp_packed *P, int64_t N, size_t *bytes);
  *   in    device, Nb x C x H x W;   out  device, Nb x M x Ho x Wo with
  *   Ho = (H + 2 pad_h - kh) / stride_h + 1, Wo likewise.
  *   ws    device workspace of at least bp_conv2d_workspace_size() bytes
- *         (256-B aligned): the listed rows of the input expanded to the
- *         K x (Nb*Ho*Wo) matrix (im2col), which the block-sparse product then
- *         reads, and the partial sums of its split work (see bp_gemm: zero-fill
- *         a new workspace).
+ *         (256-B aligned), and the partial sums of the product's split work
+ *         (see bp_gemm: zero-fill a new workspace).  Stride-1 layers with
+ *         kh * kw > 1, W and Wo <= 256 (implicit GEMM): the input copied once
+ *         to NHWC with the channels padded to a multiple of 8; the product
+ *         loads, per k-chunk (64 channels at one kernel position), one TMA box
+ *         of those channels for its tile of output rows, shifted by the kernel
+ *         position, zeros outside the input being the padding.  Other layers:
+ *         the listed rows of the input expanded to the K x (Nb*Ho*Wo) matrix
+ *         (im2col), which the product then reads.
  * Requires C*kh*kw == lay.K; dilation and groups are not supported.  The
  * input must be finite (see bp_gemm).  BP_ERR_UNSUPPORTED when kh input
  * rows padded to W + 2 pad_w exceed 12288 values, when Wo > 4096, Nb > 65535
@@ -224,8 +239,9 @@ bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, i
                     void *stream);
 
 /* Device workspace bytes bp_conv2d needs for this packed weight and input
- * shape (host output): 2 * K * (Nb*Ho*Wo rounded up to 8), rounded up to 256,
- * plus the split product's share (bp_gemm_workspace_size for N = Nb*Ho*Wo). */
+ * shape (host output): the implicit GEMM's NHWC copy, 2 * Nb * H * W *
+ * (C rounded up to 8), or the im2col matrix, 2 * K * (Nb*Ho*Wo rounded up to
+ * 8), rounded up to 256; plus the split product's share. */
 bp_status bp_conv2d_workspace_size(const bp_packed *P, int64_t Nb, int64_t C, int64_t H,
                                    int64_t W, int pad_h, int pad_w, int stride_h, int stride_w,
                                    size_t *bytes);

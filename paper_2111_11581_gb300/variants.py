@@ -1,0 +1,209 @@
+"""Measurement builds of libbp: pipeline variants behind build switches, and the
+per-stage timeline of the tensor-core product.
+
+    python -m paper_2111_11581_gb300.variants time NAME:[DEFINE,...] ...
+        builds one library per NAME with the given -D switches (e.g.
+        `base: halves:BP_GATHER_HALVES balance:BP_BALANCE`) and times each on
+        the same workloads, every build in a process of its own:
+        4096^3 bf16 at 128 x 32 blocks, keep 1/4 (the benchmark's layer),
+        4096^3 at 8 x 64 blocks, keep 1/2 (whole 64-column blocks: TMA tile
+        loads instead of gathers) and BERT-base 3072 x 768 over 8192 tokens at
+        64 x 16 blocks, keep 1/8; four rotating activation sets, 400 launches.
+
+    python -m paper_2111_11581_gb300.variants probe
+        builds and runs probes/tc_rates.cu: tcgen05.mma 128 x N x 16 issued
+        back to back from one thread (cycles per instruction for N = 256, 128,
+        64, 16) and TMA bulk copies from 1, 2 and 4 threads per SM (bytes per
+        cycle an SM ingests).
+
+    python -m paper_2111_11581_gb300.variants trace [gemm|conv3x3]
+        builds with BP_TRACE and prints CTA 0's clock64 timeline of one launch
+        of the 4096^3 layer (or of the 3x3 CONV layer: N=128, C=F=128, 16x16):
+        per pipeline stage when the control thread and a gather group found it
+        free, when the gather was issued, when the tensor-core thread saw the
+        weight tile and the rows and committed; per window and item; and the
+        global-timer start and end of every CTA.
+
+The switches (all off in the library `build()` makes): BP_TRACE (timeline),
+BP_GATHER_HALVES (both gather groups on every chunk, one barrier per half),
+BP_BALANCE (whole-item waves, then equal chunk ranges per CTA with fp32
+partial tiles).  Builds go to _build/variants/NAME next to the library.
+"""
+from __future__ import annotations
+
+import concurrent.futures as cf
+import ctypes
+import os
+import subprocess
+import sys
+
+from . import build as B
+
+OUT = os.path.join(B.HERE, "_build", "variants")
+
+
+def build_variant(name: str, defines) -> str:
+    """libbp.so built with -D<define> for each define, into _build/variants/name."""
+    out = os.path.join(OUT, name)
+    os.makedirs(out, exist_ok=True)
+    cc = B.nvcc()
+    flags = B.ARCH + ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC",
+                      "-I" + os.path.join(B.ROOT, "include"), "--expt-relaxed-constexpr"]
+    flags += ["-D" + d for d in defines if d]
+
+    def one(src):
+        obj = os.path.join(out, os.path.basename(src) + ".o")
+        r = subprocess.run([cc, *flags, "-c", src, "-o", obj], capture_output=True, text=True)
+        if r.returncode:
+            raise RuntimeError(f"nvcc failed on {src}:\n{r.stderr}")
+        return obj
+
+    with cf.ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 1)) as ex:
+        objs = list(ex.map(one, B._sources()))
+    lib = os.path.join(out, "libbp.so")
+    subprocess.run([cc, *B.ARCH, "-shared", "-o", lib, *objs], check=True)
+    return lib
+
+
+TIME_CASES = [(4096, 4096, 4096, 128, 32, 4.0, "bf16"), (4096, 4096, 4096, 8, 64, 2.0, "bf16"),
+              (3072, 768, 8192, 64, 16, 8.0, "f16")]
+
+
+def _time_in_process(lib: str):
+    import torch
+
+    from . import bp, inputs
+    bp.load(lib)
+    res = []
+    for (M, K, N, bm, bk, rate, d) in TIME_CASES:
+        dt = bp.BF16 if d == "bf16" else bp.F16
+        L = inputs.gemm_point(M, K, N, bm, bk, rate, dt)
+        W = inputs.as_torch(inputs.layer_weight(L, dt), dt).cuda()
+        sets = [torch.empty((K, N), dtype=W.dtype, device="cuda").uniform_(-1, 1)
+                for _ in range(4)]
+        lay = bp.layout(bp.BLOCK_BASED, dt, M, K, bm, bk)
+        mask = bp.prune(lay, W, rate)
+        pw = bp.pack(lay, W, mask)
+        ws = bp.gemm_workspace(pw, N)
+        Ys = [bp.gemm(pw, X, ws=ws) for X in sets]
+        ref = (W.float() * mask.float()) @ sets[0].float()
+        ok = bool(((Ys[0].float() - ref).abs() <= 1e-2 * ref.abs().clamp_min(1)).all())
+        for i in range(20):
+            bp.gemm(pw, sets[i % 4], out=Ys[i % 4], ws=ws)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n = 400
+        e0.record()
+        for i in range(n):
+            bp.gemm(pw, sets[i % 4], out=Ys[i % 4], ws=ws)
+        e1.record()
+        torch.cuda.synchronize()
+        us = e0.elapsed_time(e1) * 1000 / n
+        res.append(f"{M}x{K}x{N} bm{bm} bk{bk} r{rate:g}: {us:.2f} us "
+                   f"{2.0 * int(mask.sum()) * N / us * 1e-6:.1f} TFLOP/s ok={ok}")
+    print(" | ".join(res), flush=True)
+
+
+def _trace_in_process(lib: str, workload: str):
+    import numpy as np
+    import torch
+
+    from . import bp, inputs
+    L_ = bp.load(lib)
+    L_.bp_debug_trace_read.restype = ctypes.c_int
+    L_.bp_debug_trace_read.argtypes = [ctypes.c_void_p, ctypes.c_int]
+    L_.bp_debug_trace_clear.restype = ctypes.c_int
+    if workload == "conv3x3":
+        L = inputs.conv3x3_128()
+        dt = bp.F16
+        W = inputs.as_torch(inputs.layer_weight(L, dt).reshape(L.M, -1), dt).cuda()
+        X = inputs.as_torch(inputs.layer_input(L, dt), dt).cuda()
+        lay = bp.layout(L.scheme, dt, L.M, L.K, L.bm, L.bk, L.kh, L.kw)
+        pw = bp.pack(lay, W, bp.prune(lay, W, L.rate))
+        ws = bp.conv2d_workspace(pw, X.shape, (1, 1), (1, 1))
+        Y = bp.conv2d(pw, X, pad=(1, 1), ws=ws)
+        run = lambda: bp.conv2d(pw, X, pad=(1, 1), out=Y, ws=ws)  # noqa: E731
+    else:
+        dt = bp.BF16
+        L = inputs.gemm_point(4096, 4096, 4096, 128, 32, 4.0, dt)
+        W = inputs.as_torch(inputs.layer_weight(L, dt), dt).cuda()
+        X = inputs.as_torch(inputs.layer_input(L, dt), dt).cuda()
+        lay = bp.layout(bp.BLOCK_BASED, dt, L.M, L.K, L.bm, L.bk)
+        pw = bp.pack(lay, W, bp.prune(lay, W, L.rate))
+        ws = bp.gemm_workspace(pw, L.N)
+        Y = bp.gemm(pw, X, ws=ws)
+        run = lambda: bp.gemm(pw, X, out=Y, ws=ws)  # noqa: E731
+    for _ in range(20):
+        run()
+    torch.cuda.synchronize()
+    L_.bp_debug_trace_clear()
+    run()
+    torch.cuda.synchronize()
+    n = 512 * 8
+    buf = (ctypes.c_ulonglong * n)()
+    assert L_.bp_debug_trace_read(buf, n) == n
+    t = np.frombuffer(buf, dtype=np.uint64).reshape(512, 8).astype(np.int64)
+    stages = t[:256]
+    valid = stages[:, 5] > 0
+    t0 = stages[valid][:, [0, 1, 3]].min()
+    rel = np.where(stages > 0, stages - t0, -1)[valid]
+    print("stage ctrl_free gath_free gath_iss mma_w mma_x commit  (clock64 cycles, CTA 0)")
+    for i, r in enumerate(rel):
+        print(f"{i:5d} {r[0]:9d} {r[1]:9d} {r[2]:8d} {r[3]:6d} {r[4]:6d} {r[5]:6d}")
+    c = rel[:, 5]
+    print(f"median commit interval {np.median(np.diff(c)):.0f} cycles")
+    g = rel[rel[:, 4] >= 0]
+    if len(g):
+        print(f"median gather issue -> tensor cores see the rows {np.median(g[:, 4] - g[:, 2]):.0f}")
+    ends = t.reshape(-1)[448 * 8: 448 * 8 + 2 * 256].reshape(256, 2)
+    ends = ends[ends[:, 1] > 0]
+    if len(ends):
+        s0 = ends[:, 0].min()
+        e = (ends[:, 1] - s0) / 1000.0
+        print(f"CTA end (us after the first start): min {e.min():.1f} median "
+              f"{np.median(e):.1f} max {e.max():.1f}")
+
+
+def main(argv):
+    if len(argv) >= 1 and argv[0] == "_time":
+        _time_in_process(argv[1])
+        return
+    if len(argv) >= 1 and argv[0] == "_trace":
+        _trace_in_process(argv[1], argv[2])
+        return
+    if argv and argv[0] == "probe":
+        src = os.path.join(B.HERE, "probes", "tc_rates.cu")
+        os.makedirs(OUT, exist_ok=True)
+        exe = os.path.join(OUT, "tc_rates")
+        subprocess.run([B.nvcc(), *B.ARCH, "-O3", "-std=c++17", "-I" + os.path.join(B.ROOT, "include"),
+                        src, "-o", exe, "-lcuda"], check=True)
+        rc = 0
+        for args in (["0", "512", "256"], ["0", "512", "128"], ["0", "512", "64"],
+                     ["0", "512", "16"], ["1", "512", "256", "1"], ["1", "512", "256", "2"],
+                     ["1", "512", "256", "4"]):
+            rc |= subprocess.run([exe, *args]).returncode
+        sys.exit(rc)
+    if not argv or argv[0] not in ("time", "trace"):
+        print(__doc__)
+        sys.exit(2)
+    if argv[0] == "time":
+        variants = []
+        for a in argv[1:]:
+            name, _, fl = a.partition(":")
+            variants.append((name, [f for f in fl.split(",") if f]))
+        libs = {n: build_variant(n, f) for n, f in variants}
+        for n, _ in variants:
+            r = subprocess.run([sys.executable, "-m", "paper_2111_11581_gb300.variants", "_time",
+                                libs[n]], capture_output=True, text=True, cwd=B.ROOT)
+            print(f"[{n}] {r.stdout.strip()} {r.stderr.strip()[-400:] if r.returncode else ''}",
+                  flush=True)
+    else:
+        wl = argv[1] if len(argv) > 1 else "gemm"
+        lib = build_variant("trace", ["BP_TRACE"])
+        r = subprocess.run([sys.executable, "-m", "paper_2111_11581_gb300.variants", "_trace", lib,
+                            wl], cwd=B.ROOT)
+        sys.exit(r.returncode)
+
+
+if __name__ == "__main__":
+    main(sys.argv[1:])
