@@ -50,11 +50,16 @@
 // after issuing the weight copy.  Per window w (entries 256 + w): 0 control
 // thread at the window, 1 after copying the next window, 2 saw this window, 3
 // gather warp 0 saw it; per item i (entries 384 + i): 4 MMA thread holds a
-// free accumulator.  Entries 448 .. hold the global-timer start and end of
-// each of the first 256 CTAs.
+// free accumulator, 5 the first epilogue warp saw the finished accumulator, 6
+// it issued the item's last store.  Entries 448 .. hold the global-timer start
+// and end of each of the first 248 CTAs; entry 511: CTA 0's clock64() after
+// the grid dependency wait (0) and at exit (1).  Per 32-column output group g
+// of the first epilogue warp (entries 512 + g): 4 group start, 0 converted, 1
+// its staging box free, 2 box written and fenced, 3 store issued, 5 the next
+// group's tensor-memory load landed.
 #ifdef BP_TRACE
 namespace bp {
-constexpr int kTraceChunks = 512;
+constexpr int kTraceChunks = 1024;
 constexpr int kTraceEvents = 8;
 __device__ unsigned long long g_trace[kTraceChunks * kTraceEvents];
 }  // namespace bp
@@ -114,6 +119,7 @@ struct Params {
     int relu;
     int conv;               // 1: Y is the NCHW output of a convolution
     int ytma;               // 1: output boxes are written with TMA stores through ymap
+    int yvec;               // convolution: Ho*Wo % 8 == 0 (BP_EPI_DIRECT: 8 pixels per 16-byte store)
     int64_t M, num_slabs;
     int64_t N;              // tokens (GEMM) or Nb*Ho*Wo pixels (conv)
     int nt;                 // activation columns per tile: a multiple of 32, 64 .. 256
@@ -808,6 +814,17 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
     uint32_t yseq = 0;                       // TMA box stores issued by this warp
     int acc = 0;
     uint32_t acc_phase = 0;
+#ifdef BP_TRACE
+    int64_t titem = 0, tgrp = 0;
+#define BP_TRE(ev)                                                 \
+    do {                                                           \
+        if (warp == kEpiWarp0 && lane == 0) BP_TR(512 + tgrp, ev); \
+    } while (0)
+#else
+#define BP_TRE(ev) \
+    do {           \
+    } while (0)
+#endif
     UnitIter ui;
     Item t;
     for (ui.init(p, s.skv); ui.valid(); ui.step(p, t)) {
@@ -822,6 +839,9 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             }
             tc_fence_after();
         }
+#ifdef BP_TRACE
+        if (warp == kEpiWarp0 && lane == 0) BP_TR(384 + titem, 5);
+#endif
         const uint32_t tacc = tmem + ((uint32_t)(32 * q) << 16) + acc * p.acc_cols;
         // lane = output row of the slab; tensor-memory columns = the tile's columns
         const int64_t row0 = 32 * q;
@@ -845,6 +865,57 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
         };
         auto store = [&](const uint32_t (&pk)[16], int c0) {
             const int64_t n = t.n0 + c0;
+#ifdef BP_EPI_DIRECT
+            // (Measurement build.)  The 32 x 32 box goes through shared memory
+            // (row = lane, 64 bytes; 16-byte chunk c of row r at c ^ ((r >> 1) &
+            // 3), conflict-free both ways) and back out row by row with plain
+            // stores: per instruction 8 rows x 64 contiguous bytes, lanes 4r ..
+            // 4r + 3 on row r; the box's buffer alternates over the warp's
+            // groups.  Measured slower than the TMA box stores below on every
+            // workload (the 4096^3 layer 43.6 against 41.9 us, BERT 3072 x 768
+            // 32.1 against 25.5 us): the stores share the load/store unit with
+            // the activation gathers.
+            if (!kConv || p.yvec) {
+                const uint32_t sb = stg + (yseq & 1u) * 2048;
+                ++yseq;
+#pragma unroll
+                for (int ch = 0; ch < 4; ++ch)
+                    st_shared_v4(sb + lane * 64 + ((ch ^ ((lane >> 1) & 3)) << 4),
+                                 make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2],
+                                            pk[4 * ch + 3]));
+                __syncwarp();
+                const int c = lane & 3;
+                const int64_t nc = n + 8 * c;          // this lane's 8 columns
+                const int64_t nend = kConv ? t.n0 + t.ncols : p.N;
+                uint16_t *dst0;
+                if (kConv) {
+                    // NCHW, Ho*Wo a multiple of 8 and nc too: the 8 pixels lie in one
+                    // image, 16-byte aligned
+                    const uint32_t bb = (uint32_t)nc / (uint32_t)p.HoWo;
+                    const uint32_t hw = (uint32_t)nc - bb * (uint32_t)p.HoWo;
+                    dst0 = p.Y + ((int64_t)bb * p.M + t.slab * kSlab + row0) * p.HoWo + hw;
+                } else {
+                    dst0 = p.Y + (t.slab * kSlab + row0) * p.ldy + nc;
+                }
+                const int64_t ystride = kConv ? p.HoWo : p.ldy;
+#pragma unroll
+                for (int it = 0; it < 4; ++it) {
+                    const int rr = it * 8 + (lane >> 2);
+                    const uint4 v = ld_shared_v4(sb + rr * 64 + ((c ^ ((rr >> 1) & 3)) << 4));
+                    if (row0 + rr < t.rows && nc < nend) {
+                        uint16_t *dst = dst0 + rr * ystride;
+                        if (nc + 8 <= nend) {
+                            *reinterpret_cast<uint4 *>(dst) = v;
+                        } else {
+                            const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+                            for (int u = 0; u < 8 && nc + u < nend; ++u)
+                                dst[u] = (uint16_t)(w[u >> 1] >> (16 * (u & 1)));
+                        }
+                    }
+                }
+                return;
+            }
+#endif
             if (kConv) {
                 // NCHW output, pixel n = b*HoWo + hw is element (b, m, hw)
                 const uint32_t bb = (uint32_t)n / (uint32_t)p.HoWo;
@@ -853,10 +924,12 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                     // the 32 pixels lie in one image and in the tile: stage the box
                     // like a GEMM box (below) and store it at (hw, m, b) of the
                     // 3-D output map (a TMA store needs hw 16-byte aligned)
+                    BP_TRE(0);
                     const uint32_t sb = stg + (yseq & 1u) * 2048;
                     ++yseq;
                     if (lane == 0) bulk_wait_read<1>();
                     __syncwarp();
+                    BP_TRE(1);
 #pragma unroll
                     for (int ch = 0; ch < 4; ++ch)
                         st_shared_v4(sb + lane * 64 + ((ch ^ ((lane >> 1) & 3)) << 4),
@@ -864,11 +937,13 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                                                 pk[4 * ch + 3]));
                     fence_proxy_async_smem();
                     __syncwarp();
+                    BP_TRE(2);
                     if (lane == 0) {
                         tma_store_3d(&p.ymap, sb, (int32_t)hw, (int32_t)(t.slab * kSlab + row0),
                                      (int32_t)bb);
                         bulk_commit();
                     }
+                    BP_TRE(3);
                     return;
                 }
                 // Ho*Wo not a multiple of 8, the 32 pixels cross an image
@@ -904,20 +979,24 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             // the two boxes alternate over the warp's stores, across items (an
             // item may have an odd number of groups): the box about to be written
             // was used by the store before last
+            BP_TRE(0);
             const uint32_t sb = stg + (yseq & 1u) * 2048;
             ++yseq;
             if (lane == 0) bulk_wait_read<1>();     // the store that used this box is done
             __syncwarp();
+            BP_TRE(1);
 #pragma unroll
             for (int ch = 0; ch < 4; ++ch)
                 st_shared_v4(sb + lane * 64 + ((ch ^ ((lane >> 1) & 3)) << 4),
                              make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]));
             fence_proxy_async_smem();
             __syncwarp();
+            BP_TRE(2);
             if (lane == 0) {
                 tma_store_2d(&p.ymap, sb, (int32_t)n, (int32_t)(t.slab * kSlab + row0));
                 bulk_commit();
             }
+            BP_TRE(3);
                 };
         if (row0 < t.rows) {
             const int64_t cols = t.ncols;
@@ -1011,10 +1090,15 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                     for (int64_t c = c0; c <= c1; ++c) p.cnt[c * 4 + q] = 0;
             } else if (!kSplit || t.S == 1) {
                 for (int g = 0; g < G; ++g) {
+                    BP_TRE(4);
                     pack(r, pk);
                     if (has && g + 1 < G) tmem_ld_32x32b_x32(tacc + 32 * (g + 1), r);
                     store(pk, 32 * g);
                     if (has && g + 1 < G) tmem_ld_wait();
+                    BP_TRE(5);
+#ifdef BP_TRACE
+                    ++tgrp;
+#endif
                 }
             } else {
                 // Split item: this unit's fp32 partial rows go to its slot; the
@@ -1082,8 +1166,13 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                 acc_phase ^= 1u;
             }
         }
+#ifdef BP_TRACE
+        if (warp == kEpiWarp0 && lane == 0) BP_TR(384 + titem, 6);
+        ++titem;
+#endif
     }
     if (p.ytma && lane == 0) bulk_wait_all();    // staged output fully written before exit
+#undef BP_TRE
 }
 
 // kSplit: the launch has split items (a separate instantiation keeps the
@@ -1126,7 +1215,8 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     grid_dependency_wait();
     grid_launch_dependents();
 #ifdef BP_TRACE
-    if (threadIdx.x == 0 && blockIdx.x < 256) g_trace[448 * kTraceEvents + 2 * blockIdx.x] = globaltimer_ns();
+    if (threadIdx.x == 0 && blockIdx.x < 248) g_trace[448 * kTraceEvents + 2 * blockIdx.x] = globaltimer_ns();
+    if (threadIdx.x == 0) BP_TR(511, 0);
 #endif
     if (s.kc)
         for (int64_t i = threadIdx.x; i < p.kc_cached; i += kThreads) s.kc[i] = p.kc_ptr[i];
@@ -1161,7 +1251,8 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     __syncthreads();
     tc_fence_after();
 #ifdef BP_TRACE
-    if (threadIdx.x == 0 && blockIdx.x < 256) g_trace[448 * kTraceEvents + 2 * blockIdx.x + 1] = globaltimer_ns();
+    if (threadIdx.x == 0 && blockIdx.x < 248) g_trace[448 * kTraceEvents + 2 * blockIdx.x + 1] = globaltimer_ns();
+    if (threadIdx.x == 0) BP_TR(511, 1);
 #endif
     if (warp == kMmaWarp) tmem_dealloc(tmem, p.tmem_cols);
 }
@@ -1392,6 +1483,8 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
     }
+    p.yvec = conv && p.HoWo % 8 == 0;
+#ifndef BP_EPI_DIRECT
     if (!conv) {
         // Y (N inner, M rows) for the epilogue's 32 x 32 box stores
         const cuuint64_t gdim[2] = {(cuuint64_t)N, (cuuint64_t)P.lay.M};
@@ -1417,6 +1510,7 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
             return cudaErrorInvalidValue;
         p.ytma = 1;
     }
+#endif
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [] {

@@ -6,17 +6,44 @@
 // the 128-row slab tiles and their gathered rows, each a dependent round trip
 // to memory.  Here one CTA computes one row-block of bm rows for 32 tokens
 // straight from the compact storage of Sec. 4.3 (values of the row-block,
-// bm x K' row-major, and its kept-column list): per 128 listed columns it
-// gathers those activation rows into shared memory (16-byte cp.async) and
-// loads the row-block's weights for them, all loads of a step in flight
-// together; the 8 warps split the columns, accumulate in fp32 on the CUDA
-// cores and meet in shared memory; bias, ReLU and the round-to-nearest-even
-// cast follow.  Only kept weights enter the product, row-block by row-block,
-// as in the paper's own per-row-block kernels.
+// bm x K' row-major, and its kept-column list), on the CUDA cores in fp32;
+// only kept weights enter the product, row-block by row-block, as in the
+// paper's own per-row-block kernels.  Bias, ReLU and the round-to-nearest-even
+// cast follow.
+//
+// Such a launch is a chain of memory round trips, so the kernel keeps the
+// chain short: the row-block's range, its column indices and weights are all
+// requested at once, the range guessed as rb x (K' of an even split) -- a
+// layer pruned at one rate keeps the same number of columns in every
+// row-block -- and checked when the row-block pointers arrive (a wrong guess
+// reloads); when K is at most kStageK the CTA's 32 tokens of every activation
+// row are copied to shared memory in the same round trip, without waiting for
+// the column indices, and the product indexes them there.  Longer rows are
+// gathered by column index, 128 listed columns per step.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
 #include "bp_common.cuh"
+
+// BP_TRACE (off by default; a build for measurement only): thread 0 of each
+// of the first 256 CTAs records clock64() at its start (0), once its loads
+// are issued (1), once the row-block range arrived (2), once the step's data
+// landed (3), after the product (4) and at its end (5), and the global timer
+// at its start (6) and end (7); read back with bp_debug_small_trace_read().
+#ifdef BP_TRACE
+namespace bp {
+__device__ unsigned long long g_small_trace[256 * 8];
+}  // namespace bp
+#define BP_TS(ev, v)                                                      \
+    do {                                                                  \
+        if (threadIdx.x == 0 && blockIdx.y == 0 && blockIdx.x < 256)      \
+            bp::g_small_trace[blockIdx.x * 8 + (ev)] = (v);               \
+    } while (0)
+#else
+#define BP_TS(ev, v) \
+    do {             \
+    } while (0)
+#endif
 
 namespace bp {
 namespace {
@@ -26,6 +53,11 @@ constexpr int kSmallWarps = kSmallThreads / 32;
 constexpr int kSmallTok = 32;      // tokens per CTA
 constexpr int kSmallK = 128;       // listed columns per step
 constexpr int kSmallMaxBm = 32;
+constexpr int64_t kStageK = 1024;  // activation rows staged whole up to this K (64 KB)
+// dynamic shared memory: weights of a step, the warps' sums, the step's column
+// indices, then the activation rows (all K of them, or the step's gathered ones)
+constexpr int kOffW = 0, kOffOut = kOffW + kSmallMaxBm * kSmallK * 2;
+constexpr int kOffIdx = kOffOut + kSmallMaxBm * kSmallTok * 4, kOffX = kOffIdx + kSmallK * 4;
 
 template <bool kBf16>
 __device__ __forceinline__ float to_f(uint32_t v) {
@@ -46,26 +78,45 @@ struct SmallParams {
     const uint16_t *X;
     uint16_t *Y;
     const float *bias;
-    int64_t M, N, ldx, ldy;
+    int64_t M, K, N, ldx, ldy;
+    int64_t kp_even;     // K' of every row-block if they all kept the same count, else -1
     int bm, relu;
 };
 
+// 16-byte copies of token columns n .. n+7 of activation row k (zero past N)
+__device__ __forceinline__ void copy_tokens(uint32_t dst, const SmallParams &p, int64_t k, int64_t n) {
+    uint32_t nb = 0;
+    const uint16_t *src = p.X;
+    if (n < p.N) {
+        nb = (uint32_t)min((int64_t)16, (p.N - n) * 2);
+        src = p.X + k * p.ldx + n;
+    }
+    cp_async_16(dst, src, nb);
+}
+
 // grid: (row-blocks, token tiles of 32).  Warp w takes the listed columns
 // i = w (mod 8) of each step; lane l: tokens 4 (l % 8) .. +3, rows l / 8 + 4 j.
-template <bool kBf16>
+template <bool kBf16, bool kStage>
 __global__ void __launch_bounds__(kSmallThreads) bp_small_kernel(const __grid_constant__ SmallParams p) {
-    __shared__ __align__(16) uint16_t xs[kSmallK][kSmallTok];      // gathered rows (8 KB)
-    __shared__ __align__(16) uint16_t wsm[kSmallMaxBm][kSmallK];   // weights of the step (8 KB)
-    __shared__ float out[kSmallMaxBm][kSmallTok];                   // the warps' sums
+    extern __shared__ __align__(16) uint8_t dsm[];
+    uint16_t (*wsm)[kSmallK] = reinterpret_cast<uint16_t (*)[kSmallK]>(dsm + kOffW);
+    float (*out)[kSmallTok] = reinterpret_cast<float (*)[kSmallTok]>(dsm + kOffOut);
+    int32_t *cis = reinterpret_cast<int32_t *>(dsm + kOffIdx);
+    uint16_t (*xs)[kSmallTok] = reinterpret_cast<uint16_t (*)[kSmallTok]>(dsm + kOffX);
     const int64_t rb = blockIdx.x, n0 = (int64_t)blockIdx.y * kSmallTok;
     const int64_t r0 = rb * p.bm;
     const int rows = (int)min((int64_t)p.bm, p.M - r0);
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
     const int tq = (lane & 7) * 4, rq = lane >> 3;
+    BP_TS(0, clock64());
+    BP_TS(6, globaltimer_ns());
     for (int e = t; e < kSmallMaxBm * kSmallTok; e += kSmallThreads) (&out[0][0])[e] = 0.f;
-    __syncthreads();
-    const int64_t c0 = p.rb_ptr[rb], kp = p.rb_ptr[rb + 1] - c0;    // K' of the row-block
-    const uint16_t *wrb = p.values + (int64_t)p.bm * c0;             // rows x K' row-major
+    // the row-block's range, requested now and used once the first step's
+    // loads (issued for the guessed range) are in flight
+    const int64_t ra = p.rb_ptr[rb], rz = p.rb_ptr[rb + 1];
+    int64_t c0 = p.kp_even >= 0 ? rb * p.kp_even : ra;
+    int64_t kp = p.kp_even >= 0 ? p.kp_even : rz - ra;
+    bool first = true;
     float acc[kSmallMaxBm / 4][4];
 #pragma unroll
     for (int j = 0; j < kSmallMaxBm / 4; ++j)
@@ -73,9 +124,10 @@ __global__ void __launch_bounds__(kSmallThreads) bp_small_kernel(const __grid_co
         for (int e = 0; e < 4; ++e) acc[j][e] = 0.f;
     for (int64_t k0 = 0; k0 < kp; k0 += kSmallK) {
         const int kn = (int)min((int64_t)kSmallK, kp - k0);
+        const uint16_t *wrb = p.values + (int64_t)p.bm * c0;             // rows x K' row-major
         // All loads of the step are issued before any is used (a loop that
         // consumes each load before issuing the next serialises the round
-        // trips): the column indices and the weights, then the gathered rows.
+        // trips): the column indices and the weights, then the rows.
         constexpr int kXU = kSmallK * (kSmallTok / 8) / kSmallThreads;     // 2 copies per thread
         constexpr int kWU = kSmallMaxBm * kSmallK / 8 / kSmallThreads;     // 2 per thread
         int32_t ci[kXU];
@@ -93,28 +145,43 @@ __global__ void __launch_bounds__(kSmallThreads) bp_small_kernel(const __grid_co
             for (int q = 0; q < 8; ++q)
                 wv[u][q] = (r < rows && i + q < kn) ? wrb[(int64_t)r * kp + k0 + i + q] : (uint16_t)0;
         }
-        // Launched as a programmatic dependent: the packed weights (written by
-        // bp_pack, which synchronises) are read above while the previous
-        // kernel may still run; the activations may come from that kernel, so
-        // the first gather waits for it.
-        if (k0 == 0) {
+        if (first) {
+            first = false;
+            // Launched as a programmatic dependent: the packed weights (written
+            // by bp_pack, which synchronises) are read above while the previous
+            // kernel may still run; the activations may come from that kernel,
+            // so they are read after it.
             grid_dependency_wait();
             grid_launch_dependents();
-        }
-#pragma unroll
-        for (int u = 0; u < kXU; ++u) {
-            const int e = t + kSmallThreads * u;
-            const int i = e >> 2, q = (e & 3) * 8;
-            const int64_t n = n0 + q;
-            uint32_t nb = 0;
-            const uint16_t *src = p.X;
-            if (i < kn && n < p.N) {
-                nb = (uint32_t)min((int64_t)16, (p.N - n) * 2);
-                src = p.X + (int64_t)ci[u] * p.ldx + n;
+            if (kStage) {
+                for (int e = t; e < (int)p.K * (kSmallTok / 8); e += kSmallThreads)
+                    copy_tokens(smem_u32(&xs[e >> 2][(e & 3) * 8]), p, e >> 2, n0 + (e & 3) * 8);
+                cp_async_commit();
             }
-            cp_async_16(smem_u32(&xs[i][q]), src, nb);
+            BP_TS(1, clock64());
+            if (c0 != ra || kp != rz - ra) {
+                // the row-blocks keep different counts: start over on the real range
+                c0 = ra;
+                kp = rz - ra;
+                k0 = -kSmallK;
+                continue;
+            }
         }
-        cp_async_commit();
+        if (kStage) {
+            // the step's column indices, from the copies already in registers
+#pragma unroll
+            for (int u = 0; u < kXU; ++u)
+                if ((t & 3) == 0) cis[(t + kSmallThreads * u) >> 2] = ci[u];
+        } else {
+#pragma unroll
+            for (int u = 0; u < kXU; ++u) {
+                const int e = t + kSmallThreads * u;
+                const int i = e >> 2, q = (e & 3) * 8;
+                if (i < kn) copy_tokens(smem_u32(&xs[i][q]), p, ci[u], n0 + q);
+                else cp_async_16(smem_u32(&xs[i][q]), p.X, 0u);
+            }
+            cp_async_commit();
+        }
 #pragma unroll
         for (int u = 0; u < kWU; ++u) {
             const int e = t + kSmallThreads * u, r = e / (kSmallK / 8), i = (e % (kSmallK / 8)) * 8;
@@ -125,27 +192,34 @@ __global__ void __launch_bounds__(kSmallThreads) bp_small_kernel(const __grid_co
             pk.w = wv[u][6] | ((uint32_t)wv[u][7] << 16);
             *reinterpret_cast<uint4 *>(&wsm[r][i]) = pk;
         }
+        BP_TS(2, clock64());
         cp_async_wait_all();
         __syncthreads();
+        BP_TS(3, clock64());
         for (int i = warp; i < kn; i += kSmallWarps) {
-            const uint2 xv = *reinterpret_cast<const uint2 *>(&xs[i][tq]);
+            const int xr = kStage ? cis[i] : i;
+            const uint2 xv = *reinterpret_cast<const uint2 *>(&xs[xr][tq]);
             const float x0 = to_f<kBf16>(xv.x & 0xffffu), x1 = to_f<kBf16>(xv.x >> 16);
             const float x2 = to_f<kBf16>(xv.y & 0xffffu), x3 = to_f<kBf16>(xv.y >> 16);
 #pragma unroll
             for (int j = 0; j < kSmallMaxBm / 4; ++j) {
-                const float w = to_f<kBf16>(wsm[rq + 4 * j][i]);
-                acc[j][0] = fmaf(w, x0, acc[j][0]);
-                acc[j][1] = fmaf(w, x1, acc[j][1]);
-                acc[j][2] = fmaf(w, x2, acc[j][2]);
-                acc[j][3] = fmaf(w, x3, acc[j][3]);
+                if (rq + 4 * j < rows) {
+                    const float w = to_f<kBf16>(wsm[rq + 4 * j][i]);
+                    acc[j][0] = fmaf(w, x0, acc[j][0]);
+                    acc[j][1] = fmaf(w, x1, acc[j][1]);
+                    acc[j][2] = fmaf(w, x2, acc[j][2]);
+                    acc[j][3] = fmaf(w, x3, acc[j][3]);
+                }
             }
         }
         __syncthreads();
     }
-    if (kp == 0) {              // nothing listed: the output is the bias alone
+    if (first) {                // nothing listed: the output is the bias alone
         grid_dependency_wait();
         grid_launch_dependents();
     }
+    cp_async_wait_all();        // staged rows that no step read
+    BP_TS(4, clock64());
     // the warps' partial sums meet in shared memory
 #pragma unroll
     for (int j = 0; j < kSmallMaxBm / 4; ++j)
@@ -175,6 +249,8 @@ __global__ void __launch_bounds__(kSmallThreads) bp_small_kernel(const __grid_co
             for (int u = 0; u < 4 && n + u < p.N; ++u) dst[u] = o[u];
         }
     }
+    BP_TS(5, clock64());
+    BP_TS(7, globaltimer_ns());
 }
 
 }  // namespace
@@ -197,22 +273,52 @@ cudaError_t launch_small(const bp_packed &P, const void *X, int64_t N, int64_t l
     p.Y = static_cast<uint16_t *>(Y);
     p.bias = bias;
     p.M = P.lay.M;
+    p.K = P.lay.K;
     p.N = N;
     p.ldx = ldx;
     p.ldy = ldy;
     p.bm = P.lay.bm;
     p.relu = relu;
+    // values hold bm x K' per row-block: an even split of the total is the
+    // guess every row-block checks against its own range
+    const int64_t per_rb = (int64_t)P.lay.bm * P.num_rb;
+    p.kp_even = (per_rb > 0 && P.nnz_vals % per_rb == 0) ? P.nnz_vals / per_rb : -1;
+    const bool stage = P.lay.K <= kStageK;
+    const int smem = kOffX + (int)(stage ? P.lay.K : kSmallK) * kSmallTok * 2;
+    const bool bf16 = P.lay.dtype == BP_BF16;
+    const void *fn = stage ? (bf16 ? (const void *)bp_small_kernel<true, true> : (const void *)bp_small_kernel<false, true>)
+                           : (bf16 ? (const void *)bp_small_kernel<true, false> : (const void *)bp_small_kernel<false, false>);
+    // the staging kernels may take more than 48 KB of dynamic shared memory;
+    // allowed once per process (for the largest K staged)
+    static const cudaError_t raised = [] {
+        const int most = kOffX + (int)kStageK * kSmallTok * 2;
+        cudaError_t e = cudaFuncSetAttribute(bp_small_kernel<true, true>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(bp_small_kernel<false, true>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+        return e;
+    }();
+    if (stage && raised != cudaSuccess) return raised;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)P.num_rb, (unsigned)((N + kSmallTok - 1) / kSmallTok));
     cfg.blockDim = dim3(kSmallThreads);
+    cfg.dynamicSmemBytes = (size_t)smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return P.lay.dtype == BP_BF16 ? cudaLaunchKernelEx(&cfg, bp_small_kernel<true>, p)
-                                  : cudaLaunchKernelEx(&cfg, bp_small_kernel<false>, p);
+    void *args[] = {&p};
+    return cudaLaunchKernelExC(&cfg, fn, args);
 }
 
 }  // namespace bp
+
+#ifdef BP_TRACE
+extern "C" int bp_debug_small_trace_read(unsigned long long *host, int n) {
+    if (n > 256 * 8) n = 256 * 8;
+    return cudaMemcpyFromSymbol(host, bp::g_small_trace, n * sizeof(unsigned long long)) == cudaSuccess ? n : -1;
+}
+#endif

@@ -16,12 +16,14 @@ per-stage timeline of the tensor-core product.
         64, 16) and TMA bulk copies from 1, 2 and 4 threads per SM (bytes per
         cycle an SM ingests).
 
-    python -m paper_2111_11581_gb300.variants trace [gemm|conv3x3]
-        builds with BP_TRACE and prints CTA 0's clock64 timeline of one launch
-        of the 4096^3 layer (or of the 3x3 CONV layer: N=128, C=F=128, 16x16):
-        per pipeline stage when the control thread and a gather group found it
-        free, when the gather was issued, when the tensor-core thread saw the
-        weight tile and the rows and committed; per window and item; and the
+    python -m paper_2111_11581_gb300.variants trace [gemm|conv3x3|resnet50:LAYER|fc512]
+        builds with BP_TRACE and prints CTA 0's clock64 timeline of one launch,
+        L2 flushed before it, of the 4096^3 layer (or of the 3x3 CONV layer: N=128, C=F=128, 16x16,
+        or of one ResNet-50 layer by name): per pipeline stage when the control
+        thread and a gather group found it free, when the gather was issued,
+        when the tensor-core thread saw the weight tile and the rows and
+        committed; per item when the tensor-core thread had a free accumulator
+        and when the epilogue saw it finished and had stored it; and the
         global-timer start and end of every CTA.
 
 The switches (all off in the library `build()` makes): BP_TRACE (timeline),
@@ -113,16 +115,28 @@ def _trace_in_process(lib: str, workload: str):
     L_.bp_debug_trace_read.restype = ctypes.c_int
     L_.bp_debug_trace_read.argtypes = [ctypes.c_void_p, ctypes.c_int]
     L_.bp_debug_trace_clear.restype = ctypes.c_int
-    if workload == "conv3x3":
-        L = inputs.conv3x3_128()
-        dt = bp.F16
+    if workload == "fc512":
+        L, dt = inputs.fc512(), bp.F16
+        W = inputs.as_torch(inputs.layer_weight(L, dt), dt).cuda()
+        X = inputs.as_torch(inputs.layer_input(L, dt), dt).cuda()
+        lay = bp.layout(bp.BLOCK_BASED, dt, L.M, L.K, L.bm, L.bk)
+        pw = bp.pack(lay, W, bp.prune(lay, W, L.rate))
+        Y = bp.gemm(pw, X)
+        run = lambda: bp.gemm(pw, X, out=Y)  # noqa: E731
+    elif workload == "conv3x3" or workload.startswith("resnet50:"):
+        if workload == "conv3x3":
+            L, dt = inputs.conv3x3_128(), bp.F16
+        else:
+            name = workload.split(":", 1)[1]
+            L, dt = [l for l in inputs.resnet50_imagenet() if l.name == name][0], bp.BF16
         W = inputs.as_torch(inputs.layer_weight(L, dt).reshape(L.M, -1), dt).cuda()
         X = inputs.as_torch(inputs.layer_input(L, dt), dt).cuda()
         lay = bp.layout(L.scheme, dt, L.M, L.K, L.bm, L.bk, L.kh, L.kw)
         pw = bp.pack(lay, W, bp.prune(lay, W, L.rate))
-        ws = bp.conv2d_workspace(pw, X.shape, (1, 1), (1, 1))
-        Y = bp.conv2d(pw, X, pad=(1, 1), ws=ws)
-        run = lambda: bp.conv2d(pw, X, pad=(1, 1), out=Y, ws=ws)  # noqa: E731
+        pad, st = (L.pad, L.pad), (L.stride, L.stride)
+        ws = bp.conv2d_workspace(pw, X.shape, pad, st)
+        Y = bp.conv2d(pw, X, pad=pad, stride=st, ws=ws)
+        run = lambda: bp.conv2d(pw, X, pad=pad, stride=st, out=Y, ws=ws)  # noqa: E731
     else:
         dt = bp.BF16
         L = inputs.gemm_point(4096, 4096, 4096, 128, 32, 4.0, dt)
@@ -136,26 +150,69 @@ def _trace_in_process(lib: str, workload: str):
     for _ in range(20):
         run()
     torch.cuda.synchronize()
+    # as the workload benchmark times a launch: L2 flushed (a 256 MiB write,
+    # read back) just before it
+    flush = torch.empty(256 * 2 ** 20 // 4, dtype=torch.float32, device="cuda")
+    flush.zero_()
+    flush.sum()
+    torch.cuda.synchronize()
     L_.bp_debug_trace_clear()
+    flush.zero_()
+    flush.sum()
     run()
     torch.cuda.synchronize()
-    n = 512 * 8
+    if workload == "fc512":
+        # the short CUDA-core path: per CTA clock64 at its start, loads issued,
+        # row-block range arrived, data landed, product done, end
+        L_.bp_debug_small_trace_read.restype = ctypes.c_int
+        L_.bp_debug_small_trace_read.argtypes = [ctypes.c_void_p, ctypes.c_int]
+        sb = (ctypes.c_ulonglong * (256 * 8))()
+        assert L_.bp_debug_small_trace_read(sb, 256 * 8) == 256 * 8
+        st = np.frombuffer(sb, dtype=np.uint64).reshape(256, 8).astype(np.int64)
+        st = st[st[:, 5] > 0]
+        d = np.diff(st[:, :6], axis=1)
+        print(f"short path, {len(st)} CTAs: median cycles issue {np.median(d[:, 0]):.0f}, "
+              f"range {np.median(d[:, 1]):.0f}, data {np.median(d[:, 2]):.0f}, product "
+              f"{np.median(d[:, 3]):.0f}, epilogue {np.median(d[:, 4]):.0f}; total "
+              f"{np.median(st[:, 5] - st[:, 0]):.0f}")
+        g0 = st[:, 6].min()
+        print(f"global timer (us after the first CTA start): starts {(st[:, 6] - g0).min() / 1e3:.2f}"
+              f"..{(st[:, 6] - g0).max() / 1e3:.2f}, ends {(st[:, 7] - g0).min() / 1e3:.2f}.."
+              f"{(st[:, 7] - g0).max() / 1e3:.2f}")
+        return
+    n = 1024 * 8
     buf = (ctypes.c_ulonglong * n)()
     assert L_.bp_debug_trace_read(buf, n) == n
-    t = np.frombuffer(buf, dtype=np.uint64).reshape(512, 8).astype(np.int64)
+    t = np.frombuffer(buf, dtype=np.uint64).reshape(1024, 8).astype(np.int64)
     stages = t[:256]
     valid = stages[:, 5] > 0
-    t0 = stages[valid][:, [0, 1, 3]].min()
+    # cycles after CTA 0 passed the grid dependency wait
+    t0 = t[511, 0]
     rel = np.where(stages > 0, stages - t0, -1)[valid]
-    print("stage ctrl_free gath_free gath_iss mma_w mma_x commit  (clock64 cycles, CTA 0)")
+    print("stage ctrl_free gath_free gath_iss mma_w mma_x commit  (clock64 cycles after CTA 0's start)")
     for i, r in enumerate(rel):
         print(f"{i:5d} {r[0]:9d} {r[1]:9d} {r[2]:8d} {r[3]:6d} {r[4]:6d} {r[5]:6d}")
     c = rel[:, 5]
-    print(f"median commit interval {np.median(np.diff(c)):.0f} cycles")
+    if len(c) > 1:
+        print(f"median commit interval {np.median(np.diff(c)):.0f} cycles")
+    items = t[384:448]
+    iv = items[:, 6] > 0
+    print("item acc_free epi_saw epi_done")
+    for i, r in enumerate(items[iv]):
+        print(f"{i:4d} {r[4] - t0:8d} {r[5] - t0:7d} {r[6] - t0:8d}")
+    print(f"CTA 0 exit {t[511, 1] - t0} cycles after its start")
+    grp = t[512:1024]
+    gv = (grp[:, 4] > 0) & (grp[:, 5] > 0) & (grp[:, 3] > 0)
+    if gv.any():
+        g = grp[gv]
+        print(f"epilogue groups of warp 0 (32 columns each): {int(gv.sum())}; median cycles: "
+              f"convert {np.median(g[:, 0] - g[:, 4]):.0f}, box free {np.median(g[:, 1] - g[:, 0]):.0f}, "
+              f"write+fence {np.median(g[:, 2] - g[:, 1]):.0f}, store issue {np.median(g[:, 3] - g[:, 2]):.0f}, "
+              f"next load wait {np.median(g[:, 5] - g[:, 3]):.0f}, group {np.median(g[:, 5] - g[:, 4]):.0f}")
     g = rel[rel[:, 4] >= 0]
     if len(g):
         print(f"median gather issue -> tensor cores see the rows {np.median(g[:, 4] - g[:, 2]):.0f}")
-    ends = t.reshape(-1)[448 * 8: 448 * 8 + 2 * 256].reshape(256, 2)
+    ends = t.reshape(-1)[448 * 8: 448 * 8 + 2 * 248].reshape(248, 2)
     ends = ends[ends[:, 1] > 0]
     if len(ends):
         s0 = ends[:, 0].min()

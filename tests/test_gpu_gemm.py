@@ -88,6 +88,51 @@ def test_fc512_full_size(dtype):
     assert int(mask.sum()) == L.M * L.K // 4
 
 
+def _uneven_mask(M, K, bm, bk, seed):
+    """Block-based mask whose row-blocks keep different numbers of columns per
+    block (0 .. bk), so K' differs from row-block to row-block."""
+    rng = np.random.default_rng(seed)
+    mask = np.zeros((M, K), dtype=np.uint8)
+    for rb in range(0, M, bm):
+        keep = (rb // bm * 3) % (bk + 1)
+        for c in range(0, K, bk):
+            w = min(bk, K - c)
+            cols = rng.choice(w, size=min(keep, w), replace=False)
+            mask[rb:rb + bm, c + cols] = 1
+    return mask
+
+
+SMALL_CASES = [
+    # M, K, N, bm, bk, dtype, uneven: layers of the short CUDA-core path
+    # (bm <= 32, at most 2^24 kept multiply-adds)
+    (96, 320, 72, 16, 16, bp.F16, True),        # row-blocks keep 0 .. 16 columns per block
+    (100, 1000, 45, 32, 8, bp.BF16, True),      # ragged M and N, K just under the staged limit
+    (64, 2048, 40, 32, 32, bp.BF16, False),     # K past the staged limit: rows gathered by index
+    (50, 1536, 33, 8, 16, bp.F16, True),        # K past the limit, uneven counts
+]
+
+
+@pytest.mark.parametrize("case", SMALL_CASES, ids=lambda c: f"{c[0]}x{c[1]}x{c[2]}_b{c[3]}x{c[4]}_u{int(c[6])}")
+def test_short_path_matches_oracle(case):
+    M, K, N, bm, bk, dtype, uneven = case
+    W = inputs.normal((M, K), 0.05, dtype, M + K)
+    X = inputs.uniform((K, N), -1.0, 1.0, dtype, N)
+    b = inputs.bias(M, 0.1, 7)
+    lay = bp.layout(BB, dtype, M, K, bm, bk)
+    Wd = dev16(W, dtype)
+    if uneven:
+        mask = torch.from_numpy(_uneven_mask(M, K, bm, bk, M * N)).cuda()
+    else:
+        mask = bp.prune(lay, Wd, 8.0)
+    pw = bp.pack(lay, Wd, mask)
+    assert pw.c.nnz_vals * N <= 1 << 24
+    Y = bp.gemm(pw, dev16(X, dtype, pad_last_to=8), bias=torch.from_numpy(b).cuda(), relu=True)
+    torch.cuda.synchronize()
+    assert bp.device_status() == bp.OK
+    ref = oracle.masked_gemm(W, mask.cpu().numpy(), X, dtype, bias=b, relu=True)
+    assert_close(host_bits(Y), ref, dtype, "short path")
+
+
 SWEEP_SAMPLES = [
     # M, K, N, bm, bk, rate, dtype
     (4096, 4096, 4096, 128, 32, 4.0, bp.BF16),
