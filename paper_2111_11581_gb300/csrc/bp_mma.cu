@@ -163,6 +163,28 @@ struct Params {
     unsigned *status;
 };
 
+// Two fp32 values to one 16-bit pair (a low, b high), round to nearest even,
+// negative values to zero when kRelu (one cvt instruction).
+template <bool kBf16, bool kRelu>
+__device__ __forceinline__ uint32_t cvt_pair(float a, float b) {
+    uint32_t d;
+    if (kBf16) {
+        if (kRelu) asm("cvt.rn.relu.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(b), "f"(a));
+        else asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(b), "f"(a));
+    } else {
+        if (kRelu) asm("cvt.rn.relu.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(b), "f"(a));
+        else asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(b), "f"(a));
+    }
+    return d;
+}
+
+template <bool kBf16, bool kRelu>
+__device__ __forceinline__ void cvt_group(const uint32_t (&r)[32], float bv, uint32_t (&pk)[16]) {
+#pragma unroll
+    for (int e = 0; e < 16; ++e)
+        pk[e] = cvt_pair<kBf16, kRelu>(__uint_as_float(r[2 * e]) + bv, __uint_as_float(r[2 * e + 1]) + bv);
+}
+
 __device__ __forceinline__ uint32_t pack2(float a, float b, int dtype) {
     if (dtype == BP_BF16) {
         const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
@@ -568,7 +590,34 @@ struct WindowFiller {
     }
 };
 
-__device__ void control_thread(const Params &p, const Smem &s) {
+// Before the grid dependency wait, while the previous kernel in the stream may
+// still run: the chunk records of the first window and the weight tiles of the
+// first chunks come from the packed image (written by bp_pack, which
+// synchronises), not from anything a kernel in flight writes, so they are
+// requested now.  A weight tile only adds its bytes to its stage barrier; the
+// control thread arrives once the stage's activation loads are issued.
+// Returns the number of weight tiles requested, or -1 when the window was not
+// copied (balanced launches, whose ranges are set after the wait).
+__device__ int control_prefetch(const Params &p, const Smem &s) {
+    if (p.sk) return -1;
+    const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
+    WindowFiller wf;
+    wf.ahead.first(p, kcp, s.skv);
+    wf.filled = 0;
+    if (!wf.ahead.valid(p)) return -1;
+    const Window win = wf.ahead;
+    wf.fill(p, s, kcp);
+    const int n = (int)min((int64_t)p.stages, win.cnt);
+    for (int j = 0; j < n; ++j) {
+        if (blockIdx.x == 0 && j == p.drop_stage) return j;
+        mbar_expect_tx(&s.wfull[j], kWTileBytes);
+        bulk_g2s(smem_u32(s.w + j * kWTileBytes), p.tiles + (win.t.kc0 + win.k0 + j) * (int64_t)kWTileBytes,
+                 kWTileBytes, &s.wfull[j]);
+    }
+    return n;
+}
+
+__device__ void control_thread(const Params &p, const Smem &s, int pre) {
     const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
     Window win;
@@ -576,7 +625,13 @@ __device__ void control_thread(const Params &p, const Smem &s) {
     WindowFiller wf;
     wf.ahead = win;
     wf.filled = 0;
-    if (wf.ahead.valid(p)) wf.fill(p, s, kcp);
+    if (pre >= 0) {             // the first window was copied before the dependency wait
+        wf.filled = 1;
+        wf.ahead.next(p, kcp);
+    } else if (wf.ahead.valid(p)) {
+        wf.fill(p, s, kcp);
+    }
+    const int64_t npre = pre > 0 ? pre : 0;     // chunks whose weight tile is requested
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
@@ -616,27 +671,33 @@ __device__ void control_thread(const Params &p, const Smem &s) {
             const int nb = (int)q0.x;
             const bool tma = nb > 0;
             ++count;
+            // the weight tile of the first chunks was requested before the
+            // dependency wait
+            const bool wpre = seq < npre;
             if (p.impl && !(blockIdx.x == 0 && seq == p.drop_stage)) {
                 // implicit convolution: the weight tile and one box of 64
                 // channels at kernel position (i, j) for the tile's pixels (the
                 // padding and channels past C read as zeros)
                 const int32_t d = *reinterpret_cast<const int32_t *>(recs + j * kMetaBytes);
                 s.skind[stage] = 1u;
-                mbar_arrive_expect_tx(&s.wfull[stage], kWTileBytes + p.i_box_bytes);
-                bulk_g2s(smem_u32(s.w + stage * kWTileBytes),
-                         p.tiles + (win.t.kc0 + win.k0 + j) * (int64_t)kWTileBytes, kWTileBytes,
-                         &s.wfull[stage]);
+                mbar_arrive_expect_tx(&s.wfull[stage], (wpre ? 0u : kWTileBytes) + p.i_box_bytes);
+                if (!wpre)
+                    bulk_g2s(smem_u32(s.w + stage * kWTileBytes),
+                             p.tiles + (win.t.kc0 + win.k0 + j) * (int64_t)kWTileBytes, kWTileBytes,
+                             &s.wfull[stage]);
                 tma_load_4d(smem_u32(s.x + stage * kXTileBytes), &p.imap, (d >> 16) * 64,
                             (d & 0xff) - p.i_pw, (int32_t)win.t.h0 + ((d >> 8) & 0xff) - p.i_ph,
                             (int32_t)win.t.img0, &s.wfull[stage]);
             } else if (!(blockIdx.x == 0 && seq == p.drop_stage)) {
                 s.skind[stage] = tma ? 1u : 0u;    // read by the MMA thread after wfull
                 mbar_arrive_expect_tx(&s.wfull[stage],
-                                      kWTileBytes + (tma ? (uint32_t)p.xboxes * (kBK * 128) : 0u));
+                                      (wpre ? 0u : kWTileBytes) +
+                                          (tma ? (uint32_t)p.xboxes * (kBK * 128) : 0u));
                 BP_TR(seq, 6);
-                bulk_g2s(smem_u32(s.w + stage * kWTileBytes),
-                         p.tiles + (win.t.kc0 + win.k0 + j) * (int64_t)kWTileBytes, kWTileBytes,
-                         &s.wfull[stage]);
+                if (!wpre)
+                    bulk_g2s(smem_u32(s.w + stage * kWTileBytes),
+                             p.tiles + (win.t.kc0 + win.k0 + j) * (int64_t)kWTileBytes, kWTileBytes,
+                             &s.wfull[stage]);
                 BP_TR(seq, 7);
                 if (tma) {
                     // load b: rows y[b] .. + (8 << lg) - 1 of X into list positions
@@ -668,8 +729,12 @@ __device__ void control_thread(const Params &p, const Smem &s) {
     if (!ok) {
         raise_timeout(p, s);
         // unwinding: the copies of the last stages and the window copies may still
-        // be in flight; let them land before the CTA exits
-        for (int64_t q = count > p.stages ? count - p.stages : 0; q < count; ++q)
+        // be in flight; let them land before the CTA exits (a weight tile
+        // requested before the wait for a chunk not reached yet completes its
+        // stage once the arrival it waits for is added)
+        for (int64_t q = count; q < npre; ++q) mbar_arrive(&s.wfull[q]);
+        const int64_t reach = count > npre ? count : npre;
+        for (int64_t q = reach > p.stages ? reach - p.stages : 0; q < reach; ++q)
             if (!(blockIdx.x == 0 && q == p.drop_stage) &&
                 !mbar_wait(&s.wfull[q % p.stages], (uint32_t)((q / p.stages) & 1), kDrainNs,
                            nullptr))
@@ -830,6 +895,11 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
     for (ui.init(p, s.skv); ui.valid(); ui.step(p, t)) {
         t = ui.get(p, kcp);
         const bool has = t.nkc > 0;
+        // lane = output row of the slab; its bias is requested before the wait
+        const int64_t row0 = 32 * q;
+        const bool vrow = row0 + lane < t.rows;
+        const int64_t m = t.slab * kSlab + row0 + lane;
+        const float bv = (p.bias && vrow) ? p.bias[m] : 0.f;
         if (has) {
             // warp-uniform outcome: tcgen05.ld below is a warp-collective instruction
             const bool ok = mbar_wait(&s.tfull[acc], acc_phase, p.watchdog_ns, abort_flag);
@@ -842,25 +912,20 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
 #ifdef BP_TRACE
         if (warp == kEpiWarp0 && lane == 0) BP_TR(384 + titem, 5);
 #endif
+        // tensor-memory lanes = the warp's rows; columns = the tile's columns
         const uint32_t tacc = tmem + ((uint32_t)(32 * q) << 16) + acc * p.acc_cols;
-        // lane = output row of the slab; tensor-memory columns = the tile's columns
-        const int64_t row0 = 32 * q;
-        const bool vrow = row0 + lane < t.rows;
-        const int64_t m = t.slab * kSlab + row0 + lane;
-        const float bv = (p.bias && vrow) ? p.bias[m] : 0.f;
         // Column groups of 32: once group g's accumulators are converted (pk),
         // the tensor-memory load of group g + 1 is issued into the same
         // registers and runs while group g is stored.
         // A warp whose 32 rows are all past the slab's real rows has nothing to write.
+        // bias + ReLU + cast of a 32-column group, one branch per group
         auto pack = [&](const uint32_t (&r)[32], uint32_t (&pk)[16]) {
-#pragma unroll
-            for (int e = 0; e < 16; ++e) {
-                float a = __uint_as_float(r[2 * e]) + bv, b = __uint_as_float(r[2 * e + 1]) + bv;
-                if (p.relu) {
-                    a = fmaxf(a, 0.f);
-                    b = fmaxf(b, 0.f);
-                }
-                pk[e] = pack2(a, b, p.dtype);
+            if (p.dtype == BP_BF16) {
+                if (p.relu) cvt_group<true, true>(r, bv, pk);
+                else cvt_group<true, false>(r, bv, pk);
+            } else {
+                if (p.relu) cvt_group<false, true>(r, bv, pk);
+                else cvt_group<false, false>(r, bv, pk);
             }
         };
         auto store = [&](const uint32_t (&pk)[16], int c0) {
@@ -1208,18 +1273,24 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     }
     if (warp == kCtrlWarp && (threadIdx.x & 31) == 0)
         for (int i = 0; i < 4; ++i) prefetch_tmap(&p.xmap[i]);
-    // Launched as a programmatic dependent: everything above overlaps the end of
-    // the previous kernel in the stream; wait for it before touching global
-    // memory (it may have written the inputs, or still read the output), then
-    // let the next kernel start its own set-up as SMs come free.
+    // Launched as a programmatic dependent: the set-up overlaps the end of the
+    // previous kernel in the stream.  The packed image (written by bp_pack,
+    // which synchronises) is read before the dependency wait: the chunk
+    // pointers, the first window of chunk records and the first weight tiles.
+    // The activations, the output and the workspace are touched only after
+    // it (the previous kernel may have written the inputs, or still read the
+    // output); then the next kernel may start its own set-up as SMs come free.
+    if (s.kc)
+        for (int64_t i = threadIdx.x; i < p.kc_cached; i += kThreads) s.kc[i] = p.kc_ptr[i];
+    __syncthreads();
+    int pre = -1;
+    if (warp == kCtrlWarp && (threadIdx.x & 31) == 0) pre = control_prefetch(p, s);
     grid_dependency_wait();
     grid_launch_dependents();
 #ifdef BP_TRACE
     if (threadIdx.x == 0 && blockIdx.x < 248) g_trace[448 * kTraceEvents + 2 * blockIdx.x] = globaltimer_ns();
     if (threadIdx.x == 0) BP_TR(511, 0);
 #endif
-    if (s.kc)
-        for (int64_t i = threadIdx.x; i < p.kc_cached; i += kThreads) s.kc[i] = p.kc_ptr[i];
     if (p.sk && threadIdx.x == 0) {
         // the balanced launch's constants, once per CTA (64-bit divisions)
         const int64_t tile = p.sk_i0 / p.num_slabs;
@@ -1238,7 +1309,7 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     if (warp < kGatherWarps) {
         gather_warps(p, s);
     } else if (warp == kCtrlWarp) {
-        if ((threadIdx.x & 31) == 0) control_thread(p, s);
+        if ((threadIdx.x & 31) == 0) control_thread(p, s, pre);
         __syncwarp();
     } else if (warp == kMmaWarp) {
         if ((threadIdx.x & 31) == 0) mma_issuer(p, s, tmem);
@@ -1537,7 +1608,11 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
+#ifdef BP_NO_PDL
+    cfg.numAttrs = 0;       // (measurement build) an ordinary stream-ordered launch
+#else
     cfg.numAttrs = 1;
+#endif
     const bool parts = p.split > 1 || p.sk;
     if (conv)
         return parts ? cudaLaunchKernelEx(&cfg, bp_mma_kernel<true, true>, p)

@@ -54,10 +54,15 @@ constexpr int kSmallTok = 32;      // tokens per CTA
 constexpr int kSmallK = 128;       // listed columns per step
 constexpr int kSmallMaxBm = 32;
 constexpr int64_t kStageK = 1024;  // activation rows staged whole up to this K (64 KB)
-// dynamic shared memory: weights of a step, the warps' sums, the step's column
-// indices, then the activation rows (all K of them, or the step's gathered ones)
-constexpr int kOffW = 0, kOffOut = kOffW + kSmallMaxBm * kSmallK * 2;
-constexpr int kOffIdx = kOffOut + kSmallMaxBm * kSmallTok * 4, kOffX = kOffIdx + kSmallK * 4;
+// dynamic shared memory: weights of a step (rows padded to 136 values: the
+// four rows a warp reads at once fall in different banks), each warp's partial
+// sums, the step's column indices, then the activation rows (all K of them,
+// or the step's gathered ones)
+constexpr int kWPitch = kSmallK + 8;
+constexpr int kOffW = 0, kOffRed = kOffW + kSmallMaxBm * kWPitch * 2;
+constexpr int kOffIdx = kOffRed + kSmallWarps * kSmallMaxBm * kSmallTok * 4;
+constexpr int kOffX = kOffIdx + kSmallK * 4;
+constexpr int kMostSmem = kOffX + (int)kStageK * kSmallTok * 2;
 
 template <bool kBf16>
 __device__ __forceinline__ float to_f(uint32_t v) {
@@ -94,13 +99,15 @@ __device__ __forceinline__ void copy_tokens(uint32_t dst, const SmallParams &p, 
     cp_async_16(dst, src, nb);
 }
 
-// grid: (row-blocks, token tiles of 32).  Warp w takes the listed columns
-// i = w (mod 8) of each step; lane l: tokens 4 (l % 8) .. +3, rows l / 8 + 4 j.
+// grid: (row-blocks, token tiles of 32).  Warp w takes the column pairs
+// (2q, 2q + 1), q = w (mod 8), of each step; lane l: tokens 4 (l % 8) .. +3,
+// rows l / 8 + 4 j.  The warps' partial sums are added in warp order.
 template <bool kBf16, bool kStage>
 __global__ void __launch_bounds__(kSmallThreads) bp_small_kernel(const __grid_constant__ SmallParams p) {
     extern __shared__ __align__(16) uint8_t dsm[];
-    uint16_t (*wsm)[kSmallK] = reinterpret_cast<uint16_t (*)[kSmallK]>(dsm + kOffW);
-    float (*out)[kSmallTok] = reinterpret_cast<float (*)[kSmallTok]>(dsm + kOffOut);
+    uint16_t (*wsm)[kWPitch] = reinterpret_cast<uint16_t (*)[kWPitch]>(dsm + kOffW);
+    float (*red)[kSmallMaxBm][kSmallTok] =
+        reinterpret_cast<float (*)[kSmallMaxBm][kSmallTok]>(dsm + kOffRed);
     int32_t *cis = reinterpret_cast<int32_t *>(dsm + kOffIdx);
     uint16_t (*xs)[kSmallTok] = reinterpret_cast<uint16_t (*)[kSmallTok]>(dsm + kOffX);
     const int64_t rb = blockIdx.x, n0 = (int64_t)blockIdx.y * kSmallTok;
@@ -110,7 +117,10 @@ __global__ void __launch_bounds__(kSmallThreads) bp_small_kernel(const __grid_co
     const int tq = (lane & 7) * 4, rq = lane >> 3;
     BP_TS(0, clock64());
     BP_TS(6, globaltimer_ns());
-    for (int e = t; e < kSmallMaxBm * kSmallTok; e += kSmallThreads) (&out[0][0])[e] = 0.f;
+    // this thread's outputs in the epilogue: row t / 8, tokens 4 (t % 8) ..;
+    // its bias is requested now, with the other loads
+    const int orow = t >> 3, oq = (t & 7) * 4;
+    const float bv = (p.bias && orow < rows) ? p.bias[r0 + orow] : 0.f;
     // the row-block's range, requested now and used once the first step's
     // loads (issued for the guessed range) are in flight
     const int64_t ra = p.rb_ptr[rb], rz = p.rb_ptr[rb + 1];
@@ -196,19 +206,42 @@ __global__ void __launch_bounds__(kSmallThreads) bp_small_kernel(const __grid_co
         cp_async_wait_all();
         __syncthreads();
         BP_TS(3, clock64());
-        for (int i = warp; i < kn; i += kSmallWarps) {
-            const int xr = kStage ? cis[i] : i;
-            const uint2 xv = *reinterpret_cast<const uint2 *>(&xs[xr][tq]);
-            const float x0 = to_f<kBf16>(xv.x & 0xffffu), x1 = to_f<kBf16>(xv.x >> 16);
-            const float x2 = to_f<kBf16>(xv.y & 0xffffu), x3 = to_f<kBf16>(xv.y >> 16);
+        // column pairs: one 4-byte weight load per row serves two columns
+#pragma unroll 2
+        for (int i = 2 * warp; i + 1 < kn; i += 2 * kSmallWarps) {
+            const int xa = kStage ? cis[i] : i, xb = kStage ? cis[i + 1] : i + 1;
+            const uint2 va = *reinterpret_cast<const uint2 *>(&xs[xa][tq]);
+            const uint2 vb = *reinterpret_cast<const uint2 *>(&xs[xb][tq]);
+            const float a0 = to_f<kBf16>(va.x & 0xffffu), a1 = to_f<kBf16>(va.x >> 16);
+            const float a2 = to_f<kBf16>(va.y & 0xffffu), a3 = to_f<kBf16>(va.y >> 16);
+            const float b0 = to_f<kBf16>(vb.x & 0xffffu), b1 = to_f<kBf16>(vb.x >> 16);
+            const float b2 = to_f<kBf16>(vb.y & 0xffffu), b3 = to_f<kBf16>(vb.y >> 16);
 #pragma unroll
             for (int j = 0; j < kSmallMaxBm / 4; ++j) {
                 if (rq + 4 * j < rows) {
-                    const float w = to_f<kBf16>(wsm[rq + 4 * j][i]);
-                    acc[j][0] = fmaf(w, x0, acc[j][0]);
-                    acc[j][1] = fmaf(w, x1, acc[j][1]);
-                    acc[j][2] = fmaf(w, x2, acc[j][2]);
-                    acc[j][3] = fmaf(w, x3, acc[j][3]);
+                    const uint32_t w2 = *reinterpret_cast<const uint32_t *>(&wsm[rq + 4 * j][i]);
+                    const float wa = to_f<kBf16>(w2 & 0xffffu), wb = to_f<kBf16>(w2 >> 16);
+                    acc[j][0] = fmaf(wb, b0, fmaf(wa, a0, acc[j][0]));
+                    acc[j][1] = fmaf(wb, b1, fmaf(wa, a1, acc[j][1]));
+                    acc[j][2] = fmaf(wb, b2, fmaf(wa, a2, acc[j][2]));
+                    acc[j][3] = fmaf(wb, b3, fmaf(wa, a3, acc[j][3]));
+                }
+            }
+        }
+        if ((kn & 1) && warp == ((kn - 1) >> 1) % kSmallWarps) {
+            // odd count: the last column alone
+            const int i = kn - 1, xa = kStage ? cis[i] : i;
+            const uint2 va = *reinterpret_cast<const uint2 *>(&xs[xa][tq]);
+            const float a0 = to_f<kBf16>(va.x & 0xffffu), a1 = to_f<kBf16>(va.x >> 16);
+            const float a2 = to_f<kBf16>(va.y & 0xffffu), a3 = to_f<kBf16>(va.y >> 16);
+#pragma unroll
+            for (int j = 0; j < kSmallMaxBm / 4; ++j) {
+                if (rq + 4 * j < rows) {
+                    const float wa = to_f<kBf16>(wsm[rq + 4 * j][i]);
+                    acc[j][0] = fmaf(wa, a0, acc[j][0]);
+                    acc[j][1] = fmaf(wa, a1, acc[j][1]);
+                    acc[j][2] = fmaf(wa, a2, acc[j][2]);
+                    acc[j][3] = fmaf(wa, a3, acc[j][3]);
                 }
             }
         }
@@ -220,22 +253,32 @@ __global__ void __launch_bounds__(kSmallThreads) bp_small_kernel(const __grid_co
     }
     cp_async_wait_all();        // staged rows that no step read
     BP_TS(4, clock64());
-    // the warps' partial sums meet in shared memory
+    // each warp's partial sums to its own slice of shared memory
 #pragma unroll
     for (int j = 0; j < kSmallMaxBm / 4; ++j)
         if (rq + 4 * j < rows)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) atomicAdd(&out[rq + 4 * j][tq + e], acc[j][e]);
+            *reinterpret_cast<float4 *>(&red[warp][rq + 4 * j][tq]) =
+                make_float4(acc[j][0], acc[j][1], acc[j][2], acc[j][3]);
     __syncthreads();
-    // epilogue: + bias, ReLU, one rounding to the weight dtype; thread = (row, 4 tokens)
-    for (int e = t; e < rows * (kSmallTok / 4); e += kSmallThreads) {
-        const int r = e / (kSmallTok / 4), q = (e % (kSmallTok / 4)) * 4;
+    // epilogue: the warps' sums in warp order, + bias, ReLU, one rounding to
+    // the weight dtype; thread = (row, 4 tokens)
+    if (orow < rows) {
+        const int r = orow, q = oq;
         const int64_t m = r0 + r, n = n0 + q;
-        const float bv = p.bias ? p.bias[m] : 0.f;
+        float4 a = *reinterpret_cast<const float4 *>(&red[0][r][q]);
+#pragma unroll
+        for (int w = 1; w < kSmallWarps; ++w) {
+            const float4 v = *reinterpret_cast<const float4 *>(&red[w][r][q]);
+            a.x += v.x;
+            a.y += v.y;
+            a.z += v.z;
+            a.w += v.w;
+        }
+        const float sum[4] = {a.x, a.y, a.z, a.w};
         uint16_t o[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-            float v = out[r][q + u] + bv;
+            float v = sum[u] + bv;
             if (p.relu) v = fmaxf(v, 0.f);
             o[u] = from_f<kBf16>(v);
         }
@@ -284,22 +327,24 @@ cudaError_t launch_small(const bp_packed &P, const void *X, int64_t N, int64_t l
     const int64_t per_rb = (int64_t)P.lay.bm * P.num_rb;
     p.kp_even = (per_rb > 0 && P.nnz_vals % per_rb == 0) ? P.nnz_vals / per_rb : -1;
     const bool stage = P.lay.K <= kStageK;
-    const int smem = kOffX + (int)(stage ? P.lay.K : kSmallK) * kSmallTok * 2;
+    const int smem = kOffX + (int)(stage ? P.lay.K : kSmallK) * kSmallTok * 2;     // > 48 KB
     const bool bf16 = P.lay.dtype == BP_BF16;
     const void *fn = stage ? (bf16 ? (const void *)bp_small_kernel<true, true> : (const void *)bp_small_kernel<false, true>)
                            : (bf16 ? (const void *)bp_small_kernel<true, false> : (const void *)bp_small_kernel<false, false>);
-    // the staging kernels may take more than 48 KB of dynamic shared memory;
-    // allowed once per process (for the largest K staged)
+    // more than 48 KB of dynamic shared memory: allowed once per process (for
+    // the largest K staged)
     static const cudaError_t raised = [] {
-        const int most = kOffX + (int)kStageK * kSmallTok * 2;
-        cudaError_t e = cudaFuncSetAttribute(bp_small_kernel<true, true>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, most);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(bp_small_kernel<false, true>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+        const void *fns[4] = {(const void *)bp_small_kernel<true, true>,
+                              (const void *)bp_small_kernel<false, true>,
+                              (const void *)bp_small_kernel<true, false>,
+                              (const void *)bp_small_kernel<false, false>};
+        cudaError_t e = cudaSuccess;
+        for (const void *f : fns)
+            if (e == cudaSuccess)
+                e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, kMostSmem);
         return e;
     }();
-    if (stage && raised != cudaSuccess) return raised;
+    if (raised != cudaSuccess) return raised;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)P.num_rb, (unsigned)((N + kSmallTok - 1) / kSmallTok));
     cfg.blockDim = dim3(kSmallThreads);
@@ -309,7 +354,11 @@ cudaError_t launch_small(const bp_packed &P, const void *X, int64_t N, int64_t l
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
+#ifdef BP_NO_PDL
+    cfg.numAttrs = 0;       // (measurement build) an ordinary stream-ordered launch
+#else
     cfg.numAttrs = 1;
+#endif
     void *args[] = {&p};
     return cudaLaunchKernelExC(&cfg, fn, args);
 }

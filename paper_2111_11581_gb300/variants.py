@@ -10,6 +10,12 @@ per-stage timeline of the tensor-core product.
         loads instead of gathers) and BERT-base 3072 x 768 over 8192 tokens at
         64 x 16 blocks, keep 1/8; four rotating activation sets, 400 launches.
 
+    python -m paper_2111_11581_gb300.variants latency NAME:[DEFINE,...] ...
+        the same builds, each timing single launches as the workload benchmark
+        does (L2 flushed by a 256 MiB write, read back, then CUDA events around
+        one call; median of 10): the 512 x 512 FC layer, the 3x3 CONV layer,
+        two ResNet-50 1x1 layers and the 4096^3 layer.
+
     python -m paper_2111_11581_gb300.variants probe
         builds and runs probes/tc_rates.cu: tcgen05.mma 128 x N x 16 issued
         back to back from one thread (cycles per instruction for N = 256, 128,
@@ -29,7 +35,9 @@ per-stage timeline of the tensor-core product.
 The switches (all off in the library `build()` makes): BP_TRACE (timeline),
 BP_GATHER_HALVES (both gather groups on every chunk, one barrier per half),
 BP_BALANCE (whole-item waves, then equal chunk ranges per CTA with fp32
-partial tiles).  Builds go to _build/variants/NAME next to the library.
+partial tiles), BP_EPI_DIRECT (output boxes written back from shared memory
+with plain stores instead of TMA stores), BP_NO_PDL (ordinary launches
+instead of programmatic dependent ones).  Builds go to _build/variants/NAME next to the library.
 """
 from __future__ import annotations
 
@@ -103,6 +111,72 @@ def _time_in_process(lib: str):
         us = e0.elapsed_time(e1) * 1000 / n
         res.append(f"{M}x{K}x{N} bm{bm} bk{bk} r{rate:g}: {us:.2f} us "
                    f"{2.0 * int(mask.sum()) * N / us * 1e-6:.1f} TFLOP/s ok={ok}")
+    print(" | ".join(res), flush=True)
+
+
+LATENCY_CASES = ["fc512", "conv3x3", "resnet50:s1b1_1x1b", "resnet50:s3b2_1x1a", "gemm"]
+
+
+def _layer_call(workload: str):
+    """(run, note) for one launch of a named layer, operands on the device."""
+    import torch
+
+    from . import bp, inputs
+    if workload == "fc512":
+        L, dt = inputs.fc512(), bp.F16
+        W = inputs.as_torch(inputs.layer_weight(L, dt), dt).cuda()
+        X = inputs.as_torch(inputs.layer_input(L, dt), dt).cuda()
+        lay = bp.layout(bp.BLOCK_BASED, dt, L.M, L.K, L.bm, L.bk)
+        pw = bp.pack(lay, W, bp.prune(lay, W, L.rate))
+        Y = bp.gemm(pw, X)
+        return lambda: bp.gemm(pw, X, out=Y)
+    if workload == "gemm":
+        dt = bp.BF16
+        L = inputs.gemm_point(4096, 4096, 4096, 128, 32, 4.0, dt)
+        W = inputs.as_torch(inputs.layer_weight(L, dt), dt).cuda()
+        X = inputs.as_torch(inputs.layer_input(L, dt), dt).cuda()
+        lay = bp.layout(bp.BLOCK_BASED, dt, L.M, L.K, L.bm, L.bk)
+        pw = bp.pack(lay, W, bp.prune(lay, W, L.rate))
+        ws = bp.gemm_workspace(pw, L.N)
+        Y = bp.gemm(pw, X, ws=ws)
+        return lambda: bp.gemm(pw, X, out=Y, ws=ws)
+    if workload == "conv3x3":
+        L, dt = inputs.conv3x3_128(), bp.F16
+    else:
+        name = workload.split(":", 1)[1]
+        L, dt = [l for l in inputs.resnet50_imagenet() if l.name == name][0], bp.BF16
+    W = inputs.as_torch(inputs.layer_weight(L, dt).reshape(L.M, -1), dt).cuda()
+    X = inputs.as_torch(inputs.layer_input(L, dt), dt).cuda()
+    lay = bp.layout(L.scheme, dt, L.M, L.K, L.bm, L.bk, L.kh, L.kw)
+    pw = bp.pack(lay, W, bp.prune(lay, W, L.rate))
+    pad, st = (L.pad, L.pad), (L.stride, L.stride)
+    ws = bp.conv2d_workspace(pw, X.shape, pad, st)
+    Y = bp.conv2d(pw, X, pad=pad, stride=st, ws=ws)
+    return lambda: bp.conv2d(pw, X, pad=pad, stride=st, out=Y, ws=ws)
+
+
+def _latency_in_process(lib: str):
+    import statistics
+
+    import torch
+
+    from . import bp
+    bp.load(lib)
+    flush = torch.empty(256 * 2 ** 20 // 4, dtype=torch.float32, device="cuda")
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    res = []
+    for w in LATENCY_CASES:
+        run = _layer_call(w)
+        ts = []
+        for _ in range(12):
+            flush.zero_()
+            flush.sum()
+            ev[0].record()
+            run()
+            ev[1].record()
+            torch.cuda.synchronize()
+            ts.append(ev[0].elapsed_time(ev[1]) * 1e3)
+        res.append(f"{w}: {statistics.median(ts[2:]):.2f} us")
     print(" | ".join(res), flush=True)
 
 
@@ -225,6 +299,9 @@ def main(argv):
     if len(argv) >= 1 and argv[0] == "_time":
         _time_in_process(argv[1])
         return
+    if len(argv) >= 1 and argv[0] == "_latency":
+        _latency_in_process(argv[1])
+        return
     if len(argv) >= 1 and argv[0] == "_trace":
         _trace_in_process(argv[1], argv[2])
         return
@@ -240,18 +317,18 @@ def main(argv):
                      ["1", "512", "256", "4"]):
             rc |= subprocess.run([exe, *args]).returncode
         sys.exit(rc)
-    if not argv or argv[0] not in ("time", "trace"):
+    if not argv or argv[0] not in ("time", "latency", "trace"):
         print(__doc__)
         sys.exit(2)
-    if argv[0] == "time":
+    if argv[0] in ("time", "latency"):
         variants = []
         for a in argv[1:]:
             name, _, fl = a.partition(":")
             variants.append((name, [f for f in fl.split(",") if f]))
         libs = {n: build_variant(n, f) for n, f in variants}
         for n, _ in variants:
-            r = subprocess.run([sys.executable, "-m", "paper_2111_11581_gb300.variants", "_time",
-                                libs[n]], capture_output=True, text=True, cwd=B.ROOT)
+            r = subprocess.run([sys.executable, "-m", "paper_2111_11581_gb300.variants",
+                                "_" + argv[0], libs[n]], capture_output=True, text=True, cwd=B.ROOT)
             print(f"[{n}] {r.stdout.strip()} {r.stderr.strip()[-400:] if r.returncode else ''}",
                   flush=True)
     else:
