@@ -114,6 +114,7 @@ constexpr uint32_t kGroupThreads = kGroupWarps * 32;
 struct Params {
     CUtensorMap ymap;       // output, box 32 x 32 (x 1), 64-byte swizzle: GEMM Y as a 2-D
                             // tensor (N, M); NCHW output as a 3-D tensor (Ho*Wo, M, Nb)
+    CUtensorMap ymap64;     // the same tensor, box 64 x 32 (x 1), 128-byte swizzle
     CUtensorMap xmap[4];    // activations X (N inner, K rows), boxes 64 x (8 << i), 128-byte swizzle
     int dtype;
     int relu;
@@ -140,6 +141,7 @@ struct Params {
     CUtensorMap imap;
     int64_t i_ipt, i_rpt, i_tpi, i_HoWo, i_Wo, i_Ho, i_Nb;
     int i_ph, i_pw;
+    int i_s;                // stride 1, or 2: imap holds the input's four phases
     uint32_t i_box_bytes;
     int sk;                 // 1: balanced launch (whole items in full waves, then each CTA
                             // one equal range of the remaining items' chunks)
@@ -183,15 +185,6 @@ __device__ __forceinline__ void cvt_group(const uint32_t (&r)[32], float bv, uin
 #pragma unroll
     for (int e = 0; e < 16; ++e)
         pk[e] = cvt_pair<kBf16, kRelu>(__uint_as_float(r[2 * e]) + bv, __uint_as_float(r[2 * e + 1]) + bv);
-}
-
-__device__ __forceinline__ uint32_t pack2(float a, float b, int dtype) {
-    if (dtype == BP_BF16) {
-        const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
-        return *reinterpret_cast<const uint32_t *>(&h);
-    }
-    const __half2 h = __floats2half2_rn(a, b);
-    return *reinterpret_cast<const uint32_t *>(&h);
 }
 
 struct Smem {
@@ -679,15 +672,23 @@ __device__ void control_thread(const Params &p, const Smem &s, int pre) {
                 // channels at kernel position (i, j) for the tile's pixels (the
                 // padding and channels past C read as zeros)
                 const int32_t d = *reinterpret_cast<const int32_t *>(recs + j * kMetaBytes);
+                // window offset (di, dj) of kernel position (i, j); stride 2: the
+                // phase it falls in and the offset within that phase
+                int di = ((d >> 8) & 0xff) - p.i_ph, dj = (d & 0xff) - p.i_pw, img = 0;
+                if (p.i_s == 2) {
+                    img = (di & 1) * 2 + (dj & 1);
+                    di >>= 1;       // floor((d - phase) / 2) = floor(d / 2)
+                    dj >>= 1;
+                }
                 s.skind[stage] = 1u;
                 mbar_arrive_expect_tx(&s.wfull[stage], (wpre ? 0u : kWTileBytes) + p.i_box_bytes);
                 if (!wpre)
                     bulk_g2s(smem_u32(s.w + stage * kWTileBytes),
                              p.tiles + (win.t.kc0 + win.k0 + j) * (int64_t)kWTileBytes, kWTileBytes,
                              &s.wfull[stage]);
-                tma_load_4d(smem_u32(s.x + stage * kXTileBytes), &p.imap, (d >> 16) * 64,
-                            (d & 0xff) - p.i_pw, (int32_t)win.t.h0 + ((d >> 8) & 0xff) - p.i_ph,
-                            (int32_t)win.t.img0, &s.wfull[stage]);
+                tma_load_4d(smem_u32(s.x + stage * kXTileBytes), &p.imap, (d >> 16) * 64, dj,
+                            (int32_t)win.t.h0 + di, img * (int32_t)p.i_Nb + (int32_t)win.t.img0,
+                            &s.wfull[stage]);
             } else if (!(blockIdx.x == 0 && seq == p.drop_stage)) {
                 s.skind[stage] = tma ? 1u : 0u;    // read by the MMA thread after wfull
                 mbar_arrive_expect_tx(&s.wfull[stage],
@@ -877,6 +878,11 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
     const int q = warp & 3;                  // tensor-memory lane quadrant this warp may read
     const uint32_t stg = smem_u32(s.ystage + (warp - kEpiWarp0) * 4096);
     uint32_t yseq = 0;                       // TMA box stores issued by this warp
+    // a 64-column box whose left half (the previous group) is staged, and where
+    // it goes; whether the last store issued was such a box
+    bool pend = false, prev_big = false;
+    int64_t pn = 0;
+    uint32_t pbb = 0, phw = 0;
     int acc = 0;
     uint32_t acc_phase = 0;
 #ifdef BP_TRACE
@@ -914,6 +920,12 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
 #endif
         // tensor-memory lanes = the warp's rows; columns = the tile's columns
         const uint32_t tacc = tmem + ((uint32_t)(32 * q) << 16) + acc * p.acc_cols;
+        // convolution: (image, pixel) of the next 32-column group to store
+        uint32_t cbb = 0, chw = 0;
+        if (kConv) {
+            cbb = (uint32_t)t.n0 / (uint32_t)p.HoWo;
+            chw = (uint32_t)t.n0 - cbb * (uint32_t)p.HoWo;
+        }
         // Column groups of 32: once group g's accumulators are converted (pk),
         // the tensor-memory load of group g + 1 is issued into the same
         // registers and runs while group g is stored.
@@ -927,6 +939,55 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                 if (p.relu) cvt_group<false, true>(r, bv, pk);
                 else cvt_group<false, false>(r, bv, pk);
             }
+        };
+        // 64-column output boxes: an even group whose pair lies in the tile (and,
+        // for NCHW, in one image) is staged as the left half of a 64 x 32 box
+        // (128-byte swizzle: chunk c of row r at c ^ (r & 7)); the next group
+        // adds the right half and issues one TMA store for both.  Returns true
+        // when the group was handled here.
+        auto stage_pair = [&](const uint32_t (&pk)[16], int c0, int64_t n, uint32_t bb,
+                              uint32_t hw) -> bool {
+            if (pend) {
+                BP_TRE(0);
+                BP_TRE(1);
+                pend = false;
+#pragma unroll
+                for (int ch = 0; ch < 4; ++ch)
+                    st_shared_v4(stg + lane * 128 + (((ch + 4) ^ (lane & 7)) << 4),
+                                 make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]));
+                fence_proxy_async_smem();
+                __syncwarp();
+                BP_TRE(2);
+                if (lane == 0) {
+                    if (kConv)
+                        tma_store_3d(&p.ymap64, stg, (int32_t)phw, (int32_t)(t.slab * kSlab + row0),
+                                     (int32_t)pbb);
+                    else
+                        tma_store_2d(&p.ymap64, stg, (int32_t)pn, (int32_t)(t.slab * kSlab + row0));
+                    bulk_commit();
+                }
+                prev_big = true;
+                BP_TRE(3);
+                return true;
+            }
+            const bool pair = p.ytma && (c0 & 63) == 0 && c0 + 64 <= t.ncols &&
+                              (!kConv || (hw + 64 <= (uint32_t)p.HoWo && (hw & 7u) == 0));
+            if (!pair) return false;
+            BP_TRE(0);
+            if (lane == 0) bulk_wait_read<0>();     // every earlier store read its box
+            __syncwarp();
+            BP_TRE(1);
+#pragma unroll
+            for (int ch = 0; ch < 4; ++ch)
+                st_shared_v4(stg + lane * 128 + ((ch ^ (lane & 7)) << 4),
+                             make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]));
+            pend = true;
+            pn = n;
+            pbb = bb;
+            phw = hw;
+            BP_TRE(2);
+            BP_TRE(3);
+            return true;
         };
         auto store = [&](const uint32_t (&pk)[16], int c0) {
             const int64_t n = t.n0 + c0;
@@ -982,9 +1043,16 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             }
 #endif
             if (kConv) {
-                // NCHW output, pixel n = b*HoWo + hw is element (b, m, hw)
-                const uint32_t bb = (uint32_t)n / (uint32_t)p.HoWo;
-                const uint32_t hw = (uint32_t)n - bb * (uint32_t)p.HoWo;
+                // NCHW output, pixel n = b*HoWo + hw is element (b, m, hw); the
+                // groups are stored in order, so (b, hw) advances by 32 pixels
+                // per call from the item's first pixel (one division per item)
+                const uint32_t bb = cbb, hw = chw;
+                chw += 32;
+                while (chw >= (uint32_t)p.HoWo) {
+                    chw -= (uint32_t)p.HoWo;
+                    ++cbb;
+                }
+                if (stage_pair(pk, c0, n, bb, hw)) return;
                 if (p.ytma && hw + 32 <= (uint32_t)p.HoWo && c0 + 32 <= t.ncols && (hw & 7u) == 0) {
                     // the 32 pixels lie in one image and in the tile: stage the box
                     // like a GEMM box (below) and store it at (hw, m, b) of the
@@ -992,7 +1060,11 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                     BP_TRE(0);
                     const uint32_t sb = stg + (yseq & 1u) * 2048;
                     ++yseq;
-                    if (lane == 0) bulk_wait_read<1>();
+                    if (lane == 0) {
+                        if (prev_big) bulk_wait_read<0>();
+                        else bulk_wait_read<1>();
+                    }
+                    prev_big = false;
                     __syncwarp();
                     BP_TRE(1);
 #pragma unroll
@@ -1044,10 +1116,15 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             // the two boxes alternate over the warp's stores, across items (an
             // item may have an odd number of groups): the box about to be written
             // was used by the store before last
+            if (stage_pair(pk, c0, n, 0u, 0u)) return;
             BP_TRE(0);
             const uint32_t sb = stg + (yseq & 1u) * 2048;
             ++yseq;
-            if (lane == 0) bulk_wait_read<1>();     // the store that used this box is done
+            if (lane == 0) {                        // the store that used this box is done
+                if (prev_big) bulk_wait_read<0>();
+                else bulk_wait_read<1>();
+            }
+            prev_big = false;
             __syncwarp();
             BP_TRE(1);
 #pragma unroll
@@ -1508,6 +1585,7 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
         p.i_Nb = conv->Nb;
         p.i_ph = conv->ph;
         p.i_pw = conv->pw;
+        p.i_s = conv->sh;
     }
     p.X = static_cast<const uint16_t *>(X);
     p.ldx = ldx;
@@ -1527,11 +1605,14 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
         // NHWC input, channels padded to C8: boxes of 64 channels x Wo x hbox x
         // nbox (channels past C8 read as zero), written as K-major 128-byte rows
         // with the 128-byte swizzle
+        // (stride 2: the four phases, each ceil(H/2) x ceil(W/2), as 4 Nb images)
         const int64_t C8 = (conv->C + 7) / 8 * 8;
-        const cuuint64_t gdim[4] = {(cuuint64_t)C8, (cuuint64_t)conv->W, (cuuint64_t)conv->H,
-                                    (cuuint64_t)conv->Nb};
-        const cuuint64_t gstride[3] = {(cuuint64_t)(C8 * 2), (cuuint64_t)(conv->W * C8 * 2),
-                                       (cuuint64_t)(conv->H * conv->W * C8 * 2)};
+        const int64_t s2 = conv->sh == 2;
+        const int64_t Wi = s2 ? (conv->W + 1) / 2 : conv->W, Hi = s2 ? (conv->H + 1) / 2 : conv->H;
+        const cuuint64_t gdim[4] = {(cuuint64_t)C8, (cuuint64_t)Wi, (cuuint64_t)Hi,
+                                    (cuuint64_t)(s2 ? 4 * conv->Nb : conv->Nb)};
+        const cuuint64_t gstride[3] = {(cuuint64_t)(C8 * 2), (cuuint64_t)(Wi * C8 * 2),
+                                       (cuuint64_t)(Hi * Wi * C8 * 2)};
         const cuuint32_t hbox = (cuuint32_t)(itl.ipt > 0 ? conv->Ho : itl.rpt);
         const cuuint32_t nbox = (cuuint32_t)(itl.ipt > 0 ? itl.ipt : 1);
         const cuuint32_t box[4] = {64, (cuuint32_t)conv->Wo, hbox, nbox};
@@ -1566,6 +1647,11 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
                 CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
+        const cuuint32_t box64[2] = {64, 32};
+        if (enc(&p.ymap64, tdt, 2, Y, gdim, gstride, box64, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
         p.ytma = 1;
     } else if (p.HoWo % 8 == 0) {
         // NCHW output as (Ho*Wo, M, Nb): 32-pixel x 32-channel boxes of one
@@ -1577,6 +1663,11 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
         const cuuint32_t estride[3] = {1, 1, 1};
         if (enc(&p.ymap, tdt, 3, Y, gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
                 CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+        const cuuint32_t box64[3] = {64, 32, 1};
+        if (enc(&p.ymap64, tdt, 3, Y, gdim, gstride, box64, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
         p.ytma = 1;
