@@ -304,17 +304,26 @@ ImplicitTiles implicit_tiles(const ConvShape &cs) {
     return t;
 }
 
-// The implicit convolution serves stride-1 layers with a kh x kw > 1 window
-// (the image's section 3); strided and 1 x 1 layers take the im2col path.
+// The implicit convolution serves stride-1 and stride-2 layers with a kh x kw
+// > 1 window (the image's section 3); other strides and 1 x 1 layers take the
+// im2col path.
 bool implicit_conv_ok(const bp_packed &P, const ConvShape &cs) {
-    if ((int64_t)cs.kh * cs.kw <= 1 || cs.sh != 1 || cs.sw != 1) return false;
+    // stride 1, or stride 2 in both directions (the input staged by phases)
+    if ((int64_t)cs.kh * cs.kw <= 1 || cs.sh != cs.sw || (cs.sh != 1 && cs.sh != 2)) return false;
     if (sec3_bytes(P.lay) == 0) return false;
     if (cs.ph > 255 || cs.pw > 255 || cs.kh > 255 || cs.kw > 255) return false;
     if ((cs.C + 63) / 64 > 32767) return false;
     return implicit_tiles(cs).ok;
 }
 
+bool direct_conv_ok(const ConvShape &cs) {
+    return cs.kh == 1 && cs.kw == 1 && cs.sh == 1 && cs.sw == 1 && cs.ph == 0 && cs.pw == 0 &&
+           (cs.H * cs.W) % 8 == 0;
+}
+
 size_t nhwc8_bytes(const ConvShape &cs) {
+    if (cs.sh == 2)     // four phases of ceil(H/2) x ceil(W/2) pixels
+        return (size_t)align_up(4 * cs.Nb * cdiv(cs.H, 2) * cdiv(cs.W, 2) * align_up(cs.C, 8) * 2, 256);
     return (size_t)align_up(cs.Nb * cs.H * cs.W * align_up(cs.C, 8) * 2, 256);
 }
 
@@ -567,6 +576,10 @@ bp_status bp_conv2d_workspace_size(const bp_packed *P, int64_t Nb, int64_t C, in
         *bytes = nhwc8_bytes(cs) + plan_split(dl, N, true, &it).bytes;
         return BP_OK;
     }
+    if (direct_conv_ok(cs)) {
+        *bytes = plan_split(dl, N, true).bytes;
+        return BP_OK;
+    }
     *bytes = (size_t)align_up(P->lay.K * align_up(N, 8) * 2, 256) + plan_split(dl, N, true).bytes;
     return BP_OK;
 }
@@ -598,6 +611,15 @@ bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, i
         if (e != cudaSuccess) return BP_ERR_CUDA;
         return finish_launch(
             launch_mma(*P, dl, ws, N, 0, bias, relu, out, 0, &cs, split_ws, s, true), s);
+    }
+    if (direct_conv_ok(cs)) {
+        // 1 x 1, stride 1: the channel planes are the activation rows
+        const size_t sb = plan_split(dl, N, true).bytes;
+        if (sb && (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < sb))
+            return BP_ERR_WORKSPACE;
+        return finish_launch(launch_mma(*P, dl, in, N, cs.H * cs.W, bias, relu, out, 0, &cs,
+                                        sb ? ws : nullptr, s, false, true),
+                             s);
     }
     const int64_t ldx = align_up(N, 8);
     // workspace: the im2col matrix, then the split product's partial tiles

@@ -170,7 +170,9 @@ cudaError_t launch_im2col(const ConvShape &cs, int64_t ldx, const void *in, void
                           const int32_t *qmap, cudaStream_t s);
 int64_t im2col_row_width(const ConvShape &cs);   // staged input row length (elements)
 // NCHW input -> NHWC with the channels padded to a multiple of 8 (zeros):
-// out[b][h][w][c], C8 = roundup(C, 8) channels per pixel.
+// out[b][h][w][c], C8 = roundup(C, 8) channels per pixel.  Stride-2 layers
+// (cs.sh == 2): the four phases of the input (pixels (2h + a, 2w + c)), each
+// ceil(H/2) x ceil(W/2), phase (a, c) of image b at image (2a + c) * Nb + b.
 cudaError_t launch_nhwc8(const ConvShape &cs, const void *in, void *out, cudaStream_t s);
 // Implicit convolution (stride 1, kh * kw > 1): output tiles of whole output
 // rows.  ipt > 0: tiles of ipt whole images; else tiles of rpt rows of one
@@ -214,12 +216,16 @@ cudaError_t launch_small(const bp_packed &P, const void *X, int64_t N, int64_t l
 SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split,
                      const ImplicitTiles *it = nullptr);
 
-// With conv, X holds only the listed rows (see DevLayout::off_meta2).  ws:
-// at least plan_split(dl, N, true).bytes of 256-byte-aligned device memory,
-// or nullptr (no split).
+// With conv, X holds only the listed rows (see DevLayout::off_meta2), or
+// with direct, X is the NCHW input of a 1 x 1 stride-1 layer read in place
+// (ldx = H*W, a multiple of 8).  ws: at least plan_split(dl, N, true).bytes of
+// 256-byte-aligned device memory, or nullptr (no split).
 cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, int64_t N,
                        int64_t ldx, const float *bias, int relu, void *Y, int64_t ldy,
                        const ConvShape *conv, void *ws, cudaStream_t s,
-                       bool implicit = false);
+                       bool implicit = false, bool direct = false);
+// 1 x 1 stride-1 layers without padding whose H*W is a multiple of 8: the
+// product gathers the input's channel planes in place (no im2col)
+bool direct_conv_ok(const ConvShape &cs);
 
 }  // namespace bp

@@ -142,6 +142,10 @@ struct Params {
     int64_t i_ipt, i_rpt, i_tpi, i_HoWo, i_Wo, i_Ho, i_Nb;
     int i_ph, i_pw;
     int i_s;                // stride 1, or 2: imap holds the input's four phases
+    // 1 x 1 stride-1 convolution read in place: the activation row of channel c
+    // for pixel n = b*HW + hw is X + b*d_CHW + c*ldx + hw (ldx = HW), no load plans
+    int direct;
+    int64_t d_CHW;
     uint32_t i_box_bytes;
     int sk;                 // 1: balanced launch (whole items in full waves, then each CTA
                             // one equal range of the remaining items' chunks)
@@ -474,7 +478,13 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
         const int64_t n = win.t.n0 + lane * 8;
         const uint32_t nb =
             (lane * 8 < p.nt && n < p.N) ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
-        const uint16_t *xcol = p.X + (nb ? n : 0);
+        const uint16_t *xcol = p.X;
+        if (nb && p.direct) {
+            const int64_t b = n / p.ldx;
+            xcol = p.X + b * p.d_CHW + (n - b * p.ldx);
+        } else if (nb) {
+            xcol = p.X + n;
+        }
         // This warp's list positions of its next chunk are read from shared
         // memory before the current chunk's copies are issued: the copies fill
         // the load/store queue, and reads issued behind them would wait for it.
@@ -482,7 +492,7 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
         bool tma = false;
         auto fetch = [&](int64_t j, int32_t (&ix)[kRowsPerWarp], bool &planned) {
             const uint8_t *rec = recs + j * kMetaBytes;
-            planned = plan_loads(rec) > 0;
+            planned = plan_loads(rec) > 0 && !p.direct;
             const int32_t *l = reinterpret_cast<const int32_t *>(rec);
 #pragma unroll
             for (int i = 0; i < kRowsPerWarp; ++i) ix[i] = l[rbase + gw + kGroupWarps * i];
@@ -662,7 +672,7 @@ __device__ void control_thread(const Params &p, const Smem &s, int pre) {
             const uint4 *pv = reinterpret_cast<const uint4 *>(recs + j * kMetaBytes + kListBytes);
             const uint4 q0 = pv[0], q1 = pv[1], q2 = pv[2];
             const int nb = (int)q0.x;
-            const bool tma = nb > 0;
+            const bool tma = nb > 0 && !p.direct;
             ++count;
             // the weight tile of the first chunks was requested before the
             // dependency wait
@@ -1510,7 +1520,8 @@ SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split, const Imp
 
 cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, int64_t N,
                        int64_t ldx, const float *bias, int relu, void *Y, int64_t ldy,
-                       const ConvShape *conv, void *ws, cudaStream_t st, bool implicit) {
+                       const ConvShape *conv, void *ws, cudaStream_t st, bool implicit,
+                       bool direct) {
     Params p{};
     const uint8_t *dev = static_cast<const uint8_t *>(P.dev);
     p.dtype = P.lay.dtype;
@@ -1569,7 +1580,15 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     p.kc_ptr = reinterpret_cast<const int64_t *>(dev);
     p.tiles = dev + dl.off_tiles;
     // a convolution's X holds only the listed rows: use the compacted records
-    p.meta = dev + (conv ? dl.off_meta2 : dl.off_meta);
+    // a convolution's im2col matrix holds the listed rows only (compacted
+    // records); a 1 x 1 layer read in place uses the column indices themselves
+    p.meta = dev + (conv && !direct ? dl.off_meta2 : dl.off_meta);
+    p.direct = direct ? 1 : 0;
+    if (direct) {
+        if (!conv || conv->kh != 1 || conv->kw != 1 || ldx != conv->H * conv->W || ldx % 8)
+            return cudaErrorInvalidValue;
+        p.d_CHW = conv->C * conv->H * conv->W;
+    }
     if (implicit) {
         // section 3 of the image: K-group chunks
         p.impl = 1;
@@ -1624,7 +1643,7 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
     }
-    for (int i = 0; i < 4 && !implicit; ++i) {
+    for (int i = 0; i < 4 && !implicit && !direct; ++i) {
         // X (N inner, K rows): 64-token x (8 << i)-row boxes for runs of consecutive columns
         const cuuint64_t gdim[2] = {(cuuint64_t)N, (cuuint64_t)P.lay.K};
         const cuuint64_t gstride[1] = {(cuuint64_t)ldx * 2};

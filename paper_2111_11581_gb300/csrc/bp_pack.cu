@@ -990,9 +990,75 @@ cudaError_t launch_pack_sec3(const bp_layout &lay, const void *W, const uint8_t 
     return cudaGetLastError();
 }
 
+// Stride-2 layers: the input split into its four phases (even / odd rows x
+// even / odd columns), each an NHWC image of ceil(H/2) x ceil(W/2) pixels and
+// C8 channels.  Phase (a, c) of image b is image (2a + c) * Nb + b of the
+// output and holds input pixel (2h + a, 2w + c) at (h, w), zero past the
+// input's edge.  A stride-2 window then reads, for each kernel position, one
+// phase at a unit-stride offset.  One block: 64 channels x one input row
+// pair x 64 input columns through shared memory.
+__global__ void __launch_bounds__(256) nhwc8_phase_kernel(ConvShape cs, int64_t xchunks,
+                                                          const uint16_t *__restrict__ in,
+                                                          uint16_t *__restrict__ out) {
+    const int64_t H2 = (cs.H + 1) / 2, W2 = (cs.W + 1) / 2, C8 = (cs.C + 7) / 8 * 8;
+    const int64_t b = blockIdx.z, c0 = (int64_t)blockIdx.y * 64;
+    const int64_t r = blockIdx.x / xchunks, w0 = (blockIdx.x % xchunks) * 64;
+    __shared__ uint16_t tile[64][2][66];        // [channel][row of the pair][column] (+2 pad)
+    const bool vec = cs.W % 8 == 0;             // input rows start 16-byte aligned
+    // 64 channels x 2 rows x 64 columns, 8 columns per thread and pass
+    for (int v = threadIdx.x; v < 64 * 2 * 8; v += blockDim.x) {
+        const int ch = v >> 4, row = (v >> 3) & 1, cq = (v & 7) * 8;
+        const int64_t c = c0 + ch, h = 2 * r + row, w = w0 + cq;
+        uint16_t e[8];
+        if (c < cs.C && h < cs.H && w < cs.W) {
+            const uint16_t *src = in + ((b * cs.C + c) * cs.H + h) * cs.W + w;
+            if (vec && w + 8 <= cs.W) {
+                const uint4 q = *reinterpret_cast<const uint4 *>(src);
+                e[0] = (uint16_t)q.x; e[1] = (uint16_t)(q.x >> 16);
+                e[2] = (uint16_t)q.y; e[3] = (uint16_t)(q.y >> 16);
+                e[4] = (uint16_t)q.z; e[5] = (uint16_t)(q.z >> 16);
+                e[6] = (uint16_t)q.w; e[7] = (uint16_t)(q.w >> 16);
+            } else {
+#pragma unroll
+                for (int u = 0; u < 8; ++u) e[u] = w + u < cs.W ? src[u] : (uint16_t)0;
+            }
+        } else {
+#pragma unroll
+            for (int u = 0; u < 8; ++u) e[u] = 0;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) tile[ch][row][cq + u] = e[u];
+    }
+    __syncthreads();
+    // 4 phases x 32 phase columns x 8 groups of 8 channels, one 16-byte store each
+    for (int v = threadIdx.x; v < 4 * 32 * 8; v += blockDim.x) {
+        const int ph = v >> 8, j = (v >> 3) & 31, g = v & 7;
+        const int a = ph >> 1, cp = ph & 1;
+        const int64_t w2 = w0 / 2 + j;
+        if (w2 >= W2 || c0 + g * 8 >= C8) continue;
+        uint16_t e[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) e[u] = tile[g * 8 + u][a][2 * j + cp];
+        uint4 pk;
+        pk.x = e[0] | ((uint32_t)e[1] << 16);
+        pk.y = e[2] | ((uint32_t)e[3] << 16);
+        pk.z = e[4] | ((uint32_t)e[5] << 16);
+        pk.w = e[6] | ((uint32_t)e[7] << 16);
+        *reinterpret_cast<uint4 *>(out + ((((int64_t)ph * cs.Nb + b) * H2 + r) * W2 + w2) * C8 +
+                                   c0 + g * 8) = pk;
+    }
+}
+
 cudaError_t launch_nhwc8(const ConvShape &cs, const void *in, void *out, cudaStream_t s) {
     const int64_t HW = cs.H * cs.W, C8 = (cs.C + 7) / 8 * 8;
     if (cs.Nb * HW == 0) return cudaSuccess;
+    if (cs.sh == 2) {
+        const int64_t H2 = (cs.H + 1) / 2, xchunks = (cs.W + 63) / 64;
+        const dim3 grid((unsigned)(H2 * xchunks), (unsigned)((C8 + 63) / 64), (unsigned)cs.Nb);
+        nhwc8_phase_kernel<<<grid, 256, 0, s>>>(cs, xchunks, static_cast<const uint16_t *>(in),
+                                                static_cast<uint16_t *>(out));
+        return cudaGetLastError();
+    }
     const dim3 grid((unsigned)((HW + 63) / 64), (unsigned)((C8 + 63) / 64), (unsigned)cs.Nb);
     nhwc8_kernel<<<grid, 256, 0, s>>>(cs, static_cast<const uint16_t *>(in),
                                       static_cast<uint16_t *>(out));

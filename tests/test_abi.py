@@ -138,11 +138,19 @@ def test_conv_argument_checks_on_host(lib):
         bp.ERR_INVALID_ARG
     assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, 1, 1, 0, 1, None, 0, 256, ws, 1 << 20, 0) == \
         bp.ERR_INVALID_ARG
+    # (batches with at least 160 output tiles: launches that fill the SMs of a
+    # GPU, if one is present, without splitting, so no partial tiles are added)
     # stride 1: the implicit convolution's workspace, the input in NHWC with the
-    # channels padded to 8: 2 x 8 x 8 x 8 16-bit values
-    assert bp.bp_conv2d_workspace_size(P, 2, 8, 8, 8, 1, 1, 1, 1) == (bp.OK, 2 * 8 * 8 * 8 * 2)
-    # strided: the im2col workspace, K x roundup8(Nb*Ho*Wo) 16-bit values
-    assert bp.bp_conv2d_workspace_size(P, 3, 8, 7, 5, 0, 0, 2, 1) == (bp.OK, 72 * 32 * 2)
+    # channels padded to 8: 640 x 8 x 8 x 8 16-bit values (4 images per tile)
+    assert bp.bp_conv2d_workspace_size(P, 640, 8, 8, 8, 1, 1, 1, 1) == \
+        (bp.OK, 640 * 8 * 8 * 8 * 2)
+    # stride 2 both ways: the input's four phases, each ceil(7/2) x ceil(7/2)
+    # pixels of 8 channels (4 x 4 outputs: 16 images per tile)
+    assert bp.bp_conv2d_workspace_size(P, 2560, 8, 7, 7, 1, 1, 2, 2) == \
+        (bp.OK, 4 * 2560 * 4 * 4 * 8 * 2)
+    # other strides: the im2col workspace, K x roundup8(Nb*Ho*Wo) 16-bit values
+    assert bp.bp_conv2d_workspace_size(P, 4400, 8, 7, 5, 0, 0, 2, 1) == \
+        (bp.OK, 72 * 39600 * 2)
     assert bp.bp_conv2d_workspace_size(P, 2, 7, 8, 8, 1, 1, 1, 1)[0] == bp.ERR_INVALID_ARG
     # too small, missing or misaligned workspace
     assert bp.bp_conv2d(P, 256, 2, 8, 8, 8, 1, 1, 1, 1, None, 0, 256, ws, 2 * 8 * 8 * 8 * 2 - 1,
