@@ -8,8 +8,9 @@
  *                                                       Eq. punched, Sec. 5.1)
  *   bp_pack      dense weight + mask -> compact per-row-block storage (Sec. 4.3)
  *   bp_gemm      block-sparse GEMM  Y = (W o mask) X, fused bias/ReLU/cast
- *   bp_conv2d    block-sparse convolution (implicit GEMM for stride-1 k x k layers,
- *                im2col + the same product otherwise), same epilogue
+ *   bp_conv2d    block-sparse convolution (implicit GEMM for stride-1 and stride-2
+ *                k x k layers, 1 x 1 stride-1 layers read in place, im2col + the
+ *                same product otherwise), same epilogue
  *
  * Conventions shared by every call:
  *   - All tensor pointers are DEVICE pointers allocated by the caller; the
@@ -226,8 +227,14 @@ bp_status bp_gemm_workspace_size(const bp_packed *P, int64_t N, size_t *bytes);
  *         to NHWC with the channels padded to a multiple of 8; the product
  *         loads, per k-chunk (64 channels at one kernel position), one TMA box
  *         of those channels for its tile of output rows, shifted by the kernel
- *         position, zeros outside the input being the padding.  Other layers:
- *         the listed rows of the input expanded to the K x (Nb*Ho*Wo) matrix
+ *         position, zeros outside the input being the padding.  Stride 2 in
+ *         both directions, kh * kw > 1: the same, from the input's four
+ *         phases (even / odd rows x even / odd columns, each ceil(H/2) x
+ *         ceil(W/2) pixels, NHWC), a kernel position reading one phase.
+ *         1 x 1 stride-1 layers without padding and with H*W a multiple of 8:
+ *         the product reads the input's channel planes in place (the
+ *         workspace holds only the split partial sums).  Other layers: the
+ *         listed rows of the input expanded to the K x (Nb*Ho*Wo) matrix
  *         (im2col), which the product then reads.
  * Requires C*kh*kw == lay.K; dilation and groups are not supported.  The
  * input must be finite (see bp_gemm).  BP_ERR_UNSUPPORTED when kh input
@@ -240,8 +247,10 @@ bp_status bp_conv2d(const bp_packed *P, const void *in, int64_t Nb, int64_t C, i
 
 /* Device workspace bytes bp_conv2d needs for this packed weight and input
  * shape (host output): the implicit GEMM's NHWC copy, 2 * Nb * H * W *
- * (C rounded up to 8), or the im2col matrix, 2 * K * (Nb*Ho*Wo rounded up to
- * 8), rounded up to 256; plus the split product's share. */
+ * (C rounded up to 8) (stride 2: 2 * 4 Nb * ceil(H/2) * ceil(W/2) * (C
+ * rounded up to 8)), nothing for 1 x 1 layers read in place, or the im2col
+ * matrix, 2 * K * (Nb*Ho*Wo rounded up to 8), rounded up to 256; plus the
+ * split product's share. */
 bp_status bp_conv2d_workspace_size(const bp_packed *P, int64_t Nb, int64_t C, int64_t H,
                                    int64_t W, int pad_h, int pad_w, int stride_h, int stride_w,
                                    size_t *bytes);
