@@ -191,6 +191,18 @@ __device__ __forceinline__ void cvt_group(const uint32_t (&r)[32], float bv, uin
         pk[e] = cvt_pair<kBf16, kRelu>(__uint_as_float(r[2 * e]) + bv, __uint_as_float(r[2 * e + 1]) + bv);
 }
 
+// bias + ReLU + cast of a 32-column group, one branch per group
+__device__ __forceinline__ void cvt_any(const Params &p, const uint32_t (&r)[32], float bv,
+                                        uint32_t (&pk)[16]) {
+    if (p.dtype == BP_BF16) {
+        if (p.relu) cvt_group<true, true>(r, bv, pk);
+        else cvt_group<true, false>(r, bv, pk);
+    } else {
+        if (p.relu) cvt_group<false, true>(r, bv, pk);
+        else cvt_group<false, false>(r, bv, pk);
+    }
+}
+
 struct Smem {
     uint8_t *w;          // stages x kWTileBytes
     uint8_t *x;          // stages x kXTileBytes
@@ -203,6 +215,7 @@ struct Smem {
     uint64_t *tempty;    // [2] accumulator drained
     uint64_t *drain;     // [1]
     uint64_t *fixbar;    // [4] balanced launch: a partial tile's quadrant landed (per epilogue warp)
+    uint64_t *ffull;     // the CTA's final item's accumulator is complete (single use)
     uint64_t *pfull;     // [kWinBufs] a window of chunk records landed (TMA byte count)
     uint64_t *pempty;    // [kWinBufs] the gather warps and the control thread are done with it
     uint32_t *skind;     // [stages] 1: the stage's activations come from TMA tile loads
@@ -229,7 +242,8 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
     s.tempty = s.tfull + 2;
     s.drain = s.tempty + 2;
     s.fixbar = s.drain + 1;
-    s.pfull = s.fixbar + 4;
+    s.ffull = s.fixbar + 4;
+    s.pfull = s.ffull + 1;
     s.pempty = s.pfull + kWinBufs;
     s.skind = reinterpret_cast<uint32_t *>(s.pempty + kWinBufs);
     s.tmem_base = s.skind + p.stages;
@@ -245,7 +259,7 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
 
 size_t smem_bytes(int64_t stages, uint32_t ystage_bytes, int64_t kc_cached) {
     return 1024 + (size_t)stages * (kWTileBytes + kXTileBytes) + ystage_bytes +
-           ((2 + kFullPerStage) * (size_t)stages + 9 + 2 * kWinBufs) * 8 + 4 * (size_t)stages + 8 + 8 + 32 + 128 +
+           ((2 + kFullPerStage) * (size_t)stages + 10 + 2 * kWinBufs) * 8 + 4 * (size_t)stages + 8 + 8 + 32 + 128 +
            (size_t)kWinBufs * kWinBytes + 8 * (size_t)kc_cached;
 }
 
@@ -438,6 +452,17 @@ struct Window {
     }
     __device__ __forceinline__ bool valid(const Params &) const { return ui.valid(); }
 };
+
+// The CTA's final item: its last work unit, when it has chunks and the launch
+// splits nothing.  By the time its accumulator is complete every pipeline
+// stage is idle, and the gather warps share its epilogue with the epilogue
+// warps (each warp can read the tensor-memory lanes of quadrant warp % 4).
+__device__ __forceinline__ bool final_unit(const Params &p, const UnitIter &ui, const Item &t) {
+    if (p.split > 1 || p.sk || t.nkc == 0) return false;
+    UnitIter nx = ui;
+    nx.step(p, t);
+    return !nx.valid();
+}
 
 // Load plan of a chunk record (see DevLayout): number of tile loads.
 __device__ __forceinline__ int plan_loads(const uint8_t *rec) {
@@ -869,6 +894,7 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
         }
         if (!ok) break;
         umma_commit(&s.tfull[acc]);
+        if (final_unit(p, ui, t)) umma_commit(s.ffull);
         if (++acc == 2) {
             acc = 0;
             acc_phase ^= 1u;
@@ -880,13 +906,19 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
 }
 
 // ------------------------------------------------------------------ epilogue
+// slot 0: an epilogue warp, every item; slots 1, 2: gather warps 0-3 and 4-7
+// after their last gather, the final item only.  The final item's 64-column
+// pairs k go to slot k mod 3 of the warps of each quadrant.
 template <bool kSplit, bool kConv>
-__device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
+__device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem, int slot) {
     const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int q = warp & 3;                  // tensor-memory lane quadrant this warp may read
-    const uint32_t stg = smem_u32(s.ystage + (warp - kEpiWarp0) * 4096);
+    // 4 KB of staging per warp: the epilogue's own area, or for a gather warp
+    // the idle activation stage area
+    uint8_t *const stgp = slot == 0 ? s.ystage + (warp - kEpiWarp0) * 4096 : s.x + warp * 4096;
+    const uint32_t stg = smem_u32(stgp);
     uint32_t yseq = 0;                       // TMA box stores issued by this warp
     // a 64-column box whose left half (the previous group) is staged, and where
     // it goes; whether the last store issued was such a box
@@ -911,14 +943,35 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
     for (ui.init(p, s.skv); ui.valid(); ui.step(p, t)) {
         t = ui.get(p, kcp);
         const bool has = t.nkc > 0;
+        const bool fin = !kSplit && final_unit(p, ui, t);
+        if (slot > 0 && !fin) {
+            if (has && ++acc == 2) {      // the accumulator this item used
+                acc = 0;
+                acc_phase ^= 1u;
+            }
+            continue;
+        }
         // lane = output row of the slab; its bias is requested before the wait
         const int64_t row0 = 32 * q;
         const bool vrow = row0 + lane < t.rows;
         const int64_t m = t.slab * kSlab + row0 + lane;
         const float bv = (p.bias && vrow) ? p.bias[m] : 0.f;
         if (has) {
+#ifdef BP_EPI_WARM
+            {
+                // (measurement build) the conversion once on dummy data while the
+                // accumulator is still being computed
+                uint32_t dr[32], dp[16];
+#pragma unroll
+                for (int e = 0; e < 32; ++e) dr[e] = (uint32_t)(lane + e);
+                cvt_any(p, dr, bv, dp);
+#pragma unroll
+                for (int e = 0; e < 16; ++e) asm volatile("" ::"r"(dp[e]));
+            }
+#endif
             // warp-uniform outcome: tcgen05.ld below is a warp-collective instruction
-            const bool ok = mbar_wait(&s.tfull[acc], acc_phase, p.watchdog_ns, abort_flag);
+            const bool ok = slot > 0 ? mbar_wait(s.ffull, 0, p.watchdog_ns, abort_flag)
+                                     : mbar_wait(&s.tfull[acc], acc_phase, p.watchdog_ns, abort_flag);
             if (!__all_sync(0xffffffffu, ok)) {
                 raise_timeout(p, s);
                 break;
@@ -930,26 +983,22 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
 #endif
         // tensor-memory lanes = the warp's rows; columns = the tile's columns
         const uint32_t tacc = tmem + ((uint32_t)(32 * q) << 16) + acc * p.acc_cols;
+        // this warp's groups: all, or for the final item the 64-column pairs
+        // k = slot (mod 3): first group and the step between pairs
+        const int g0 = fin ? 2 * slot : 0, pstep = fin ? 3 : 1;
         // convolution: (image, pixel) of the next 32-column group to store
         uint32_t cbb = 0, chw = 0;
         if (kConv) {
-            cbb = (uint32_t)t.n0 / (uint32_t)p.HoWo;
-            chw = (uint32_t)t.n0 - cbb * (uint32_t)p.HoWo;
+            const uint32_t n1 = (uint32_t)t.n0 + 32u * (uint32_t)g0;
+            cbb = n1 / (uint32_t)p.HoWo;
+            chw = n1 - cbb * (uint32_t)p.HoWo;
         }
         // Column groups of 32: once group g's accumulators are converted (pk),
         // the tensor-memory load of group g + 1 is issued into the same
         // registers and runs while group g is stored.
         // A warp whose 32 rows are all past the slab's real rows has nothing to write.
         // bias + ReLU + cast of a 32-column group, one branch per group
-        auto pack = [&](const uint32_t (&r)[32], uint32_t (&pk)[16]) {
-            if (p.dtype == BP_BF16) {
-                if (p.relu) cvt_group<true, true>(r, bv, pk);
-                else cvt_group<true, false>(r, bv, pk);
-            } else {
-                if (p.relu) cvt_group<false, true>(r, bv, pk);
-                else cvt_group<false, false>(r, bv, pk);
-            }
-        };
+        auto pack = [&](const uint32_t (&r)[32], uint32_t (&pk)[16]) { cvt_any(p, r, bv, pk); };
         // 64-column output boxes: an even group whose pair lies in the tile (and,
         // for NCHW, in one image) is staged as the left half of a 64 x 32 box
         // (128-byte swizzle: chunk c of row r at c ^ (r & 7)); the next group
@@ -1097,7 +1146,7 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                 // boundary or the tile's end: stage the 32 x 32 box (lane = channel row, 80-byte
                 // rows), then write it with lanes along the pixels, one
                 // coalesced 64-byte store per channel
-                uint8_t *box = s.ystage + (warp - kEpiWarp0) * 4096;
+                uint8_t *box = stgp;
                 // the box overlaps both TMA staging boxes: their stores must
                 // have read them
                 if (p.ytma && lane == 0) bulk_wait_read<0>();
@@ -1150,12 +1199,12 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
             }
             BP_TRE(3);
                 };
-        if (row0 < t.rows) {
-            const int64_t cols = t.ncols;
-            const int G = (int)((cols + 31) / 32);
+        const int64_t cols = t.ncols;
+        const int G = (int)((cols + 31) / 32);
+        if (row0 < t.rows && g0 < G) {
             uint32_t r[32], pk[16];
             if (has) {
-                tmem_ld_32x32b_x32(tacc, r);
+                tmem_ld_32x32b_x32(tacc + 32 * g0, r);
                 tmem_ld_wait();
             } else {
 #pragma unroll
@@ -1241,16 +1290,28 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                 if (lane == 0 && okw)
                     for (int64_t c = c0; c <= c1; ++c) p.cnt[c * 4 + q] = 0;
             } else if (!kSplit || t.S == 1) {
-                for (int g = 0; g < G; ++g) {
+                for (int g = g0; g < G;) {
+                    // the next group of this warp: the pair's second, or the
+                    // first of its next pair
+                    const int gn = (g & 1) == 0 ? g + 1 : g + 1 + 2 * (pstep - 1);
                     BP_TRE(4);
                     pack(r, pk);
-                    if (has && g + 1 < G) tmem_ld_32x32b_x32(tacc + 32 * (g + 1), r);
+                    if (has && gn < G) tmem_ld_32x32b_x32(tacc + 32 * gn, r);
                     store(pk, 32 * g);
-                    if (has && g + 1 < G) tmem_ld_wait();
+                    if (kConv && gn != g + 1) {
+                        // skipped pairs (their pixels) before the next group
+                        chw += 32u * (uint32_t)(gn - g - 1);
+                        while (chw >= (uint32_t)p.HoWo) {
+                            chw -= (uint32_t)p.HoWo;
+                            ++cbb;
+                        }
+                    }
+                    if (has && gn < G) tmem_ld_wait();
                     BP_TRE(5);
 #ifdef BP_TRACE
                     ++tgrp;
 #endif
+                    g = gn;
                 }
             } else {
                 // Split item: this unit's fp32 partial rows go to its slot; the
@@ -1310,7 +1371,7 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem) {
                 }
             }
         }
-        if (has) {
+        if (has && slot == 0) {
             tc_fence_before();
             mbar_arrive(&s.tempty[acc]);
             if (++acc == 2) {
@@ -1347,6 +1408,7 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
         }
         mbar_init(s.drain, 1);
         for (int i = 0; i < 4; ++i) mbar_init(&s.fixbar[i], 1);
+        mbar_init(s.ffull, 1);
         for (int i = 0; i < kWinBufs; ++i) {
             mbar_init(&s.pfull[i], 1);
             mbar_init(&s.pempty[i], kGatherWarps + 1);
@@ -1395,6 +1457,8 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
 
     if (warp < kGatherWarps) {
         gather_warps(p, s);
+        // then a share of the final item's output (pipeline stages idle by then)
+        if (!kSplit) epilogue<kSplit, kConv>(p, s, tmem, 1 + (warp >> 2));
     } else if (warp == kCtrlWarp) {
         if ((threadIdx.x & 31) == 0) control_thread(p, s, pre);
         __syncwarp();
@@ -1402,7 +1466,7 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
         if ((threadIdx.x & 31) == 0) mma_issuer(p, s, tmem);
         __syncwarp();
     } else {
-        epilogue<kSplit, kConv>(p, s, tmem);
+        epilogue<kSplit, kConv>(p, s, tmem, 0);
     }
 
     tc_fence_before();

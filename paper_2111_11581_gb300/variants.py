@@ -22,7 +22,7 @@ per-stage timeline of the tensor-core product.
         64, 16) and TMA bulk copies from 1, 2 and 4 threads per SM (bytes per
         cycle an SM ingests).
 
-    python -m paper_2111_11581_gb300.variants trace [gemm|conv3x3|resnet50:LAYER|fc512]
+    python -m paper_2111_11581_gb300.variants trace [gemm|conv3x3|resnet50:LAYER|fc512] [DEFINE ...]
         builds with BP_TRACE and prints CTA 0's clock64 timeline of one launch,
         L2 flushed before it, of the 4096^3 layer (or of the 3x3 CONV layer: N=128, C=F=128, 16x16,
         or of one ResNet-50 layer by name): per pipeline stage when the control
@@ -37,7 +37,8 @@ BP_GATHER_HALVES (both gather groups on every chunk, one barrier per half),
 BP_BALANCE (whole-item waves, then equal chunk ranges per CTA with fp32
 partial tiles), BP_EPI_DIRECT (output boxes written back from shared memory
 with plain stores instead of TMA stores), BP_NO_PDL (ordinary launches
-instead of programmatic dependent ones).  Builds go to _build/variants/NAME next to the library.
+instead of programmatic dependent ones), BP_EPI_WARM (the epilogue runs its
+conversion once on dummy data while it waits for an accumulator).  Builds go to _build/variants/NAME next to the library.
 """
 from __future__ import annotations
 
@@ -283,6 +284,10 @@ def _trace_in_process(lib: str, workload: str):
               f"convert {np.median(g[:, 0] - g[:, 4]):.0f}, box free {np.median(g[:, 1] - g[:, 0]):.0f}, "
               f"write+fence {np.median(g[:, 2] - g[:, 1]):.0f}, store issue {np.median(g[:, 3] - g[:, 2]):.0f}, "
               f"next load wait {np.median(g[:, 5] - g[:, 3]):.0f}, group {np.median(g[:, 5] - g[:, 4]):.0f}")
+        print("first groups: start, convert, box free, write, issue, load wait (cycles after CTA 0's start / durations)")
+        for k, r in enumerate(g[:8]):
+            print(f"  {k}: {r[4] - t0:7d} {r[0] - r[4]:5d} {r[1] - r[0]:5d} {r[2] - r[1]:5d} "
+                  f"{r[3] - r[2]:5d} {r[5] - r[3]:5d}")
     g = rel[rel[:, 4] >= 0]
     if len(g):
         print(f"median gather issue -> tensor cores see the rows {np.median(g[:, 4] - g[:, 2]):.0f}")
@@ -333,7 +338,8 @@ def main(argv):
                   flush=True)
     else:
         wl = argv[1] if len(argv) > 1 else "gemm"
-        lib = build_variant("trace", ["BP_TRACE"])
+        extra = [d for d in argv[2:] if d]
+        lib = build_variant("trace" + "".join("_" + d.lower() for d in extra), ["BP_TRACE"] + extra)
         r = subprocess.run([sys.executable, "-m", "paper_2111_11581_gb300.variants", "_trace", lib,
                             wl], cwd=B.ROOT)
         sys.exit(r.returncode)
