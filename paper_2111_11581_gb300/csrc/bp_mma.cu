@@ -54,9 +54,9 @@
 // it issued the item's last store.  Entries 448 .. hold the global-timer start
 // and end of each of the first 248 CTAs; entry 511: CTA 0's clock64() after
 // the grid dependency wait (0) and at exit (1).  Per 32-column output group g
-// of the first epilogue warp (entries 512 + g): 4 group start, 0 converted, 1
-// its staging box free, 2 box written and fenced, 3 store issued, 5 the next
-// group's tensor-memory load landed.
+// of the first epilogue warp (entries 512 + g): 4 group start, 6 converted, 7
+// next group's tensor-memory load issued, 0 store entered, 1 its staging box
+// free, 2 box written and fenced, 3 store issued, 5 the next load landed.
 #ifdef BP_TRACE
 namespace bp {
 constexpr int kTraceChunks = 1024;
@@ -957,18 +957,6 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem, int slot
         const int64_t m = t.slab * kSlab + row0 + lane;
         const float bv = (p.bias && vrow) ? p.bias[m] : 0.f;
         if (has) {
-#ifdef BP_EPI_WARM
-            {
-                // (measurement build) the conversion once on dummy data while the
-                // accumulator is still being computed
-                uint32_t dr[32], dp[16];
-#pragma unroll
-                for (int e = 0; e < 32; ++e) dr[e] = (uint32_t)(lane + e);
-                cvt_any(p, dr, bv, dp);
-#pragma unroll
-                for (int e = 0; e < 16; ++e) asm volatile("" ::"r"(dp[e]));
-            }
-#endif
             // warp-uniform outcome: tcgen05.ld below is a warp-collective instruction
             const bool ok = slot > 0 ? mbar_wait(s.ffull, 0, p.watchdog_ns, abort_flag)
                                      : mbar_wait(&s.tfull[acc], acc_phase, p.watchdog_ns, abort_flag);
@@ -1296,7 +1284,9 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem, int slot
                     const int gn = (g & 1) == 0 ? g + 1 : g + 1 + 2 * (pstep - 1);
                     BP_TRE(4);
                     pack(r, pk);
+                    BP_TRE(6);
                     if (has && gn < G) tmem_ld_32x32b_x32(tacc + 32 * gn, r);
+                    BP_TRE(7);
                     store(pk, 32 * g);
                     if (kConv && gn != g + 1) {
                         // skipped pairs (their pixels) before the next group

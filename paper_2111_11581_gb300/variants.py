@@ -37,8 +37,7 @@ BP_GATHER_HALVES (both gather groups on every chunk, one barrier per half),
 BP_BALANCE (whole-item waves, then equal chunk ranges per CTA with fp32
 partial tiles), BP_EPI_DIRECT (output boxes written back from shared memory
 with plain stores instead of TMA stores), BP_NO_PDL (ordinary launches
-instead of programmatic dependent ones), BP_EPI_WARM (the epilogue runs its
-conversion once on dummy data while it waits for an accumulator).  Builds go to _build/variants/NAME next to the library.
+instead of programmatic dependent ones).  Builds go to _build/variants/NAME next to the library.
 """
 from __future__ import annotations
 
@@ -284,10 +283,11 @@ def _trace_in_process(lib: str, workload: str):
               f"convert {np.median(g[:, 0] - g[:, 4]):.0f}, box free {np.median(g[:, 1] - g[:, 0]):.0f}, "
               f"write+fence {np.median(g[:, 2] - g[:, 1]):.0f}, store issue {np.median(g[:, 3] - g[:, 2]):.0f}, "
               f"next load wait {np.median(g[:, 5] - g[:, 3]):.0f}, group {np.median(g[:, 5] - g[:, 4]):.0f}")
-        print("first groups: start, convert, box free, write, issue, load wait (cycles after CTA 0's start / durations)")
+        print("first groups: start, convert, load issue, to store, box free, write, issue, load wait "
+              "(cycles after CTA 0's start / durations)")
         for k, r in enumerate(g[:8]):
-            print(f"  {k}: {r[4] - t0:7d} {r[0] - r[4]:5d} {r[1] - r[0]:5d} {r[2] - r[1]:5d} "
-                  f"{r[3] - r[2]:5d} {r[5] - r[3]:5d}")
+            print(f"  {k}: {r[4] - t0:7d} {r[6] - r[4]:5d} {r[7] - r[6]:5d} {r[0] - r[7]:5d} "
+                  f"{r[1] - r[0]:5d} {r[2] - r[1]:5d} {r[3] - r[2]:5d} {r[5] - r[3]:5d}")
     g = rel[rel[:, 4] >= 0]
     if len(g):
         print(f"median gather issue -> tensor cores see the rows {np.median(g[:, 4] - g[:, 2]):.0f}")
