@@ -19,8 +19,11 @@ per-stage timeline of the tensor-core product.
     python -m paper_2111_11581_gb300.variants probe
         builds and runs probes/tc_rates.cu: tcgen05.mma 128 x N x 16 issued
         back to back from one thread (cycles per instruction for N = 256, 128,
-        64, 16) and TMA bulk copies from 1, 2 and 4 threads per SM (bytes per
-        cycle an SM ingests).
+        64, 16), TMA bulk copies from 1, 2 and 4 threads per SM (bytes per
+        cycle an SM ingests), the stage ring without data (cycles per 64-column
+        chunk for 2-6 stages, with and without the per-stage fences) and
+        back-to-back MMAs while other warps copy into shared memory (bulk or
+        cp.async rows).
 
     python -m paper_2111_11581_gb300.variants trace [gemm|conv3x3|resnet50:LAYER|fc512] [DEFINE ...]
         builds with BP_TRACE and prints CTA 0's clock64 timeline of one launch,
@@ -319,7 +322,41 @@ def main(argv):
         rc = 0
         for args in (["0", "512", "256"], ["0", "512", "128"], ["0", "512", "64"],
                      ["0", "512", "16"], ["1", "512", "256", "1"], ["1", "512", "256", "2"],
-                     ["1", "512", "256", "4"]):
+                     ["1", "512", "256", "4"],
+                     # stage ring without data: stages, fences
+                     ["2", "4096", "256", "4", "0"], ["2", "4096", "256", "4", "1"],
+                     ["2", "4096", "256", "4", "3"], ["2", "4096", "256", "6", "1"],
+                     ["2", "4096", "256", "2", "1"], ["2", "4096", "256", "4", "5"],
+                     ["2", "2048", "256", "4", "2049"],
+                     ["2", "2048", "256", "4", "2053"], ["2", "4096", "128", "4", "1"],
+                     # what a commit costs: groups of 2 / 4 / 8 MMAs
+                     ["4", "2048", "256", "4", "2"], ["4", "2048", "256", "4", "0"],
+                     ["4", "2048", "256", "4", "1"], ["4", "4096", "256", "2", "0"],
+                     ["4", "1024", "256", "8", "0"], ["4", "1024", "256", "8", "1"],
+                     # the row gather alone against its footprint (MB) and row pitch (KB)
+                     ["5", "2048", "16", "8", "0"], ["5", "2048", "16", "8", "8"],
+                     ["5", "2048", "64", "8", "8"], ["5", "2048", "256", "8", "8"],
+                     ["5", "2048", "64", "4", "8"], ["5", "2048", "64", "2", "8"],
+                     # gathers beside a bulk-copy stream (the product's mix, no tensor core)
+                     ["6", "2048", "64", "6", "0"], ["6", "2048", "64", "6", "1"],
+                     ["6", "2048", "64", "6", "2"], ["6", "2048", "64", "4", "0"],
+                     ["6", "2048", "64", "4", "2"],
+                     # the product's stage ring with its data, no tensor core
+                     ["7", "4096", "256", "4", "0"], ["7", "4096", "256", "4", "1"],
+                     ["7", "4096", "256", "4", "2"], ["7", "4096", "256", "4", "3"],
+                     ["7", "4096", "256", "4", "4"], ["7", "4096", "256", "4", "8"],
+                     ["7", "4096", "128", "4", "0"], ["7", "4096", "256", "3", "0"],
+                     ["7", "4096", "256", "4", "17"], ["7", "4096", "256", "8", "33"],
+                     ["7", "4096", "256", "8", "49"], ["7", "4096", "256", "8", "32"],
+                     ["7", "4096", "256", "6", "33"], ["7", "4096", "128", "4", "1"],
+                     ["7", "4096", "256", "4", "65"], ["7", "4096", "256", "4", "129"],
+                     ["7", "4096", "256", "4", "64"], ["7", "4096", "256", "8", "97"],
+                     ["7", "4096", "256", "4", "256"], ["7", "4096", "256", "4", "257"],
+                     ["7", "4096", "256", "8", "289"],
+                     # MMAs against concurrent copies: bulk, then cp.async rows
+                     ["3", "512", "256", "1", "0"], ["3", "512", "256", "2", "0"],
+                     ["3", "512", "256", "2", "4"], ["3", "512", "256", "4", "4"],
+                     ["3", "512", "256", "6", "4"]):
             rc |= subprocess.run([exe, *args]).returncode
         sys.exit(rc)
     if not argv or argv[0] not in ("time", "latency", "trace"):
