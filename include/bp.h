@@ -188,13 +188,15 @@ bp_status bp_pack(const bp_layout *lay, const void *W, const uint8_t *mask, bp_p
  *   relu  0 / 1
  *   Y     device, M x N row-major (ldy >= N, multiple of 8)
  *   ws    device workspace of bp_gemm_workspace_size() bytes (256-B aligned),
- *         or NULL: with it, the work that would leave SMs idle in the last
- *         wave (or when there is little work) is split along k and its fp32
- *         partial sums are added in the workspace; without it nothing is
- *         split (same result up to fp32 summation order).  Zero-fill a new
- *         workspace (and again after a BP_ERR_TIMEOUT); the kernel leaves it
- *         ready for the next call.  Calls that may overlap on the GPU need
- *         separate workspaces.
+ *         or NULL: with it, a launch with fewer (128-row slab, column tile)
+ *         items than SMs splits each item along k and its units add their
+ *         fp32 partial sums into one accumulator tile per item in the
+ *         workspace (atomic vector adds, so the order of those fp32 adds, and
+ *         rarely the last bit of the rounded output, can differ from call to
+ *         call); without it nothing is split (same result up to fp32
+ *         summation order).  Zero-fill a new workspace (and again after a
+ *         BP_ERR_TIMEOUT); the kernel leaves it zeroed for the next call.
+ *         Calls that may overlap on the GPU need separate workspaces.
  * Any bm: weights are processed in slabs of 128 rows (see bp_packed::dev).
  * Small layers with row-blocks of at most 32 rows (nnz_vals * N <= 2^24) take
  * a short path instead: one CTA per (row-block, 32 tokens) on the compact

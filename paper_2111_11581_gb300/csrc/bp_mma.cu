@@ -57,6 +57,11 @@
 // of the first epilogue warp (entries 512 + g): 4 group start, 6 converted, 7
 // next group's tensor-memory load issued, 0 store entered, 1 its staging box
 // free, 2 box written and fenced, 3 store issued, 5 the next load landed.
+// Split launches, per epilogue warp of quadrant q (entries 1000 + q): 0 its
+// reductions start, 1 issued, 2 fenced, 3 arrival counted (CTA 0), and for
+// the last arrival of split item 0 (any CTA, its own clock): 4 the sums
+// landed in shared memory, 5 the output stores start, 6 the output stored and
+// the tile zeroed; entries 1004 + q: each column group stored.
 #ifdef BP_TRACE
 namespace bp {
 constexpr int kTraceChunks = 1024;
@@ -129,8 +134,8 @@ struct Params {
     int64_t full_items;     // the first full_items items are single work units
     int split;              // units per later item (k-chunk ranges)
     int64_t num_units;      // full_items + (num_items - full_items) * split
-    float *part;            // split items: fp32 partial tiles, [item][unit][128][256];
-                            // balanced launches: one tile per CTA
+    float *part;            // split items: one fp32 accumulator tile per item, [item][128][256];
+                            // balanced launches: one partial tile per CTA
     int32_t *cnt;           // split items: arrivals per (item, row quadrant); balanced
                             // launches: per (CTA, row quadrant) "partial written" flags
     // implicit convolution (stride 1): X is the NHWC input with channels padded
@@ -1139,13 +1144,65 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem, int slot
                 // have read them
                 if (p.ytma && lane == 0) bulk_wait_read<0>();
                 __syncwarp();                      // the previous box has been read
+                const int rmax = (int)min((int64_t)32, t.rows - row0);
+                // Ho*Wo dividing 32 and the group starting at an image: the group
+                // holds whole images, and each image's 32 channels x Ho*Wo pixels
+                // are one run of 64 Ho*Wo contiguous bytes of the NCHW output
+                // (16-byte aligned when M is a multiple of 8).  Lane r (channel
+                // row) puts its Ho*Wo values of image i at (i * 32 + r) * Ho*Wo
+                // of the staging area, which thus holds the runs back to back,
+                // and the warp copies them out with 16-byte loads and stores.
+                // (One 2-byte store per lane and channel took ~3,000 cycles per
+                // group on 2 x 2 images.)
+                {
+                    const uint32_t HW = (uint32_t)p.HoWo;
+                    const int64_t cols = min((int64_t)32, t.n0 + t.ncols - n);
+                    if (hw == 0u && HW < 32u && (32u % HW) == 0u && rmax == 32 && (p.M & 7) == 0 &&
+                        cols > 0 && cols % HW == 0) {
+                        const int lg = __ffs((int)HW) - 1;            // HW is a power of two
+                        const uint32_t sb = smem_u32(box);
+                        if (lg == 0) {
+#pragma unroll
+                            for (int i = 0; i < 32; ++i)
+                                st_shared_u16(sb + (i * 32 + lane) * 2, (uint16_t)(pk[i >> 1] >> (16 * (i & 1))));
+                        } else if (lg == 1) {
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) st_shared_u32(sb + (i * 64 + lane * 2) * 2, pk[i]);
+                        } else if (lg == 2) {
+#pragma unroll
+                            for (int i = 0; i < 8; ++i)
+                                st_shared_v2(sb + (i * 128 + lane * 4) * 2, pk[2 * i], pk[2 * i + 1]);
+                        } else if (lg == 3) {
+#pragma unroll
+                            for (int i = 0; i < 4; ++i)
+                                st_shared_v4(sb + (i * 256 + lane * 8) * 2,
+                                             make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]));
+                        } else {
+#pragma unroll
+                            for (int i = 0; i < 2; ++i)
+#pragma unroll
+                                for (int h = 0; h < 2; ++h)
+                                    st_shared_v4(sb + (i * 512 + lane * 16 + h * 8) * 2,
+                                                 make_uint4(pk[8 * i + 4 * h], pk[8 * i + 4 * h + 1],
+                                                            pk[8 * i + 4 * h + 2], pk[8 * i + 4 * h + 3]));
+                        }
+                        __syncwarp();
+                        const int total = (int)cols * 4;               // 16-byte pieces
+                        uint16_t *ybase = p.Y + ((int64_t)bb * p.M + t.slab * kSlab + row0) * HW;
+                        for (int k = lane; k < total; k += 32) {
+                            const int i = k >> (lg + 2), off = k & ((4 << lg) - 1);
+                            *reinterpret_cast<uint4 *>(ybase + (int64_t)i * p.M * HW + off * 8) =
+                                ld_shared_v4(sb + k * 16);
+                        }
+                        return;
+                    }
+                }
 #pragma unroll
                 for (int ch = 0; ch < 4; ++ch)
                     st_shared_v4(smem_u32(box + lane * 80 + ch * 16),
                                  make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]));
                 __syncwarp();
                 const int64_t nn = n + lane;
-                const int rmax = (int)min((int64_t)32, t.rows - row0);
                 // only the tile's own pixels: an implicit convolution's tile
                 // holds fewer pixels than the MMA's N
                 if (nn < t.n0 + t.ncols && rmax > 0) {
@@ -1304,61 +1361,94 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem, int slot
                     g = gn;
                 }
             } else {
-                // Split item: this unit's fp32 partial rows go to its slot; the
-                // unit whose arrival completes the (item, quadrant) count sums
-                // all slots and writes the output (no unit waits for another).
-                // Slot layout per quadrant: [group][8 float4][lane], so each
-                // warp access is 512 contiguous bytes.
-                float4 *slot = reinterpret_cast<float4 *>(p.part) +
-                               ((t.j * t.S + t.s) * 4 + q) * kQuad + lane;
-                for (int g = 0; g < G; ++g) {
+                // Split item: the units of an item add their fp32 partial rows
+                // into the item's accumulator tile in the workspace with vector
+                // reductions (no value returned, so no unit waits on them); the
+                // unit whose arrival completes the (item, quadrant) count reads
+                // the sum back, zeroes the tile again for the next launch and
+                // writes the output.  No unit waits for another.  Tile layout
+                // per quadrant: [group][8 float4][lane], so each warp access is
+                // 512 contiguous bytes.  (Summing per-unit partial tiles in the
+                // last unit instead left that unit reading S x 128 KB alone,
+                // latency-bound: 20-30 us on the 512-filter VGG-16 layers.)
+                float4 *acc4 = reinterpret_cast<float4 *>(p.part) + (t.j * 4 + q) * kQuad;
+#ifdef BP_TRACE
+#define BP_TRS(ev)                                                                     \
+    do {                                                                               \
+        if (lane == 0 && ((ev) < 4 ? blockIdx.x == 0 : t.j == 0))                       \
+            bp::g_trace[(1000 + q) * bp::kTraceEvents + (ev)] = clock64();             \
+    } while (0)
+#else
+#define BP_TRS(ev) \
+    do {           \
+    } while (0)
+#endif
+                BP_TRS(0);
+                if (has) {
+                    for (int g = 0; g < G; ++g) {
 #pragma unroll
-                    for (int e = 0; e < 8; ++e)
-                        __stcg(slot + (g * 8 + e) * 32,
-                               make_float4(__uint_as_float(r[4 * e]), __uint_as_float(r[4 * e + 1]),
-                                           __uint_as_float(r[4 * e + 2]), __uint_as_float(r[4 * e + 3])));
-                    if (has && g + 1 < G) {
-                        tmem_ld_32x32b_x32(tacc + 32 * (g + 1), r);
-                        tmem_ld_wait();
+                        for (int e = 0; e < 8; ++e)
+                            red_add_f32x4(acc4 + (g * 8 + e) * 32 + lane, __uint_as_float(r[4 * e]),
+                                          __uint_as_float(r[4 * e + 1]), __uint_as_float(r[4 * e + 2]),
+                                          __uint_as_float(r[4 * e + 3]));
+                        if (g + 1 < G) {
+                            tmem_ld_32x32b_x32(tacc + 32 * (g + 1), r);
+                            tmem_ld_wait();
+                        }
                     }
                 }
+                BP_TRS(1);
                 __threadfence();
                 __syncwarp();
+                BP_TRS(2);
                 int last = 0;
                 if (lane == 0) last = atomicAdd(p.cnt + t.j * 4 + q, 1) == t.S - 1;
+                BP_TRS(3);
                 if (__shfl_sync(0xffffffffu, last, 0)) {
                     __threadfence();
                     if (lane == 0) p.cnt[t.j * 4 + q] = 0;     // zero again for the next launch
-                    const float4 *base = reinterpret_cast<const float4 *>(p.part) +
-                                         (t.j * t.S * 4 + q) * kQuad + lane;
-                    for (int g = 0; g < G; ++g) {
-                        float4 a[8];
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) a[e] = __ldcg(base + (g * 8 + e) * 32);
-                        for (int u = 1; u < t.S; ++u) {
-                            float4 v[8];
-#pragma unroll
-                            for (int e = 0; e < 8; ++e)
-                                v[e] = __ldcg(base + (int64_t)u * 4 * kQuad + (g * 8 + e) * 32);
+                    // Every CTA of a split launch runs one unit, so its activation
+                    // stages are idle now: the quadrant's 32 KB of sums come in
+                    // with one TMA bulk copy (plain loads, 8 per lane in flight,
+                    // would take a round trip per column group).
+                    uint8_t *qbuf = s.w + q * (kQuad * 16);    // inside the stage area (checked at launch)
+                    bool okw = true;
+                    if (lane == 0) {
+                        fence_proxy_async_global();
+                        mbar_arrive_expect_tx(&s.fixbar[q], (uint32_t)(kQuad * 16));
+                        bulk_g2s(smem_u32(qbuf), acc4, (uint32_t)(kQuad * 16), &s.fixbar[q]);
+                    }
+                    okw = mbar_wait(&s.fixbar[q], 0, p.watchdog_ns, abort_flag);
+                    BP_TRS(4);
+                    if (!__all_sync(0xffffffffu, okw)) {
+                        raise_timeout(p, s);
+                    } else {
+                        BP_TRS(5);
+                        const float4 *sm4 = reinterpret_cast<const float4 *>(qbuf) + lane;
+                        for (int g = 0; g < G; ++g) {
 #pragma unroll
                             for (int e = 0; e < 8; ++e) {
-                                a[e].x += v[e].x;
-                                a[e].y += v[e].y;
-                                a[e].z += v[e].z;
-                                a[e].w += v[e].w;
+                                const float4 v = sm4[(g * 8 + e) * 32];
+                                r[4 * e] = __float_as_uint(v.x);
+                                r[4 * e + 1] = __float_as_uint(v.y);
+                                r[4 * e + 2] = __float_as_uint(v.z);
+                                r[4 * e + 3] = __float_as_uint(v.w);
                             }
+                            pack(r, pk);
+                            store(pk, 32 * g);
+#ifdef BP_TRACE
+                            if (lane == 0 && g < 8 && t.j == 0)
+                                bp::g_trace[(1004 + q) * bp::kTraceEvents + g] = clock64();
+#endif
                         }
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            r[4 * e] = __float_as_uint(a[e].x);
-                            r[4 * e + 1] = __float_as_uint(a[e].y);
-                            r[4 * e + 2] = __float_as_uint(a[e].z);
-                            r[4 * e + 3] = __float_as_uint(a[e].w);
-                        }
-                        pack(r, pk);
-                        store(pk, 32 * g);
+                        // the copy has read the tile: zero it for the next launch
+                        // (after the output, which the next layer waits for)
+                        for (int i = 0; i < 8 * 8; ++i)
+                            __stcg(acc4 + i * 32 + lane, make_float4(0.f, 0.f, 0.f, 0.f));
+                        BP_TRS(6);
                     }
                 }
+#undef BP_TRS
             }
         }
         if (has && slot == 0) {
@@ -1565,9 +1655,10 @@ SplitPlan plan_split(const DevLayout &dl, int64_t N, bool allow_split, const Imp
 #endif
     sp.units = sp.full + (sp.items - sp.full) * sp.split;
     if (sp.split > 1) {
-        const int64_t slots = (sp.items - sp.full) * sp.split;
-        sp.bytes = (size_t)((slots * kSlab * kNT * 4 + 255) / 256 * 256 +
-                            ((sp.items - sp.full) * 16 + 255) / 256 * 256);
+        // one fp32 accumulator tile per split item, then its arrival counters
+        const int64_t tiles = sp.items - sp.full;
+        sp.bytes = (size_t)((tiles * kSlab * kNT * 4 + 255) / 256 * 256 +
+                            (tiles * 16 + 255) / 256 * 256);
     }
     return sp;
 }
@@ -1609,13 +1700,13 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
                                             (int64_t)sp.units * kSlab * kNT * 4);
     }
     if (sp.split > 1) {
-        // partial tiles, then the arrival counters (zero on entry: the caller
-        // zero-fills a new workspace, and each item's last unit zeroes its
-        // counters again)
-        const int64_t slots = (sp.items - sp.full) * sp.split;
+        // accumulator tiles, then the arrival counters (zero on entry: the
+        // caller zero-fills a new workspace, and each item's last unit zeroes
+        // its tile and counters again)
+        const int64_t tiles = sp.items - sp.full;
         p.part = static_cast<float *>(ws);
         p.cnt = reinterpret_cast<int32_t *>(static_cast<uint8_t *>(ws) +
-                                            (slots * kSlab * kNT * 4 + 255) / 256 * 256);
+                                            (tiles * kSlab * kNT * 4 + 255) / 256 * 256);
     }
     p.ystage_bytes = 4 * 4096;     // per epilogue warp: two 2 KB boxes (GEMM) or one (conv)
     // shared memory: stages, output staging, barriers, index ring, and a copy of
@@ -1627,6 +1718,11 @@ cudaError_t launch_mma(const bp_packed &P, const DevLayout &dl, const void *X, i
     };
     p.stages = stages_for(0);
     if (p.stages < 2) return cudaErrorInvalidValue;
+    // a split or balanced launch's last unit stages four 32 KB quadrants of
+    // fp32 sums in the stage area
+    if ((sp.split > 1 || sp.balanced) &&
+        p.stages * (int64_t)(kWTileBytes + kXTileBytes) < 4 * (int64_t)kSlab / 4 * kNT * 4)
+        return cudaErrorInvalidValue;
     const int64_t kc_entries = p.num_slabs + 1;
     p.kc_cached = (kc_entries <= kMaxCachedKc && stages_for(kc_entries) == p.stages) ? kc_entries : 0;
     p.acc_cols = kNT;

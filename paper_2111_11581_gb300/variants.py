@@ -25,7 +25,7 @@ per-stage timeline of the tensor-core product.
         back-to-back MMAs while other warps copy into shared memory (bulk or
         cp.async rows).
 
-    python -m paper_2111_11581_gb300.variants trace [gemm|conv3x3|resnet50:LAYER|fc512] [DEFINE ...]
+    python -m paper_2111_11581_gb300.variants trace [gemm|conv3x3|resnet50:LAYER|vgg16:LAYER|fc512] [DEFINE ...]
         builds with BP_TRACE and prints CTA 0's clock64 timeline of one launch,
         L2 flushed before it, of the 4096^3 layer (or of the 3x3 CONV layer: N=128, C=F=128, 16x16,
         or of one ResNet-50 layer by name): per pipeline stage when the control
@@ -200,9 +200,12 @@ def _trace_in_process(lib: str, workload: str):
         pw = bp.pack(lay, W, bp.prune(lay, W, L.rate))
         Y = bp.gemm(pw, X)
         run = lambda: bp.gemm(pw, X, out=Y)  # noqa: E731
-    elif workload == "conv3x3" or workload.startswith("resnet50:"):
+    elif workload == "conv3x3" or workload.startswith(("resnet50:", "vgg16:")):
         if workload == "conv3x3":
             L, dt = inputs.conv3x3_128(), bp.F16
+        elif workload.startswith("vgg16:"):
+            name = workload.split(":", 1)[1]
+            L, dt = [l for l in inputs.vgg16_cifar() if l.name == name][0], bp.F16
         else:
             name = workload.split(":", 1)[1]
             L, dt = [l for l in inputs.resnet50_imagenet() if l.name == name][0], bp.BF16
@@ -291,6 +294,17 @@ def _trace_in_process(lib: str, workload: str):
         for k, r in enumerate(g[:8]):
             print(f"  {k}: {r[4] - t0:7d} {r[6] - r[4]:5d} {r[7] - r[6]:5d} {r[0] - r[7]:5d} "
                   f"{r[1] - r[0]:5d} {r[2] - r[1]:5d} {r[3] - r[2]:5d} {r[5] - r[3]:5d}")
+    sp = t[1000:1004]
+    if (sp[:, 3] > 0).any():
+        print("split epilogue per quadrant, CTA 0 (cycles after its start): reductions start, "
+              "issued, fenced, counted; item 0's last arrival (cycles after its sums landed): "
+              "output stores start, stored + tile zeroed, each group stored")
+        for q, r in enumerate(sp):
+            line = f"  q{q}: " + " ".join(f"{v - t0:7d}" if v > 0 else "      -" for v in r[:4])
+            if r[4] > 0:
+                gs = t[1004 + q]
+                line += " | " + " ".join(f"{v - r[4]:7d}" for v in list(r[5:7]) + list(gs) if v > 0)
+            print(line)
     g = rel[rel[:, 4] >= 0]
     if len(g):
         print(f"median gather issue -> tensor cores see the rows {np.median(g[:, 4] - g[:, 2]):.0f}")

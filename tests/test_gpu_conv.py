@@ -60,6 +60,12 @@ CASES = [
     # shared memory, 8-column groups spanning two images, a partial last group
     (24, 16, 3, 3, 11, 7, 7, 1, 1, BPU, 8, 4, 3.0, bp.BF16),
     (16, 24, 3, 3, 10, 6, 6, 1, 1, BPU, 8, 4, 3.0, bp.F16),
+    # Ho*Wo dividing 32: each 32-pixel output group holds whole images, written
+    # as 16-byte runs of 32 channels x Ho*Wo; few items, so the launches split
+    (256, 64, 3, 3, 40, 2, 2, 1, 1, BPU, 8, 4, 8.0, bp.BF16),   # 2x2, two slabs
+    (160, 32, 3, 3, 33, 1, 1, 1, 1, BPU, 8, 4, 3.0, bp.F16),    # 1x1 outputs, 32-row second slab
+    (64, 24, 3, 3, 50, 1, 2, 1, 1, BPU, 8, 4, 3.0, bp.BF16),    # 1x2
+    (96, 16, 3, 3, 45, 2, 4, 1, 1, BPU, 16, 8, 4.0, bp.F16),    # 2x4
 ]
 
 
