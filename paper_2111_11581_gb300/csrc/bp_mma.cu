@@ -208,6 +208,43 @@ __device__ __forceinline__ void cvt_any(const Params &p, const uint32_t (&r)[32]
     }
 }
 
+// Whole images of an NCHW output: lane r (channel row) of a 32-column group
+// holds Ho*Wo consecutive values of each of `imgs` images (packed pairs in pk,
+// Ho*Wo a power of two below 32) and writes them at yl + i * istride (its
+// channel's place in image i's run of 32 channels x Ho*Wo pixels), so that
+// every warp store is one contiguous piece of 64 Ho*Wo bytes.  Loops are
+// unrolled to their bound so that pk stays in registers.
+__device__ __forceinline__ void store_images(uint16_t *yl, int64_t istride, uint32_t HW, int imgs,
+                                             const uint32_t (&pk)[16]) {
+    if (HW == 1u) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+            if (i < imgs) yl[i * istride] = (uint16_t)(pk[i >> 1] >> (16 * (i & 1)));
+    } else if (HW == 2u) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+            if (i < imgs) *reinterpret_cast<uint32_t *>(yl + i * istride) = pk[i];
+    } else if (HW == 4u) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            if (i < imgs) *reinterpret_cast<uint2 *>(yl + i * istride) = make_uint2(pk[2 * i], pk[2 * i + 1]);
+    } else if (HW == 8u) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            if (i < imgs)
+                *reinterpret_cast<uint4 *>(yl + i * istride) =
+                    make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+    } else {
+#pragma unroll
+        for (int i = 0; i < 2; ++i)
+            if (i < imgs) {
+                uint4 *d = reinterpret_cast<uint4 *>(yl + i * istride);
+                d[0] = make_uint4(pk[8 * i], pk[8 * i + 1], pk[8 * i + 2], pk[8 * i + 3]);
+                d[1] = make_uint4(pk[8 * i + 4], pk[8 * i + 5], pk[8 * i + 6], pk[8 * i + 7]);
+            }
+    }
+}
+
 struct Smem {
     uint8_t *w;          // stages x kWTileBytes
     uint8_t *x;          // stages x kXTileBytes
@@ -1097,12 +1134,16 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem, int slot
             if (kConv) {
                 // NCHW output, pixel n = b*HoWo + hw is element (b, m, hw); the
                 // groups are stored in order, so (b, hw) advances by 32 pixels
-                // per call from the item's first pixel (one division per item)
+                // per call from the item's first pixel
                 const uint32_t bb = cbb, hw = chw;
-                chw += 32;
-                while (chw >= (uint32_t)p.HoWo) {
-                    chw -= (uint32_t)p.HoWo;
-                    ++cbb;
+                {
+                    // one division instead of a loop per image passed (images of
+                    // a few pixels pass eight per group; the loop's dependent
+                    // steps on the captured counters cost ~850 cycles on 2 x 2)
+                    const uint32_t nh = chw + 32u, HWu = (uint32_t)p.HoWo;
+                    const uint32_t adv = nh >= HWu ? nh / HWu : 0u;
+                    cbb += adv;
+                    chw = nh - adv * HWu;
                 }
                 if (stage_pair(pk, c0, n, bb, hw)) return;
                 if (p.ytma && hw + 32 <= (uint32_t)p.HoWo && c0 + 32 <= t.ncols && (hw & 7u) == 0) {
@@ -1139,64 +1180,28 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem, int slot
                 // boundary or the tile's end: stage the 32 x 32 box (lane = channel row, 80-byte
                 // rows), then write it with lanes along the pixels, one
                 // coalesced 64-byte store per channel
+                const int rmax = (int)min((int64_t)32, t.rows - row0);
+                // Ho*Wo dividing 32 and the group starting at an image: the group
+                // holds whole images, and each image's 32 channels x Ho*Wo pixels
+                // are one run of 64 Ho*Wo contiguous bytes of the NCHW output,
+                // written from registers (store_images).  (One 2-byte store per
+                // lane and channel, pixels across lanes, took ~3,000 cycles per
+                // group on 2 x 2 images.)
+                {
+                    const uint32_t HW = (uint32_t)p.HoWo;
+                    const int64_t cols = min((int64_t)32, t.n0 + t.ncols - n);
+                    if (hw == 0u && HW < 32u && (32u % HW) == 0u && rmax == 32 && cols > 0 &&
+                        cols % HW == 0) {
+                        store_images(p.Y + ((int64_t)bb * p.M + t.slab * kSlab + row0 + lane) * HW,
+                                     (int64_t)p.M * HW, HW, (int)(cols / HW), pk);
+                        return;
+                    }
+                }
                 uint8_t *box = stgp;
                 // the box overlaps both TMA staging boxes: their stores must
                 // have read them
                 if (p.ytma && lane == 0) bulk_wait_read<0>();
                 __syncwarp();                      // the previous box has been read
-                const int rmax = (int)min((int64_t)32, t.rows - row0);
-                // Ho*Wo dividing 32 and the group starting at an image: the group
-                // holds whole images, and each image's 32 channels x Ho*Wo pixels
-                // are one run of 64 Ho*Wo contiguous bytes of the NCHW output
-                // (16-byte aligned when M is a multiple of 8).  Lane r (channel
-                // row) puts its Ho*Wo values of image i at (i * 32 + r) * Ho*Wo
-                // of the staging area, which thus holds the runs back to back,
-                // and the warp copies them out with 16-byte loads and stores.
-                // (One 2-byte store per lane and channel took ~3,000 cycles per
-                // group on 2 x 2 images.)
-                {
-                    const uint32_t HW = (uint32_t)p.HoWo;
-                    const int64_t cols = min((int64_t)32, t.n0 + t.ncols - n);
-                    if (hw == 0u && HW < 32u && (32u % HW) == 0u && rmax == 32 && (p.M & 7) == 0 &&
-                        cols > 0 && cols % HW == 0) {
-                        const int lg = __ffs((int)HW) - 1;            // HW is a power of two
-                        const uint32_t sb = smem_u32(box);
-                        if (lg == 0) {
-#pragma unroll
-                            for (int i = 0; i < 32; ++i)
-                                st_shared_u16(sb + (i * 32 + lane) * 2, (uint16_t)(pk[i >> 1] >> (16 * (i & 1))));
-                        } else if (lg == 1) {
-#pragma unroll
-                            for (int i = 0; i < 16; ++i) st_shared_u32(sb + (i * 64 + lane * 2) * 2, pk[i]);
-                        } else if (lg == 2) {
-#pragma unroll
-                            for (int i = 0; i < 8; ++i)
-                                st_shared_v2(sb + (i * 128 + lane * 4) * 2, pk[2 * i], pk[2 * i + 1]);
-                        } else if (lg == 3) {
-#pragma unroll
-                            for (int i = 0; i < 4; ++i)
-                                st_shared_v4(sb + (i * 256 + lane * 8) * 2,
-                                             make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]));
-                        } else {
-#pragma unroll
-                            for (int i = 0; i < 2; ++i)
-#pragma unroll
-                                for (int h = 0; h < 2; ++h)
-                                    st_shared_v4(sb + (i * 512 + lane * 16 + h * 8) * 2,
-                                                 make_uint4(pk[8 * i + 4 * h], pk[8 * i + 4 * h + 1],
-                                                            pk[8 * i + 4 * h + 2], pk[8 * i + 4 * h + 3]));
-                        }
-                        __syncwarp();
-                        const int total = (int)cols * 4;               // 16-byte pieces
-                        uint16_t *ybase = p.Y + ((int64_t)bb * p.M + t.slab * kSlab + row0) * HW;
-                        for (int k = lane; k < total; k += 32) {
-                            const int i = k >> (lg + 2), off = k & ((4 << lg) - 1);
-                            *reinterpret_cast<uint4 *>(ybase + (int64_t)i * p.M * HW + off * 8) =
-                                ld_shared_v4(sb + k * 16);
-                        }
-                        return;
-                    }
-                }
 #pragma unroll
                 for (int ch = 0; ch < 4; ++ch)
                     st_shared_v4(smem_u32(box + lane * 80 + ch * 16),
@@ -1347,11 +1352,10 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem, int slot
                     store(pk, 32 * g);
                     if (kConv && gn != g + 1) {
                         // skipped pairs (their pixels) before the next group
-                        chw += 32u * (uint32_t)(gn - g - 1);
-                        while (chw >= (uint32_t)p.HoWo) {
-                            chw -= (uint32_t)p.HoWo;
-                            ++cbb;
-                        }
+                        const uint32_t nh = chw + 32u * (uint32_t)(gn - g - 1), HWu = (uint32_t)p.HoWo;
+                        const uint32_t adv = nh >= HWu ? nh / HWu : 0u;
+                        cbb += adv;
+                        chw = nh - adv * HWu;
                     }
                     if (has && gn < G) tmem_ld_wait();
                     BP_TRE(5);
@@ -1425,6 +1429,19 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem, int slot
                     } else {
                         BP_TRS(5);
                         const float4 *sm4 = reinterpret_cast<const float4 *>(qbuf) + lane;
+                        // an NCHW output whose groups hold whole images: the runs
+                        // are written here directly (the generic store path
+                        // reloads its spilled per-item state every group, ~800
+                        // cycles of round trips per group)
+                        const uint32_t HWw = kConv ? (uint32_t)p.HoWo : 0u;
+                        const bool whole = kConv && HWw < 32u && (32u % HWw) == 0u &&
+                                           (uint32_t)t.n0 % HWw == 0u && row0 + 32 <= t.rows;
+                        uint16_t *yw = nullptr;
+                        int64_t iw = 0;
+                        if (whole) {
+                            iw = (int64_t)p.M * HWw;
+                            yw = p.Y + (((int64_t)t.n0 / HWw) * p.M + t.slab * kSlab + row0 + lane) * HWw;
+                        }
                         for (int g = 0; g < G; ++g) {
 #pragma unroll
                             for (int e = 0; e < 8; ++e) {
@@ -1435,7 +1452,12 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem, int slot
                                 r[4 * e + 3] = __float_as_uint(v.w);
                             }
                             pack(r, pk);
-                            store(pk, 32 * g);
+                            if (whole) {
+                                const int cols = (int)min((int64_t)32, t.ncols - 32 * g);
+                                store_images(yw + (int64_t)(32 / HWw) * g * iw, iw, HWw, cols / (int)HWw, pk);
+                            } else {
+                                store(pk, 32 * g);
+                            }
 #ifdef BP_TRACE
                             if (lane == 0 && g < 8 && t.j == 0)
                                 bp::g_trace[(1004 + q) * bp::kTraceEvents + g] = clock64();
