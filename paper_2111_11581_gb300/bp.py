@@ -90,6 +90,11 @@ def load(path: str = LIB_PATH):
         for name, (res, args) in sig.items():
             f = getattr(lib, name)
             f.restype, f.argtypes = res, args
+        # BP_WATCHDOG_NS: the bound on every kernel wait (bp_set_watchdog_ns),
+        # e.g. raised under a profiler that replays each launch many times
+        wd = os.environ.get("BP_WATCHDOG_NS")
+        if wd:
+            lib.bp_set_watchdog_ns(int(float(wd)))
         _lib = lib
         return lib
 

@@ -192,23 +192,27 @@ __global__ void __launch_bounds__(320, 1) probe(const __grid_constant__ PP p) {
         // waits spin on test_wait; 512 / 1024 the gather warps poll for a free
         // stage from lane 0 only / with a back-off sleep; 2048 the consumer
         // releases a stage before its hold; 4096 it holds by sleeping in a
-        // loop, 8192 with one sleep, 16384 with a chain of FMAs.  Cycles per
-        // 64-row chunk.
+        // loop, 8192 with one sleep, 16384 with a chain of FMAs; 32768 two
+        // chunks per stage (128 rows, 32 KB tile, 1,024-cycle hold, at most 2
+        // stages).  Cycles per 64-row chunk.
         const int S = p.nthreads;
         const bool half = (p.flags & 32) != 0, all8 = (p.flags & 16) != 0;
-        const int rows_per = half ? 32 : 64;
-        const uint32_t wbytes = half ? 8192u : 16384u, xbytes = half ? 16384u : 32768u;
-        const uint32_t xcn = half ? 4096u : 8192u;          // bytes per 64-token group
+        const bool dbl = (p.flags & 32768) != 0;          // two chunks per stage (128 rows)
+        const int rows_per = half ? 32 : dbl ? 128 : 64;
+        const uint32_t wbytes = half ? 8192u : dbl ? 32768u : 16384u;
+        const uint32_t xbytes = half ? 16384u : dbl ? 65536u : 32768u;
+        const uint32_t xcn = half ? 4096u : dbl ? 16384u : 8192u;   // bytes per 64-token group
         uint64_t *full = bars + 16, *wfull = bars + 24, *empty = bars + 32;
         const uint8_t *X = p.W;
         const int64_t n0 = (p.flags & 8) ? 0 : (int64_t)(blockIdx.x % 16) * 256;
         auto row_of = [&](int c, int i) -> int64_t {
             const uint32_t h = (uint32_t)(c * 2654435761u) ^ (uint32_t)(blockIdx.x * 40503u) ^ (uint32_t)(i * 97u);
             if (p.flags & 4) return (int64_t)((h * 2246822519u) >> 20);                 // 0 .. 4095
-            const int64_t b = (int64_t)(((uint32_t)(c * 2654435761u) ^ (uint32_t)(blockIdx.x * 40503u)) % 3840u);
+            const int64_t b = (int64_t)(((uint32_t)(c * 2654435761u) ^ (uint32_t)(blockIdx.x * 40503u)) %
+                                        (uint32_t)(4096 - 4 * rows_per));
             return b + 4 * i + ((h >> 7) & 3);                                            // < 4096
         };
-        const int chunks = half ? 2 * p.iters : p.iters;
+        const int chunks = half ? 2 * p.iters : dbl ? p.iters / 2 : p.iters;
         // flag 256: every wait spins on mbarrier.test_wait instead of try_wait
         const bool spin = (p.flags & 256) != 0;
         auto wait = [&](uint64_t *bar, uint32_t parity) -> bool {
@@ -306,7 +310,7 @@ __global__ void __launch_bounds__(320, 1) probe(const __grid_constant__ PP p) {
             if (!ok) atomicOr(p.err, 512u);
         } else if (warp == 9 && lane == 0) {
             bool ok = true;
-            const long long hold = half ? 256 : 512;
+            const long long hold = half ? 256 : dbl ? 1024 : 512;
             const unsigned long long t0 = clock64();
             for (int c = 0; c < chunks && ok; ++c) {
                 const int s = c % S;
@@ -486,8 +490,9 @@ int main(int argc, char **argv) {
     if (N < 16 || N > 256 || N % 16 || nth < 1 || nth > 8 || iters < 1 || test < 0 || test > 7)
         return 2;
     if (test != 4 && test != 5 && test != 6 && test != 7 && nth > 6) return 2;
-    if (test == 7 && (nth < 2 || nth > ((flags & 32) ? 8 : 4) || (N != 128 && N != 256) || flags < 0 ||
-                      flags > 32767 || (flags & 192) == 192 || ((flags & 64) && nth < 4))) return 2;
+    if (test == 7 && (nth < 2 || nth > ((flags & 32) ? 8 : (flags & 32768) ? 2 : 4) ||
+                      (N != 128 && N != 256) || flags < 0 || flags > 65535 || (flags & 192) == 192 ||
+                      ((flags & 64) && nth < 4) || ((flags & 32) && (flags & 32768)))) return 2;
     if (test == 5 && (flags < 0 || flags > 64 || (flags & (flags - 1)) || (N & (N - 1)))) return 2;
     if (test == 6 && (nth > 6 || flags < 0 || flags > 2 || N < 64 || (N & (N - 1)))) return 2;
     if (test == 4 && nth != 2 && nth != 4 && nth != 8) return 2;   // MMAs per group
