@@ -205,11 +205,14 @@ __global__ void __launch_bounds__(320, 1) probe(const __grid_constant__ PP p) {
         uint64_t *full = bars + 16, *wfull = bars + 24, *empty = bars + 32;
         const uint8_t *X = p.W;
         const int64_t n0 = (p.flags & 8) ? 0 : (int64_t)(blockIdx.x % 16) * 256;
-        auto row_of = [&](int c, int i) -> int64_t {
+        // a chunk's first row (one division per chunk, outside the row loop)
+        const uint32_t span = (uint32_t)(4096 - 4 * rows_per);
+        auto base_of = [&](int c) -> int64_t {
+            return (int64_t)(((uint32_t)(c * 2654435761u) ^ (uint32_t)(blockIdx.x * 40503u)) % span);
+        };
+        auto row_of = [&](int c, int64_t b, int i) -> int64_t {
             const uint32_t h = (uint32_t)(c * 2654435761u) ^ (uint32_t)(blockIdx.x * 40503u) ^ (uint32_t)(i * 97u);
             if (p.flags & 4) return (int64_t)((h * 2246822519u) >> 20);                 // 0 .. 4095
-            const int64_t b = (int64_t)(((uint32_t)(c * 2654435761u) ^ (uint32_t)(blockIdx.x * 40503u)) %
-                                        (uint32_t)(4096 - 4 * rows_per));
             return b + 4 * i + ((h >> 7) & 3);                                            // < 4096
         };
         const int chunks = half ? 2 * p.iters : dbl ? p.iters / 2 : p.iters;
@@ -265,8 +268,9 @@ __global__ void __launch_bounds__(320, 1) probe(const __grid_constant__ PP p) {
                 if (rec) tr[0] = clock64();
                 const uint32_t xs = smem_u32(base + S * wbytes + s * xbytes);
                 if (lane * 8 < p.N) {
+                    const int64_t b = base_of(c);
                     for (int r = gw; r < rows_per; r += gwarps) {
-                        const int64_t row = row_of(c, r);
+                        const int64_t row = row_of(c, b, r);
                         cp_async_16_full(xs + cn * xcn + r * 128 + ((jj ^ (r & 7)) << 4),
                                          X + (row * 4096 + n0 + lane * 8) * 2);
                     }
