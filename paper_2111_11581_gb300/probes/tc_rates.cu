@@ -319,10 +319,23 @@ __global__ void __launch_bounds__(320, 1) probe(const __grid_constant__ PP p) {
             for (int c = 0; c < chunks && ok; ++c) {
                 const int s = c % S;
                 const uint32_t ph = (uint32_t)((c / S) & 1);
-                ok = wait(&wfull[s], ph) && wait(&full[s], ph);
+                unsigned long long *tq = p.out + 4 * gridDim.x + 448 + (int64_t)c * 4;
+                if (blockIdx.x == 0 && c < 64) tq[0] = clock64();
+                ok = wait(&wfull[s], ph);
+                if (blockIdx.x == 0 && c < 64) tq[1] = clock64();
+                ok = ok && wait(&full[s], ph);
+                if (blockIdx.x == 0 && c < 64) tq[2] = clock64();
                 if (!ok) break;
                 unsigned long long *tr = p.out + 4 * gridDim.x + (int64_t)c * 4;
                 if (blockIdx.x == 0 && c < 64) tr[2] = clock64();
+                // CTA 0: was the next stage's data already complete before this
+                // stage's hold began (1), or only later (0)?
+                if (blockIdx.x == 0 && c < 64 && c + 1 < chunks) {
+                    const int s1 = (c + 1) % S;
+                    const uint32_t ph1 = (uint32_t)(((c + 1) / S) & 1);
+                    p.out[4 * gridDim.x + 384 + c] =
+                        (mbar_test_wait(&wfull[s1], ph1) && mbar_test_wait(&full[s1], ph1)) ? 1ull : 0ull;
+                }
                 // flag 2048: release the stage first, then hold (the hold then
                 // delays only the consumer); flag 4096: hold by sleeping
                 if (p.flags & 2048) mbar_arrive(&empty[s]);
@@ -341,11 +354,12 @@ __global__ void __launch_bounds__(320, 1) probe(const __grid_constant__ PP p) {
                 }
                 if (blockIdx.x == 0 && c < 64) tr[3] = clock64();
                 if (!(p.flags & 2048)) mbar_arrive(&empty[s]);
+                if (blockIdx.x == 0 && c < 64) tq[3] = clock64();
             }
             p.out[blockIdx.x] = clock64() - t0;
             if (!ok) atomicOr(p.err, 1024u);
         }
-    } else if (p.test == 4) {    } else if (p.test == 4) {
+    } else if (p.test == 4) {
         // back-to-back MMAs in groups of `per` (2, 4 or 8), a commit after each
         // group (flag 2: none), groups alternating between two accumulators
         // (flag 1); nothing waits on the commits until the end
@@ -510,14 +524,14 @@ int main(int argc, char **argv) {
     cudaMemset(W, 0, wbytes);
     unsigned long long *out = nullptr;
     unsigned *err = nullptr;
-    cudaMalloc(&out, (4 * sms + 384) * 8);
+    cudaMalloc(&out, (4 * sms + 704) * 8);
     cudaMalloc(&err, 4);
     cudaMemset(err, 0, 4);
     PP p{test, iters, N, nth, flags, W, out, err};
     const int smem = 1024 + kData + 1024;
     cudaFuncSetAttribute(probe, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     for (int w = 0; w < 3; ++w) {
-        cudaMemset(out, 0, (4 * sms + 384) * 8);
+        cudaMemset(out, 0, (4 * sms + 704) * 8);
         probe<<<sms, 320, smem>>>(p);
         if (cudaDeviceSynchronize() != cudaSuccess) {
             printf("cuda error\n");
@@ -551,8 +565,18 @@ int main(int argc, char **argv) {
                nth, N, flags, avg / iters, herr);
         if (getenv("TC_RING_TRACE")) {
             // CTA 0: per chunk, producer saw the stage free / issued, consumer saw the data / released
-            std::vector<unsigned long long> t(384);
-            cudaMemcpy(t.data(), out + 4 * sms, 384 * 8, cudaMemcpyDeviceToHost);
+            std::vector<unsigned long long> t(704);
+            cudaMemcpy(t.data(), out + 4 * sms, 704 * 8, cudaMemcpyDeviceToHost);
+            // consumer: release -> (loop) -> wfull wait done -> full wait done
+            for (int c = 10; c < 14; ++c)
+                printf("  consumer chunk %d: arrive %lld, to next wait start %lld, wfull wait %lld, full wait %lld\n", c,
+                       (long long)(t[448 + 4 * c + 3] - t[4 * c + 3]),
+                       (long long)(t[448 + 4 * (c + 1)] - t[448 + 4 * c + 3]),
+                       (long long)(t[448 + 4 * (c + 1) + 1] - t[448 + 4 * (c + 1)]),
+                       (long long)(t[448 + 4 * (c + 1) + 2] - t[448 + 4 * (c + 1) + 1]));
+            int ready = 0;
+            for (int c = 8; c < 40; ++c) ready += (int)t[384 + c];
+            printf("  next stage already complete before the hold: %d of 32 chunks\n", ready);
             const unsigned long long z = t[2];
             for (int c = 0; c < 32; ++c)
                 printf("  chunk %2d: free %7lld issued %7lld data %7lld released %7lld; warps issued "
