@@ -322,6 +322,28 @@ __device__ __forceinline__ void umma_f16_ss(uint32_t d_tmem, uint64_t a_desc, ui
         : "memory");
 }
 
+// Four MMAs of K=16 into one accumulator, issued back to back from one asm
+// block: A and B descriptors advance by da / db per step, and the first MMA
+// accumulates iff `accumulate` (the later ones always).  The descriptors are
+// formed before the first issue, so no other instruction sits between the
+// MMAs: the tensor pipe takes the next MMA only as the previous one drains,
+// and each instruction placed between two MMAs delays the stream.
+__device__ __forceinline__ void umma_f16_ss_x4(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                               uint64_t da, uint64_t db, uint32_t idesc,
+                                               uint32_t accumulate) {
+    const uint64_t a1 = a_desc + da, a2 = a_desc + 2 * da, a3 = a_desc + 3 * da;
+    const uint64_t b1 = b_desc + db, b2 = b_desc + 2 * db, b3 = b_desc + 3 * db;
+    asm volatile(
+        "{\n .reg .pred p, q;\n setp.ne.b32 p, %10, 0;\n setp.eq.b32 q, %10, %10;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %5, %9, p;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %2, %6, %9, q;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %3, %7, %9, q;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %4, %8, %9, q;\n}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(a1), "l"(a2), "l"(a3), "l"(b_desc), "l"(b1), "l"(b2), "l"(b3), "r"(idesc),
+        "r"(accumulate)
+        : "memory");
+}
+
 // Arrive once on `bar` when every tcgen05.mma issued so far by this thread is done.
 __device__ __forceinline__ void umma_commit(uint64_t *bar) {
     asm volatile(

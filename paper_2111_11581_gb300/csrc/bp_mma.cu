@@ -87,6 +87,22 @@ constexpr int kMaxStages = 8;
 constexpr int kWin = 16;               // chunk records per shared-memory window
 constexpr int kWinBufs = 3;            // windows in shared memory (one being filled ahead)
 constexpr uint32_t kWinBytes = kWin * kMetaBytes;
+constexpr uint32_t kCwinBytes = 256;        // one Window record (size checked below)
+constexpr int kWmeta = 6;                   // int64 words of a window descriptor
+// Window descriptor flags (Smem::wmeta word 3).
+constexpr uint32_t kWinFirst = 1;       // the window starts its unit
+constexpr uint32_t kWinLast = 2;        // the window ends its unit
+constexpr uint32_t kWinFinal = 4;       // the unit is the CTA's final one
+// Stage flags (Smem::sflag): how the stage's activations were loaded and where
+// its chunk sits in its work unit.  Only the scheduler warp decodes work units
+// (into window descriptors, Smem::wmeta, which the control thread and the
+// gather warps follow); the tensor-core thread follows the stage flags the
+// control thread sets.
+constexpr uint32_t kStageTma = 1;       // activations loaded by TMA (no proxy fence needed)
+constexpr uint32_t kStageFirst = 2;     // first chunk of its unit: a fresh accumulator
+constexpr uint32_t kStageLast = 4;      // last chunk of its unit: the accumulator is complete
+constexpr uint32_t kStageFinal = 8;     // last chunk of the CTA's final unit
+constexpr uint32_t kStageEnd = 16;      // no more chunks: the stage holds nothing
 constexpr int64_t kMaxCachedKc = 2048; // kc_ptr entries kept in shared memory at most
 constexpr int64_t kMaxSmem = 232448;   // dynamic shared memory per CTA (227 KB)
 constexpr int kNT = 256;               // activation columns per tile at most (the MMA's N)
@@ -98,23 +114,23 @@ constexpr int kGatherWarps = 8;
 constexpr int kCtrlWarp = 8;
 constexpr int kMmaWarp = 9;
 constexpr int kEpiWarp0 = 10;
-constexpr int kThreads = (kEpiWarp0 + 4) * 32;
-// The gather warps form kGatherGroups groups.  By default the groups take
-// turns: group g gathers the chunks whose sequence number is g modulo
-// kGatherGroups, so one group issues copies while another waits for its next
-// stage.  With BP_GATHER_HALVES group h gathers rows 32h .. 32h+31 of every
-// chunk instead, each half signalling a barrier of its own, and the tensor
-// cores start on the first half while the second is still landing.
+constexpr int kSchedWarp = kEpiWarp0 + 4;   // decodes the windows ahead (lane 0)
+constexpr int kThreads = (kSchedWarp + 1) * 32;
+// The gather warps form kGatherGroups groups that take turns: group g
+// gathers the chunks whose sequence number is g modulo kGatherGroups, so one
+// group issues copies while another waits for its next stage.
 constexpr int kGatherGroups = 2;
 constexpr int kGroupWarps = kGatherWarps / kGatherGroups;
-#ifdef BP_GATHER_HALVES
-constexpr int kRowsPerWarp = 32 / kGroupWarps;      // list positions per warp and chunk
-constexpr int kFullPerStage = 2;
-#else
 constexpr int kRowsPerWarp = 64 / kGroupWarps;      // list positions per warp and chunk
-constexpr int kFullPerStage = 1;
-#endif
 constexpr uint32_t kGroupThreads = kGroupWarps * 32;
+// One barrier per stage tells the tensor-core thread that the stage is
+// loaded: the control thread arrives once (with the stage's TMA byte count)
+// and the chunk's gather group kGroupThreads times, each thread when its
+// copies have landed, or lane 0 of each warp for its warp when the chunk has
+// a load plan (TMA brings its rows).  A second barrier for the gathered rows
+// costs the tensor-core thread another wait per chunk, 100-150 cycles even
+// when its phase has already completed.
+constexpr uint32_t kStageArrivals = kGroupThreads + 1;
 
 struct Params {
     CUtensorMap ymap;       // output, box 32 x 32 (x 1), 64-byte swizzle: GEMM Y as a 2-D
@@ -249,9 +265,8 @@ struct Smem {
     uint8_t *w;          // stages x kWTileBytes
     uint8_t *x;          // stages x kXTileBytes
     uint8_t *ystage;     // GEMM: 4 epilogue warps x 2 buffers x 2 KB
-    uint64_t *full;      // [stages] gathered activation rows landed (256 arrivals; used by
-                         // chunks without a load plan only)
-    uint64_t *wfull;     // [stages] weight tile (+ TMA-loaded activations) landed
+    uint64_t *wfull;     // [stages] the stage is loaded: weight tile, TMA-loaded activations
+                         // and gathered rows (kStageArrivals arrivals + the TMA bytes)
     uint64_t *empty;     // [stages] tensor cores done with the stage
     uint64_t *tfull;     // [2] accumulator ready for the epilogue
     uint64_t *tempty;    // [2] accumulator drained
@@ -260,11 +275,22 @@ struct Smem {
     uint64_t *ffull;     // the CTA's final item's accumulator is complete (single use)
     uint64_t *pfull;     // [kWinBufs] a window of chunk records landed (TMA byte count)
     uint64_t *pempty;    // [kWinBufs] the gather warps and the control thread are done with it
-    uint32_t *skind;     // [stages] 1: the stage's activations come from TMA tile loads
+    uint32_t *sflag;     // [stages] what the stage holds (kStage* bits), set by the control
+                         // thread before its arrival on wfull
     uint32_t *tmem_base;
     int *abort_flag;
+    int64_t *gprog;      // [kGatherWarps + 1] per gather warp: 1 + the sequence number of the
+                         // last chunk it arrived for; [kGatherWarps]: warps out of their loop
     int64_t *skv;        // [4] balanced launch: chunk position of item sk_i0, chunks from
                          // there on, this CTA's range [lo, hi) (set in the prologue)
+    int64_t *wmeta;      // [kWinBufs][kWmeta] per window buffer, written before the
+                         // arrival on pfull: chunks in the window (0: no more windows),
+                         // the tile's first token column, the window's first chunk
+                         // position, kWin* flags, and the implicit convolution's first
+                         // output row and image
+    uint8_t *cwin;       // [sizeof(Window)] window 1, decoded before the dependency wait
+    int *pre;            // weight tiles requested before the dependency wait (-1: the
+                         // first window was not requested then)
     uint8_t *win;        // [kWinBufs][kWinBytes] chunk records of the current windows
     int64_t *kc;         // [kc_cached] copy of kc_ptr, or nullptr
 };
@@ -277,8 +303,7 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
     s.x = base + p.stages * kWTileBytes;
     s.ystage = s.x + p.stages * kXTileBytes;
     uint8_t *b = s.ystage + p.ystage_bytes;
-    s.full = reinterpret_cast<uint64_t *>(b);
-    s.wfull = s.full + kFullPerStage * p.stages;
+    s.wfull = reinterpret_cast<uint64_t *>(b);
     s.empty = s.wfull + p.stages;
     s.tfull = s.empty + p.stages;
     s.tempty = s.tfull + 2;
@@ -287,13 +312,17 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
     s.ffull = s.fixbar + 4;
     s.pfull = s.ffull + 1;
     s.pempty = s.pfull + kWinBufs;
-    s.skind = reinterpret_cast<uint32_t *>(s.pempty + kWinBufs);
-    s.tmem_base = s.skind + p.stages;
+    s.sflag = reinterpret_cast<uint32_t *>(s.pempty + kWinBufs);
+    s.tmem_base = s.sflag + p.stages;
     s.abort_flag = reinterpret_cast<int *>(s.tmem_base + 1);
-    s.skv = reinterpret_cast<int64_t *>(
+    s.gprog = reinterpret_cast<int64_t *>(
         (reinterpret_cast<uintptr_t>(s.abort_flag + 1) + 7) & ~static_cast<uintptr_t>(7));
+    s.skv = s.gprog + kGatherWarps + 1;
+    s.wmeta = s.skv + 4;
+    s.cwin = reinterpret_cast<uint8_t *>(s.wmeta + kWmeta * kWinBufs);
+    s.pre = reinterpret_cast<int *>(s.cwin + kCwinBytes);
     // TMA bulk copies need a 16-byte-aligned destination: round up to 128 bytes
-    const uintptr_t after = reinterpret_cast<uintptr_t>(s.skv + 4);
+    const uintptr_t after = reinterpret_cast<uintptr_t>(s.pre + 2);
     s.win = reinterpret_cast<uint8_t *>((after + 127) & ~static_cast<uintptr_t>(127));
     s.kc = p.kc_cached ? reinterpret_cast<int64_t *>(s.win + kWinBufs * kWinBytes) : nullptr;
     return s;
@@ -301,7 +330,8 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, const Params &p) {
 
 size_t smem_bytes(int64_t stages, uint32_t ystage_bytes, int64_t kc_cached) {
     return 1024 + (size_t)stages * (kWTileBytes + kXTileBytes) + ystage_bytes +
-           ((2 + kFullPerStage) * (size_t)stages + 10 + 2 * kWinBufs) * 8 + 4 * (size_t)stages + 8 + 8 + 32 + 128 +
+           (2 * (size_t)stages + 10 + 2 * kWinBufs) * 8 + 4 * (size_t)stages + 8 + 8 +
+           8 * (kGatherWarps + 1) + 32 + 8 * kWmeta * kWinBufs + kCwinBytes + 8 + 128 +
            (size_t)kWinBufs * kWinBytes + 8 * (size_t)kc_cached;
 }
 
@@ -494,6 +524,7 @@ struct Window {
     }
     __device__ __forceinline__ bool valid(const Params &) const { return ui.valid(); }
 };
+static_assert(sizeof(Window) <= kCwinBytes, "window record");
 
 // The CTA's final item: its last work unit, when it has chunks and the launch
 // splits nothing.  By the time its accumulator is complete every pipeline
@@ -514,35 +545,30 @@ __device__ __forceinline__ int plan_loads(const uint8_t *rec) {
 // ------------------------------------------------------------------ gather warps
 __device__ void gather_warps(const Params &p, const Smem &s) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
-    Window win;
-    win.first(p, kcp, s.skv);
     const int group = warp / kGroupWarps, gw = warp % kGroupWarps;
     const int nst = (int)p.stages;
-#ifdef BP_GATHER_HALVES
-    constexpr int kStep = 1;    // every chunk
-    const int rbase = 32 * group;
-    int gst = 0;
-#else
     constexpr int kStep = kGatherGroups;
     constexpr int rbase = 0;
     int gst = group;            // stage of this group's next chunk (sequence number group + 2i)
-#endif
     uint32_t gph = 0;
     int64_t count = 0, wseq = 0;
     bool ok = true;
-    for (; win.valid(p) && ok; win.next(p, kcp), ++wseq) {
+    for (;; ++wseq) {
         const int buf = (int)(wseq % kWinBufs);
         // outcomes of waits are made warp-uniform, so the warp leaves the loop as one
         ok = __all_sync(0xffffffffu, mbar_wait(&s.pfull[buf], (uint32_t)((wseq / kWinBufs) & 1),
                                               p.watchdog_ns, abort_flag));
         if (!ok) break;
         if (warp == 0 && lane == 0) BP_TR(256 + wseq, 3);
+        // the window's descriptor, written by the control thread before its
+        // arrival on pfull
+        const int64_t wcnt = s.wmeta[kWmeta * buf], wn0 = s.wmeta[kWmeta * buf + 1];
+        if (wcnt == 0) break;       // no more windows
         const uint8_t *recs = s.win + buf * kWinBytes;
         // the tile's token columns: 16 bytes (8 columns) per lane, lanes past
         // the tile's width idle
-        const int64_t n = win.t.n0 + lane * 8;
+        const int64_t n = wn0 + lane * 8;
         const uint32_t nb =
             (lane * 8 < p.nt && n < p.N) ? (uint32_t)min((int64_t)16, (p.N - n) * 2) : 0u;
         const uint16_t *xcol = p.X;
@@ -565,16 +591,12 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
             for (int i = 0; i < kRowsPerWarp; ++i) ix[i] = l[rbase + gw + kGroupWarps * i];
         };
         const int64_t base = count;         // sequence number of the window's first chunk
-#ifdef BP_GATHER_HALVES
-        int64_t j = 0;
-#else
         int64_t j = (group - base % kGatherGroups + kGatherGroups) % kGatherGroups;
-#endif
-        if (j < win.cnt) fetch(j, idx, tma);
-        for (; j < win.cnt; j += kStep) {
+        if (j < wcnt) fetch(j, idx, tma);
+        for (; j < wcnt; j += kStep) {
             int32_t nidx[kRowsPerWarp];
             bool ntma = false;
-            if (j + kStep < win.cnt) fetch(j + kStep, nidx, ntma);
+            if (j + kStep < wcnt) fetch(j + kStep, nidx, ntma);
             const int64_t seq = base + j;
             // stage = seq mod stages, phase = its ring pass parity (kept
             // incrementally: a 64-bit division per chunk sits on the issue path)
@@ -586,15 +608,17 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
                 gph ^= 1u;
             }
             const bool drop = blockIdx.x == 0 && seq == p.drop_stage;
-            // A planned chunk is loaded and signalled by the control thread; the
-            // group still waits for its stage (lane 0 alone), which keeps it at
-            // most one phase of the stage barriers ahead of the tensor cores.
+            // A planned chunk is loaded by the control thread; the group still
+            // waits for its stage (lane 0 alone) and arrives on it, lane 0 for
+            // the warp, which keeps it at most one phase of the stage barriers
+            // ahead of the tensor cores.
             ok = __all_sync(0xffffffffu,
                             (!tma || lane == 0)
                                 ? mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)
                                 : true);
             if (!ok) break;
             if (gw == 0 && lane == 0) BP_TR(seq, 1);
+            if (tma && !drop && lane == 0) mbar_arrive_cnt(&s.wfull[stage], 32);
             if (!tma && !drop) {
                 // 64 rows x nt columns: one warp instruction per row segment
                 const uint32_t xs = smem_u32(s.x + stage * kXTileBytes);
@@ -618,37 +642,60 @@ __device__ void gather_warps(const Params &p, const Smem &s) {
                         }
                     }
                 }
-                // Signal the stage once this thread's copies have landed, without
+                // Arrive on the stage once this thread's copies have landed, without
                 // blocking.  The tile was written through the generic proxy; the
                 // tensor-core thread orders it before its async-proxy reads with a
                 // proxy fence after acquiring the barrier.
-                cp_async_arrive_noinc(&s.full[kFullPerStage * stage + (kFullPerStage - 1) * group]);
+                cp_async_arrive_noinc(&s.wfull[stage]);
                 if (gw == 0 && lane == 0) BP_TR(seq, 2);
             }
+            // progress for the control thread's unwinding (after the arrivals)
+            if (lane == 0) *reinterpret_cast<volatile int64_t *>(&s.gprog[warp]) = seq + 1;
 #pragma unroll
             for (int i = 0; i < kRowsPerWarp; ++i) idx[i] = nidx[i];
             tma = ntma;
         }
-        count = base + win.cnt;
+        count = base + wcnt;
         if (!ok) break;
         __syncwarp();        // the lanes' reads of the window precede lane 0's release
         if (lane == 0) mbar_arrive(&s.pempty[buf]);
     }
     if (!ok) raise_timeout(p, s);
     cp_async_wait_all();
+    __syncwarp();
+    if (lane == 0) {
+        __threadfence_block();
+        atomicAdd(reinterpret_cast<unsigned long long *>(&s.gprog[kGatherWarps]), 1ull);
+    }
 }
 
 // ------------------------------------------------------------------ control thread
 struct WindowFiller {
-    Window ahead;        // next window to copy into shared memory
+    Window ahead;        // next window to copy into shared memory (decoded)
     int64_t filled;      // windows copied so far
+    // Requests window `filled` (= ahead) into its buffer with its descriptor;
+    // past the last window, the end marker (a descriptor of 0 chunks).  Then
+    // decodes the window after it.
     __device__ __forceinline__ void fill(const Params &p, const Smem &s, const int64_t *kcp) {
         const int buf = (int)(filled % kWinBufs);
+        int64_t *wm = s.wmeta + kWmeta * buf;
+        ++filled;
+        if (!ahead.valid(p)) {
+            wm[0] = 0;
+            mbar_arrive(&s.pfull[buf]);
+            return;
+        }
+        wm[0] = ahead.cnt;
+        wm[1] = ahead.t.n0;
+        wm[2] = ahead.t.kc0 + ahead.k0;
+        wm[3] = (ahead.k0 == 0 ? kWinFirst : 0u) | (ahead.k0 + ahead.cnt == ahead.t.nkc ? kWinLast : 0u) |
+                (final_unit(p, ahead.ui, ahead.t) ? kWinFinal : 0u);
+        wm[4] = ahead.t.h0;
+        wm[5] = ahead.t.img0;
         const uint32_t bytes = (uint32_t)ahead.cnt * kMetaBytes;
         mbar_arrive_expect_tx(&s.pfull[buf], bytes);
         bulk_g2s(smem_u32(s.win + buf * kWinBytes),
                  p.meta + (ahead.t.kc0 + ahead.k0) * kMetaBytes, bytes, &s.pfull[buf]);
-        ++filled;
         ahead.next(p, kcp);
     }
     // the CTA is unwinding: let the window copies that may be in flight land first
@@ -664,8 +711,9 @@ struct WindowFiller {
 // still run: the chunk records of the first window and the weight tiles of the
 // first chunks come from the packed image (written by bp_pack, which
 // synchronises), not from anything a kernel in flight writes, so they are
-// requested now.  A weight tile only adds its bytes to its stage barrier; the
-// control thread arrives once the stage's activation loads are issued.
+// requested now, and window 1 is decoded (kept in cwin for the scheduler
+// warp).  A weight tile only adds its bytes to its stage barrier; the control
+// thread arrives once the stage's activation loads are issued.
 // Returns the number of weight tiles requested, or -1 when the window was not
 // copied (balanced launches, whose ranges are set after the wait).
 __device__ int control_prefetch(const Params &p, const Smem &s) {
@@ -677,6 +725,7 @@ __device__ int control_prefetch(const Params &p, const Smem &s) {
     if (!wf.ahead.valid(p)) return -1;
     const Window win = wf.ahead;
     wf.fill(p, s, kcp);
+    *reinterpret_cast<Window *>(s.cwin) = wf.ahead;
     const int n = (int)min((int64_t)p.stages, win.cnt);
     for (int j = 0; j < n; ++j) {
         if (blockIdx.x == 0 && j == p.drop_stage) return j;
@@ -687,54 +736,81 @@ __device__ int control_prefetch(const Params &p, const Smem &s) {
     return n;
 }
 
-__device__ void control_thread(const Params &p, const Smem &s, int pre) {
+// The scheduler warp's lane 0: requests the CTA's windows of chunk records in
+// order, each with its descriptor, as the buffers come free (the window after
+// the last one is the end marker).  It is the only role that decodes work
+// units, and it runs up to kWinBufs - 1 windows ahead of the others, so the
+// decoding (cold code, run once per window) stays off their paths.
+__device__ void scheduler_thread(const Params &p, const Smem &s) {
     const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
     volatile int *abort_flag = s.abort_flag;
-    Window win;
-    win.first(p, kcp, s.skv);
     WindowFiller wf;
-    wf.ahead = win;
-    wf.filled = 0;
-    if (pre >= 0) {             // the first window was copied before the dependency wait
+    if (*s.pre >= 0) {          // window 0 was requested before the dependency wait
+        wf.ahead = *reinterpret_cast<const Window *>(s.cwin);
         wf.filled = 1;
-        wf.ahead.next(p, kcp);
-    } else if (wf.ahead.valid(p)) {
-        wf.fill(p, s, kcp);
+    } else {
+        wf.ahead.first(p, kcp, s.skv);
+        wf.filled = 0;
     }
+    bool ok = true;
+    for (;;) {
+        // window `filled` goes to the buffer released by window filled - kWinBufs
+        const int64_t prev = wf.filled - kWinBufs;
+        if (prev >= 0 && !mbar_wait(&s.pempty[prev % kWinBufs], (uint32_t)((prev / kWinBufs) & 1),
+                                    p.watchdog_ns, abort_flag)) {
+            ok = false;
+            break;
+        }
+        const bool end = !wf.ahead.valid(p);
+        wf.fill(p, s, kcp);
+        if (end) break;
+    }
+    if (!ok) raise_timeout(p, s);
+    // the last window copies land before the CTA can exit, whether or not a
+    // consumer reached them
+    wf.drain(p, s);
+}
+
+// The control thread follows the window descriptors: per chunk it waits for
+// the stage, sets the stage's flags and issues its TMA loads.  After the last
+// chunk a stage flagged kStageEnd tells the tensor-core thread to stop.
+__device__ void control_thread(const Params &p, const Smem &s, int pre) {
+    volatile int *abort_flag = s.abort_flag;
     const int64_t npre = pre > 0 ? pre : 0;     // chunks whose weight tile is requested
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
-    int64_t count = 0, wseq = 0;
-    for (; win.valid(p) && ok; win.next(p, kcp), ++wseq) {
+    int64_t count = 0;
+    for (int64_t wseq = 0;; ++wseq) {
         const int buf = (int)(wseq % kWinBufs);
         BP_TR(256 + wseq, 0);
-        // copy the next window into the buffer released by window wseq - 2
-        if (wf.ahead.valid(p)) {
-            const int64_t prev = wf.filled - kWinBufs;
-            if (prev >= 0 && !mbar_wait(&s.pempty[prev % kWinBufs],
-                                        (uint32_t)((prev / kWinBufs) & 1), p.watchdog_ns,
-                                        abort_flag)) {
-                ok = false;
-                break;
-            }
-            wf.fill(p, s, kcp);
-        }
-        BP_TR(256 + wseq, 1);
         if (!mbar_wait(&s.pfull[buf], (uint32_t)((wseq / kWinBufs) & 1), p.watchdog_ns,
                        abort_flag)) {
             ok = false;
             break;
         }
         BP_TR(256 + wseq, 2);
+        const int64_t *wm = s.wmeta + kWmeta * buf;
+        const int64_t wcnt = wm[0];
+        if (wcnt == 0) break;       // no more windows
+        const int64_t wn0 = wm[1], wc0 = wm[2];
+        const uint32_t wfl = (uint32_t)wm[3];
+        const int32_t wh0 = (int32_t)wm[4], wimg0 = (int32_t)wm[5];
         const uint8_t *recs = s.win + buf * kWinBytes;
-        for (int64_t j = 0; j < win.cnt; ++j) {
+        // flags of the window's chunks: the unit's first and last chunk, and
+        // whether the unit is the CTA's final one
+        const uint32_t ufin = (wfl & kWinFinal) ? kStageFinal : 0u;
+        const int64_t jfirst = (wfl & kWinFirst) ? 0 : -1, jlast = (wfl & kWinLast) ? wcnt - 1 : -1;
+        for (int64_t j = 0; j < wcnt; ++j) {
             const int64_t seq = count;
+            BP_TR(seq, 4);
             if (!mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)) {
                 ok = false;
                 break;
             }
             BP_TR(seq, 0);
+            const uint32_t uflag =
+                (j == jfirst ? kStageFirst : 0u) | (j == jlast ? kStageLast | ufin : 0u);
             // the plan: words 0..11 in three 16-byte loads
             const uint4 *pv = reinterpret_cast<const uint4 *>(recs + j * kMetaBytes + kListBytes);
             const uint4 q0 = pv[0], q1 = pv[1], q2 = pv[2];
@@ -757,24 +833,24 @@ __device__ void control_thread(const Params &p, const Smem &s, int pre) {
                     di >>= 1;       // floor((d - phase) / 2) = floor(d / 2)
                     dj >>= 1;
                 }
-                s.skind[stage] = 1u;
+                s.sflag[stage] = kStageTma | uflag;
                 mbar_arrive_expect_tx(&s.wfull[stage], (wpre ? 0u : kWTileBytes) + p.i_box_bytes);
                 if (!wpre)
                     bulk_g2s(smem_u32(s.w + stage * kWTileBytes),
-                             p.tiles + (win.t.kc0 + win.k0 + j) * (int64_t)kWTileBytes, kWTileBytes,
+                             p.tiles + (wc0 + j) * (int64_t)kWTileBytes, kWTileBytes,
                              &s.wfull[stage]);
                 tma_load_4d(smem_u32(s.x + stage * kXTileBytes), &p.imap, (d >> 16) * 64, dj,
-                            (int32_t)win.t.h0 + di, img * (int32_t)p.i_Nb + (int32_t)win.t.img0,
+                            wh0 + di, img * (int32_t)p.i_Nb + wimg0,
                             &s.wfull[stage]);
             } else if (!(blockIdx.x == 0 && seq == p.drop_stage)) {
-                s.skind[stage] = tma ? 1u : 0u;    // read by the MMA thread after wfull
+                s.sflag[stage] = (tma ? kStageTma : 0u) | uflag;  // read by the MMA thread after wfull
                 mbar_arrive_expect_tx(&s.wfull[stage],
                                       (wpre ? 0u : kWTileBytes) +
                                           (tma ? (uint32_t)p.xboxes * (kBK * 128) : 0u));
                 BP_TR(seq, 6);
                 if (!wpre)
                     bulk_g2s(smem_u32(s.w + stage * kWTileBytes),
-                             p.tiles + (win.t.kc0 + win.k0 + j) * (int64_t)kWTileBytes, kWTileBytes,
+                             p.tiles + (wc0 + j) * (int64_t)kWTileBytes, kWTileBytes,
                              &s.wfull[stage]);
                 BP_TR(seq, 7);
                 if (tma) {
@@ -791,7 +867,7 @@ __device__ void control_thread(const Params &p, const Smem &s, int pre) {
                         const CUtensorMap *map = &p.xmap[(d >> 4) & 3u];
 #pragma unroll
                         for (int cn = 0; cn < p.xboxes; ++cn)
-                            tma_load_2d(dst + cn * 8192, map, (int32_t)(win.t.n0 + cn * 64),
+                            tma_load_2d(dst + cn * 8192, map, (int32_t)(wn0 + cn * 64),
                                         (int32_t)ys[b], &s.wfull[stage]);
                     }
                 }
@@ -804,20 +880,48 @@ __device__ void control_thread(const Params &p, const Smem &s, int pre) {
         if (!ok) break;
         mbar_arrive(&s.pempty[buf]);
     }
+    if (ok) {
+        // no more chunks: the end marker for the tensor-core thread
+        if (mbar_wait(&s.empty[stage], phase ^ 1u, p.watchdog_ns, abort_flag)) {
+            s.sflag[stage] = kStageEnd;
+            mbar_arrive_cnt(&s.wfull[stage], kStageArrivals);
+        } else {
+            ok = false;
+        }
+    }
     if (!ok) {
         raise_timeout(p, s);
         // unwinding: the copies of the last stages and the window copies may still
-        // be in flight; let them land before the CTA exits (a weight tile
-        // requested before the wait for a chunk not reached yet completes its
-        // stage once the arrival it waits for is added)
-        for (int64_t q = count; q < npre; ++q) mbar_arrive(&s.wfull[q]);
+        // be in flight; let them land before the CTA exits.  A stage completes
+        // once its TMA bytes have landed and its arrivals are in: the ones of
+        // gather warps that left their loop before the chunk, and this thread's
+        // own for a chunk whose weight tile was requested before the dependency
+        // wait but not reached, are added here.  The gather warps leave once
+        // they see the abort flag; their progress is read after they have.
+        const volatile int64_t *gprog = s.gprog;
+        {
+            uint64_t deadline = 0;
+            for (uint32_t it = 1; gprog[kGatherWarps] < kGatherWarps; ++it) {
+                __nanosleep(64);
+                if ((it & 15u) == 0u) {
+                    const uint64_t now = globaltimer_ns();
+                    if (deadline == 0) deadline = now + kDrainNs;
+                    else if (now > deadline) break;
+                }
+            }
+        }
         const int64_t reach = count > npre ? count : npre;
-        for (int64_t q = reach > p.stages ? reach - p.stages : 0; q < reach; ++q)
-            if (!(blockIdx.x == 0 && q == p.drop_stage) &&
-                !mbar_wait(&s.wfull[q % p.stages], (uint32_t)((q / p.stages) & 1), kDrainNs,
+        for (int64_t q = reach > p.stages ? reach - p.stages : 0; q < reach; ++q) {
+            if (blockIdx.x == 0 && q == p.drop_stage) continue;
+            uint32_t missing = q >= count ? 1u : 0u;
+            const int g0 = (int)(q % kGatherGroups) * kGroupWarps;
+            for (int w = g0; w < g0 + kGroupWarps; ++w)
+                if (gprog[w] <= q) missing += 32u;
+            if (missing) mbar_arrive_cnt(&s.wfull[q % p.stages], missing);
+            if (!mbar_wait(&s.wfull[q % p.stages], (uint32_t)((q / p.stages) & 1), kDrainNs,
                            nullptr))
                 atomicOr(p.status, kDevTimeout);
-        wf.drain(p, s);
+        }
     }
 }
 
@@ -825,14 +929,15 @@ __device__ void control_thread(const Params &p, const Smem &s, int pre) {
 __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
     // Everything the loop needs lives in registers: the per-chunk path is a
     // chain of dependent barrier probes and issues, so any reload from the
-    // parameter bank or shared memory adds to every chunk.
-    const int64_t *kcp = s.kc ? s.kc : p.kc_ptr;
+    // parameter bank or shared memory adds to every chunk.  The thread decodes
+    // no work units: each stage's flags (set by the control thread) say where
+    // its chunk sits in its unit, and a stage flagged kStageEnd ends the loop.
     volatile int *abort_flag = s.abort_flag;
     const uint64_t wdog = p.watchdog_ns;
     const int nst = (int)p.stages;
     const uint32_t acc_cols = p.acc_cols;
-    uint64_t *const wfull = s.wfull, *const full = s.full, *const empty = s.empty;
-    const volatile uint32_t *const skind = s.skind;
+    uint64_t *const wfull = s.wfull, *const empty = s.empty;
+    const volatile uint32_t *const sflag = s.sflag;
     // B: MN-major activation rows, or for the implicit convolution K-major
     // pixel rows (both with the 128-byte swizzle)
     const uint32_t idesc = make_idesc(p.dtype == BP_BF16, false, !p.impl, kSlab, p.nt);
@@ -846,101 +951,66 @@ __device__ void mma_issuer(const Params &p, const Smem &s, uint32_t tmem) {
     const uint32_t xkstep = p.impl ? 32u >> 4 : 2048u >> 4;
     int stage = 0;
     uint32_t phase = 0;
-    uint32_t gphase = 0;     // per gather barrier: parity of its next fill (bit = barrier)
     int acc = 0;
     uint32_t acc_phase = 0;
-    bool ok = true;
+    uint32_t d = tmem;
 #ifdef BP_TRACE
     int64_t tseq = 0, titem = 0;
 #else
     constexpr int64_t tseq = 0;
 #endif
-    UnitIter ui;
-    Item t;
-    for (ui.init(p, s.skv); ui.valid() && ok; ui.step(p, t)) {
-        t = ui.get(p, kcp);
-        if (t.nkc == 0) continue;
-        if (!mbar_wait(&s.tempty[acc], acc_phase ^ 1u, wdog, abort_flag)) {
+    bool ready = mbar_test_wait(&wfull[0], 0);
+    for (;;) {
+        if (!ready && !mbar_wait(&wfull[stage], phase, wdog, abort_flag)) {
             raise_timeout(p, s);
             break;
         }
-#ifdef BP_TRACE
-        BP_TR(384 + titem, 4);
-        ++titem;
-#endif
-        tc_fence_after();
-        const uint32_t d = tmem + acc * acc_cols;
-        bool ready = mbar_test_wait(&wfull[stage], phase);
-        for (int64_t kc = 0; kc < t.nkc; ++kc) {
-            if (!ready && !mbar_wait(&wfull[stage], phase, wdog, abort_flag)) {
+        BP_TR(tseq, 3);
+        const uint32_t f = sflag[stage];
+        if (f & kStageEnd) break;
+        // gathered rows: order their generic-proxy (cp.async) writes, acquired
+        // through the barrier, before the tensor core's async-proxy reads
+        if (!(f & kStageTma)) fence_proxy_async_smem();
+        if (f & kStageFirst) {
+            // a unit's first chunk: the next accumulator, once drained
+            if (!mbar_wait(&s.tempty[acc], acc_phase ^ 1u, wdog, abort_flag)) {
                 raise_timeout(p, s);
-                ok = false;
                 break;
             }
-            BP_TR(tseq, 3);
-            const bool gathered = skind[stage] == 0u;
-            // gathered rows: wait for them, then order their generic-proxy
-            // (cp.async) writes, acquired through the barrier, before the tensor
-            // core's async-proxy reads
-            const uint32_t fb = kFullPerStage * stage;
-            if (gathered) {
-                if (!mbar_wait(&full[fb], (gphase >> fb) & 1u, wdog, abort_flag)) {
-                    raise_timeout(p, s);
-                    ok = false;
-                    break;
-                }
-                gphase ^= 1u << fb;
-                fence_proxy_async_smem();
-                BP_TR(tseq, 4);
-            }
-            // order the MMAs below after the barrier waits above
-            tc_fence_after();
-            const uint64_t wd = wdesc0 + (uint32_t)(stage * (kWTileBytes >> 4));
-            const uint64_t xd = xdesc0 + (uint32_t)(stage * (kXTileBytes >> 4));
-            const int nstage = stage + 1 == nst ? 0 : stage + 1;
-            const uint32_t nphase = stage + 1 == nst ? phase ^ 1u : phase;
-            // probe the next chunk's barrier now: the answer is needed only after
-            // the MMAs below have been issued
-            ready = kc + 1 < t.nkc && mbar_test_wait(&wfull[nstage], nphase);
-#ifdef BP_GATHER_HALVES
-#pragma unroll
-            for (int kk = 0; kk < 2; ++kk)
-                umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * xkstep, idesc,
-                            (kc > 0 || kk > 0) ? 1u : 0u);
-            if (gathered) {
-                if (!mbar_wait(&full[fb + 1], (gphase >> (fb + 1)) & 1u, wdog, abort_flag)) {
-                    raise_timeout(p, s);
-                    ok = false;
-                    break;
-                }
-                gphase ^= 1u << (fb + 1);
-                fence_proxy_async_smem();
-                tc_fence_after();
-            }
-#pragma unroll
-            for (int kk = 2; kk < 4; ++kk)
-                umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * xkstep, idesc, 1u);
-#else
-#pragma unroll
-            for (int kk = 0; kk < kBK / 16; ++kk)
-                umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * xkstep, idesc,
-                            (kc > 0 || kk > 0) ? 1u : 0u);
-#endif
-            umma_commit(&empty[stage]);
-            BP_TR(tseq, 5);
 #ifdef BP_TRACE
-            ++tseq;
+            BP_TR(384 + titem, 4);
+            ++titem;
 #endif
-            stage = nstage;
-            phase = nphase;
+            d = tmem + acc * acc_cols;
         }
-        if (!ok) break;
-        umma_commit(&s.tfull[acc]);
-        if (final_unit(p, ui, t)) umma_commit(s.ffull);
-        if (++acc == 2) {
-            acc = 0;
-            acc_phase ^= 1u;
+        // order the MMAs below after the barrier waits above
+        tc_fence_after();
+        const uint64_t wd = wdesc0 + (uint32_t)(stage * (kWTileBytes >> 4));
+        const uint64_t xd = xdesc0 + (uint32_t)(stage * (kXTileBytes >> 4));
+        const int nstage = stage + 1 == nst ? 0 : stage + 1;
+        const uint32_t nphase = stage + 1 == nst ? phase ^ 1u : phase;
+        // probe the next stage now: the answer is needed only after the MMAs
+        // below have been issued
+        ready = mbar_test_wait(&wfull[nstage], nphase);
+        const uint32_t acc0 = (f & kStageFirst) ? 0u : 1u;
+#pragma unroll
+        for (int kk = 0; kk < kBK / 16; ++kk)
+            umma_f16_ss(d, wd + kk * (32 >> 4), xd + kk * xkstep, idesc, kk > 0 ? 1u : acc0);
+        umma_commit(&empty[stage]);
+        BP_TR(tseq, 5);
+#ifdef BP_TRACE
+        ++tseq;
+#endif
+        if (f & kStageLast) {
+            umma_commit(&s.tfull[acc]);
+            if (f & kStageFinal) umma_commit(s.ffull);
+            if (++acc == 2) {
+                acc = 0;
+                acc_phase ^= 1u;
+            }
         }
+        stage = nstage;
+        phase = nphase;
     }
     // all issued tensor-core work must finish before tensor memory is freed
     umma_commit(s.drain);
@@ -1433,7 +1503,7 @@ __device__ void epilogue(const Params &p, const Smem &s, uint32_t tmem, int slot
                         // are written here directly (the generic store path
                         // reloads its spilled per-item state every group, ~800
                         // cycles of round trips per group)
-                        const uint32_t HWw = kConv ? (uint32_t)p.HoWo : 0u;
+                        const uint32_t HWw = kConv ? (uint32_t)p.HoWo : 1u;
                         const bool whole = kConv && HWw < 32u && (32u % HWw) == 0u &&
                                            (uint32_t)t.n0 % HWw == 0u && row0 + 32 <= t.rows;
                         uint16_t *yw = nullptr;
@@ -1500,8 +1570,7 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     const int warp = threadIdx.x >> 5;
     if (threadIdx.x == 0) {
         for (int i = 0; i < p.stages; ++i) {
-            for (int h = 0; h < kFullPerStage; ++h) mbar_init(&s.full[kFullPerStage * i + h], kGroupThreads);
-            mbar_init(&s.wfull[i], 1);
+            mbar_init(&s.wfull[i], kStageArrivals);
             mbar_init(&s.empty[i], 1);
         }
         for (int i = 0; i < 2; ++i) {
@@ -1516,6 +1585,7 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
             mbar_init(&s.pempty[i], kGatherWarps + 1);
         }
         *s.abort_flag = 0;
+        for (int i = 0; i <= kGatherWarps; ++i) s.gprog[i] = 0;
         fence_mbar_init();
     }
     if (warp == kMmaWarp) {
@@ -1535,7 +1605,10 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
         for (int64_t i = threadIdx.x; i < p.kc_cached; i += kThreads) s.kc[i] = p.kc_ptr[i];
     __syncthreads();
     int pre = -1;
-    if (warp == kCtrlWarp && (threadIdx.x & 31) == 0) pre = control_prefetch(p, s);
+    if (warp == kCtrlWarp && (threadIdx.x & 31) == 0) {
+        pre = control_prefetch(p, s);
+        *s.pre = pre;           // read by the scheduler warp after the barrier below
+    }
     grid_dependency_wait();
     grid_launch_dependents();
 #ifdef BP_TRACE
@@ -1567,8 +1640,11 @@ __global__ void __launch_bounds__(kThreads, 1) bp_mma_kernel(const __grid_consta
     } else if (warp == kMmaWarp) {
         if ((threadIdx.x & 31) == 0) mma_issuer(p, s, tmem);
         __syncwarp();
-    } else {
+    } else if (warp < kSchedWarp) {
         epilogue<kSplit, kConv>(p, s, tmem, 0);
+    } else {
+        if ((threadIdx.x & 31) == 0) scheduler_thread(p, s);
+        __syncwarp();
     }
 
     tc_fence_before();

@@ -26,6 +26,22 @@
 //           chunk, two gather groups, a consumer that releases each stage):
 //           cycles per chunk against the rows' spread, the tiles shared
 //           between CTAs, the weight copies and the hold time;
+//   test 8: groups of four 128 x N x 16 MMAs and a commit (one 64-column
+//           chunk) with the tensor-core thread's per-chunk work between the
+//           groups (flags: 1 tcgen05.fence::after_thread_sync, 2
+//           fence.proxy.async, 4 try_wait on a completed barrier, 8 test_wait
+//           on a completed barrier, 16 a dependent shared-memory load, 32 a
+//           chain of 32 dependent integer operations, 64 a clock64 store to
+//           global memory, 128 test_wait on an incomplete barrier; 256: that
+//           work after the group's second MMA instead of before its first;
+//           512: clock64 read before and after each group, to time its issue;
+//           1024: meanwhile warps 2-9 poll a barrier that never completes;
+//           2048: meanwhile warps 2-7 gather 512-byte rows with cp.async;
+//           4096: the groups' operands rotate over four 48 KB stages, as in
+//           the product, instead of one resident A and B; 8192: no work
+//           function at all between the groups; 16384: eight rarely taken
+//           branches between the groups, each around a nanosleep):
+//           cycles per group (and how long the thread takes to issue one);
 //   test 3: test 0's back-to-back MMAs while 1..6 other warps copy into a
 //           separate shared-memory area (TMA bulk copies of 16 KB, or with
 //           flag 4 one warp-wide 512-byte cp.async row per instruction, 16
@@ -44,12 +60,72 @@ using namespace bp;
 constexpr uint64_t kLim = 1000000000ull;
 constexpr int kData = 4 * 49152;    // shared-memory data area (test 7: four 48 KB stages)
 
+struct PP;
+template <int kCode>
+__device__ __forceinline__ void t8_loop(const PP &p, uint32_t tmem, uint64_t a0, uint64_t b0, uint32_t idesc,
+                                        uint64_t *bars, const volatile uint32_t *vz, bool &ok);
 struct PP {
     int test, iters, N, nthreads, flags;
     const uint8_t *W;
     unsigned long long *out;    // [2 * gridDim.x]: per CTA cycles (and test 3: bytes copied, cycles)
     unsigned *err;
 };
+
+// test 8 with nthreads = code >= 2: the groups with one kind of per-group code
+// present in the loop, run when flag bit (code - 2) is set: 2 tcgen05 fence,
+// 3 try_wait (bounded wait) on a completed barrier, 4 test_wait, 5 proxy
+// fence, 6 a shared-memory load feeding the descriptor, 7 a clock64 store,
+// 8 a 32-op integer chain; with the operands rotating over four 48 KB stages
+// and the K step and first accumulate flag read at run time, as in the
+// product: 9 descriptors formed between the MMAs, 10 the four MMAs from one
+// asm block with their descriptors formed first
+template <int kCode>
+__device__ __forceinline__ void t8_loop(const PP &p, uint32_t tmem, uint64_t a0, uint64_t b0, uint32_t idesc,
+                                        uint64_t *bars, const volatile uint32_t *vz, bool &ok) {
+    const bool on = (p.flags >> (kCode - 2)) & 1;
+    uint32_t x = 1;
+    if (kCode >= 9) {
+        const uint64_t da = 2 + (uint64_t)(p.flags & 1), db = 128 + (uint64_t)(p.flags & 2);
+        for (int c = 0; c < p.iters; ++c) {
+            const uint32_t so = (uint32_t)(c & 3) * (49152u >> 4);
+            const uint64_t a = a0 + so, b = b0 + so;
+            const uint32_t acc0 = (c & 15) ? 1u : (uint32_t)(p.flags >> 2) & 1u;
+            if (kCode == 9) {
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk)
+                    umma_f16_ss(tmem, a + kk * da, b + kk * db, idesc, kk > 0 ? 1u : acc0);
+            } else {
+                umma_f16_ss_x4(tmem, a, b, da, db, idesc, acc0);
+            }
+            umma_commit(&bars[c & 7]);
+        }
+        return;
+    }
+    for (int c = 0; c < p.iters; ++c) {
+        uint32_t off = 0;
+        if (on) {
+            if (kCode == 2) tc_fence_after();
+            if (kCode == 3) ok &= mbar_wait(&bars[14], 0, kLim, nullptr);
+            if (kCode == 4) ok &= mbar_test_wait(&bars[14], 0);
+            if (kCode == 5) fence_proxy_async_smem();
+            if (kCode == 6) off += *vz;
+            if (kCode == 7) p.out[4 * gridDim.x + (c & 255)] = clock64();
+            if (kCode == 8) {
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                    asm volatile("mad.lo.u32 %0, %0, 3, %1;" : "+r"(x) : "r"((uint32_t)c));
+                uint32_t z;
+                asm volatile("and.b32 %0, %1, 0;" : "=r"(z) : "r"(x));
+                off += z;
+            }
+        }
+        umma_f16_ss(tmem, a0 + off, b0, idesc, 1u);
+        umma_f16_ss(tmem, a0 + 2, b0 + 128, idesc, 1u);
+        umma_f16_ss(tmem, a0 + 4, b0 + 256, idesc, 1u);
+        umma_f16_ss(tmem, a0 + 6, b0 + 384, idesc, 1u);
+        umma_commit(&bars[c & 7]);
+    }
+}
 
 __global__ void __launch_bounds__(320, 1) probe(const __grid_constant__ PP p) {
     extern __shared__ __align__(1024) uint8_t raw[];
@@ -70,6 +146,7 @@ __global__ void __launch_bounds__(320, 1) probe(const __grid_constant__ PP p) {
         for (int i = 24; i < 40; ++i) mbar_init(&bars[i], 1);
         fence_mbar_init();
         tbase[1] = 0;           // test 3: the MMA thread's "done" flag
+        tbase[2] = 0;           // test 8: a zero read from shared memory
     }
     for (int i = threadIdx.x; i < kData / 16; i += blockDim.x)
         reinterpret_cast<uint4 *>(base)[i] = make_uint4(0, 0, 0, 0);
@@ -389,6 +466,132 @@ __global__ void __launch_bounds__(320, 1) probe(const __grid_constant__ PP p) {
             p.out[blockIdx.x] = clock64() - t0;
             if (!ok) atomicOr(p.err, 64u);
         }
+    } else if (p.test == 8) {
+        if (threadIdx.x == 0) {
+            mbar_arrive(&bars[14]);     // completes its phase 0
+            const uint32_t idesc = make_idesc(true, false, true, 128, p.N);
+            const uint64_t a0 = make_sdesc_sw128(smem_u32(base), 16, 1024);
+            const uint64_t b0 = make_sdesc_sw128(smem_u32(base + 16384), 8192, 1024);
+            const volatile uint32_t *vz = tbase + 2;
+            const int f = p.flags;
+            uint32_t x = 1;
+            bool ok = true;
+            unsigned long long issue = 0;
+            auto work = [&](int c, uint32_t &off) {
+                if (f & 1) tc_fence_after();
+                if (f & 2) fence_proxy_async_smem();
+                if (f & 4) ok &= mbar_wait(&bars[14], 0, kLim, nullptr);
+                if (f & 8) ok &= mbar_test_wait(&bars[14], 0);
+                if (f & 16) off += *vz;
+                if (f & 32) {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i)
+                        asm volatile("mad.lo.u32 %0, %0, 3, %1;" : "+r"(x) : "r"((uint32_t)c));
+                    uint32_t z;
+                    asm volatile("and.b32 %0, %1, 0;" : "=r"(z) : "r"(x));
+                    off += z;
+                }
+                if (f & 64) p.out[4 * gridDim.x + (c & 255)] = clock64();
+                if (f & 128) ok &= !mbar_test_wait(&bars[13], 0);
+            };
+            const unsigned long long t0 = clock64();
+            if (p.nthreads >= 2) {
+                switch (p.nthreads) {
+                    case 2: t8_loop<2>(p, tmem, a0, b0, idesc, bars, vz, ok); break;
+                    case 3: t8_loop<3>(p, tmem, a0, b0, idesc, bars, vz, ok); break;
+                    case 4: t8_loop<4>(p, tmem, a0, b0, idesc, bars, vz, ok); break;
+                    case 5: t8_loop<5>(p, tmem, a0, b0, idesc, bars, vz, ok); break;
+                    case 6: t8_loop<6>(p, tmem, a0, b0, idesc, bars, vz, ok); break;
+                    case 7: t8_loop<7>(p, tmem, a0, b0, idesc, bars, vz, ok); break;
+                    case 8: t8_loop<8>(p, tmem, a0, b0, idesc, bars, vz, ok); break;
+                    case 9: t8_loop<9>(p, tmem, a0, b0, idesc, bars, vz, ok); break;
+                    default: t8_loop<10>(p, tmem, a0, b0, idesc, bars, vz, ok); break;
+                }
+            } else if (f & 256) {
+                // the work between the group's second and third MMA
+                for (int c = 0; c < p.iters; ++c) {
+                    uint32_t off = 0;
+                    umma_f16_ss(tmem, a0, b0, idesc, 1u);
+                    umma_f16_ss(tmem, a0 + 2, b0 + 128, idesc, 1u);
+                    work(c, off);
+                    umma_f16_ss(tmem, a0 + 4 + off, b0 + 256, idesc, 1u);
+                    umma_f16_ss(tmem, a0 + 6, b0 + 384, idesc, 1u);
+                    umma_commit(&bars[c & 7]);
+                }
+            } else if (f & 512) {
+                for (int c = 0; c < p.iters; ++c) {
+                    uint32_t off = 0;
+                    const unsigned long long ti = clock64();
+                    work(c, off);
+                    umma_f16_ss(tmem, a0 + off, b0, idesc, 1u);
+                    umma_f16_ss(tmem, a0 + 2, b0 + 128, idesc, 1u);
+                    umma_f16_ss(tmem, a0 + 4, b0 + 256, idesc, 1u);
+                    umma_f16_ss(tmem, a0 + 6, b0 + 384, idesc, 1u);
+                    umma_commit(&bars[c & 7]);
+                    issue += clock64() - ti;
+                }
+            } else if (f & 8192) {
+                for (int c = 0; c < p.iters; ++c) {
+                    if (f & 16384) {
+#pragma unroll
+                        for (int k = 0; k < 8; ++k)
+                            if (c == -1 - k * p.iters) asm volatile("nanosleep.u32 0;");
+                    }
+                    umma_f16_ss(tmem, a0, b0, idesc, 1u);
+                    umma_f16_ss(tmem, a0 + 2, b0 + 128, idesc, 1u);
+                    umma_f16_ss(tmem, a0 + 4, b0 + 256, idesc, 1u);
+                    umma_f16_ss(tmem, a0 + 6, b0 + 384, idesc, 1u);
+                    umma_commit(&bars[c & 7]);
+                }
+            } else if (f & 4096) {
+                // stage st: A at st * 48 KB, B 16 KB after it (descriptor units of 16 B)
+                for (int c = 0; c < p.iters; ++c) {
+                    uint32_t off = 0;
+                    work(c, off);
+                    const uint32_t so = (uint32_t)(c & 3) * (49152u >> 4);
+                    const uint64_t a = make_sdesc_sw128(smem_u32(base), 16, 1024) + so;
+                    const uint64_t b = make_sdesc_sw128(smem_u32(base + 16384), 8192, 1024) + so;
+                    umma_f16_ss(tmem, a + off, b, idesc, 1u);
+                    umma_f16_ss(tmem, a + 2, b + 128, idesc, 1u);
+                    umma_f16_ss(tmem, a + 4, b + 256, idesc, 1u);
+                    umma_f16_ss(tmem, a + 6, b + 384, idesc, 1u);
+                    umma_commit(&bars[c & 7]);
+                }
+            } else {
+                for (int c = 0; c < p.iters; ++c) {
+                    uint32_t off = 0;
+                    work(c, off);
+                    umma_f16_ss(tmem, a0 + off, b0, idesc, 1u);
+                    umma_f16_ss(tmem, a0 + 2, b0 + 128, idesc, 1u);
+                    umma_f16_ss(tmem, a0 + 4, b0 + 256, idesc, 1u);
+                    umma_f16_ss(tmem, a0 + 6, b0 + 384, idesc, 1u);
+                    umma_commit(&bars[c & 7]);
+                }
+            }
+            umma_commit(&bars[15]);
+            ok &= mbar_wait(&bars[15], 0, kLim, nullptr);
+            p.out[blockIdx.x] = clock64() - t0;
+            p.out[gridDim.x + blockIdx.x] = issue;
+            *reinterpret_cast<volatile uint32_t *>(tbase + 1) = 1u;
+            if (!ok) atomicOr(p.err, 128u);
+        } else if (warp >= 2 && (p.flags & 1024)) {
+            // pollers: a barrier nobody arrives on, until the MMA thread is done
+            const volatile uint32_t *done = tbase + 1;
+            const uint32_t a = smem_u32(&bars[12]);
+            for (int it = 0; it < (1 << 24) && !*done; ++it) (void)mbar_try_wait(a, 0);
+        } else if (warp >= 2 && warp <= 7 && (p.flags & 2048)) {
+            // copiers: 16 rows of 512 B per batch into their own 8 KB areas
+            const volatile uint32_t *done = tbase + 1;
+            const uint32_t dst = smem_u32(base + 65536 + (warp - 2) * 8192);
+            for (int it = 0; it < (1 << 20) && !*done; ++it) {
+#pragma unroll
+                for (int r = 0; r < 16; ++r) {
+                    const int64_t row = ((int64_t)blockIdx.x * 131 + it * 16 + r + warp * 977) % 16384;
+                    cp_async_16_full(dst + r * 512 + lane * 16, p.W + row * 512 + lane * 16);
+                }
+                cp_async_wait_all();
+            }
+        }
     } else if (p.test == 2) {
         // stage ring without data: full[s] = bars[s], empty[s] = bars[8 + s]
         const int S = p.nthreads;
@@ -505,9 +708,10 @@ int main(int argc, char **argv) {
     const int N = argc > 3 ? atoi(argv[3]) : 256;
     const int nth = argc > 4 ? atoi(argv[4]) : 1;
     const int flags = argc > 5 ? atoi(argv[5]) : 0;
-    if (N < 16 || N > 256 || N % 16 || nth < 1 || nth > 8 || iters < 1 || test < 0 || test > 7)
+    if (N < 16 || N > 256 || N % 16 || nth < 1 || nth > (test == 8 ? 10 : 8) || iters < 1 || test < 0 ||
+        test > 8)
         return 2;
-    if (test != 4 && test != 5 && test != 6 && test != 7 && nth > 6) return 2;
+    if (test != 4 && test != 5 && test != 6 && test != 7 && test != 8 && nth > 6) return 2;
     if (test == 7 && (nth < 2 || nth > ((flags & 32) ? 8 : (flags & 32768) ? 2 : 4) ||
                       (N != 128 && N != 256) || flags < 0 || flags > 65535 || (flags & 192) == 192 ||
                       ((flags & 64) && nth < 4) || ((flags & 32) && (flags & 32768)))) return 2;
@@ -515,6 +719,8 @@ int main(int argc, char **argv) {
     if (test == 6 && (nth > 6 || flags < 0 || flags > 2 || N < 64 || (N & (N - 1)))) return 2;
     if (test == 4 && nth != 2 && nth != 4 && nth != 8) return 2;   // MMAs per group
     if (test == 2 && (nth < 2 || nth > 6)) return 2;     // stages
+    if (test == 8 && (flags < 0 || flags > 32767 || (flags & 3072) == 3072 ||
+                      ((flags & 4096) && (flags & 2048)))) return 2;
     int sms = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
     uint8_t *W = nullptr;
@@ -594,6 +800,9 @@ int main(int argc, char **argv) {
     else if (test == 5)
         printf("cp.async rows of 512 B from %d warp(s), pitch %d B over %d MB: %.1f bytes per cycle "
                "per SM (err %u)\n", nth, flags > 0 ? flags * 1024 : 512, N, cyc > 0 ? byt / cyc : 0.0, herr);
+    else if (test == 8)
+        printf("mma groups of 4 x (128 x %d x 16) + commit, per-group work %d (code %d): %.1f cycles per "
+               "group, %.1f to issue one (err %u)\n", N, flags, nth, avg / iters, byt / sms / iters, herr);
     else if (test == 4)
         printf("mma 128 x %d x 16 in groups of %d, %s, %s: %.1f cycles per instruction (err %u)\n",
                N, nth, (flags & 2) ? "no commits" : "a commit per group",

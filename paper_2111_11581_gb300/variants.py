@@ -3,7 +3,7 @@ per-stage timeline of the tensor-core product.
 
     python -m paper_2111_11581_gb300.variants time NAME:[DEFINE,...] ...
         builds one library per NAME with the given -D switches (e.g.
-        `base: halves:BP_GATHER_HALVES balance:BP_BALANCE`) and times each on
+        `base: balance:BP_BALANCE`) and times each on
         the same workloads, every build in a process of its own:
         4096^3 bf16 at 128 x 32 blocks, keep 1/4 (the benchmark's layer),
         4096^3 at 8 x 64 blocks, keep 1/2 (whole 64-column blocks: TMA tile
@@ -25,18 +25,20 @@ per-stage timeline of the tensor-core product.
         back-to-back MMAs while other warps copy into shared memory (bulk or
         cp.async rows).
 
-    python -m paper_2111_11581_gb300.variants trace [gemm|conv3x3|resnet50:LAYER|vgg16:LAYER|fc512] [DEFINE ...]
+    python -m paper_2111_11581_gb300.variants trace [gemm|gemm8|conv3x3|resnet50:LAYER|vgg16:LAYER|fc512][+warm] [DEFINE ...]
         builds with BP_TRACE and prints CTA 0's clock64 timeline of one launch,
-        L2 flushed before it, of the 4096^3 layer (or of the 3x3 CONV layer: N=128, C=F=128, 16x16,
-        or of one ResNet-50 layer by name): per pipeline stage when the control
+        L2 flushed before it, of the 4096^3 layer (bm=128 bk=32 at 4x; gemm8:
+        bm=8 bk=64 at 2x; or of the 3x3 CONV layer: N=128, C=F=128, 16x16, or
+        of one ResNet-50 / VGG-16 layer by name); with +warm, of the last of
+        three back-to-back launches instead: per pipeline stage when the control
         thread and a gather group found it free, when the gather was issued,
-        when the tensor-core thread saw the weight tile and the rows and
-        committed; per item when the tensor-core thread had a free accumulator
-        and when the epilogue saw it finished and had stored it; and the
-        global-timer start and end of every CTA.
+        when the tensor-core thread saw the stage loaded and committed; per
+        window when the control thread and the gather warps had its records;
+        per item when the tensor-core thread had a free accumulator and when
+        the epilogue saw it finished and had stored it; and the global-timer
+        start and end of every CTA.
 
 The switches (all off in the library `build()` makes): BP_TRACE (timeline),
-BP_GATHER_HALVES (both gather groups on every chunk, one barrier per half),
 BP_BALANCE (whole-item waves, then equal chunk ranges per CTA with fp32
 partial tiles), BP_EPI_DIRECT (output boxes written back from shared memory
 with plain stores instead of TMA stores), BP_NO_PDL (ordinary launches
@@ -187,6 +189,12 @@ def _trace_in_process(lib: str, workload: str):
     import numpy as np
     import torch
 
+    # WORKLOAD+warm: the last of three back-to-back launches, no flush (code,
+    # parameters and the packed image in L2, the start overlapping the previous
+    # launch as in a timing loop)
+    warm = workload.endswith("+warm")
+    workload = workload.removesuffix("+warm")
+
     from . import bp, inputs
     L_ = bp.load(lib)
     L_.bp_debug_trace_read.restype = ctypes.c_int
@@ -219,7 +227,8 @@ def _trace_in_process(lib: str, workload: str):
         run = lambda: bp.conv2d(pw, X, pad=pad, stride=st, out=Y, ws=ws)  # noqa: E731
     else:
         dt = bp.BF16
-        L = inputs.gemm_point(4096, 4096, 4096, 128, 32, 4.0, dt)
+        L = (inputs.gemm_point(4096, 4096, 4096, 8, 64, 2.0, dt) if workload == "gemm8" else
+             inputs.gemm_point(4096, 4096, 4096, 128, 32, 4.0, dt))
         W = inputs.as_torch(inputs.layer_weight(L, dt), dt).cuda()
         X = inputs.as_torch(inputs.layer_input(L, dt), dt).cuda()
         lay = bp.layout(bp.BLOCK_BASED, dt, L.M, L.K, L.bm, L.bk)
@@ -237,9 +246,13 @@ def _trace_in_process(lib: str, workload: str):
     flush.sum()
     torch.cuda.synchronize()
     L_.bp_debug_trace_clear()
-    flush.zero_()
-    flush.sum()
-    run()
+    if warm:
+        for _ in range(3):
+            run()
+    else:
+        flush.zero_()
+        flush.sum()
+        run()
     torch.cuda.synchronize()
     if workload == "fc512":
         # the short CUDA-core path: per CTA clock64 at its start, loads issued,
@@ -269,12 +282,21 @@ def _trace_in_process(lib: str, workload: str):
     # cycles after CTA 0 passed the grid dependency wait
     t0 = t[511, 0]
     rel = np.where(stages > 0, stages - t0, -1)[valid]
-    print("stage ctrl_free gath_free gath_iss mma_w mma_x commit  (clock64 cycles after CTA 0's start)")
+    print("stage ctrl_wait ctrl_free ctrl_arr ctrl_w gath_free gath_iss mma_w commit  (clock64 "
+          "cycles after CTA 0's start; control: waits for the stage, has it, arrived, weight "
+          "tile issued)")
     for i, r in enumerate(rel):
-        print(f"{i:5d} {r[0]:9d} {r[1]:9d} {r[2]:8d} {r[3]:6d} {r[4]:6d} {r[5]:6d}")
+        print(f"{i:5d} {r[4]:9d} {r[0]:9d} {r[6]:8d} {r[7]:6d} {r[1]:9d} {r[2]:8d} {r[3]:6d} {r[5]:6d}")
     c = rel[:, 5]
     if len(c) > 1:
         print(f"median commit interval {np.median(np.diff(c)):.0f} cycles")
+    wins = t[256:384]
+    wv = wins[:, 2] > 0
+    if wv.any():
+        print("window ctrl_top ctrl_recs ctrl_next gath_recs  (control: loop top, this window's "
+              "records landed, next window requested; gather warp 0: records landed)")
+        for i, r in enumerate(wins[wv]):
+            print(f"{i:6d} {r[0] - t0:8d} {r[2] - t0:9d} {r[1] - t0:9d} {r[3] - t0:9d}")
     items = t[384:448]
     iv = items[:, 6] > 0
     print("item acc_free epi_saw epi_done")
