@@ -21,9 +21,12 @@ per-stage timeline of the tensor-core product.
         back to back from one thread (cycles per instruction for N = 256, 128,
         64, 16), TMA bulk copies from 1, 2 and 4 threads per SM (bytes per
         cycle an SM ingests), the stage ring without data (cycles per 64-column
-        chunk for 2-6 stages, with and without the per-stage fences) and
+        chunk for 2-6 stages, with and without the per-stage fences),
         back-to-back MMAs while other warps copy into shared memory (bulk or
-        cp.async rows).
+        cp.async rows), and groups of four MMAs and a commit with the
+        tensor-core thread's per-chunk work placed between them (barrier
+        probes, fences, loads, descriptor arithmetic; other warps polling or
+        copying meanwhile).
 
     python -m paper_2111_11581_gb300.variants trace [gemm|gemm8|conv3x3|resnet50:LAYER|vgg16:LAYER|fc512][+warm] [DEFINE ...]
         builds with BP_TRACE and prints CTA 0's clock64 timeline of one launch,
@@ -377,6 +380,14 @@ def main(argv):
                      ["6", "2048", "64", "6", "0"], ["6", "2048", "64", "6", "1"],
                      ["6", "2048", "64", "6", "2"], ["6", "2048", "64", "4", "0"],
                      ["6", "2048", "64", "4", "2"],
+                     # what per-group work between MMA groups costs the issue stream
+                     ["8", "2048", "256", "1", "0"], ["8", "2048", "256", "2", "1"],
+                     ["8", "2048", "256", "3", "2"], ["8", "2048", "256", "4", "4"],
+                     ["8", "2048", "256", "5", "8"], ["8", "2048", "256", "6", "16"],
+                     ["8", "2048", "256", "9", "0"], ["8", "2048", "256", "10", "0"],
+                     ["8", "2048", "256", "1", "8192"], ["8", "2048", "256", "1", "9216"],
+                     ["8", "2048", "256", "1", "10240"], ["8", "2048", "256", "1", "1028"],
+                     ["8", "2048", "256", "1", "2052"],
                      # the product's stage ring with its data, no tensor core
                      ["7", "4096", "256", "4", "0"], ["7", "4096", "256", "4", "1"],
                      ["7", "4096", "256", "4", "2"], ["7", "4096", "256", "4", "3"],
