@@ -84,7 +84,7 @@ __device__ __forceinline__ void t8_loop(const PP &p, uint32_t tmem, uint64_t a0,
                                         uint64_t *bars, const volatile uint32_t *vz, bool &ok) {
     const bool on = (p.flags >> (kCode - 2)) & 1;
     uint32_t x = 1;
-    if (kCode >= 9) {
+    if constexpr (kCode >= 9) {
         const uint64_t da = 2 + (uint64_t)(p.flags & 1), db = 128 + (uint64_t)(p.flags & 2);
         for (int c = 0; c < p.iters; ++c) {
             const uint32_t so = (uint32_t)(c & 3) * (49152u >> 4);
@@ -99,8 +99,7 @@ __device__ __forceinline__ void t8_loop(const PP &p, uint32_t tmem, uint64_t a0,
             }
             umma_commit(&bars[c & 7]);
         }
-        return;
-    }
+    } else {
     for (int c = 0; c < p.iters; ++c) {
         uint32_t off = 0;
         if (on) {
@@ -124,6 +123,7 @@ __device__ __forceinline__ void t8_loop(const PP &p, uint32_t tmem, uint64_t a0,
         umma_f16_ss(tmem, a0 + 4, b0 + 256, idesc, 1u);
         umma_f16_ss(tmem, a0 + 6, b0 + 384, idesc, 1u);
         umma_commit(&bars[c & 7]);
+    }
     }
 }
 
