@@ -754,7 +754,7 @@ def run_workload(args):
                           f" cols {chunks * 64}", file=sys.stderr, flush=True)
         if bp.device_status() != bp.OK:
             raise RuntimeError("kernel watchdog fired")
-        out["timing"] = "device time of bp_conv2d (im2col + product), median of 9, L2 flushed"
+        out["timing"] = "device time of bp_conv2d (NHWC copy or im2col, then the product), median of 9, L2 flushed"
         print(json.dumps(out), flush=True)
         return
     elif name == "sweep":
