@@ -22,6 +22,7 @@ import ctypes
 import hashlib
 import json
 import os
+import re
 import statistics
 import sys
 import threading
@@ -54,10 +55,16 @@ def read_peaks() -> dict:
 
 
 def kernel_source_sha() -> str:
+    """Hash of the product kernel's code: its sources with comments and
+    whitespace removed, so that a comment-only edit keeps a recorded ncu
+    figure valid and any code change invalidates it."""
     h = hashlib.sha256()
     for f in ("bp_mma.cu", "bp_common.cuh", "bp_internal.h"):
-        with open(os.path.join(ROOT, "paper_2111_11581_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2111_11581_gb300", "csrc", f)) as fh:
+            src = fh.read()
+        src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+        src = re.sub(r"//[^\n]*", " ", src)
+        h.update("".join(src.split()).encode())
     return h.hexdigest()[:16]
 
 

@@ -1,5 +1,6 @@
-// Block-sparse product on the sm_103a tensor cores (bp_gemm, and bp_conv2d on
-// its im2col matrix).
+// Block-sparse product on the sm_103a tensor cores (bp_gemm, and bp_conv2d:
+// the implicit GEMM over an NHWC copy of the input, the NCHW planes in place
+// for 1 x 1 layers, or an im2col matrix).
 //
 // The packed weight is a sequence of 128-row slabs; a slab's column list is
 // the union of its rows' kept columns (Sec. 4.3: the rows of a row-block keep
@@ -14,18 +15,26 @@
 //               16-byte cp.async straight into the swizzled layout (one
 //               512-byte row segment per warp instruction), signalled with
 //               cp.async.mbarrier.arrive.noinc so no thread blocks on them;
-//   warp 8      control (one thread): copies the chunks' records (index list
-//               + load plan) into shared memory a window of kWin chunks at a
-//               time, one window ahead (TMA bulk copies), copies each stage's
-//               weight tile (TMA bulk), and when a chunk's list is made of runs
-//               of consecutive columns (its plan, built at pack time) loads the
-//               activation rows of each run with TMA tile loads;
+//   warp 8      control (one thread): per chunk, once its stage is free, sets
+//               the stage's flags, copies its weight tile (TMA bulk), and when
+//               the chunk's list is made of runs of consecutive columns (its
+//               plan, built at pack time) loads the activation rows of each
+//               run with TMA tile loads;
 //   warp 9      MMA issuer: tcgen05.mma 128 x 256 x 16 into one of two fp32
 //               accumulators in tensor memory (the epilogue of a tile
-//               overlaps the MMAs of the next);
+//               overlaps the MMAs of the next), following the stage flags;
 //   warps 10-13 epilogue: tcgen05.ld, + bias, ReLU, round to fp16/bf16, then
 //               TMA tensor stores of 32 x 32 boxes staged in shared memory
-//               (GEMM), or direct stores into the NCHW output (convolution).
+//               (GEMM), or direct stores into the NCHW output (convolution);
+//   warp 14     scheduler (one thread): the only role that decodes work
+//               units; copies the chunks' records (index list + load plan)
+//               into shared memory a window of kWin chunks at a time, with a
+//               descriptor the control thread and the gather warps follow,
+//               up to two windows ahead (TMA bulk copies).
+//
+// One mbarrier per stage says that the stage is loaded (the control thread's
+// arrival with the TMA byte count, and the gather group's arrivals); the
+// tensor-core thread's commit frees it.
 //
 // Every wait is bounded (see mbar_wait); on expiry the kernel records
 // kDevTimeout in the device status word, drains its own copies and tensor
@@ -45,11 +54,11 @@
 // clock64() at fixed points of each of its first kTraceChunks pipeline stages,
 // read back with bp_debug_trace_read().  Events per stage: 0 control thread
 // found the stage free, 1 gather group found it free, 2 gather group issued
-// its copies, 3 MMA thread saw the weight tile, 4 MMA thread saw the gathered
-// rows, 5 MMA thread committed the stage, 6 and 7 control thread before /
-// after issuing the weight copy.  Per window w (entries 256 + w): 0 control
-// thread at the window, 1 after copying the next window, 2 saw this window, 3
-// gather warp 0 saw it; per item i (entries 384 + i): 4 MMA thread holds a
+// its copies, 3 MMA thread saw the stage loaded, 4 control thread started
+// waiting for the stage, 5 MMA thread committed the stage, 6 and 7 control
+// thread before / after issuing the weight copy.  Per window w (entries 256 +
+// w): 0 control thread at the window, 2 it saw the window's records, 3 gather
+// warp 0 saw them; per item i (entries 384 + i): 4 MMA thread holds a
 // free accumulator, 5 the first epilogue warp saw the finished accumulator, 6
 // it issued the item's last store.  Entries 448 .. hold the global-timer start
 // and end of each of the first 248 CTAs; entry 511: CTA 0's clock64() after
