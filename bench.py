@@ -70,7 +70,7 @@ def kernel_source_sha() -> str:
 
 def recorded_traffic(workload: str):
     """DRAM bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel source; else None."""
+    on the current kernel code (see kernel_source_sha); else None."""
     p = os.path.join(ROOT, "profiles", "ncu_traffic.json")
     if not os.path.exists(p):
         return None
@@ -362,7 +362,7 @@ def run_ours(args):
     roof = {"bound": bound, "achieved": round(achieved, 2), "peak": peak, "unit": UNIT,
             "frac": round(achieved / peak, 4), "traffic": recorded_traffic(workload_name()),
             "traffic_note": "dram__bytes_read.sum + dram__bytes_write.sum of one launch under "
-                            "ncu (null unless taken on the current kernel source); the "
+                            "ncu (null unless taken on the current kernel code); the "
                             "output's write-back to DRAM happens after the kernel ends (Y "
                             "stays in L2), so it reads below the algorithmic bytes",
             "peak_source": f"{peaks['_source']} (bf16 burst)",
