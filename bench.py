@@ -54,13 +54,15 @@ def read_peaks() -> dict:
             "_source": "fallback"}
 
 
-def kernel_source_sha() -> str:
-    """Hash of the product kernel's code: its sources with comments and
-    whitespace removed, so that a comment-only edit keeps a recorded ncu
-    figure valid and any code change invalidates it."""
+def kernel_source_sha(csrc: str | None = None) -> str:
+    """Hash of the product kernel's code: its sources (in `csrc`, by default
+    the package's) with comments and whitespace removed, so that a
+    comment-only edit keeps a recorded ncu figure valid and any code change
+    invalidates it."""
+    csrc = csrc or os.path.join(ROOT, "paper_2111_11581_gb300", "csrc")
     h = hashlib.sha256()
     for f in ("bp_mma.cu", "bp_common.cuh", "bp_internal.h"):
-        with open(os.path.join(ROOT, "paper_2111_11581_gb300", "csrc", f)) as fh:
+        with open(os.path.join(csrc, f)) as fh:
             src = fh.read()
         src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
         src = re.sub(r"//[^\n]*", " ", src)

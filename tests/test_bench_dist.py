@@ -1,7 +1,8 @@
 """Host logic of the multi-rank benchmark on CPU: world_size-2 gloo ranks
 combine their local times and work the way bench.py does (whole-job units
 over the slowest rank's time), only rank 0 of the reference arm runs, and
-`bench.py --gpus 2` started without torchrun launches two ranks itself."""
+`bench.py --gpus 2` started without torchrun launches two ranks itself; and
+the key of the recorded ncu traffic follows the kernel's code only."""
 import json
 import os
 import socket
@@ -102,3 +103,24 @@ def test_gpus_flag_must_match_the_launch(monkeypatch):
                        cwd=ROOT)
     assert r.returncode != 0
     assert "WORLD_SIZE" in r.stderr
+
+
+def test_kernel_source_hash_ignores_comments_only(tmp_path):
+    """The recorded ncu traffic is keyed on the product kernel's code: a
+    comment or whitespace edit keeps the key, a code edit changes it."""
+    import shutil
+
+    sys.path.insert(0, ROOT)
+    import bench
+
+    src = os.path.join(ROOT, "paper_2111_11581_gb300", "csrc")
+    for f in ("bp_mma.cu", "bp_common.cuh", "bp_internal.h"):
+        shutil.copy(os.path.join(src, f), tmp_path / f)
+    base = bench.kernel_source_sha(str(tmp_path))
+    assert base == bench.kernel_source_sha()
+    p = tmp_path / "bp_internal.h"
+    text = p.read_text()
+    p.write_text("// a note\n/* a block\n   comment */\n" + text.replace("\n", "\n\n", 3))
+    assert bench.kernel_source_sha(str(tmp_path)) == base
+    p.write_text(text + "\nconstexpr int kUnused = 1;\n")
+    assert bench.kernel_source_sha(str(tmp_path)) != base
